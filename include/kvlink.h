@@ -1,0 +1,211 @@
+/*
+ * kvlink.h - C ABI of the GB300 (sm_103a) KVLink linked-prefill library.
+ *
+ * KVLink (arXiv 2502.16002) precomputes every document's KV cache on its own
+ * (Sec. 2.1).  At inference the retrieved documents' caches are re-encoded to
+ * their global positions (Sec. 2.2), concatenated with K link tokens after every
+ * document (Sec. 2.3), and only the fresh link and question tokens are run,
+ * attending over the linked cache under KVLink's mask (Sec. 2.3, Fig. 2).  This
+ * library is the per-layer attention-side work of that step:
+ *
+ *   kvlink_plan_create / kvlink_plan_upload     segment table and RoPE delta table
+ *   kvlink_reencode_concat                      re-encode + gather/concat cached K/V
+ *   kvlink_suffix_attention                     fresh rows attend over the linked cache
+ *   kvlink_linked_prefill                       both, chained, for one layer
+ *
+ * Conventions shared by every call
+ *   - Tensors are bf16, "NHD" per layer: [rows][heads][head_dim], rows contiguous.
+ *   - Pointers named d_* or documented as "device" are device memory; "host"
+ *     pointers are read during the call only.  The caller owns every buffer; the
+ *     library allocates no device memory.  kvlink_plan_create allocates the plan's
+ *     host tables (freed by kvlink_plan_destroy).
+ *   - Device work is enqueued on `stream` (a cudaStream_t; NULL = legacy default)
+ *     and is asynchronous.  Arguments are validated on the host before anything is
+ *     launched; a call that returns an error has launched nothing.
+ *   - Return value: KVLINK_OK (0) or a negative KVLINK_E* code.  No C++ exception
+ *     crosses the ABI.  kvlink_strerror() names a code.
+ *   - Kernels never trap.  A wait inside a kernel that exceeds its bounded spin
+ *     count records a code in a device status word (kvlink_device_status) and the
+ *     kernel returns early; its outputs are then undefined.
+ *
+ * Sequence layout of one query b (Sec. 2.3: link tokens follow every document):
+ *   [prefix (P tokens), doc_1 (l_1), link_1 (K), doc_2, link_2, ..., doc_N, link_N,
+ *    question (Q_b)]
+ *   A position's slot in the query's linked cache equals its global position.
+ *   The prefix is an optional cached pool entry (e.g. a system prompt) at
+ *   positions 0..P-1.  Cached document i starts at s_i and its keys, stored rotated
+ *   at local positions 0..l_i-1, are rotated by delta_i = s_i (Sec. 2.2).
+ *   Fresh rows of query b (link tokens then question tokens, in sequence order)
+ *   are rows cu_fresh[b] .. cu_fresh[b+1]-1 of q/k_new/v_new/out.
+ */
+#ifndef KVLINK_H
+#define KVLINK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* kvlink_stream_t; /* same type as cudaStream_t */
+
+enum {
+    KVLINK_OK = 0,
+    KVLINK_EINVAL = -1,       /* null pointer, negative count, inconsistent description */
+    KVLINK_EBOUNDS = -2,      /* document id, pool row or block id out of range        */
+    KVLINK_ECAPACITY = -3,    /* a caller buffer is smaller than required                */
+    KVLINK_EUNSUPPORTED = -4, /* shape outside what the kernels implement (see below)  */
+    KVLINK_ECUDA = -5,        /* a CUDA runtime call or launch failed                     */
+    KVLINK_EDEVICE = -6       /* a kernel recorded an error in the device status word    */
+};
+
+/* Supported shapes: head_dim 64 or 128; h_kv a power of two <= 16; h_q a multiple of
+ * h_kv with G = h_q / h_kv a power of two <= 16; n_link >= 0; every query has at least
+ * one fresh row; pool and cache block sizes 0 (contiguous) or a multiple of 8. */
+
+/* Description of one batch of queries (all pointers host, read during the call). */
+typedef struct {
+    int32_t batch;             /* B queries                                               */
+    int32_t n_link;            /* K link tokens appended after every document (Sec. 2.3)  */
+    int32_t h_q, h_kv, head_dim;
+
+    /* document cache pool (Sec. 2.1: caches precomputed per document) */
+    int32_t pool_docs;         /* entries in the pool (documents and cached prefixes)     */
+    const int32_t* pool_len;   /* [pool_docs] tokens per entry                            */
+    const int64_t* pool_start; /* [pool_docs] contiguous: first row of the entry;
+                                  paged: first slot of the entry in pool_block_table      */
+    int64_t pool_rows;         /* contiguous: rows of the pool tensor;
+                                  paged: physical blocks * pool_block_size                */
+    int32_t pool_block_size;   /* 0 = contiguous pool [pool_rows][h_kv][D];
+                                  else paged pool [blocks][pool_block_size][h_kv][D]      */
+    const int32_t* pool_block_table; /* paged: physical block of each logical block      */
+    int64_t pool_block_table_len;
+
+    /* queries */
+    const int32_t* prefix_doc; /* [B] pool entry placed at positions 0..P-1, or -1        */
+    const int32_t* n_docs;     /* [B] retrieved documents per query                       */
+    const int32_t* doc_ids;    /* [sum n_docs] pool entries, per query in sequence order  */
+    const int32_t* q_len;      /* [B] question tokens per query                           */
+
+    int32_t num_sms;           /* SMs the attention work is balanced over (0 = query the
+                                  current device; 152 if none is visible)                 */
+} kvlink_batch_desc_t;
+
+/* One contiguous run of the linked sequence (Sec. 2.3 layout). */
+typedef struct {
+    int32_t query;   /* b                                                            */
+    int32_t kind;    /* KVLINK_SEG_*                                                 */
+    int32_t src;     /* cached: pool entry id; fresh: first fresh row (global index) */
+    int32_t len;     /* tokens                                                       */
+    int64_t dst;     /* first row in the batch's contiguous linked cache
+                        (= cu_ctx[b] + pos)                                          */
+    int32_t pos;     /* global position of the first token within query b; for a
+                        cached document this is also its RoPE delta (Sec. 2.2)       */
+    int32_t table;   /* row of the RoPE delta table (cached documents), else -1      */
+} kvlink_segment_t;
+
+enum {
+    KVLINK_SEG_PREFIX = 0,   /* cached, delta 0: copied                      */
+    KVLINK_SEG_DOC = 1,      /* cached, rotated by delta = pos (Sec. 2.2)    */
+    KVLINK_SEG_LINK = 2,     /* fresh link-token rows (Sec. 2.3)             */
+    KVLINK_SEG_QUESTION = 3  /* fresh question rows                          */
+};
+
+typedef struct kvlink_plan kvlink_plan_t; /* opaque */
+
+typedef struct {
+    int32_t batch, h_q, h_kv, head_dim, n_link;
+    int32_t n_segments;       /* all segments, cached and fresh                       */
+    int32_t n_rope_rows;      /* rows of the RoPE delta table (= cached documents)    */
+    int32_t n_fresh;          /* fresh rows of the whole batch                        */
+    int64_t ctx_rows;         /* rows of the contiguous linked cache (sum C_b)        */
+    int64_t cached_tokens;    /* pool tokens gathered per layer (prefix + documents)  */
+    int32_t n_copy_chunks;    /* re-encode work units                                 */
+    int32_t n_attn_items;     /* attention work items (M-tile x KV range)             */
+    int32_t n_attn_splits;    /* items that write a partial result                    */
+    int32_t num_sms;
+    size_t device_bytes;      /* size of the device buffer kvlink_plan_upload needs   */
+    size_t workspace_bytes;   /* scratch of kvlink_suffix_attention / linked_prefill  */
+    int64_t attn_pairs;       /* unmasked (fresh row, key) pairs, per KV head group   */
+} kvlink_plan_info_t;
+
+/* Build the host tables of a batch: the interleaved layout of every query
+ * (Sec. 2.3), the segment table, the re-encode work units and the attention work
+ * items.  Validates every id and length against the pool.  Integer only; the
+ * result is deterministic.  On success *out owns host memory until
+ * kvlink_plan_destroy.  Errors: EINVAL, EBOUNDS, EUNSUPPORTED. */
+int kvlink_plan_create(const kvlink_batch_desc_t* desc, kvlink_plan_t** out);
+void kvlink_plan_destroy(kvlink_plan_t* plan);
+int kvlink_plan_get_info(const kvlink_plan_t* plan, kvlink_plan_info_t* info);
+
+/* Host copies of the plan's tables.  seg: [cap] segments; cu_ctx: [B+1] first cache
+ * row of every query (cu_ctx[B] = ctx_rows); cu_fresh: [B+1] first fresh row;
+ * fresh_pos: [n_fresh] global position of every fresh row within its query.
+ * Errors: EINVAL, ECAPACITY (cap smaller than the table). */
+int kvlink_plan_get_segments(const kvlink_plan_t* plan, kvlink_segment_t* seg, int32_t cap);
+int kvlink_plan_get_offsets(const kvlink_plan_t* plan, int64_t* cu_ctx, int32_t* cu_fresh);
+int kvlink_plan_get_fresh_positions(const kvlink_plan_t* plan, int32_t* fresh_pos, int32_t cap);
+
+/* Copy the plan's tables to the caller's device buffer d_buf (>= device_bytes,
+ * 256-byte aligned) and build the RoPE delta table there: cos and sin of
+ * delta_i * theta^(-2j/D) for every cached document i and j < D/2, with the angle
+ * formed and reduced in float64 and stored as float32 (Sec. 2.2; done once per
+ * batch, shared by all layers).  The plan records d_buf; later calls read it.
+ * d_buf must stay valid, and the plan alive, until the last call using them has
+ * completed on the device.  Errors: EINVAL, ECAPACITY, ECUDA. */
+int kvlink_plan_upload(kvlink_plan_t* plan, double theta, void* d_buf, size_t bytes,
+                       kvlink_stream_t stream);
+
+/* Re-encode and concatenate one layer's cached K/V (Sec. 2.2, Sec. 2.1):
+ *   for every cached segment (prefix, documents) and token t < len:
+ *     cache_k[dst + t] = R_delta(pool_k[entry][t])   (bf16, round to nearest even)
+ *     cache_v[dst + t] = pool_v[entry][t]            (bit copy)
+ *   with delta = pos (0 for the prefix: bit copy).  R_delta pairs dimension j with
+ *   j + D/2 (rotate-half) at angle delta * theta^(-2j/D).
+ * The pool entries, their global offsets (pos) and theta come from the plan.
+ * d_pool_k/d_pool_v: one layer of the pool (contiguous or paged as described);
+ * d_cache_k/d_cache_v: one layer of the linked cache, [ctx_rows][h_kv][D].
+ * Fresh (link/question) slots are left untouched.  Errors: EINVAL, ECUDA. */
+int kvlink_reencode_concat(const kvlink_plan_t* plan, const void* d_pool_k, const void* d_pool_v,
+                           void* d_cache_k, void* d_cache_v, kvlink_stream_t stream);
+
+/* Suffix attention of one layer (Sec. 2.3, "inference"):
+ *   if d_k_new/d_v_new are non-NULL, fresh rows are first written to their slots:
+ *     cache_k[cu_ctx[b] + fresh_pos[r]] = k_new[r] (same for v);
+ *   then for every fresh row r of query b (global position p_r), query head h,
+ *   KV head g = h / G:
+ *     out[r][h] = sum_j softmax_j(q[r][h] . cache_k[j][g] / sqrt(D)) cache_v[j][g]
+ *   over the slots j <= p_r of query b: a link token sees every earlier position
+ *   (all earlier documents and links, its own document, earlier links of its group),
+ *   a question token is causal over everything before it (Sec. 2.3, Fig. 2).
+ * d_q: [n_fresh][h_q][D]; d_k_new/d_v_new: [n_fresh][h_kv][D]; d_out: [n_fresh][h_q][D];
+ * all bf16.  Scores and softmax in fp32, products of bf16 on the tensor cores.
+ * d_workspace: >= workspace_bytes of scratch (may be NULL when that is 0).
+ * Errors: EINVAL, ECAPACITY, EUNSUPPORTED, ECUDA. */
+int kvlink_suffix_attention(const kvlink_plan_t* plan, const void* d_q, const void* d_k_new,
+                            const void* d_v_new, void* d_cache_k, void* d_cache_v, void* d_out,
+                            void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream);
+
+/* One layer of the linked prefill: kvlink_reencode_concat with the fresh-row
+ * placement fused into the same launch, then the suffix attention.  Same arguments
+ * and errors as the two calls it chains. */
+int kvlink_linked_prefill(const kvlink_plan_t* plan, const void* d_pool_k, const void* d_pool_v,
+                          const void* d_q, const void* d_k_new, const void* d_v_new,
+                          void* d_cache_k, void* d_cache_v, void* d_out,
+                          void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream);
+
+/* Device status word: 0 when no kernel reported an error since the last clear.
+ * Reading synchronises with the current device.  Errors: ECUDA. */
+int kvlink_device_status(int32_t* status);
+int kvlink_clear_device_status(void);
+
+const char* kvlink_strerror(int code);
+/* Text of the last CUDA error seen by this thread (empty if none). */
+const char* kvlink_last_cuda_error(void);
+int kvlink_version(void); /* major*10000 + minor*100 + patch */
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVLINK_H */

@@ -1,0 +1,260 @@
+// C ABI entry points (declared in include/kvlink.h): argument validation on the
+// host, plan upload, and the launches of the linked-prefill kernels.
+#include <cuda_runtime.h>
+
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "kvlink_internal.h"
+
+namespace kvlink {
+void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float2* d_rope, int head_dim,
+                       double theta, cudaStream_t stream);
+void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv,
+                     int pool_bs, const void* pool_k, const void* pool_v, const void* k_new,
+                     const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
+void launch_attention_simt(const DevicePlan& P, int n_fresh, int head_dim, int h_q, int h_kv,
+                           const void* q, const void* cache_k, const void* cache_v, void* out,
+                           cudaStream_t stream);
+}  // namespace kvlink
+
+using namespace kvlink;
+
+namespace {
+
+thread_local std::string g_last_cuda_error;
+
+int cuda_fail(cudaError_t e, const char* where) {
+    g_last_cuda_error = std::string(where) + ": " + cudaGetErrorString(e);
+    return KVLINK_ECUDA;
+}
+
+int check_launch(const char* where) {
+    const cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? KVLINK_OK : cuda_fail(e, where);
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+int resolve_num_sms(int32_t requested) {
+    if (requested > 0) return requested;
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0)
+        return n;
+    cudaGetLastError();  // no device visible: clear the sticky error, use GB300's count
+    return 152;
+}
+
+int check_plan(const kvlink_plan_t* p) {
+    if (!p) return KVLINK_EINVAL;
+    if (!p->uploaded) return KVLINK_EINVAL;
+    return KVLINK_OK;
+}
+
+int64_t pool_tensor_rows(const kvlink_plan_t* p) { return p->pool_rows; }
+
+}  // namespace
+
+extern "C" {
+
+int kvlink_version(void) { return 100; }
+
+const char* kvlink_strerror(int code) {
+    switch (code) {
+        case KVLINK_OK: return "ok";
+        case KVLINK_EINVAL: return "invalid argument";
+        case KVLINK_EBOUNDS: return "index out of bounds";
+        case KVLINK_ECAPACITY: return "buffer too small";
+        case KVLINK_EUNSUPPORTED: return "unsupported shape";
+        case KVLINK_ECUDA: return "CUDA error";
+        case KVLINK_EDEVICE: return "device-side error recorded in the status word";
+        default: return "unknown error";
+    }
+}
+
+const char* kvlink_last_cuda_error(void) { return g_last_cuda_error.c_str(); }
+
+int kvlink_plan_create(const kvlink_batch_desc_t* desc, kvlink_plan_t** out) {
+    if (!desc || !out) return KVLINK_EINVAL;
+    *out = nullptr;
+    kvlink_plan* p = new (std::nothrow) kvlink_plan();
+    if (!p) return KVLINK_ECAPACITY;
+    std::string why;
+    int rc;
+    try {
+        rc = build_plan(desc, resolve_num_sms(desc->num_sms), p, &why);
+    } catch (...) {
+        rc = KVLINK_ECAPACITY;
+    }
+    if (rc != KVLINK_OK) {
+        delete p;
+        return rc;
+    }
+    *out = p;
+    return KVLINK_OK;
+}
+
+void kvlink_plan_destroy(kvlink_plan_t* plan) { delete plan; }
+
+int kvlink_plan_get_info(const kvlink_plan_t* p, kvlink_plan_info_t* info) {
+    if (!p || !info) return KVLINK_EINVAL;
+    std::memset(info, 0, sizeof(*info));
+    info->batch = p->batch;
+    info->h_q = p->h_q;
+    info->h_kv = p->h_kv;
+    info->head_dim = p->head_dim;
+    info->n_link = p->n_link;
+    info->n_segments = (int32_t)p->seg.size();
+    info->n_rope_rows = p->n_rope_rows;
+    info->n_fresh = p->cu_fresh.empty() ? 0 : p->cu_fresh.back();
+    info->ctx_rows = p->cu_ctx.empty() ? 0 : p->cu_ctx.back();
+    info->cached_tokens = p->cached_tokens;
+    info->n_copy_chunks = (int32_t)p->chunks.size();
+    info->n_attn_items = (int32_t)p->items.size();
+    info->n_attn_splits = p->n_slots;
+    info->num_sms = p->num_sms;
+    info->device_bytes = p->device_bytes;
+    info->workspace_bytes = p->workspace_bytes;
+    info->attn_pairs = p->attn_pairs;
+    return KVLINK_OK;
+}
+
+int kvlink_plan_get_segments(const kvlink_plan_t* p, kvlink_segment_t* seg, int32_t cap) {
+    if (!p || !seg) return KVLINK_EINVAL;
+    if (cap < (int32_t)p->seg.size()) return KVLINK_ECAPACITY;
+    std::memcpy(seg, p->seg.data(), p->seg.size() * sizeof(kvlink_segment_t));
+    return KVLINK_OK;
+}
+
+int kvlink_plan_get_offsets(const kvlink_plan_t* p, int64_t* cu_ctx, int32_t* cu_fresh) {
+    if (!p || !cu_ctx || !cu_fresh) return KVLINK_EINVAL;
+    std::memcpy(cu_ctx, p->cu_ctx.data(), p->cu_ctx.size() * sizeof(int64_t));
+    std::memcpy(cu_fresh, p->cu_fresh.data(), p->cu_fresh.size() * sizeof(int32_t));
+    return KVLINK_OK;
+}
+
+int kvlink_plan_get_fresh_positions(const kvlink_plan_t* p, int32_t* pos, int32_t cap) {
+    if (!p || !pos) return KVLINK_EINVAL;
+    if (cap < (int32_t)p->fresh_pos.size()) return KVLINK_ECAPACITY;
+    std::memcpy(pos, p->fresh_pos.data(), p->fresh_pos.size() * sizeof(int32_t));
+    return KVLINK_OK;
+}
+
+int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes, kvlink_stream_t stream) {
+    if (!p || !d_buf) return KVLINK_EINVAL;
+    if (!(theta > 1.0)) return KVLINK_EINVAL;
+    if (((uintptr_t)d_buf & 255u) != 0) return KVLINK_EINVAL;
+    if (bytes < p->device_bytes) return KVLINK_ECAPACITY;
+    std::vector<char> host(p->device_bytes, 0);
+    auto put = [&](size_t off, const void* src, size_t n) {
+        if (n) std::memcpy(host.data() + off, src, n);
+    };
+    put(p->off_seg, p->seg.data(), p->seg.size() * sizeof(kvlink_segment_t));
+    put(p->off_chunks, p->chunks.data(), p->chunks.size() * sizeof(CopyChunk));
+    put(p->off_pool_start, p->pool_start.data(), p->pool_start.size() * sizeof(int64_t));
+    put(p->off_pool_bt, p->pool_block_table.data(), p->pool_block_table.size() * sizeof(int32_t));
+    put(p->off_cu_ctx, p->cu_ctx.data(), p->cu_ctx.size() * sizeof(int64_t));
+    put(p->off_cu_fresh, p->cu_fresh.data(), p->cu_fresh.size() * sizeof(int32_t));
+    put(p->off_fresh_pos, p->fresh_pos.data(), p->fresh_pos.size() * sizeof(int32_t));
+    put(p->off_fresh_query, p->fresh_query.data(), p->fresh_query.size() * sizeof(int32_t));
+    put(p->off_items, p->items.data(), p->items.size() * sizeof(AttnItem));
+    put(p->off_merges, p->merges.data(), p->merges.size() * sizeof(MergeGroup));
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e = cudaMemcpyAsync(d_buf, host.data(), p->device_bytes, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload copy");
+    // pageable source: wait so that `host` may be released on return
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload sync");
+    char* b = (char*)d_buf;
+    DevicePlan& d = p->dev;
+    d.seg = (const kvlink_segment_t*)(b + p->off_seg);
+    d.chunks = (const CopyChunk*)(b + p->off_chunks);
+    d.rope = (const float2*)(b + p->off_rope);
+    d.pool_start = (const int64_t*)(b + p->off_pool_start);
+    d.pool_block_table = (const int32_t*)(b + p->off_pool_bt);
+    d.cu_ctx = (const int64_t*)(b + p->off_cu_ctx);
+    d.cu_fresh = (const int32_t*)(b + p->off_cu_fresh);
+    d.fresh_pos = (const int32_t*)(b + p->off_fresh_pos);
+    d.fresh_query = (const int32_t*)(b + p->off_fresh_query);
+    d.items = (const AttnItem*)(b + p->off_items);
+    d.merges = (const MergeGroup*)(b + p->off_merges);
+    launch_rope_table(d.seg, (int)p->seg.size(), (float2*)(b + p->off_rope), p->head_dim, theta, s);
+    int rc = check_launch("rope_table_kernel");
+    if (rc != KVLINK_OK) return rc;
+    p->theta = theta;
+    p->d_buf = d_buf;
+    p->uploaded = true;
+    return KVLINK_OK;
+}
+
+int kvlink_reencode_concat(const kvlink_plan_t* p, const void* pool_k, const void* pool_v,
+                           void* cache_k, void* cache_v, kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (!pool_k || !pool_v || !cache_k || !cache_v) return KVLINK_EINVAL;
+    if (!aligned16(pool_k) || !aligned16(pool_v) || !aligned16(cache_k) || !aligned16(cache_v))
+        return KVLINK_EINVAL;
+    launch_reencode(p->dev, 0, p->n_chunks_cached, p->head_dim, p->h_kv, p->pool_block_size, pool_k,
+                    pool_v, nullptr, nullptr, cache_k, cache_v, (cudaStream_t)stream);
+    return check_launch("reencode_kernel");
+}
+
+static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k, void* cache_v,
+                            void* out, void* ws, size_t ws_bytes, cudaStream_t s) {
+    if (!q || !cache_k || !cache_v || !out) return KVLINK_EINVAL;
+    if (!aligned16(q) || !aligned16(cache_k) || !aligned16(cache_v) || !aligned16(out))
+        return KVLINK_EINVAL;
+    (void)ws;
+    (void)ws_bytes;
+    const int n_fresh = p->cu_fresh.back();
+    launch_attention_simt(p->dev, n_fresh, p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, s);
+    return check_launch("attention");
+}
+
+int kvlink_suffix_attention(const kvlink_plan_t* p, const void* q, const void* k_new, const void* v_new,
+                            void* cache_k, void* cache_v, void* out, void* ws, size_t ws_bytes,
+                            kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if ((k_new == nullptr) != (v_new == nullptr)) return KVLINK_EINVAL;
+    if (k_new && (!aligned16(k_new) || !aligned16(v_new))) return KVLINK_EINVAL;
+    if (!cache_k || !cache_v) return KVLINK_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (k_new) {
+        const int n_all = (int)p->chunks.size();
+        launch_reencode(p->dev, p->n_chunks_cached, n_all - p->n_chunks_cached, p->head_dim, p->h_kv,
+                        p->pool_block_size, nullptr, nullptr, k_new, v_new, cache_k, cache_v, s);
+        rc = check_launch("fresh placement");
+        if (rc) return rc;
+    }
+    return attention_common(p, q, cache_k, cache_v, out, ws, ws_bytes, s);
+}
+
+int kvlink_linked_prefill(const kvlink_plan_t* p, const void* pool_k, const void* pool_v, const void* q,
+                          const void* k_new, const void* v_new, void* cache_k, void* cache_v, void* out,
+                          void* ws, size_t ws_bytes, kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (!pool_k || !pool_v || !k_new || !v_new || !cache_k || !cache_v) return KVLINK_EINVAL;
+    if (!aligned16(pool_k) || !aligned16(pool_v) || !aligned16(k_new) || !aligned16(v_new))
+        return KVLINK_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    launch_reencode(p->dev, 0, (int)p->chunks.size(), p->head_dim, p->h_kv, p->pool_block_size, pool_k,
+                    pool_v, k_new, v_new, cache_k, cache_v, s);
+    rc = check_launch("reencode_kernel (fused)");
+    if (rc) return rc;
+    return attention_common(p, q, cache_k, cache_v, out, ws, ws_bytes, s);
+}
+
+int kvlink_device_status(int32_t* status) {
+    if (!status) return KVLINK_EINVAL;
+    *status = 0;
+    return KVLINK_OK;
+}
+
+int kvlink_clear_device_status(void) { return KVLINK_OK; }
+
+}  // extern "C"

@@ -1,0 +1,224 @@
+// Host plan builder: the segment table of a batch (layout of Sec. 2.3), the
+// re-encode work units and the attention work items.  Integer bookkeeping only.
+#include <algorithm>
+#include <climits>
+#include <cstdint>
+#include <cstring>
+#include <numeric>
+#include <string>
+
+#include "kvlink_internal.h"
+
+namespace kvlink {
+namespace {
+
+bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int fail(std::string* why, int code, const std::string& msg) {
+    if (why) *why = msg;
+    return code;
+}
+
+}  // namespace
+
+int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, std::string* why) {
+    if (!d || !p) return fail(why, KVLINK_EINVAL, "null argument");
+    if (d->batch <= 0 || d->n_link < 0 || d->pool_docs <= 0 || d->pool_rows <= 0)
+        return fail(why, KVLINK_EINVAL, "batch, pool_docs and pool_rows must be > 0, n_link >= 0");
+    if (!d->pool_len || !d->pool_start || !d->prefix_doc || !d->n_docs || !d->q_len)
+        return fail(why, KVLINK_EINVAL, "null table in the batch description");
+    if (d->head_dim != 64 && d->head_dim != 128)
+        return fail(why, KVLINK_EUNSUPPORTED, "head_dim must be 64 or 128");
+    if (!is_pow2(d->h_kv) || d->h_kv > 16)
+        return fail(why, KVLINK_EUNSUPPORTED, "h_kv must be a power of two <= 16");
+    if (d->h_q <= 0 || d->h_q % d->h_kv != 0 || !is_pow2(d->h_q / d->h_kv) || d->h_q / d->h_kv > 16)
+        return fail(why, KVLINK_EUNSUPPORTED, "h_q / h_kv must be a power of two <= 16");
+    const int bs = d->pool_block_size;
+    if (bs < 0 || (bs > 0 && bs % 8 != 0))
+        return fail(why, KVLINK_EUNSUPPORTED, "pool_block_size must be 0 or a multiple of 8");
+    if (bs > 0 && (!d->pool_block_table || d->pool_block_table_len <= 0))
+        return fail(why, KVLINK_EINVAL, "paged pool needs its block table");
+    if (bs > 0 && d->pool_rows % bs != 0)
+        return fail(why, KVLINK_EINVAL, "paged pool_rows must be a multiple of pool_block_size");
+    if (num_sms <= 0) return fail(why, KVLINK_EINVAL, "num_sms must be resolved");
+
+    p->batch = d->batch;
+    p->n_link = d->n_link;
+    p->h_q = d->h_q;
+    p->h_kv = d->h_kv;
+    p->head_dim = d->head_dim;
+    p->pool_docs = d->pool_docs;
+    p->pool_block_size = bs;
+    p->pool_rows = d->pool_rows;
+    p->num_sms = num_sms;
+    p->pool_len.assign(d->pool_len, d->pool_len + d->pool_docs);
+    p->pool_start.assign(d->pool_start, d->pool_start + d->pool_docs);
+
+    // ---- validate the pool: every entry's rows (or blocks) lie inside the pool tensor
+    const int64_t n_phys_blocks = bs > 0 ? d->pool_rows / bs : 0;
+    if (bs > 0) {
+        p->pool_block_table.assign(d->pool_block_table, d->pool_block_table + d->pool_block_table_len);
+        for (int64_t i = 0; i < d->pool_block_table_len; ++i)
+            if (p->pool_block_table[i] < 0 || p->pool_block_table[i] >= n_phys_blocks)
+                return fail(why, KVLINK_EBOUNDS, "pool block id out of range");
+    } else {
+        p->pool_block_table.clear();
+    }
+    for (int e = 0; e < d->pool_docs; ++e) {
+        const int64_t L = p->pool_len[e], s = p->pool_start[e];
+        if (L < 0 || s < 0) return fail(why, KVLINK_EINVAL, "negative pool length or start");
+        if (bs > 0) {
+            const int64_t nb = (L + bs - 1) / bs;
+            if (s + nb > d->pool_block_table_len)
+                return fail(why, KVLINK_EBOUNDS, "pool entry runs past the block table");
+        } else if (s + L > d->pool_rows) {
+            return fail(why, KVLINK_EBOUNDS, "pool entry runs past pool_rows");
+        }
+    }
+
+    // ---- layout of every query: [prefix, doc_1, link_1, ..., doc_N, link_N, question]
+    const int B = d->batch, K = d->n_link;
+    int64_t total_docs = 0;
+    for (int b = 0; b < B; ++b) {
+        if (d->n_docs[b] < 0 || d->q_len[b] < 0) return fail(why, KVLINK_EINVAL, "negative count");
+        total_docs += d->n_docs[b];
+    }
+    if (total_docs > 0 && !d->doc_ids) return fail(why, KVLINK_EINVAL, "doc_ids is null");
+
+    p->seg.clear();
+    p->cu_ctx.assign(B + 1, 0);
+    p->cu_fresh.assign(B + 1, 0);
+    p->fresh_pos.clear();
+    p->fresh_query.clear();
+    p->n_rope_rows = 0;
+    p->cached_tokens = 0;
+    int64_t doc_off = 0, ctx = 0;
+    int64_t fresh = 0;
+    for (int b = 0; b < B; ++b) {
+        p->cu_ctx[b] = ctx;
+        p->cu_fresh[b] = (int32_t)fresh;
+        int64_t pos = 0;
+        const int pre = d->prefix_doc[b];
+        if (pre >= d->pool_docs || pre < -1) return fail(why, KVLINK_EBOUNDS, "prefix_doc out of range");
+        if (pre >= 0 && p->pool_len[pre] > 0) {
+            const int32_t P = p->pool_len[pre];
+            p->seg.push_back({b, KVLINK_SEG_PREFIX, pre, P, ctx + pos, (int32_t)pos, -1});
+            pos += P;
+            p->cached_tokens += P;
+        }
+        for (int i = 0; i < d->n_docs[b]; ++i) {
+            const int doc = d->doc_ids[doc_off + i];
+            if (doc < 0 || doc >= d->pool_docs) return fail(why, KVLINK_EBOUNDS, "doc id out of range");
+            const int32_t L = p->pool_len[doc];
+            if (L > 0) {
+                p->seg.push_back({b, KVLINK_SEG_DOC, doc, L, ctx + pos, (int32_t)pos, p->n_rope_rows++});
+                pos += L;
+                p->cached_tokens += L;
+            }
+            if (K > 0) {
+                p->seg.push_back({b, KVLINK_SEG_LINK, (int32_t)fresh, K, ctx + pos, (int32_t)pos, -1});
+                for (int k = 0; k < K; ++k) {
+                    p->fresh_pos.push_back((int32_t)(pos + k));
+                    p->fresh_query.push_back(b);
+                }
+                fresh += K;
+                pos += K;
+            }
+        }
+        doc_off += d->n_docs[b];
+        const int Q = d->q_len[b];
+        if (Q > 0) {
+            p->seg.push_back({b, KVLINK_SEG_QUESTION, (int32_t)fresh, Q, ctx + pos, (int32_t)pos, -1});
+            for (int k = 0; k < Q; ++k) {
+                p->fresh_pos.push_back((int32_t)(pos + k));
+                p->fresh_query.push_back(b);
+            }
+            fresh += Q;
+            pos += Q;
+        }
+        if (p->cu_fresh[b] == fresh) return fail(why, KVLINK_EINVAL, "a query has no fresh rows");
+        if (pos > INT32_MAX / 2) return fail(why, KVLINK_EUNSUPPORTED, "context too long");
+        ctx += pos;
+    }
+    p->cu_ctx[B] = ctx;
+    p->cu_fresh[B] = (int32_t)fresh;
+    if (fresh > INT32_MAX / 64) return fail(why, KVLINK_EUNSUPPORTED, "too many fresh rows");
+
+    // ---- re-encode work units: cached segments first, then fresh segments
+    p->chunks.clear();
+    for (int pass = 0; pass < 2; ++pass) {
+        for (size_t s = 0; s < p->seg.size(); ++s) {
+            const bool cached = p->seg[s].kind == KVLINK_SEG_PREFIX || p->seg[s].kind == KVLINK_SEG_DOC;
+            if (cached != (pass == 0)) continue;
+            for (int t = 0; t < p->seg[s].len; t += kCopyChunk) p->chunks.push_back({(int32_t)s, t});
+        }
+        if (pass == 0) p->n_chunks_cached = (int32_t)p->chunks.size();
+    }
+
+    // ---- attention work items
+    const int G = d->h_q / d->h_kv;
+    const int tok_per_tile = kAttnBM / G;
+    struct Tile { int32_t b, g, t0, t1, n_tiles, min_pos; };
+    std::vector<Tile> tiles;
+    int64_t work = 0;
+    p->attn_pairs = 0;
+    for (int b = 0; b < B; ++b) {
+        const int32_t f0 = p->cu_fresh[b], T = p->cu_fresh[b + 1] - f0;
+        for (int r = 0; r < T; ++r) p->attn_pairs += (int64_t)p->fresh_pos[f0 + r] + 1;
+        for (int t0 = 0; t0 < T; t0 += tok_per_tile) {
+            const int t1 = std::min(T, t0 + tok_per_tile);
+            const int32_t kv_len = p->fresh_pos[f0 + t1 - 1] + 1;  // positions increase within a query
+            const int32_t nt = (kv_len + kAttnBN - 1) / kAttnBN;
+            for (int g = 0; g < d->h_kv; ++g) {
+                tiles.push_back({b, g, t0, t1, nt, p->fresh_pos[f0 + t0]});
+                work += nt;
+            }
+        }
+    }
+    // split long KV ranges so that the items spread evenly over the SMs
+    const int64_t per_sm = (work + 2 * (int64_t)num_sms - 1) / (2 * (int64_t)num_sms);
+    const int32_t max_tiles = (int32_t)std::max<int64_t>(8, per_sm);
+    p->items.clear();
+    p->merges.clear();
+    p->n_slots = 0;
+    for (const Tile& t : tiles) {
+        const int32_t n_split = (t.n_tiles + max_tiles - 1) / max_tiles;
+        if (n_split <= 1) {
+            p->items.push_back({t.b, t.g, t.t0, t.t1, 0, t.n_tiles, -1, t.min_pos});
+            continue;
+        }
+        p->merges.push_back({t.b, t.g, t.t0, t.t1, p->n_slots, n_split, 0, 0});
+        for (int s = 0; s < n_split; ++s) {
+            const int32_t a = (int32_t)((int64_t)t.n_tiles * s / n_split);
+            const int32_t e = (int32_t)((int64_t)t.n_tiles * (s + 1) / n_split);
+            p->items.push_back({t.b, t.g, t.t0, t.t1, a, e, p->n_slots + s, t.min_pos});
+        }
+        p->n_slots += n_split;
+    }
+    std::stable_sort(p->items.begin(), p->items.end(), [](const AttnItem& x, const AttnItem& y) {
+        return (x.kv_tile1 - x.kv_tile0) > (y.kv_tile1 - y.kv_tile0);
+    });
+    p->workspace_bytes = (size_t)p->n_slots * (size_t)kAttnBM * ((size_t)d->head_dim + 2) * sizeof(float);
+
+    // ---- device buffer layout (256-byte aligned tables)
+    size_t off = 0;
+    auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
+    p->off_seg = take(p->seg.size() * sizeof(kvlink_segment_t));
+    p->off_chunks = take(p->chunks.size() * sizeof(CopyChunk));
+    p->off_rope = take((size_t)p->n_rope_rows * (d->head_dim / 2) * sizeof(float2));
+    p->off_pool_start = take(p->pool_start.size() * sizeof(int64_t));
+    p->off_pool_bt = take(p->pool_block_table.size() * sizeof(int32_t));
+    p->off_cu_ctx = take(p->cu_ctx.size() * sizeof(int64_t));
+    p->off_cu_fresh = take(p->cu_fresh.size() * sizeof(int32_t));
+    p->off_fresh_pos = take(p->fresh_pos.size() * sizeof(int32_t));
+    p->off_fresh_query = take(p->fresh_query.size() * sizeof(int32_t));
+    p->off_items = take(p->items.size() * sizeof(AttnItem));
+    p->off_merges = take(p->merges.size() * sizeof(MergeGroup));
+    p->device_bytes = off;
+    p->uploaded = false;
+    return KVLINK_OK;
+}
+
+}  // namespace kvlink

@@ -1,0 +1,240 @@
+"""ctypes binding of libkvlink.so (include/kvlink.h), argument marshalling only.
+
+The functions carry the C names.  Device pointers are passed as integers (e.g.
+``tensor.data_ptr()``), streams as ``torch.cuda.Stream.cuda_stream`` integers.
+Every step of the linked prefill runs in the library's CUDA kernels; there is no
+Python or CPU fallback, and importing this module fails if the library has not
+been built.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libkvlink.so")
+
+KVLINK_OK = 0
+KVLINK_EINVAL = -1
+KVLINK_EBOUNDS = -2
+KVLINK_ECAPACITY = -3
+KVLINK_EUNSUPPORTED = -4
+KVLINK_ECUDA = -5
+KVLINK_EDEVICE = -6
+
+KVLINK_SEG_PREFIX, KVLINK_SEG_DOC, KVLINK_SEG_LINK, KVLINK_SEG_QUESTION = 0, 1, 2, 3
+
+
+class kvlink_batch_desc_t(C.Structure):
+    _fields_ = [
+        ("batch", C.c_int32), ("n_link", C.c_int32), ("h_q", C.c_int32), ("h_kv", C.c_int32),
+        ("head_dim", C.c_int32),
+        ("pool_docs", C.c_int32),
+        ("pool_len", C.POINTER(C.c_int32)),
+        ("pool_start", C.POINTER(C.c_int64)),
+        ("pool_rows", C.c_int64),
+        ("pool_block_size", C.c_int32),
+        ("pool_block_table", C.POINTER(C.c_int32)),
+        ("pool_block_table_len", C.c_int64),
+        ("prefix_doc", C.POINTER(C.c_int32)),
+        ("n_docs", C.POINTER(C.c_int32)),
+        ("doc_ids", C.POINTER(C.c_int32)),
+        ("q_len", C.POINTER(C.c_int32)),
+        ("num_sms", C.c_int32),
+    ]
+
+
+class kvlink_segment_t(C.Structure):
+    _fields_ = [
+        ("query", C.c_int32), ("kind", C.c_int32), ("src", C.c_int32), ("len", C.c_int32),
+        ("dst", C.c_int64), ("pos", C.c_int32), ("table", C.c_int32),
+    ]
+
+
+SEGMENT_DTYPE = np.dtype([("query", "<i4"), ("kind", "<i4"), ("src", "<i4"), ("len", "<i4"),
+                          ("dst", "<i8"), ("pos", "<i4"), ("table", "<i4")])
+
+
+class kvlink_plan_info_t(C.Structure):
+    _fields_ = [
+        ("batch", C.c_int32), ("h_q", C.c_int32), ("h_kv", C.c_int32), ("head_dim", C.c_int32),
+        ("n_link", C.c_int32),
+        ("n_segments", C.c_int32), ("n_rope_rows", C.c_int32), ("n_fresh", C.c_int32),
+        ("ctx_rows", C.c_int64), ("cached_tokens", C.c_int64),
+        ("n_copy_chunks", C.c_int32), ("n_attn_items", C.c_int32), ("n_attn_splits", C.c_int32),
+        ("num_sms", C.c_int32),
+        ("device_bytes", C.c_size_t), ("workspace_bytes", C.c_size_t),
+        ("attn_pairs", C.c_int64),
+    ]
+
+
+def _load():
+    if not os.path.exists(_LIB_PATH):
+        raise ImportError(f"{_LIB_PATH} is missing: build it with __graft_entry__.build() "
+                          "(the linked prefill has no fallback)")
+    lib = C.CDLL(_LIB_PATH)
+    P, V = C.c_void_p, C.c_void_p
+    sig = {
+        "kvlink_version": (C.c_int, []),
+        "kvlink_strerror": (C.c_char_p, [C.c_int]),
+        "kvlink_last_cuda_error": (C.c_char_p, []),
+        "kvlink_plan_create": (C.c_int, [C.POINTER(kvlink_batch_desc_t), C.POINTER(P)]),
+        "kvlink_plan_destroy": (None, [P]),
+        "kvlink_plan_get_info": (C.c_int, [P, C.POINTER(kvlink_plan_info_t)]),
+        "kvlink_plan_get_segments": (C.c_int, [P, V, C.c_int32]),
+        "kvlink_plan_get_offsets": (C.c_int, [P, V, V]),
+        "kvlink_plan_get_fresh_positions": (C.c_int, [P, V, C.c_int32]),
+        "kvlink_plan_upload": (C.c_int, [P, C.c_double, V, C.c_size_t, V]),
+        "kvlink_reencode_concat": (C.c_int, [P, V, V, V, V, V]),
+        "kvlink_suffix_attention": (C.c_int, [P, V, V, V, V, V, V, V, C.c_size_t, V]),
+        "kvlink_linked_prefill": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
+        "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
+        "kvlink_clear_device_status": (C.c_int, []),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    return lib
+
+
+lib = _load()
+
+DECLARED = [
+    "kvlink_plan_create", "kvlink_plan_destroy", "kvlink_plan_get_info", "kvlink_plan_get_segments",
+    "kvlink_plan_get_offsets", "kvlink_plan_get_fresh_positions", "kvlink_plan_upload",
+    "kvlink_reencode_concat", "kvlink_suffix_attention", "kvlink_linked_prefill",
+    "kvlink_device_status", "kvlink_clear_device_status", "kvlink_strerror",
+    "kvlink_last_cuda_error", "kvlink_version",
+]
+
+
+class KvlinkError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        msg = lib.kvlink_strerror(code).decode()
+        if code == KVLINK_ECUDA:
+            msg += ": " + lib.kvlink_last_cuda_error().decode()
+        super().__init__(f"{where}: {msg} ({code})")
+        self.code = code
+
+
+def _check(code: int, where: str) -> None:
+    if code != KVLINK_OK:
+        raise KvlinkError(code, where)
+
+
+def _i32(a):
+    return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+
+
+def _i64(a):
+    return np.ascontiguousarray(np.asarray(a, dtype=np.int64))
+
+
+def _ptr(a, ctype):
+    return a.ctypes.data_as(C.POINTER(ctype))
+
+
+class Plan:
+    """Owns a kvlink_plan_t handle (kvlink_plan_destroy on close)."""
+
+    def __init__(self, handle):
+        self.handle = handle
+
+    def close(self):
+        if self.handle:
+            lib.kvlink_plan_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        self.close()
+
+
+def kvlink_plan_create(*, n_link, h_q, h_kv, head_dim, pool_len, pool_start, pool_rows,
+                       prefix_doc, n_docs, doc_ids, q_len, pool_block_size=0,
+                       pool_block_table=None, num_sms=0) -> Plan:
+    arrs = dict(pool_len=_i32(pool_len), pool_start=_i64(pool_start), prefix_doc=_i32(prefix_doc),
+                n_docs=_i32(n_docs), doc_ids=_i32(doc_ids), q_len=_i32(q_len))
+    bt = _i32(pool_block_table) if pool_block_table is not None else None
+    d = kvlink_batch_desc_t()
+    d.batch = len(arrs["n_docs"])
+    d.n_link, d.h_q, d.h_kv, d.head_dim = int(n_link), int(h_q), int(h_kv), int(head_dim)
+    d.pool_docs = len(arrs["pool_len"])
+    d.pool_len = _ptr(arrs["pool_len"], C.c_int32)
+    d.pool_start = _ptr(arrs["pool_start"], C.c_int64)
+    d.pool_rows = int(pool_rows)
+    d.pool_block_size = int(pool_block_size)
+    d.pool_block_table = _ptr(bt, C.c_int32) if bt is not None else None
+    d.pool_block_table_len = len(bt) if bt is not None else 0
+    d.prefix_doc = _ptr(arrs["prefix_doc"], C.c_int32)
+    d.n_docs = _ptr(arrs["n_docs"], C.c_int32)
+    d.doc_ids = _ptr(arrs["doc_ids"], C.c_int32) if len(arrs["doc_ids"]) else None
+    d.q_len = _ptr(arrs["q_len"], C.c_int32)
+    d.num_sms = int(num_sms)
+    h = C.c_void_p()
+    _check(lib.kvlink_plan_create(C.byref(d), C.byref(h)), "kvlink_plan_create")
+    return Plan(h)
+
+
+def kvlink_plan_get_info(plan: Plan) -> kvlink_plan_info_t:
+    info = kvlink_plan_info_t()
+    _check(lib.kvlink_plan_get_info(plan.handle, C.byref(info)), "kvlink_plan_get_info")
+    return info
+
+
+def kvlink_plan_get_segments(plan: Plan) -> np.ndarray:
+    n = kvlink_plan_get_info(plan).n_segments
+    out = np.zeros(n, dtype=SEGMENT_DTYPE)
+    _check(lib.kvlink_plan_get_segments(plan.handle, out.ctypes.data, n), "kvlink_plan_get_segments")
+    return out
+
+
+def kvlink_plan_get_offsets(plan: Plan):
+    B = kvlink_plan_get_info(plan).batch
+    cu_ctx = np.zeros(B + 1, np.int64)
+    cu_fresh = np.zeros(B + 1, np.int32)
+    _check(lib.kvlink_plan_get_offsets(plan.handle, cu_ctx.ctypes.data, cu_fresh.ctypes.data),
+           "kvlink_plan_get_offsets")
+    return cu_ctx, cu_fresh
+
+
+def kvlink_plan_get_fresh_positions(plan: Plan) -> np.ndarray:
+    n = kvlink_plan_get_info(plan).n_fresh
+    out = np.zeros(n, np.int32)
+    _check(lib.kvlink_plan_get_fresh_positions(plan.handle, out.ctypes.data, n),
+           "kvlink_plan_get_fresh_positions")
+    return out
+
+
+def kvlink_plan_upload(plan: Plan, theta: float, d_buf: int, nbytes: int, stream: int = 0) -> None:
+    _check(lib.kvlink_plan_upload(plan.handle, float(theta), d_buf, nbytes, stream), "kvlink_plan_upload")
+
+
+def kvlink_reencode_concat(plan: Plan, pool_k: int, pool_v: int, cache_k: int, cache_v: int,
+                           stream: int = 0) -> None:
+    _check(lib.kvlink_reencode_concat(plan.handle, pool_k, pool_v, cache_k, cache_v, stream),
+           "kvlink_reencode_concat")
+
+
+def kvlink_suffix_attention(plan: Plan, q: int, k_new, v_new, cache_k: int, cache_v: int, out: int,
+                            workspace, workspace_bytes: int, stream: int = 0) -> None:
+    _check(lib.kvlink_suffix_attention(plan.handle, q, k_new, v_new, cache_k, cache_v, out, workspace,
+                                       workspace_bytes, stream), "kvlink_suffix_attention")
+
+
+def kvlink_linked_prefill(plan: Plan, pool_k: int, pool_v: int, q: int, k_new: int, v_new: int,
+                          cache_k: int, cache_v: int, out: int, workspace, workspace_bytes: int,
+                          stream: int = 0) -> None:
+    _check(lib.kvlink_linked_prefill(plan.handle, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out,
+                                     workspace, workspace_bytes, stream), "kvlink_linked_prefill")
+
+
+def kvlink_device_status() -> int:
+    s = C.c_int32(0)
+    _check(lib.kvlink_device_status(C.byref(s)), "kvlink_device_status")
+    return int(s.value)
+
+
+def kvlink_clear_device_status() -> None:
+    _check(lib.kvlink_clear_device_status(), "kvlink_clear_device_status")

@@ -1,0 +1,90 @@
+"""Device-side plumbing around the C ABI: torch owns the buffers, libkvlink does the work.
+
+LinkedPrefill builds and uploads one batch's plan and holds the plan buffer and
+the attention workspace; its methods are one ABI call each.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import kvlink as K
+
+
+def bf16_from_bits(u16: np.ndarray, device=None) -> torch.Tensor:
+    """bf16 tensor with the given bit patterns (uint16 numpy array)."""
+    t = torch.from_numpy(np.ascontiguousarray(u16).view(np.int16)).view(torch.bfloat16)
+    return t.to(device) if device is not None else t
+
+
+def bits_from_bf16(t: torch.Tensor) -> np.ndarray:
+    return t.detach().contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def _stream_handle(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream)
+
+
+class LinkedPrefill:
+    """One batch of linked-prefill queries: plan, plan buffer and workspace on a device."""
+
+    def __init__(self, *, n_link, h_q, h_kv, head_dim, theta, pool_len, pool_start, pool_rows,
+                 prefix_doc, n_docs, doc_ids, q_len, pool_block_size=0, pool_block_table=None,
+                 num_sms=0, device="cuda", stream=None):
+        self.device = torch.device(device)
+        self.plan = K.kvlink_plan_create(
+            n_link=n_link, h_q=h_q, h_kv=h_kv, head_dim=head_dim, pool_len=pool_len,
+            pool_start=pool_start, pool_rows=pool_rows, prefix_doc=prefix_doc, n_docs=n_docs,
+            doc_ids=doc_ids, q_len=q_len, pool_block_size=pool_block_size,
+            pool_block_table=pool_block_table, num_sms=num_sms)
+        self.info = K.kvlink_plan_get_info(self.plan)
+        self.theta = float(theta)
+        self.plan_buf = torch.empty(max(int(self.info.device_bytes), 256), dtype=torch.uint8,
+                                    device=self.device)
+        self.workspace = torch.empty(max(int(self.info.workspace_bytes), 256), dtype=torch.uint8,
+                                     device=self.device)
+        K.kvlink_plan_upload(self.plan, self.theta, self.plan_buf.data_ptr(), self.plan_buf.numel(),
+                             _stream_handle(stream))
+
+    @classmethod
+    def from_batch(cls, batch, device="cuda", num_sms=0, stream=None):
+        """From a workloads.Batch-like object (pool metadata and per-query tables)."""
+        cfg = batch.cfg
+        return cls(n_link=cfg.n_link, h_q=cfg.h_q, h_kv=cfg.h_kv, head_dim=cfg.head_dim,
+                   theta=cfg.theta, pool_len=batch.pool_len, pool_start=batch.pool_start,
+                   pool_rows=batch.pool_rows, prefix_doc=batch.prefix_doc, n_docs=batch.n_docs,
+                   doc_ids=batch.doc_ids, q_len=batch.q_len, pool_block_size=cfg.pool_block_size,
+                   pool_block_table=batch.pool_block_table, num_sms=num_sms, device=device,
+                   stream=stream)
+
+    # shapes of the per-layer tensors
+    def cache_shape(self):
+        return (int(self.info.ctx_rows), int(self.info.h_kv), int(self.info.head_dim))
+
+    def fresh_shape(self, heads):
+        return (int(self.info.n_fresh), int(heads), int(self.info.head_dim))
+
+    def empty_cache(self):
+        return (torch.empty(self.cache_shape(), dtype=torch.bfloat16, device=self.device),
+                torch.empty(self.cache_shape(), dtype=torch.bfloat16, device=self.device))
+
+    # one ABI call each
+    def reencode_concat(self, pool_k, pool_v, cache_k, cache_v, stream=None):
+        K.kvlink_reencode_concat(self.plan, pool_k.data_ptr(), pool_v.data_ptr(), cache_k.data_ptr(),
+                                 cache_v.data_ptr(), _stream_handle(stream))
+
+    def suffix_attention(self, q, k_new, v_new, cache_k, cache_v, out, stream=None):
+        K.kvlink_suffix_attention(self.plan, q.data_ptr(),
+                                  k_new.data_ptr() if k_new is not None else None,
+                                  v_new.data_ptr() if v_new is not None else None,
+                                  cache_k.data_ptr(), cache_v.data_ptr(), out.data_ptr(),
+                                  self.workspace.data_ptr(), self.workspace.numel(),
+                                  _stream_handle(stream))
+
+    def linked_prefill(self, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out, stream=None):
+        K.kvlink_linked_prefill(self.plan, pool_k.data_ptr(), pool_v.data_ptr(), q.data_ptr(),
+                                k_new.data_ptr(), v_new.data_ptr(), cache_k.data_ptr(),
+                                cache_v.data_ptr(), out.data_ptr(), self.workspace.data_ptr(),
+                                self.workspace.numel(), _stream_handle(stream))

@@ -1,0 +1,160 @@
+"""Host-side tests of the C ABI (no GPU): symbol exports, the segment table and
+offsets against the oracle's layout (bit-exact), attention work coverage, and
+argument validation."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle as O
+import workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def K():
+    from paper_2502_16002_gb300.build import build
+
+    build()
+    from paper_2502_16002_gb300 import kvlink
+
+    return kvlink
+
+
+def _declared_functions():
+    src = open(os.path.join(ROOT, "include", "kvlink.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(kvlink_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_function(K):
+    names = _declared_functions()
+    assert len(names) >= 15
+    lib = ctypes.CDLL(K._LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(K.DECLARED)
+
+
+def _plan(K, batch, **over):
+    cfg = batch.cfg
+    kw = dict(n_link=cfg.n_link, h_q=cfg.h_q, h_kv=cfg.h_kv, head_dim=cfg.head_dim,
+              pool_len=batch.pool_len, pool_start=batch.pool_start, pool_rows=batch.pool_rows,
+              prefix_doc=batch.prefix_doc, n_docs=batch.n_docs, doc_ids=batch.doc_ids,
+              q_len=batch.q_len, pool_block_size=cfg.pool_block_size,
+              pool_block_table=batch.pool_block_table, num_sms=152)
+    kw.update(over)
+    return K.kvlink_plan_create(**kw)
+
+
+def _oracle_layout(batch, b):
+    cfg = batch.cfg
+    P = int(batch.pool_len[batch.prefix_doc[b]]) if batch.prefix_doc[b] >= 0 else 0
+    return O.linked_layout(P, [int(batch.pool_len[d]) for d in batch.docs_of(b)], cfg.n_link,
+                           int(batch.q_len[b]))
+
+
+@pytest.mark.parametrize("cfg_index", [1, 2, 3, 4, 5])
+def test_segment_table_matches_oracle_layout(K, cfg_index):
+    batch = W.draw_batch(W.get_config(cfg_index))
+    plan = _plan(K, batch)
+    seg = K.kvlink_plan_get_segments(plan)
+    cu_ctx, cu_fresh = K.kvlink_plan_get_offsets(plan)
+    fpos = K.kvlink_plan_get_fresh_positions(plan)
+    ctx = fresh = 0
+    for b in range(batch.cfg.batch):
+        lay = _oracle_layout(batch, b)
+        assert cu_ctx[b] == ctx and cu_fresh[b] == fresh
+        # expected segments, in sequence order
+        exp = []
+        if lay.prefix_len:
+            exp.append((K.KVLINK_SEG_PREFIX, int(batch.prefix_doc[b]), lay.prefix_len, 0))
+        f = fresh
+        for i, d in enumerate(batch.docs_of(b)):
+            exp.append((K.KVLINK_SEG_DOC, int(d), int(lay.doc_len[i]), int(lay.doc_start[i])))
+            if batch.cfg.n_link:
+                exp.append((K.KVLINK_SEG_LINK, f, batch.cfg.n_link, int(lay.link_pos[i, 0])))
+                f += batch.cfg.n_link
+        exp.append((K.KVLINK_SEG_QUESTION, f, int(batch.q_len[b]), int(lay.question_pos[0])))
+        mine = seg[seg["query"] == b]
+        got = [(int(s["kind"]), int(s["src"]), int(s["len"]), int(s["pos"])) for s in mine]
+        assert got == exp
+        assert np.array_equal(mine["dst"], ctx + mine["pos"])
+        T = len(lay.fresh_pos)
+        assert np.array_equal(fpos[fresh: fresh + T], lay.fresh_pos)
+        ctx += lay.total
+        fresh += T
+    assert cu_ctx[-1] == ctx and cu_fresh[-1] == fresh
+    info = K.kvlink_plan_get_info(plan)
+    assert info.ctx_rows == ctx and info.n_fresh == fresh
+    docs = seg[seg["kind"] == K.KVLINK_SEG_DOC]
+    assert np.array_equal(np.sort(docs["table"]), np.arange(len(docs)))
+    assert info.attn_pairs == int(np.sum(fpos.astype(np.int64) + 1))
+
+
+def _items(K, plan):
+    """Attention items and merge groups, read back from the plan's device-buffer image."""
+    import paper_2502_16002_gb300.kvlink as KK
+    # items are not exported by the ABI; re-derive coverage from the public info instead
+    return KK.kvlink_plan_get_info(plan)
+
+
+@pytest.mark.parametrize("cfg_index", [1, 2, 3, 4, 5])
+def test_attention_work_counts(K, cfg_index):
+    batch = W.draw_batch(W.get_config(cfg_index))
+    plan = _plan(K, batch)
+    info = K.kvlink_plan_get_info(plan)
+    cfg = batch.cfg
+    tok_per_tile = 128 // cfg.group
+    m_tiles = sum(-(-int(t) // tok_per_tile) for t in batch.n_fresh)
+    assert info.n_attn_items >= m_tiles * cfg.h_kv
+    assert info.workspace_bytes == info.n_attn_splits * 128 * (cfg.head_dim + 2) * 4
+
+
+def test_invalid_arguments_are_rejected_before_launch(K):
+    batch = W.draw_batch(W.get_config(1))
+    with pytest.raises(K.KvlinkError) as e:
+        _plan(K, batch, doc_ids=np.asarray([0, 5], np.int32))
+    assert e.value.code == K.KVLINK_EBOUNDS
+    with pytest.raises(K.KvlinkError) as e:
+        _plan(K, batch, head_dim=96)
+    assert e.value.code == K.KVLINK_EUNSUPPORTED
+    with pytest.raises(K.KvlinkError) as e:
+        _plan(K, batch, h_q=6)
+    assert e.value.code == K.KVLINK_EUNSUPPORTED
+    with pytest.raises(K.KvlinkError) as e:
+        _plan(K, batch, pool_rows=100)            # docs need 128 rows
+    assert e.value.code == K.KVLINK_EBOUNDS
+    with pytest.raises(K.KvlinkError) as e:
+        _plan(K, batch, prefix_doc=np.asarray([7], np.int32))
+    assert e.value.code == K.KVLINK_EBOUNDS
+    with pytest.raises(K.KvlinkError) as e:
+        _plan(K, batch, q_len=np.asarray([0], np.int32), n_link=0)   # no fresh rows
+    assert e.value.code == K.KVLINK_EINVAL
+    plan = _plan(K, batch)
+    info = K.kvlink_plan_get_info(plan)
+    with pytest.raises(K.KvlinkError) as e:       # too small: rejected before any CUDA call
+        K.kvlink_plan_upload(plan, 1e4, 1 << 20, info.device_bytes - 1, 0)
+    assert e.value.code == K.KVLINK_ECAPACITY
+    with pytest.raises(K.KvlinkError) as e:       # not uploaded yet
+        K.kvlink_reencode_concat(plan, 256, 256, 256, 256, 0)
+    assert e.value.code == K.KVLINK_EINVAL
+
+
+def test_paged_pool_block_ids_are_validated(K):
+    batch = W.draw_batch(W.get_config(5))
+    bt = batch.pool_block_table.copy()
+    bt[3] = batch.pool_rows // 16            # one past the last physical block
+    with pytest.raises(K.KvlinkError) as e:
+        _plan(K, batch, pool_block_table=bt)
+    assert e.value.code == K.KVLINK_EBOUNDS
+
+
+def test_plan_is_deterministic(K):
+    batch = W.draw_batch(W.get_config(3))
+    a = K.kvlink_plan_get_segments(_plan(K, batch))
+    b = K.kvlink_plan_get_segments(_plan(K, batch))
+    assert a.tobytes() == b.tobytes()
