@@ -2,9 +2,8 @@
 precomputed document caches, and the suffix attention of link and question tokens
 (arXiv 2502.16002, Sec. 2.2-2.3), behind the C ABI in include/kvlink.h.
 
-Importing this package loads libkvlink.so and fails if it has not been built.
+`paper_2502_16002_gb300.kvlink` (the binding) and `.runtime` load libkvlink.so
+on import and fail if it has not been built (`paper_2502_16002_gb300.build`);
+there is no fallback.
 """
-from . import kvlink  # noqa: F401  (loads the CUDA library; no fallback)
-from .kvlink import KvlinkError  # noqa: F401
-
-__all__ = ["kvlink", "KvlinkError"]
+__all__ = ["kvlink", "runtime", "build"]
