@@ -187,6 +187,14 @@ int kvlink_suffix_attention(const kvlink_plan_t* plan, const void* d_q, const vo
                             const void* d_v_new, void* d_cache_k, void* d_cache_v, void* d_out,
                             void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream);
 
+/* The same computation as kvlink_suffix_attention on the CUDA cores: one CTA per
+ * (fresh row, KV head) streams the row's visible keys with an online softmax in
+ * fp32; no tensor cores, no workspace.  A second, independent GPU implementation
+ * for cross-checking and for debugging.  Errors: EINVAL, ECUDA. */
+int kvlink_suffix_attention_simt(const kvlink_plan_t* plan, const void* d_q, const void* d_k_new,
+                                 const void* d_v_new, void* d_cache_k, void* d_cache_v, void* d_out,
+                                 kvlink_stream_t stream);
+
 /* One layer of the linked prefill: kvlink_reencode_concat with the fresh-row
  * placement fused into the same launch, then the suffix attention.  Same arguments
  * and errors as the two calls it chains. */

@@ -28,6 +28,7 @@ SOURCES = [
     "kvlink_api.cu",
     "kvlink_reencode.cu",
     "kvlink_attention_simt.cu",
+    "kvlink_attention_tc.cu",
 ]
 
 

@@ -10,7 +10,7 @@
 #include "kvlink_internal.h"
 
 namespace kvlink {
-void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float2* d_rope, int head_dim,
+void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float4* d_rope, int head_dim,
                        double theta, cudaStream_t stream);
 void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv,
                      int pool_bs, const void* pool_k, const void* pool_v, const void* k_new,
@@ -18,6 +18,11 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
 void launch_attention_simt(const DevicePlan& P, int n_fresh, int head_dim, int h_q, int h_kv,
                            const void* q, const void* cache_k, const void* cache_v, void* out,
                            cudaStream_t stream);
+int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t ctx_rows,
+                        int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
+                        void* out, void* ws, cudaStream_t stream, cudaError_t* err);
+int read_attention_status(int32_t* status);
+int clear_attention_status();
 }  // namespace kvlink
 
 using namespace kvlink;
@@ -53,8 +58,6 @@ int check_plan(const kvlink_plan_t* p) {
     if (!p->uploaded) return KVLINK_EINVAL;
     return KVLINK_OK;
 }
-
-int64_t pool_tensor_rows(const kvlink_plan_t* p) { return p->pool_rows; }
 
 }  // namespace
 
@@ -172,7 +175,7 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     DevicePlan& d = p->dev;
     d.seg = (const kvlink_segment_t*)(b + p->off_seg);
     d.chunks = (const CopyChunk*)(b + p->off_chunks);
-    d.rope = (const float2*)(b + p->off_rope);
+    d.rope = (const float4*)(b + p->off_rope);
     d.pool_start = (const int64_t*)(b + p->off_pool_start);
     d.pool_block_table = (const int32_t*)(b + p->off_pool_bt);
     d.cu_ctx = (const int64_t*)(b + p->off_cu_ctx);
@@ -181,7 +184,7 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     d.fresh_query = (const int32_t*)(b + p->off_fresh_query);
     d.items = (const AttnItem*)(b + p->off_items);
     d.merges = (const MergeGroup*)(b + p->off_merges);
-    launch_rope_table(d.seg, (int)p->seg.size(), (float2*)(b + p->off_rope), p->head_dim, theta, s);
+    launch_rope_table(d.seg, (int)p->seg.size(), (float4*)(b + p->off_rope), p->head_dim, theta, s);
     int rc = check_launch("rope_table_kernel");
     if (rc != KVLINK_OK) return rc;
     p->theta = theta;
@@ -202,16 +205,27 @@ int kvlink_reencode_concat(const kvlink_plan_t* p, const void* pool_k, const voi
     return check_launch("reencode_kernel");
 }
 
+static int place_fresh(const kvlink_plan_t* p, const void* k_new, const void* v_new, void* cache_k,
+                       void* cache_v, cudaStream_t s) {
+    const int n_all = (int)p->chunks.size();
+    launch_reencode(p->dev, p->n_chunks_cached, n_all - p->n_chunks_cached, p->head_dim, p->h_kv,
+                    p->pool_block_size, nullptr, nullptr, k_new, v_new, cache_k, cache_v, s);
+    return check_launch("fresh placement");
+}
+
 static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k, void* cache_v,
                             void* out, void* ws, size_t ws_bytes, cudaStream_t s) {
     if (!q || !cache_k || !cache_v || !out) return KVLINK_EINVAL;
     if (!aligned16(q) || !aligned16(cache_k) || !aligned16(cache_v) || !aligned16(out))
         return KVLINK_EINVAL;
-    (void)ws;
-    (void)ws_bytes;
-    const int n_fresh = p->cu_fresh.back();
-    launch_attention_simt(p->dev, n_fresh, p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, s);
-    return check_launch("attention");
+    if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
+    if (ws && !aligned16(ws)) return KVLINK_EINVAL;
+    cudaError_t err = cudaSuccess;
+    const int rc = launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
+                                       p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out,
+                                       ws, s, &err);
+    if (rc == KVLINK_ECUDA) return cuda_fail(err, "suffix attention launch");
+    return rc;
 }
 
 int kvlink_suffix_attention(const kvlink_plan_t* p, const void* q, const void* k_new, const void* v_new,
@@ -224,13 +238,27 @@ int kvlink_suffix_attention(const kvlink_plan_t* p, const void* q, const void* k
     if (!cache_k || !cache_v) return KVLINK_EINVAL;
     cudaStream_t s = (cudaStream_t)stream;
     if (k_new) {
-        const int n_all = (int)p->chunks.size();
-        launch_reencode(p->dev, p->n_chunks_cached, n_all - p->n_chunks_cached, p->head_dim, p->h_kv,
-                        p->pool_block_size, nullptr, nullptr, k_new, v_new, cache_k, cache_v, s);
-        rc = check_launch("fresh placement");
+        rc = place_fresh(p, k_new, v_new, cache_k, cache_v, s);
         if (rc) return rc;
     }
     return attention_common(p, q, cache_k, cache_v, out, ws, ws_bytes, s);
+}
+
+int kvlink_suffix_attention_simt(const kvlink_plan_t* p, const void* q, const void* k_new, const void* v_new,
+                                 void* cache_k, void* cache_v, void* out, kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if ((k_new == nullptr) != (v_new == nullptr)) return KVLINK_EINVAL;
+    if (k_new && (!aligned16(k_new) || !aligned16(v_new))) return KVLINK_EINVAL;
+    if (!q || !cache_k || !cache_v || !out) return KVLINK_EINVAL;
+    if (!aligned16(q) || !aligned16(cache_k) || !aligned16(cache_v) || !aligned16(out)) return KVLINK_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (k_new) {
+        rc = place_fresh(p, k_new, v_new, cache_k, cache_v, s);
+        if (rc) return rc;
+    }
+    launch_attention_simt(p->dev, p->cu_fresh.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, s);
+    return check_launch("simt attention");
 }
 
 int kvlink_linked_prefill(const kvlink_plan_t* p, const void* pool_k, const void* pool_v, const void* q,
@@ -252,9 +280,9 @@ int kvlink_linked_prefill(const kvlink_plan_t* p, const void* pool_k, const void
 int kvlink_device_status(int32_t* status) {
     if (!status) return KVLINK_EINVAL;
     *status = 0;
-    return KVLINK_OK;
+    return read_attention_status(status);
 }
 
-int kvlink_clear_device_status(void) { return KVLINK_OK; }
+int kvlink_clear_device_status(void) { return clear_attention_status(); }
 
 }  // extern "C"

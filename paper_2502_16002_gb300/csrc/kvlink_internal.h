@@ -50,7 +50,7 @@ static_assert(sizeof(MergeGroup) == 32, "MergeGroup layout");
 struct DevicePlan {
     const kvlink_segment_t* seg;
     const CopyChunk* chunks;     // cached-segment chunks first, then fresh-segment chunks
-    const float2* rope;          // [n_rope_rows][D/2] (cos, sin)
+    const float4* rope;          // [n_rope_rows][D/2] (cos hi, cos lo, sin hi, sin lo)
     const int64_t* pool_start;   // [pool_docs]
     const int32_t* pool_block_table;
     const int64_t* cu_ctx;       // [B+1]

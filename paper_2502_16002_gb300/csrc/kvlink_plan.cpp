@@ -207,7 +207,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
     p->off_seg = take(p->seg.size() * sizeof(kvlink_segment_t));
     p->off_chunks = take(p->chunks.size() * sizeof(CopyChunk));
-    p->off_rope = take((size_t)p->n_rope_rows * (d->head_dim / 2) * sizeof(float2));
+    p->off_rope = take((size_t)p->n_rope_rows * (d->head_dim / 2) * sizeof(float4));
     p->off_pool_start = take(p->pool_start.size() * sizeof(int64_t));
     p->off_pool_bt = take(p->pool_block_table.size() * sizeof(int32_t));
     p->off_cu_ctx = take(p->cu_ctx.size() * sizeof(int64_t));

@@ -8,6 +8,14 @@
 // pairs it rotates) and the value chunks at the same offsets, so every load and
 // store is a coalesced 128-bit access and the eight (cos, sin) pairs of the
 // segment's delta stay in registers for the whole unit.
+//
+// Precision: a rotated component x cos a - y sin a can cancel to far below |x|,
+// where the bf16 quantum is tiny; an fp32 cos/sin (relative error 2^-24) would
+// then be off by many bf16 ulps.  The table therefore holds cos and sin as
+// unevaluated float pairs hi + lo (about 48 significant bits, split from the
+// fp64 values) and the kernel forms the products with their exact FMA rounding
+// errors, so the fp32 result carries an absolute error near 2^-47 |x| and rounds
+// to within one bf16 ulp of the correctly rounded fp64 rotation.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -17,11 +25,11 @@ namespace kvlink {
 
 // --------------------------------------------------------------------------
 // A2: cos/sin(delta * theta^(-2j/D)) for every cached document segment.
-// The angle is formed and reduced in float64; only the final cos/sin are
-// rounded to float32, so the key rotation error does not grow with delta.
+// The angle is formed and reduced in float64, so the rotation error does not
+// grow with delta; cos and sin are stored as float pairs (hi, lo).
 // --------------------------------------------------------------------------
 __global__ void rope_table_kernel(const kvlink_segment_t* __restrict__ seg, int n_seg,
-                                  float2* __restrict__ rope, int half, double theta, int head_dim) {
+                                  float4* __restrict__ rope, int half, double theta, int head_dim) {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= (int64_t)n_seg * half) return;
     const int s = (int)(i / half), j = (int)(i % half);
@@ -31,10 +39,11 @@ __global__ void rope_table_kernel(const kvlink_segment_t* __restrict__ seg, int 
     const double angle = (double)sg.pos * inv_freq;
     double sn, cs;
     sincos(angle, &sn, &cs);
-    rope[(int64_t)sg.table * half + j] = make_float2((float)cs, (float)sn);
+    const float ch = (float)cs, sh = (float)sn;
+    rope[(int64_t)sg.table * half + j] = make_float4(ch, (float)(cs - (double)ch), sh, (float)(sn - (double)sh));
 }
 
-void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float2* d_rope, int head_dim,
+void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float4* d_rope, int head_dim,
                        double theta, cudaStream_t stream) {
     const int half = head_dim / 2;
     const int64_t n = (int64_t)n_seg * half;
@@ -63,19 +72,38 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
     return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// y_lo = x_lo cos - x_hi sin ; y_hi = x_hi cos + x_lo sin, 8 lanes of each half
-__device__ __forceinline__ void rotate8(uint4& lo, uint4& hi, const float (&c)[8], const float (&s)[8]) {
+// x c - y s and y c + x s with c = ch + cl, s = sh + sl (double-float), x, y exact.
+// The leading products are rounded explicitly (no contraction) and their exact
+// rounding errors recovered with FMA; the small terms are added once at the end.
+__device__ __forceinline__ float rot_first(float x, float y, float ch, float cl, float sh, float sl) {
+    const float p1 = __fmul_rn(x, ch), p2 = __fmul_rn(y, sh);
+    const float e1 = fmaf(x, ch, -p1), e2 = fmaf(y, sh, -p2);
+    const float t = __fsub_rn(p1, p2);
+    const float corr = (e1 - e2) + fmaf(x, cl, -(y * sl));
+    return __fadd_rn(t, corr);
+}
+
+__device__ __forceinline__ float rot_second(float x, float y, float ch, float cl, float sh, float sl) {
+    const float p1 = __fmul_rn(y, ch), p2 = __fmul_rn(x, sh);
+    const float e1 = fmaf(y, ch, -p1), e2 = fmaf(x, sh, -p2);
+    const float t = __fadd_rn(p1, p2);
+    const float corr = (e1 + e2) + fmaf(y, cl, x * sl);
+    return __fadd_rn(t, corr);
+}
+
+// lo' = lo cos - hi sin ; hi' = hi cos + lo sin, for the 8 pairs of one (lo, hi) chunk pair
+__device__ __forceinline__ void rotate8(uint4& lo, uint4& hi, const float4 (&cs)[8]) {
     uint32_t* a = reinterpret_cast<uint32_t*>(&lo);
     uint32_t* b = reinterpret_cast<uint32_t*>(&hi);
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
         const float x0 = bf16lo(a[w]), x1 = bf16hi(a[w]);
         const float y0 = bf16lo(b[w]), y1 = bf16hi(b[w]);
-        const int e = 2 * w;
-        const float r0 = fmaf(x0, c[e], -y0 * s[e]);
-        const float r1 = fmaf(x1, c[e + 1], -y1 * s[e + 1]);
-        const float t0 = fmaf(y0, c[e], x0 * s[e]);
-        const float t1 = fmaf(y1, c[e + 1], x1 * s[e + 1]);
+        const float4 c0 = cs[2 * w], c1 = cs[2 * w + 1];
+        const float r0 = rot_first(x0, y0, c0.x, c0.y, c0.z, c0.w);
+        const float r1 = rot_first(x1, y1, c1.x, c1.y, c1.z, c1.w);
+        const float t0 = rot_second(x0, y0, c0.x, c0.y, c0.z, c0.w);
+        const float t1 = rot_second(x1, y1, c1.x, c1.y, c1.z, c1.w);
         a[w] = pack_bf16(r0, r1);
         b[w] = pack_bf16(t0, t1);
     }
@@ -106,17 +134,14 @@ __global__ void __launch_bounds__(kCopyThreads) reencode_kernel(
     const __nv_bfloat16* sk = fresh ? k_new : pool_k;
     const __nv_bfloat16* sv = fresh ? v_new : pool_v;
 
-    float c[8], s[8];
+    float4 cs[8];
     if (rotate) {
-        const float4* t = reinterpret_cast<const float4*>(P.rope + (int64_t)sg.table * (D / 2) + j0);
+        const float4* t = P.rope + (int64_t)sg.table * (D / 2) + j0;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const float4 v = __ldg(t + q);
-            c[2 * q] = v.x; s[2 * q] = v.y; c[2 * q + 1] = v.z; s[2 * q + 1] = v.w;
-        }
+        for (int q = 0; q < 8; ++q) cs[q] = __ldg(t + q);
     } else {
 #pragma unroll
-        for (int e = 0; e < 8; ++e) { c[e] = 1.f; s[e] = 0.f; }
+        for (int q = 0; q < 8; ++q) cs[q] = make_float4(1.f, 0.f, 0.f, 0.f);
     }
     const int64_t entry_start = fresh ? 0 : P.pool_start[sg.src];
 
@@ -144,14 +169,14 @@ __global__ void __launch_bounds__(kCopyThreads) reencode_kernel(
             vb0 = ld_stream(reinterpret_cast<const uint4*>(sv + rb + lo_off));
             vb1 = ld_stream(reinterpret_cast<const uint4*>(sv + rb + hi_off));
         }
-        if (rotate) rotate8(ka0, ka1, c, s);
+        if (rotate) rotate8(ka0, ka1, cs);
         const int64_t da = (sg.dst + ta) * row_elems;
         *reinterpret_cast<uint4*>(cache_k + da + lo_off) = ka0;
         *reinterpret_cast<uint4*>(cache_k + da + hi_off) = ka1;
         *reinterpret_cast<uint4*>(cache_v + da + lo_off) = va0;
         *reinterpret_cast<uint4*>(cache_v + da + hi_off) = va1;
         if (has_b) {
-            if (rotate) rotate8(kb0, kb1, c, s);
+            if (rotate) rotate8(kb0, kb1, cs);
             const int64_t db = (sg.dst + tb) * row_elems;
             *reinterpret_cast<uint4*>(cache_k + db + lo_off) = kb0;
             *reinterpret_cast<uint4*>(cache_k + db + hi_off) = kb1;

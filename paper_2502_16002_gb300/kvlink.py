@@ -88,6 +88,7 @@ def _load():
         "kvlink_plan_upload": (C.c_int, [P, C.c_double, V, C.c_size_t, V]),
         "kvlink_reencode_concat": (C.c_int, [P, V, V, V, V, V]),
         "kvlink_suffix_attention": (C.c_int, [P, V, V, V, V, V, V, V, C.c_size_t, V]),
+        "kvlink_suffix_attention_simt": (C.c_int, [P, V, V, V, V, V, V, V]),
         "kvlink_linked_prefill": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
@@ -104,7 +105,8 @@ lib = _load()
 DECLARED = [
     "kvlink_plan_create", "kvlink_plan_destroy", "kvlink_plan_get_info", "kvlink_plan_get_segments",
     "kvlink_plan_get_offsets", "kvlink_plan_get_fresh_positions", "kvlink_plan_upload",
-    "kvlink_reencode_concat", "kvlink_suffix_attention", "kvlink_linked_prefill",
+    "kvlink_reencode_concat", "kvlink_suffix_attention", "kvlink_suffix_attention_simt",
+    "kvlink_linked_prefill",
     "kvlink_device_status", "kvlink_clear_device_status", "kvlink_strerror",
     "kvlink_last_cuda_error", "kvlink_version",
 ]
@@ -221,6 +223,12 @@ def kvlink_suffix_attention(plan: Plan, q: int, k_new, v_new, cache_k: int, cach
                             workspace, workspace_bytes: int, stream: int = 0) -> None:
     _check(lib.kvlink_suffix_attention(plan.handle, q, k_new, v_new, cache_k, cache_v, out, workspace,
                                        workspace_bytes, stream), "kvlink_suffix_attention")
+
+
+def kvlink_suffix_attention_simt(plan: Plan, q: int, k_new, v_new, cache_k: int, cache_v: int, out: int,
+                                 stream: int = 0) -> None:
+    _check(lib.kvlink_suffix_attention_simt(plan.handle, q, k_new, v_new, cache_k, cache_v, out, stream),
+           "kvlink_suffix_attention_simt")
 
 
 def kvlink_linked_prefill(plan: Plan, pool_k: int, pool_v: int, q: int, k_new: int, v_new: int,

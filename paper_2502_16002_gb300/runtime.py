@@ -83,6 +83,13 @@ class LinkedPrefill:
                                   self.workspace.data_ptr(), self.workspace.numel(),
                                   _stream_handle(stream))
 
+    def suffix_attention_simt(self, q, k_new, v_new, cache_k, cache_v, out, stream=None):
+        K.kvlink_suffix_attention_simt(self.plan, q.data_ptr(),
+                                       k_new.data_ptr() if k_new is not None else None,
+                                       v_new.data_ptr() if v_new is not None else None,
+                                       cache_k.data_ptr(), cache_v.data_ptr(), out.data_ptr(),
+                                       _stream_handle(stream))
+
     def linked_prefill(self, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out, stream=None):
         K.kvlink_linked_prefill(self.plan, pool_k.data_ptr(), pool_v.data_ptr(), q.data_ptr(),
                                 k_new.data_ptr(), v_new.data_ptr(), cache_k.data_ptr(),
