@@ -130,9 +130,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + C::N_BARS);
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(tmem_holder + 1);
 
-    // after a recorded failure, later launches return at once instead of waiting out their bounds
-    if (*reinterpret_cast<volatile int32_t*>(&g_attn_status) != 0) return;
-
     const AttnItem it = P.items[blockIdx.x];
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int n_tiles = it.kv_tile1 - it.kv_tile0;
@@ -151,7 +148,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         mbar_init(bar_p_full, kSoftmaxWarps);
         mbar_init(bar_o_done, 1);
         mbar_init(bar_drain, 1);
-        *abort_flag = 0;
+        // after a recorded failure, later launches skip their work instead of waiting out their bounds
+        *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_attn_status) != 0 ? 1 : 0;
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
@@ -167,8 +165,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
+    const bool skip = *abort_flag != 0;  // written before the barrier: uniform across the CTA
 
-    if (warp == kTmaWarp) {
+    if (skip) {
+        // nothing issued: fall through to the teardown
+    } else if (warp == kTmaWarp) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             const int g = it.kv_head;
