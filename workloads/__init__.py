@@ -16,6 +16,7 @@ from .draw import (
     pool_kv,
     fresh_qkv,
     cache_block_tables,
+    normal_bf16_torch,
 )
 
 __all__ = [
@@ -30,4 +31,5 @@ __all__ = [
     "pool_kv",
     "fresh_qkv",
     "cache_block_tables",
+    "normal_bf16_torch",
 ]
