@@ -151,7 +151,7 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.set_device(dev)
     cfg = W.get_config(args.config)
     batch = W.draw_batch(cfg, seed=rank)           # every rank serves its own batch
-    L = cfg.layers
+    L = args.layers or cfg.layers
     lp = LinkedPrefill.from_batch(batch, device=dev)
     info = lp.info
     ctx, T = int(info.ctx_rows), int(info.n_fresh)
@@ -326,46 +326,48 @@ def run_ours(args, rank, world, local_rank):
 
 # ------------------------------------------------------------------ CPU oracle (baseline)
 
-def oracle_sample(cfg, n_samples=None, max_seconds=20.0):
+def oracle_sample(cfg, n_layers=None, max_seconds=20.0):
     """Time the fp64 oracle on (query, layer) samples of the workload.
 
-    Returns (us per query over all layers, seconds spent, description)."""
+    Layers are taken in the order 0, L-1, L/2, ...; within a layer every query is run
+    until max_seconds of oracle time have been spent.  Returns (us per query over all
+    layers, seconds spent, description)."""
     import oracle
 
     batch = W.draw_batch(cfg)
-    samples = [(0, 0), (cfg.batch - 1, cfg.layers - 1), (cfg.batch // 2, cfg.layers // 2),
-               (0, cfg.layers - 1)]
-    if n_samples is not None:
-        samples = samples[:n_samples]
-    times = []
-    spent = 0.0
-    done = []
-    for b, layer in samples:
+    layers = [0, cfg.layers - 1, cfg.layers // 2, cfg.layers // 4][: (n_layers or 4)]
+    layers = list(dict.fromkeys(layers))
+    times, done, spent = [], [], 0.0
+    for layer in layers:
         pk, pv = W.pool_kv(batch, layer)
         q, kn, vn = W.fresh_qkv(batch, layer)
-        t0 = time.perf_counter()
-        oracle.oracle_query_layer(batch, b, pk, pv, q, kn, vn)
-        dt = time.perf_counter() - t0
-        times.append(dt)
-        done.append((b, layer))
-        spent += dt
+        for b in range(cfg.batch):
+            t0 = time.perf_counter()
+            oracle.oracle_query_layer(batch, b, pk, pv, q, kn, vn)
+            dt = time.perf_counter() - t0
+            times.append(dt)
+            done.append((b, layer))
+            spent += dt
+            if spent > max_seconds:
+                break
         if spent > max_seconds:
             break
     per_query_layer = float(np.mean(times))
-    desc = (f"{len(done)} (query, layer) samples {done} of {cfg.name}: full re-encode/concat of the "
-            f"query's cache and attention of all its fresh rows and heads in fp64; "
-            f"value = mean per (query, layer) x {cfg.layers} layers")
+    desc = (f"{len(done)} (query, layer) samples over layers {sorted(set(l for _, l in done))} of "
+            f"{cfg.name}: full re-encode/concat of the query's cache and attention of all its fresh "
+            f"rows and heads in fp64 (numpy, BLAS threads); value = mean per (query, layer) x "
+            f"{cfg.layers} layers")
     return per_query_layer * cfg.layers * 1e6, spent, desc
 
 
 def run_reference(args):
     cfg = W.get_config(args.config)
     for _ in range(args.warmup):
-        oracle_sample(cfg, n_samples=1)
+        oracle_sample(cfg, n_layers=1, max_seconds=0.0)
     vals = []
     t_all = 0.0
     for _ in range(args.steps):
-        v, s, desc = oracle_sample(cfg, n_samples=1)
+        v, s, desc = oracle_sample(cfg, n_layers=1, max_seconds=0.0)
         vals.append(v)
         t_all += s
     value = float(np.mean(vals))
@@ -383,9 +385,11 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
-    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", type=int, default=3)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="layers per step (default: the workload's); fewer only for small profiling runs")
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
