@@ -1,24 +1,27 @@
 // Suffix attention on the tcgen05 tensor cores (Sec. 2.3, "inference").
 //
-// Work item = one M-tile of 128 rows (128/G fresh tokens x the G query heads
-// that share one KV head) of one query, over a range of 128-key tiles of that
-// query's linked cache.  Rows are (token, head) pairs, so the G heads of a
-// GQA group share every K/V tile load.
+// Work item = one M-tile of up to 128 rows (up to 128/G fresh tokens x the G
+// query heads that share one KV head) of one query, over a range of 128-key
+// tiles of that query's linked cache.  Rows are (token, head) pairs, so the G
+// heads of a GQA group share every K/V tile load.
 //
-// Warp roles (192 threads, one CTA per SM, 512 TMEM columns):
+// Warp roles (224 threads, one CTA per SM, 512 TMEM columns):
 //   warps 0-3  softmax + epilogue; thread r owns row r = TMEM lane r
-//   warp 4     TMA producer: Q once, then K and V tiles into an NS-stage ring
+//   warp 4     TMA: Q once, then K tiles into an NK-stage ring
 //   warp 5     TMEM allocation and the single MMA-issuing thread
-// Per KV tile j:
-//   S_j = Q K_j^T          tcgen05.mma, SMEM x SMEM -> TMEM (double-buffered S)
-//   P_j = exp2(S_j*c - m)  softmax warps: TMEM -> registers -> bf16 P in SMEM
-//   O  += P_j V_j          tcgen05.mma, SMEM x SMEM -> TMEM (V read MN-major)
-// The running max m is only raised when it grows by more than 2^8, so the O
-// accumulator in TMEM is rescaled rarely; m, l stay per thread in registers.
-// The mask keeps key slot j for a row at global position p iff j <= p, and is
-// only evaluated on tiles that reach past the tile's smallest row position.
-// Items whose KV range was split write unnormalised partials (O, m, l) to the
-// workspace; attn_merge_kernel combines them.
+//   warp 6     TMA: V tiles into an NV-stage ring
+// Per KV tile j (TMEM: three S/P buffers of 128 columns, then O):
+//   S_j = Q K_j^T           tcgen05.mma SMEM x SMEM -> S buffer j%3
+//   P_j = exp2(S_j c - m)   softmax warps: TMEM -> registers -> bf16 P written back
+//                           over the first 64 columns of the same buffer
+//   O  += P_j V_j           tcgen05.mma TMEM x SMEM (P from TMEM, V read MN-major)
+// S_j is issued only after PV_{j-3} has finished reading the buffer, so up to
+// three tiles are in flight and the softmax never waits on a PV except to
+// rescale O.  The running max m is raised only when it grows by more than 2^8,
+// so that rescale is rare.  The mask keeps key slot j for a row at global
+// position p iff j <= p, and is evaluated only on tiles that reach past the
+// tile's smallest row position.  Items whose KV range was split write
+// unnormalised partials (O, m, l) to the workspace; attn_merge_kernel combines them.
 //
 // Every mbarrier wait is bounded in time.  On expiry the kernel records
 // kAttnStatusWaitTimeout in its status word, the other roles leave their loops,
@@ -37,10 +40,11 @@ using namespace sm100;
 
 static __device__ int32_t g_attn_status;
 
-constexpr int kTcThreads = 192;
+constexpr int kTcThreads = 224;
 constexpr int kSoftmaxWarps = 4;
-constexpr int kTmaWarp = 4;
+constexpr int kTmaKWarp = 4;
 constexpr int kMmaWarp = 5;
+constexpr int kTmaVWarp = 6;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 constexpr int32_t kAttnStatusWaitTimeout = 0x41;
@@ -49,20 +53,24 @@ constexpr float kRescaleThreshold = 8.0f;         // log2 units: rescale O when 
 template <int D>
 struct TcCfg {
     static constexpr int ATOMS = D / 64;                 // 128-byte swizzle atoms along head_dim
-    static constexpr int NS = (D == 128) ? 2 : 4;        // K/V ring stages
+    static constexpr int NK = (D == 128) ? 3 : 5;        // K ring stages
+    static constexpr int NV = (D == 128) ? 3 : 5;        // V ring stages
+    static constexpr int NB = 3;                         // S/P buffers in TMEM
     static constexpr uint32_t ATOM_BYTES = 128 * 128;    // [128 rows][64 bf16]
     static constexpr uint32_t Q_BYTES = ATOMS * ATOM_BYTES;
     static constexpr uint32_t KV_BYTES = ATOMS * ATOM_BYTES;
-    static constexpr uint32_t P_BYTES = 2 * ATOM_BYTES;  // [128 rows][128 keys] bf16
     static constexpr uint32_t OFF_Q = 0;
     static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
-    static constexpr uint32_t OFF_V = OFF_K + NS * KV_BYTES;
-    static constexpr uint32_t OFF_P = OFF_V + NS * KV_BYTES;
-    static constexpr uint32_t OFF_BAR = OFF_P + P_BYTES;
-    // q_full, k_full[NS], v_full[NS], kv_empty[NS], s_full[2], s_free[2], p_full, o_done, drain
-    static constexpr int N_BARS = 1 + 3 * NS + 4 + 3;
+    static constexpr uint32_t OFF_V = OFF_K + NK * KV_BYTES;
+    static constexpr uint32_t OFF_BAR = OFF_V + NV * KV_BYTES;
+    // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB], p_full[NB], o_done[NB], drain
+    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 3 * NB + 1;
     static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
-    static constexpr uint32_t TMEM_S0 = 0, TMEM_S1 = 128, TMEM_O = 256;
+    // TMEM columns: S/P buffers then the O accumulator
+    static constexpr uint32_t TMEM_S = 0;                // buffer b at b * 128
+    static constexpr uint32_t TMEM_O = NB * kAttnBN;
+    static_assert(TMEM_O + D <= kTmemCols, "TMEM budget");
+    static_assert(SMEM_BYTES <= 232448, "shared memory budget");
 };
 
 // Wait for phase `parity` of `bar`; false if another role aborted or the time limit passed.
@@ -102,8 +110,23 @@ __device__ __forceinline__ uint32_t pack2_bf16(float a, float b) {
     return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
-    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+// TMA producer loop for one ring (K or V): tiles j = 0..n-1 of the item's key range.
+template <int STAGES, int ATOMS>
+__device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes, const CUtensorMap* map,
+                                             uint64_t* full, uint64_t* empty, int n, int g, int key_row0,
+                                             volatile int32_t* abort_flag) {
+    int issued = 0;
+    for (int j = 0; j < n; ++j) {
+        const int st = j % STAGES;
+        if (!wait_bar(empty + st, ((j / STAGES) & 1) ^ 1, abort_flag)) break;
+        mbar_arrive_expect_tx(full + st, stage_bytes);
+#pragma unroll
+        for (int a = 0; a < ATOMS; ++a)
+            tma_load_3d(ring + st * stage_bytes + a * (128 * 128), map, a * 64, g, key_row0 + j * kAttnBN, full + st);
+        issued = j + 1;
+    }
+    // no copy may still be in flight when the CTA leaves
+    for (int j = issued - STAGES > 0 ? issued - STAGES : 0; j < issued; ++j) drain_bar(full + j % STAGES, (j / STAGES) & 1);
 }
 
 template <int D, int G>
@@ -112,21 +135,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                    const __grid_constant__ CUtensorMap tm_v, DevicePlan P, __nv_bfloat16* __restrict__ out,
                    float* __restrict__ ws, int h_q, float scale_log2) {
     using C = TcCfg<D>;
-    constexpr int NS = C::NS;
+    constexpr int NK = C::NK, NV = C::NV, NB = C::NB;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
 
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
     uint64_t* bar_q_full = bars;
-    uint64_t* bar_k_full = bars + 1;
-    uint64_t* bar_v_full = bars + 1 + NS;
-    uint64_t* bar_kv_empty = bars + 1 + 2 * NS;
-    uint64_t* bar_s_full = bars + 1 + 3 * NS;
-    uint64_t* bar_s_free = bar_s_full + 2;
-    uint64_t* bar_p_full = bar_s_free + 2;
-    uint64_t* bar_o_done = bar_p_full + 1;
-    uint64_t* bar_drain = bar_o_done + 1;
+    uint64_t* bar_k_full = bar_q_full + 1;
+    uint64_t* bar_k_empty = bar_k_full + NK;
+    uint64_t* bar_v_full = bar_k_empty + NK;
+    uint64_t* bar_v_empty = bar_v_full + NV;
+    uint64_t* bar_s_full = bar_v_empty + NV;
+    uint64_t* bar_p_full = bar_s_full + NB;
+    uint64_t* bar_o_done = bar_p_full + NB;
+    uint64_t* bar_drain = bar_o_done + NB;
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + C::N_BARS);
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(tmem_holder + 1);
 
@@ -135,19 +158,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int n_tiles = it.kv_tile1 - it.kv_tile0;
 
     if (threadIdx.x == 0) {
-        mbar_init(bar_q_full, 1);
-        for (int s = 0; s < NS; ++s) {
-            mbar_init(bar_k_full + s, 1);
-            mbar_init(bar_v_full + s, 1);
-            mbar_init(bar_kv_empty + s, 1);
+        for (int i = 0; i < C::N_BARS; ++i) {
+            const bool p_full = bars + i >= bar_p_full && bars + i < bar_p_full + NB;
+            mbar_init(bars + i, p_full ? kSoftmaxWarps : 1);
         }
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(bar_s_full + i, 1);
-            mbar_init(bar_s_free + i, kSoftmaxWarps);
-        }
-        mbar_init(bar_p_full, kSoftmaxWarps);
-        mbar_init(bar_o_done, 1);
-        mbar_init(bar_drain, 1);
         // after a recorded failure, later launches skip their work instead of waiting out their bounds
         *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_attn_status) != 0 ? 1 : 0;
         fence_mbar_init();
@@ -156,7 +170,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         tmem_alloc(tmem_holder, kTmemCols);
         tmem_relinquish();
     }
-    if (warp == kTmaWarp && lane == 0) {
+    if (warp == kTmaKWarp && lane == 0) {
         prefetch_tensormap(&tm_q);
         prefetch_tensormap(&tm_k);
         prefetch_tensormap(&tm_v);
@@ -166,80 +180,65 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
     const bool skip = *abort_flag != 0;  // written before the barrier: uniform across the CTA
+    const int key_row0 = (int)P.cu_ctx[it.query] + it.kv_tile0 * kAttnBN;
 
     if (skip) {
         // nothing issued: fall through to the teardown
-    } else if (warp == kTmaWarp) {
-        // ------------------------------------------------------------ TMA producer
+    } else if (warp == kTmaKWarp) {
+        // ------------------------------------------------------------ Q, then the K ring
         if (lane == 0) {
-            const int g = it.kv_head;
             const int q_row0 = P.cu_fresh[it.query] + it.tok0;
-            const int key_row0 = (int)P.cu_ctx[it.query] + it.kv_tile0 * kAttnBN;
             mbar_arrive_expect_tx(bar_q_full, C::Q_BYTES);
 #pragma unroll
             for (int a = 0; a < C::ATOMS; ++a)
-                tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &tm_q, a * 64, g * G, q_row0, bar_q_full);
-            int issued = 0;
-            for (int j = 0; j < n_tiles; ++j) {
-                const int st = j % NS;
-                if (!wait_bar(bar_kv_empty + st, ((j / NS) & 1) ^ 1, abort_flag)) break;
-                const int key = key_row0 + j * kAttnBN;
-                mbar_arrive_expect_tx(bar_k_full + st, C::KV_BYTES);
-#pragma unroll
-                for (int a = 0; a < C::ATOMS; ++a)
-                    tma_load_3d(smem + C::OFF_K + st * C::KV_BYTES + a * C::ATOM_BYTES, &tm_k, a * 64, g, key,
-                                bar_k_full + st);
-                mbar_arrive_expect_tx(bar_v_full + st, C::KV_BYTES);
-#pragma unroll
-                for (int a = 0; a < C::ATOMS; ++a)
-                    tma_load_3d(smem + C::OFF_V + st * C::KV_BYTES + a * C::ATOM_BYTES, &tm_v, a * 64, g, key,
-                                bar_v_full + st);
-                issued = j + 1;
-            }
-            // no copy may still be in flight when the CTA leaves
+                tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &tm_q, a * 64, it.kv_head * G, q_row0, bar_q_full);
+            produce_ring<NK, C::ATOMS>(smem + C::OFF_K, C::KV_BYTES, &tm_k, bar_k_full, bar_k_empty, n_tiles,
+                                       it.kv_head, key_row0, abort_flag);
             drain_bar(bar_q_full, 0);
-            for (int j = issued - NS > 0 ? issued - NS : 0; j < issued; ++j) {
-                drain_bar(bar_k_full + j % NS, (j / NS) & 1);
-                drain_bar(bar_v_full + j % NS, (j / NS) & 1);
-            }
         }
+    } else if (warp == kTmaVWarp) {
+        // ------------------------------------------------------------ the V ring
+        if (lane == 0)
+            produce_ring<NV, C::ATOMS>(smem + C::OFF_V, C::KV_BYTES, &tm_v, bar_v_full, bar_v_empty, n_tiles,
+                                       it.kv_head, key_row0, abort_flag);
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
             constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
             const uint32_t sQ = smem_u32(smem + C::OFF_Q);
-            const uint32_t sP = smem_u32(smem + C::OFF_P);
             bool ok = wait_bar(bar_q_full, 0, abort_flag);
+            // O += P_i V_i, P_i (bf16) read from its S buffer in TMEM
             auto issue_pv = [&](int i) -> bool {
-                const int st = i % NS;
-                if (!wait_bar(bar_p_full, i & 1, abort_flag)) return false;
-                if (!wait_bar(bar_v_full + st, (i / NS) & 1, abort_flag)) return false;
+                const int b = i % NB, sv = i % NV;
+                if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag)) return false;
+                if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag)) return false;
                 tc_fence_after();
-                const uint32_t sV = smem_u32(smem + C::OFF_V + st * C::KV_BYTES);
+                const uint32_t sV = smem_u32(smem + C::OFF_V + sv * C::KV_BYTES);
+                const uint32_t pcol = tmem + C::TMEM_S + b * kAttnBN;
 #pragma unroll
-                for (int kk = 0; kk < kAttnBN / 16; ++kk) {
-                    const uint64_t a = sdesc_sw128(sP + (kk >> 2) * C::ATOM_BYTES + (kk & 3) * 32, 16, 1024);
-                    const uint64_t b = sdesc_sw128(sV + kk * 16 * 128, C::ATOM_BYTES, 1024);
-                    mma_bf16_ss(tmem + C::TMEM_O, a, b, idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
-                }
-                mma_commit(bar_o_done);
-                mma_commit(bar_kv_empty + st);
+                for (int kk = 0; kk < kAttnBN / 16; ++kk)
+                    mma_bf16_ts(tmem + C::TMEM_O, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, C::ATOM_BYTES, 1024),
+                                idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
+                mma_commit(bar_o_done + b);
+                mma_commit(bar_v_empty + sv);
                 return true;
             };
             for (int j = 0; ok && j < n_tiles; ++j) {
-                const int st = j % NS, sb = j & 1;
-                if (!(ok = wait_bar(bar_k_full + st, (j / NS) & 1, abort_flag))) break;
-                if (!(ok = wait_bar(bar_s_free + sb, ((j >> 1) & 1) ^ 1, abort_flag))) break;
+                const int sk = j % NK, b = j % NB;
+                if (!(ok = wait_bar(bar_k_full + sk, (j / NK) & 1, abort_flag))) break;
+                // buffer b last held P_{j-NB}: its PV must have finished reading it
+                if (j >= NB && !(ok = wait_bar(bar_o_done + b, ((j - NB) / NB) & 1, abort_flag))) break;
                 tc_fence_after();
-                const uint32_t sK = smem_u32(smem + C::OFF_K + st * C::KV_BYTES);
+                const uint32_t sK = smem_u32(smem + C::OFF_K + sk * C::KV_BYTES);
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t koff = (kk >> 2) * C::ATOM_BYTES + (kk & 3) * 32;
-                    mma_bf16_ss(tmem + (sb ? C::TMEM_S1 : C::TMEM_S0), sdesc_sw128(sQ + koff, 16, 1024),
+                    mma_bf16_ss(tmem + C::TMEM_S + b * kAttnBN, sdesc_sw128(sQ + koff, 16, 1024),
                                 sdesc_sw128(sK + koff, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
                 }
-                mma_commit(bar_s_full + sb);
+                mma_commit(bar_s_full + b);
+                mma_commit(bar_k_empty + sk);
                 if (j >= 1) ok = issue_pv(j - 1);
             }
             if (ok && n_tiles > 0) ok = issue_pv(n_tiles - 1);
@@ -247,53 +246,41 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             drain_bar(bar_drain, 0);
         }
     } else {
-        // ------------------------------------------------------------ softmax + epilogue
+        // ------------------------------------------------------------ softmax + epilogue (warps 0-3)
         const int r = threadIdx.x;  // tile row == TMEM lane
         const int tok = it.tok0 + r / G;
         const bool valid = tok < it.tok1;
         const int frow = P.cu_fresh[it.query] + tok;
         const int pos = valid ? P.fresh_pos[frow] : 0x7fffffff;
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-        const uint32_t sP = smem_u32(smem + C::OFF_P);
         float m = -INFINITY, l = 0.f;
         bool ok = true;
         for (int j = 0; j < n_tiles; ++j) {
-            const int sb = j & 1;
-            if (!(ok = warp_wait(bar_s_full + sb, (j >> 1) & 1, abort_flag))) break;
+            const int b = j % NB;
+            if (!(ok = warp_wait(bar_s_full + b, (j / NB) & 1, abort_flag))) break;
             tc_fence_after();
             uint32_t s[128];
-            const uint32_t s_col = tmem + lane_base + (sb ? C::TMEM_S1 : C::TMEM_S0);
+            const uint32_t s_col = tmem + lane_base + C::TMEM_S + b * kAttnBN;
             tmem_ld32(s_col + 0, *reinterpret_cast<uint32_t(*)[32]>(s + 0));
             tmem_ld32(s_col + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
             tmem_ld32(s_col + 64, *reinterpret_cast<uint32_t(*)[32]>(s + 64));
             tmem_ld32(s_col + 96, *reinterpret_cast<uint32_t(*)[32]>(s + 96));
             tmem_ld_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar_s_free + sb);
 
-            float x[128];
+            // raw row max (scale > 0 commutes with max); masked slots become -inf
             const int key0 = (it.kv_tile0 + j) * kAttnBN;
-            float mt = -INFINITY;
+            float mx = -INFINITY;
             if (key0 + kAttnBN - 1 > it.min_pos) {
 #pragma unroll
                 for (int c = 0; c < 128; ++c) {
-                    x[c] = (key0 + c > pos) ? -INFINITY : __uint_as_float(s[c]) * scale_log2;
-                    mt = fmaxf(mt, x[c]);
+                    if (key0 + c > pos) s[c] = __float_as_uint(-INFINITY);
+                    mx = fmaxf(mx, __uint_as_float(s[c]));
                 }
             } else {
 #pragma unroll
-                for (int c = 0; c < 128; ++c) {
-                    x[c] = __uint_as_float(s[c]) * scale_log2;
-                    mt = fmaxf(mt, x[c]);
-                }
+                for (int c = 0; c < 128; ++c) mx = fmaxf(mx, __uint_as_float(s[c]));
             }
-            const float m_new = fmaxf(m, mt);
-            if (j > 0) {
-                // PV_{j-1} complete: P may be overwritten and O is stable
-                if (!(ok = warp_wait(bar_o_done, (j - 1) & 1, abort_flag))) break;
-                tc_fence_after();
-            }
+            const float m_new = fmaxf(m, mx * scale_log2);
             const bool resc = m_new > m + kRescaleThreshold;
             float alpha = 1.f;
             if (resc) {
@@ -302,6 +289,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 m = m_new;
             }
             if (j > 0 && __any_sync(0xffffffffu, resc)) {
+                // O is touched only while no PV is in flight: PV_{j-1} done, PV_j not yet issued
+                if (!(ok = warp_wait(bar_o_done + (j - 1) % NB, ((j - 1) / NB) & 1, abort_flag))) break;
+                tc_fence_after();
 #pragma unroll
                 for (int c4 = 0; c4 < D / 32; ++c4) {
                     uint32_t o[32];
@@ -312,29 +302,27 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
                     tmem_st32(o_col, o);
                 }
-                tmem_st_wait();
             }
             const float mu = (m == -INFINITY) ? 0.f : m;
             float rs = 0.f;
+            uint32_t pk[64];
 #pragma unroll
-            for (int cc = 0; cc < 16; ++cc) {
-                float p[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    p[e] = ex2_approx(x[cc * 8 + e] - mu);
-                    rs += p[e];
-                }
-                const uint32_t addr = sP + (cc >> 3) * C::ATOM_BYTES + r * 128 + ((((cc & 7) ^ (r & 7))) << 4);
-                st_shared_v4(addr, pack2_bf16(p[0], p[1]), pack2_bf16(p[2], p[3]), pack2_bf16(p[4], p[5]),
-                             pack2_bf16(p[6], p[7]));
+            for (int c = 0; c < 64; ++c) {
+                const float p0 = ex2_approx(fmaf(__uint_as_float(s[2 * c]), scale_log2, -mu));
+                const float p1 = ex2_approx(fmaf(__uint_as_float(s[2 * c + 1]), scale_log2, -mu));
+                rs += p0 + p1;
+                pk[c] = pack2_bf16(p0, p1);
             }
             l += rs;
-            fence_proxy_async_smem();
+            // P_j (bf16) over the first 64 columns of its S buffer, read there by the PV MMA
+            tmem_st32(s_col + 0, *reinterpret_cast<uint32_t(*)[32]>(pk + 0));
+            tmem_st32(s_col + 32, *reinterpret_cast<uint32_t(*)[32]>(pk + 32));
+            tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar_p_full);
+            if (lane == 0) mbar_arrive(bar_p_full + b);
         }
-        if (ok && n_tiles > 0) ok = warp_wait(bar_o_done, (n_tiles - 1) & 1, abort_flag);
+        if (ok && n_tiles > 0) ok = warp_wait(bar_o_done + (n_tiles - 1) % NB, ((n_tiles - 1) / NB) & 1, abort_flag);
         if (ok) {
             tc_fence_after();
             if (it.slot < 0) {

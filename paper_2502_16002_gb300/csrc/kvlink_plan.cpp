@@ -158,6 +158,8 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     }
 
     // ---- attention work items
+    // M-tiles of one (query, KV head) split the query's fresh tokens into near-equal
+    // runs of at most kAttnBM / G tokens; a tile's key range ends at its last token.
     const int G = d->h_q / d->h_kv;
     const int tok_per_tile = kAttnBM / G;
     struct Tile { int32_t b, g, t0, t1, n_tiles, min_pos; };
@@ -167,11 +169,12 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     for (int b = 0; b < B; ++b) {
         const int32_t f0 = p->cu_fresh[b], T = p->cu_fresh[b + 1] - f0;
         for (int r = 0; r < T; ++r) p->attn_pairs += (int64_t)p->fresh_pos[f0 + r] + 1;
-        for (int t0 = 0; t0 < T; t0 += tok_per_tile) {
-            const int t1 = std::min(T, t0 + tok_per_tile);
-            const int32_t kv_len = p->fresh_pos[f0 + t1 - 1] + 1;  // positions increase within a query
-            const int32_t nt = (kv_len + kAttnBN - 1) / kAttnBN;
-            for (int g = 0; g < d->h_kv; ++g) {
+        const int n_mt = (T + tok_per_tile - 1) / tok_per_tile;
+        for (int g = 0; g < d->h_kv; ++g) {
+            for (int mt = 0; mt < n_mt; ++mt) {
+                const int t0 = (int)((int64_t)T * mt / n_mt), t1 = (int)((int64_t)T * (mt + 1) / n_mt);
+                const int32_t kv_len = p->fresh_pos[f0 + t1 - 1] + 1;  // positions increase within a query
+                const int32_t nt = (kv_len + kAttnBN - 1) / kAttnBN;
                 tiles.push_back({b, g, t0, t1, nt, p->fresh_pos[f0 + t0]});
                 work += nt;
             }
@@ -197,9 +200,23 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         }
         p->n_slots += n_split;
     }
-    std::stable_sort(p->items.begin(), p->items.end(), [](const AttnItem& x, const AttnItem& y) {
-        return (x.kv_tile1 - x.kv_tile0) > (y.kv_tile1 - y.kv_tile0);
-    });
+    // Launch order: the items of one (query, KV head) stay adjacent, so that CTAs running
+    // at the same time read the same K/V tiles (served from L2 after the first); groups
+    // go longest first, and so do the items inside a group.
+    {
+        std::vector<int64_t> group_cost((size_t)B * d->h_kv, 0);
+        for (const AttnItem& it : p->items)
+            group_cost[(size_t)it.query * d->h_kv + it.kv_head] =
+                std::max<int64_t>(group_cost[(size_t)it.query * d->h_kv + it.kv_head], it.kv_tile1 - it.kv_tile0);
+        std::stable_sort(p->items.begin(), p->items.end(), [&](const AttnItem& x, const AttnItem& y) {
+            const int64_t gx = group_cost[(size_t)x.query * d->h_kv + x.kv_head];
+            const int64_t gy = group_cost[(size_t)y.query * d->h_kv + y.kv_head];
+            if (gx != gy) return gx > gy;
+            if (x.query != y.query) return x.query < y.query;
+            if (x.kv_head != y.kv_head) return x.kv_head < y.kv_head;
+            return (x.kv_tile1 - x.kv_tile0) > (y.kv_tile1 - y.kv_tile0);
+        });
+    }
     p->workspace_bytes = (size_t)p->n_slots * (size_t)kAttnBM * ((size_t)d->head_dim + 2) * sizeof(float);
 
     // ---- device buffer layout (256-byte aligned tables)
