@@ -63,57 +63,81 @@ def _cores():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 200 ms while running."""
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms in a background reader.
 
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    Each line is stamped when it arrives; summary() keeps the samples that fall inside
+    the window marked with start() / stop()."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, gpu_index: int):
         self.gpu = gpu_index
         self.proc = None
-        self.out = None
+        self.lines = []
+        self.t0 = self.t1 = None
 
     def __enter__(self):
+        import threading
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
                  "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except (FileNotFoundError, OSError):
             self.proc = None
+            return self
+
+        def reader():
+            for line in self.proc.stdout:
+                self.lines.append((time.time(), line))
+
+        self.thread = threading.Thread(target=reader, daemon=True)
+        self.thread.start()
+        time.sleep(0.5)  # let the first samples arrive before the timed region
         return self
+
+    def start(self):
+        self.t0 = time.time()
+
+    def stop(self):
+        self.t1 = time.time()
 
     def __exit__(self, *a):
         if self.proc is None:
             return
+        time.sleep(0.3)
         self.proc.terminate()
         try:
-            self.out, _ = self.proc.communicate(timeout=5)
+            self.proc.wait(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
-            self.out, _ = self.proc.communicate()
+        self.thread.join(timeout=5)
 
     def summary(self):
-        if not self.out:
+        if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        sm, mx, reasons = [], None, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in self.out.strip().splitlines():
+        sm, mx, reasons, n_all = [], None, set(), 0
+        for t, line in self.lines:
             f = [x.strip() for x in line.split(",")]
-            if len(f) < 9:
+            if len(f) < 8:
+                continue
+            n_all += 1
+            if self.t0 is not None and not (self.t0 - 0.2 <= t <= self.t1 + 0.2):
                 continue
             try:
-                sm.append(float(f[1]))
-                mx = float(f[2])
+                sm.append(float(f[0]))
+                mx = float(f[1])
             except ValueError:
                 continue
-            for n, v in zip(names, f[5:9]):
+            for n, v in zip(names, f[4:8]):
                 if v.lower().startswith("active"):
                     reasons.add(n)
         if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": sorted(reasons)}
-        load = [s for s in sm if s > 0.5 * (mx or max(sm))] or sm
-        return {"sm_mhz": statistics.median(load), "sm_max_mhz": mx, "reasons": sorted(reasons),
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": 0,
+                    "samples_total": n_all}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
                 "samples": len(sm)}
 
 
@@ -201,11 +225,13 @@ def run_ours(args, rank, world, local_rank):
     with ClockSampler(local_rank) as clk:
         barrier()
         torch.cuda.synchronize(dev)
+        clk.start()
         e0.record(stream)
         for _ in range(args.steps):
             step()
         e1.record(stream)
         torch.cuda.synchronize(dev)
+        clk.stop()
         barrier()
     ms_total = max_over_ranks(e0.elapsed_time(e1))
     ms_per_step = ms_total / args.steps
@@ -214,10 +240,11 @@ def run_ours(args, rank, world, local_rank):
     assert K.kvlink_device_status() == 0
 
     # ---- per-kernel pass: same work through the separate calls, events around each
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(L * args.steps)]
+    k_steps = min(args.steps, 20)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(L * k_steps)]
     torch.cuda.synchronize(dev)
     i = 0
-    for _ in range(args.steps):
+    for _ in range(k_steps):
         for l in range(L):
             a, b_, c = ev[i]
             a.record(stream)
@@ -385,8 +412,8 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--config", type=int, default=3)
     ap.add_argument("--layers", type=int, default=0,
                     help="layers per step (default: the workload's); fewer only for small profiling runs")

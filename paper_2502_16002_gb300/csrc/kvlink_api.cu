@@ -12,9 +12,11 @@
 namespace kvlink {
 void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float4* d_rope, int head_dim,
                        double theta, cudaStream_t stream);
-void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv,
-                     int pool_bs, const void* pool_k, const void* pool_v, const void* k_new,
-                     const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
+void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv, int num_sms,
+                     const void* pool_k, const void* pool_v, const void* k_new, const void* v_new, void* cache_k,
+                     void* cache_v, cudaStream_t stream);
+int read_copy_status(int32_t* status);
+int clear_copy_status();
 void launch_attention_simt(const DevicePlan& P, int n_fresh, int head_dim, int h_q, int h_kv,
                            const void* q, const void* cache_k, const void* cache_v, void* out,
                            cudaStream_t stream);
@@ -200,8 +202,8 @@ int kvlink_reencode_concat(const kvlink_plan_t* p, const void* pool_k, const voi
     if (!pool_k || !pool_v || !cache_k || !cache_v) return KVLINK_EINVAL;
     if (!aligned16(pool_k) || !aligned16(pool_v) || !aligned16(cache_k) || !aligned16(cache_v))
         return KVLINK_EINVAL;
-    launch_reencode(p->dev, 0, p->n_chunks_cached, p->head_dim, p->h_kv, p->pool_block_size, pool_k,
-                    pool_v, nullptr, nullptr, cache_k, cache_v, (cudaStream_t)stream);
+    launch_reencode(p->dev, 0, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, pool_k, pool_v, nullptr,
+                    nullptr, cache_k, cache_v, (cudaStream_t)stream);
     return check_launch("reencode_kernel");
 }
 
@@ -209,7 +211,7 @@ static int place_fresh(const kvlink_plan_t* p, const void* k_new, const void* v_
                        void* cache_v, cudaStream_t s) {
     const int n_all = (int)p->chunks.size();
     launch_reencode(p->dev, p->n_chunks_cached, n_all - p->n_chunks_cached, p->head_dim, p->h_kv,
-                    p->pool_block_size, nullptr, nullptr, k_new, v_new, cache_k, cache_v, s);
+                    p->num_sms, nullptr, nullptr, k_new, v_new, cache_k, cache_v, s);
     return check_launch("fresh placement");
 }
 
@@ -270,8 +272,8 @@ int kvlink_linked_prefill(const kvlink_plan_t* p, const void* pool_k, const void
     if (!aligned16(pool_k) || !aligned16(pool_v) || !aligned16(k_new) || !aligned16(v_new))
         return KVLINK_EINVAL;
     cudaStream_t s = (cudaStream_t)stream;
-    launch_reencode(p->dev, 0, (int)p->chunks.size(), p->head_dim, p->h_kv, p->pool_block_size, pool_k,
-                    pool_v, k_new, v_new, cache_k, cache_v, s);
+    launch_reencode(p->dev, 0, (int)p->chunks.size(), p->head_dim, p->h_kv, p->num_sms, pool_k, pool_v, k_new,
+                    v_new, cache_k, cache_v, s);
     rc = check_launch("reencode_kernel (fused)");
     if (rc) return rc;
     return attention_common(p, q, cache_k, cache_v, out, ws, ws_bytes, s);
@@ -279,10 +281,16 @@ int kvlink_linked_prefill(const kvlink_plan_t* p, const void* pool_k, const void
 
 int kvlink_device_status(int32_t* status) {
     if (!status) return KVLINK_EINVAL;
-    *status = 0;
-    return read_attention_status(status);
+    int32_t a = 0, c = 0;
+    int rc = read_attention_status(&a);
+    if (rc == KVLINK_OK) rc = read_copy_status(&c);
+    *status = a != 0 ? a : c;
+    return rc;
 }
 
-int kvlink_clear_device_status(void) { return clear_attention_status(); }
+int kvlink_clear_device_status(void) {
+    const int rc = clear_attention_status();
+    return rc != KVLINK_OK ? rc : clear_copy_status();
+}
 
 }  // extern "C"

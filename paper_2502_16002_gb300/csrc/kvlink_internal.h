@@ -13,14 +13,26 @@ namespace kvlink {
 
 constexpr int kAttnBM = 128;     // (fresh token, query head) rows per attention tile
 constexpr int kAttnBN = 128;     // keys per KV tile
-constexpr int kCopyChunk = 32;   // tokens per re-encode work unit
-constexpr int kCopyThreads = 256;
+constexpr int kCopyStageBytes = 32768;   // K (or V) bytes of one re-encode work unit
+constexpr int kCopyMaxTokens = 128;
 
-// One re-encode work unit: tokens [t0, t0 + kCopyChunk) of segment `seg`.
+// Tokens per re-encode work unit for a given K row size (H_kv * D * 2 bytes).
+inline int copy_chunk_tokens(int row_bytes) {
+    int t = kCopyStageBytes / row_bytes;
+    return t < 8 ? 8 : (t > kCopyMaxTokens ? kCopyMaxTokens : t);
+}
+
+// One re-encode work unit: n consecutive tokens whose K/V rows are contiguous both in
+// the source (pool or fresh rows) and in the linked cache.  Resolved on the host.
 struct CopyChunk {
-    int32_t seg;
-    int32_t t0;
+    int64_t src_row;   // first source row (pool row, or fresh row for LINK/QUESTION)
+    int64_t dst_row;   // first linked-cache row
+    int32_t n;         // tokens
+    int32_t kind;      // KVLINK_SEG_*
+    int32_t table;     // RoPE delta table row (documents), else -1
+    int32_t seg;       // segment index
 };
+static_assert(sizeof(CopyChunk) == 32, "CopyChunk layout");
 
 // One attention work item: an M-tile of (token, head) rows of one query and KV head,
 // over KV tiles [kv_tile0, kv_tile1).

@@ -146,13 +146,29 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     p->cu_fresh[B] = (int32_t)fresh;
     if (fresh > INT32_MAX / 64) return fail(why, KVLINK_EUNSUPPORTED, "too many fresh rows");
 
-    // ---- re-encode work units: cached segments first, then fresh segments
+    // ---- re-encode work units: cached segments first, then fresh segments.  A unit never
+    // crosses a pool block, so its source rows, like its cache rows, are contiguous.
     p->chunks.clear();
+    const int ct = copy_chunk_tokens(d->h_kv * d->head_dim * 2);
     for (int pass = 0; pass < 2; ++pass) {
         for (size_t s = 0; s < p->seg.size(); ++s) {
-            const bool cached = p->seg[s].kind == KVLINK_SEG_PREFIX || p->seg[s].kind == KVLINK_SEG_DOC;
+            const kvlink_segment_t& sg = p->seg[s];
+            const bool cached = sg.kind == KVLINK_SEG_PREFIX || sg.kind == KVLINK_SEG_DOC;
             if (cached != (pass == 0)) continue;
-            for (int t = 0; t < p->seg[s].len; t += kCopyChunk) p->chunks.push_back({(int32_t)s, t});
+            for (int t = 0; t < sg.len;) {
+                int n = std::min(ct, sg.len - t);
+                int64_t src;
+                if (!cached) {
+                    src = (int64_t)sg.src + t;
+                } else if (bs == 0) {
+                    src = p->pool_start[sg.src] + t;
+                } else {
+                    n = std::min(n, bs - t % bs);
+                    src = (int64_t)p->pool_block_table[p->pool_start[sg.src] + t / bs] * bs + t % bs;
+                }
+                p->chunks.push_back({src, sg.dst + t, n, sg.kind, sg.table, (int32_t)s});
+                t += n;
+            }
         }
         if (pass == 0) p->n_chunks_cached = (int32_t)p->chunks.size();
     }

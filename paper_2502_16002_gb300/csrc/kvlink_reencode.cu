@@ -1,13 +1,11 @@
 // RoPE delta table (Sec. 2.2, once per batch) and the re-encode + concat kernel
 // (Sec. 2.2 positional re-encoding, Sec. 2.1 concatenation of the caches).
 //
-// The re-encode kernel is a streaming copy bound by HBM bandwidth.  One CTA takes
-// one work unit: kCopyChunk tokens of one segment.  A thread owns a fixed
-// (KV head, j0) slot across the unit's tokens: it moves the 16-byte key chunks
-// holding dimensions j0..j0+7 and j0+D/2..j0+D/2+7 (the two halves of the RoPE
-// pairs it rotates) and the value chunks at the same offsets, so every load and
-// store is a coalesced 128-bit access and the eight (cos, sin) pairs of the
-// segment's delta stay in registers for the whole unit.
+// The re-encode kernel is a streaming copy bound by HBM bandwidth.  Work units are
+// runs of tokens whose K/V rows are contiguous in the source and in the linked
+// cache (resolved on the host).  A persistent CTA per SM pipelines its units
+// through a 3-stage shared-memory ring with bulk (TMA) copies: global -> shared
+// loads, an in-place rotation of the document keys, shared -> global stores.
 //
 // Precision: a rotated component x cos a - y sin a can cancel to far below |x|,
 // where the bf16 quantum is tiny; an fp32 cos/sin (relative error 2^-24) would
@@ -20,6 +18,7 @@
 #include <cuda_runtime.h>
 
 #include "kvlink_internal.h"
+#include "kvlink_sm100.cuh"
 
 namespace kvlink {
 
@@ -54,16 +53,8 @@ void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float4* d_rope,
 }
 
 // --------------------------------------------------------------------------
-// A3 + A4: re-encode/copy one work unit per CTA.
+// Rotation of one (lo, hi) pair of 16-byte key chunks: 8 RoPE pairs (j, j + D/2).
 // --------------------------------------------------------------------------
-__device__ __forceinline__ uint4 ld_stream(const uint4* p) {
-    uint4 r;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-                 : "l"(p));
-    return r;
-}
-
 __device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
@@ -109,96 +100,193 @@ __device__ __forceinline__ void rotate8(uint4& lo, uint4& hi, const float4 (&cs)
     }
 }
 
-template <int D>
-__global__ void __launch_bounds__(kCopyThreads) reencode_kernel(
-    DevicePlan P, int chunk_base, int h_kv, int pool_bs,
-    const __nv_bfloat16* __restrict__ pool_k, const __nv_bfloat16* __restrict__ pool_v,
-    const __nv_bfloat16* __restrict__ k_new, const __nv_bfloat16* __restrict__ v_new,
-    __nv_bfloat16* __restrict__ cache_k, __nv_bfloat16* __restrict__ cache_v) {
-    constexpr int UPH = D / 16;  // (lo, hi) chunk pairs per head
-    const int U = h_kv * UPH;    // pairs per token (divides kCopyThreads)
-    const int TP = kCopyThreads / U;
-    const CopyChunk ch = P.chunks[chunk_base + blockIdx.x];
-    const kvlink_segment_t sg = P.seg[ch.seg];
-    const int n = min(kCopyChunk, sg.len - ch.t0);
-    const int unit = threadIdx.x % U;
-    const int tok = threadIdx.x / U;
-    const int head = unit / UPH;
-    const int j0 = (unit % UPH) * 8;
-    const int64_t row_elems = (int64_t)h_kv * D;
-    const int64_t lo_off = (int64_t)head * D + j0;
-    const int64_t hi_off = lo_off + D / 2;
+// --------------------------------------------------------------------------
+// A3 + A4: persistent re-encode/copy through a shared-memory ring.
+// --------------------------------------------------------------------------
+constexpr int kCopyConsumers = 128;                  // 4 warps rotate keys in shared memory
+constexpr int kCopyThreads = 32 + kCopyConsumers;    // + 1 producer warp
+constexpr int kCopyStages = 3;
+constexpr uint64_t kCopyWaitLimitNs = 2000000000ull;
+constexpr int32_t kCopyStatusWaitTimeout = 0x21;
 
-    const bool fresh = sg.kind == KVLINK_SEG_LINK || sg.kind == KVLINK_SEG_QUESTION;
-    const bool rotate = sg.kind == KVLINK_SEG_DOC;
-    const __nv_bfloat16* sk = fresh ? k_new : pool_k;
-    const __nv_bfloat16* sv = fresh ? v_new : pool_v;
+static __device__ int32_t g_copy_status;
 
-    float4 cs[8];
-    if (rotate) {
-        const float4* t = P.rope + (int64_t)sg.table * (D / 2) + j0;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) cs[q] = __ldg(t + q);
-    } else {
-#pragma unroll
-        for (int q = 0; q < 8; ++q) cs[q] = make_float4(1.f, 0.f, 0.f, 0.f);
-    }
-    const int64_t entry_start = fresh ? 0 : P.pool_start[sg.src];
+struct CopySmem {
+    static constexpr uint32_t STAGE = 2 * kCopyStageBytes;   // K then V
+    static constexpr uint32_t OFF_BAR = kCopyStages * STAGE;
+    static constexpr uint32_t BYTES = OFF_BAR + 2 * kCopyStages * 8 + 16 + 128;
+};
 
-    auto src_row = [&](int tt) -> int64_t {
-        if (fresh) return (int64_t)sg.src + tt;
-        if (pool_bs == 0) return entry_start + tt;
-        return (int64_t)P.pool_block_table[entry_start + tt / pool_bs] * pool_bs + tt % pool_bs;
-    };
-
-    // two tokens per iteration: all eight 16-byte loads are issued before any store
-    for (int t = tok; t < n; t += 2 * TP) {
-        const int ta = ch.t0 + t;
-        const bool has_b = t + TP < n;
-        const int tb = ta + TP;
-        const int64_t ra = src_row(ta) * row_elems;
-        const int64_t rb = has_b ? src_row(tb) * row_elems : ra;
-        uint4 ka0 = ld_stream(reinterpret_cast<const uint4*>(sk + ra + lo_off));
-        uint4 ka1 = ld_stream(reinterpret_cast<const uint4*>(sk + ra + hi_off));
-        const uint4 va0 = ld_stream(reinterpret_cast<const uint4*>(sv + ra + lo_off));
-        const uint4 va1 = ld_stream(reinterpret_cast<const uint4*>(sv + ra + hi_off));
-        uint4 kb0, kb1, vb0, vb1;
-        if (has_b) {
-            kb0 = ld_stream(reinterpret_cast<const uint4*>(sk + rb + lo_off));
-            kb1 = ld_stream(reinterpret_cast<const uint4*>(sk + rb + hi_off));
-            vb0 = ld_stream(reinterpret_cast<const uint4*>(sv + rb + lo_off));
-            vb1 = ld_stream(reinterpret_cast<const uint4*>(sv + rb + hi_off));
-        }
-        if (rotate) rotate8(ka0, ka1, cs);
-        const int64_t da = (sg.dst + ta) * row_elems;
-        *reinterpret_cast<uint4*>(cache_k + da + lo_off) = ka0;
-        *reinterpret_cast<uint4*>(cache_k + da + hi_off) = ka1;
-        *reinterpret_cast<uint4*>(cache_v + da + lo_off) = va0;
-        *reinterpret_cast<uint4*>(cache_v + da + hi_off) = va1;
-        if (has_b) {
-            if (rotate) rotate8(kb0, kb1, cs);
-            const int64_t db = (sg.dst + tb) * row_elems;
-            *reinterpret_cast<uint4*>(cache_k + db + lo_off) = kb0;
-            *reinterpret_cast<uint4*>(cache_k + db + hi_off) = kb1;
-            *reinterpret_cast<uint4*>(cache_v + db + lo_off) = vb0;
-            *reinterpret_cast<uint4*>(cache_v + db + hi_off) = vb1;
+__device__ __forceinline__ bool copy_wait(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
+    if (sm100::mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = sm100::globaltimer_ns();
+    while (true) {
+        if (sm100::mbar_try_wait(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (sm100::globaltimer_ns() - t0 > kCopyWaitLimitNs) {
+            *abort_flag = 1;
+            atomicCAS(&g_copy_status, 0, kCopyStatusWaitTimeout);
+            return false;
         }
     }
 }
 
-void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv,
-                     int pool_bs, const void* pool_k, const void* pool_v, const void* k_new,
-                     const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream) {
+__device__ __forceinline__ void copy_drain(uint64_t* bar, uint32_t parity) {
+    const uint64_t t0 = sm100::globaltimer_ns();
+    while (!sm100::mbar_try_wait(bar, parity))
+        if (sm100::globaltimer_ns() - t0 > kCopyWaitLimitNs) {
+            atomicCAS(&g_copy_status, 0, kCopyStatusWaitTimeout);
+            return;
+        }
+}
+
+// CTA b handles the contiguous range of work units [n*b/grid, n*(b+1)/grid).
+// Producer (warp 0, one thread): bulk-loads a unit's K rows and V rows into a stage.
+// Consumers (warps 1-4): rotate the unit's keys in place when it is a document (each
+// thread keeps a fixed (head, j0) slot and its eight double-float cos/sin pairs), then
+// one thread bulk-stores K and V to the linked cache and frees the stage once the
+// stores have read it.  V is never touched by the threads.
+template <int D>
+__global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
+    const CopyChunk* __restrict__ chunks, int n_chunks, const float4* __restrict__ rope, int h_kv,
+    const __nv_bfloat16* __restrict__ pool_k, const __nv_bfloat16* __restrict__ pool_v,
+    const __nv_bfloat16* __restrict__ k_new, const __nv_bfloat16* __restrict__ v_new,
+    __nv_bfloat16* __restrict__ cache_k, __nv_bfloat16* __restrict__ cache_v) {
+    using namespace sm100;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    uint8_t* smem = smem_raw + ((128u - (raw_addr & 127u)) & 127u);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + CopySmem::OFF_BAR);
+    uint64_t* empty = full + kCopyStages;
+    volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(empty + kCopyStages);
+
+    const int c_begin = (int)((int64_t)n_chunks * blockIdx.x / gridDim.x);
+    const int c_end = (int)((int64_t)n_chunks * (blockIdx.x + 1) / gridDim.x);
+    const int64_t row_elems = (int64_t)h_kv * D;
+    const uint32_t row_bytes = (uint32_t)(row_elems * 2);
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kCopyStages; ++i) {
+            mbar_init(full + i, 1);
+            mbar_init(empty + i, 1);
+        }
+        *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_copy_status) != 0 ? 1 : 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (*abort_flag) return;  // uniform: written before the barrier
+
+    if (threadIdx.x < 32) {
+        // ------------------------------------------------------------ producer
+        if (threadIdx.x == 0) {
+            int issued = 0;
+            for (int c = c_begin, i = 0; c < c_end; ++c, ++i) {
+                const int st = i % kCopyStages;
+                if (!copy_wait(empty + st, ((i / kCopyStages) & 1) ^ 1, abort_flag)) break;
+                const CopyChunk ch = chunks[c];
+                const bool fresh = ch.kind == KVLINK_SEG_LINK || ch.kind == KVLINK_SEG_QUESTION;
+                const __nv_bfloat16* sk = (fresh ? k_new : pool_k) + ch.src_row * row_elems;
+                const __nv_bfloat16* sv = (fresh ? v_new : pool_v) + ch.src_row * row_elems;
+                const uint32_t bytes = (uint32_t)ch.n * row_bytes;
+                uint8_t* stage = smem + st * CopySmem::STAGE;
+                mbar_arrive_expect_tx(full + st, 2 * bytes);
+                bulk_load(stage, sk, bytes, full + st);
+                bulk_load(stage + kCopyStageBytes, sv, bytes, full + st);
+                issued = i + 1;
+            }
+            // no load may still be in flight when the CTA leaves
+            for (int i = issued - kCopyStages > 0 ? issued - kCopyStages : 0; i < issued; ++i)
+                copy_drain(full + i % kCopyStages, (i / kCopyStages) & 1);
+        }
+        return;
+    }
+
+    // ---------------------------------------------------------------- consumers
+    const int tc = threadIdx.x - 32;
+    constexpr int UPH = D / 16;                // (lo, hi) chunk pairs per head
+    const int U = h_kv * UPH;                  // pairs per token, a power of two <= 128
+    const int TPP = kCopyConsumers / U;        // tokens per pass
+    const int unit = tc % U;
+    const int tok0 = tc / U;
+    const int head = unit / UPH;
+    const int j0 = (unit % UPH) * 8;
+    const uint32_t lo_off = (uint32_t)(head * D + j0) * 2;
+    int cur_table = -1;
+    float4 cs[8];
+    for (int c = c_begin, i = 0; c < c_end; ++c, ++i) {
+        const int st = i % kCopyStages;
+        copy_wait(full + st, (i / kCopyStages) & 1, abort_flag);
+        named_bar_sync(1, kCopyConsumers);
+        if (*abort_flag) break;  // uniform: every consumer passed the barrier first
+        const CopyChunk ch = chunks[c];
+        uint8_t* stage = smem + st * CopySmem::STAGE;
+        if (ch.kind == KVLINK_SEG_DOC) {
+            if (ch.table != cur_table) {
+                const float4* t = rope + (int64_t)ch.table * (D / 2) + j0;
+#pragma unroll
+                for (int q = 0; q < 8; ++q) cs[q] = __ldg(t + q);
+                cur_table = ch.table;
+            }
+            for (int t = tok0; t < ch.n; t += TPP) {
+                uint4* lo = reinterpret_cast<uint4*>(stage + (uint32_t)t * row_bytes + lo_off);
+                uint4* hi = reinterpret_cast<uint4*>(stage + (uint32_t)t * row_bytes + lo_off + D);
+                uint4 a = *lo, b = *hi;
+                rotate8(a, b, cs);
+                *lo = a;
+                *hi = b;
+            }
+            fence_proxy_async_smem();  // the bulk store reads these writes through the async proxy
+        }
+        named_bar_sync(1, kCopyConsumers);
+        if (tc == 0) {
+            const uint32_t bytes = (uint32_t)ch.n * row_bytes;
+            bulk_store(cache_k + ch.dst_row * row_elems, stage, bytes);
+            bulk_store(cache_v + ch.dst_row * row_elems, stage + kCopyStageBytes, bytes);
+            bulk_commit();
+            bulk_wait_read<1>();  // the previous unit's stores have read their stage
+            if (i > 0) mbar_arrive(empty + (i - 1) % kCopyStages);
+        }
+    }
+    if (tc == 0) bulk_wait<0>();
+}
+
+void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv, int num_sms,
+                     const void* pool_k, const void* pool_v, const void* k_new, const void* v_new, void* cache_k,
+                     void* cache_v, cudaStream_t stream) {
     if (n_chunks <= 0) return;
     using bf = __nv_bfloat16;
-    if (head_dim == 128)
-        reencode_kernel<128><<<n_chunks, kCopyThreads, 0, stream>>>(
-            P, chunk_base, h_kv, pool_bs, (const bf*)pool_k, (const bf*)pool_v, (const bf*)k_new,
-            (const bf*)v_new, (bf*)cache_k, (bf*)cache_v);
-    else
-        reencode_kernel<64><<<n_chunks, kCopyThreads, 0, stream>>>(
-            P, chunk_base, h_kv, pool_bs, (const bf*)pool_k, (const bf*)pool_v, (const bf*)k_new,
-            (const bf*)v_new, (bf*)cache_k, (bf*)cache_v);
+    const int grid = n_chunks < num_sms ? n_chunks : num_sms;
+    const CopyChunk* ch = P.chunks + chunk_base;
+    if (head_dim == 128) {
+        static bool attr = false;
+        if (!attr) {
+            cudaFuncSetAttribute(reencode_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)CopySmem::BYTES);
+            attr = true;
+        }
+        reencode_kernel<128><<<grid, kCopyThreads, CopySmem::BYTES, stream>>>(
+            ch, n_chunks, P.rope, h_kv, (const bf*)pool_k, (const bf*)pool_v, (const bf*)k_new, (const bf*)v_new,
+            (bf*)cache_k, (bf*)cache_v);
+    } else {
+        static bool attr = false;
+        if (!attr) {
+            cudaFuncSetAttribute(reencode_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)CopySmem::BYTES);
+            attr = true;
+        }
+        reencode_kernel<64><<<grid, kCopyThreads, CopySmem::BYTES, stream>>>(
+            ch, n_chunks, P.rope, h_kv, (const bf*)pool_k, (const bf*)pool_v, (const bf*)k_new, (const bf*)v_new,
+            (bf*)cache_k, (bf*)cache_v);
+    }
+}
+
+int read_copy_status(int32_t* status) {
+    return cudaMemcpyFromSymbol(status, g_copy_status, sizeof(int32_t)) == cudaSuccess ? KVLINK_OK : KVLINK_ECUDA;
+}
+
+int clear_copy_status() {
+    const int32_t z = 0;
+    return cudaMemcpyToSymbol(g_copy_status, &z, sizeof(int32_t)) == cudaSuccess ? KVLINK_OK : KVLINK_ECUDA;
 }
 
 }  // namespace kvlink
