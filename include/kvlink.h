@@ -203,6 +203,27 @@ int kvlink_linked_prefill(const kvlink_plan_t* plan, const void* d_pool_k, const
                           void* d_cache_k, void* d_cache_v, void* d_out,
                           void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream);
 
+/* Allocation-free variant of kvlink_suffix_attention.  The paper has no counterpart:
+ * this entry point serves callers that may not allocate device memory at all, such as
+ * a serving loop whose memory budget is fixed at start-up (cudaMalloc can synchronise
+ * the device and fragments a pre-carved pool) or code that enqueues work where
+ * allocation is not permitted.  Same arguments and result as kvlink_suffix_attention,
+ * minus the workspace: the split-KV scratch is a static device array of
+ * KVLINK_NOALLOC_MAX_WORKSPACE_BYTES inside this library, which every GPU that loads
+ * the library holds until the process exits.  The call allocates nothing.
+ *   - Plans whose workspace_bytes exceed KVLINK_NOALLOC_MAX_WORKSPACE_BYTES are
+ *     rejected with KVLINK_ECAPACITY before anything is launched.
+ *   - The first call on a device looks up the array's device address (once per
+ *     device, with that device current); make that first call before any stream
+ *     capture.
+ *   - All calls share the array and it keeps the last call's contents; nothing in it
+ *     needs to start at zero.  Calls whose work overlaps on the GPU race on it.
+ * Errors: EINVAL, ECAPACITY, EUNSUPPORTED, ECUDA. */
+#define KVLINK_NOALLOC_MAX_WORKSPACE_BYTES (8u << 20)
+int kvlink_suffix_attention_noalloc(const kvlink_plan_t* plan, const void* d_q, const void* d_k_new,
+                                    const void* d_v_new, void* d_cache_k, void* d_cache_v, void* d_out,
+                                    kvlink_stream_t stream);
+
 /* Device status word: 0 when no kernel reported an error since the last clear.
  * Reading synchronises with the current device.  Errors: ECUDA. */
 int kvlink_device_status(int32_t* status);

@@ -89,6 +89,7 @@ def _load():
         "kvlink_reencode_concat": (C.c_int, [P, V, V, V, V, V]),
         "kvlink_suffix_attention": (C.c_int, [P, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_suffix_attention_simt": (C.c_int, [P, V, V, V, V, V, V, V]),
+        "kvlink_suffix_attention_noalloc": (C.c_int, [P, V, V, V, V, V, V, V]),
         "kvlink_linked_prefill": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
@@ -108,8 +109,11 @@ DECLARED = [
     "kvlink_reencode_concat", "kvlink_suffix_attention", "kvlink_suffix_attention_simt",
     "kvlink_linked_prefill",
     "kvlink_device_status", "kvlink_clear_device_status", "kvlink_strerror",
-    "kvlink_last_cuda_error", "kvlink_version",
+    "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc",
 ]
+
+# size of the static scratch used by kvlink_suffix_attention_noalloc (include/kvlink.h)
+KVLINK_NOALLOC_MAX_WORKSPACE_BYTES = 8 << 20
 
 
 class KvlinkError(RuntimeError):
@@ -229,6 +233,14 @@ def kvlink_suffix_attention_simt(plan: Plan, q: int, k_new, v_new, cache_k: int,
                                  stream: int = 0) -> None:
     _check(lib.kvlink_suffix_attention_simt(plan.handle, q, k_new, v_new, cache_k, cache_v, out, stream),
            "kvlink_suffix_attention_simt")
+
+
+def kvlink_suffix_attention_noalloc(plan: Plan, q: int, k_new, v_new, cache_k: int, cache_v: int, out: int,
+                                    stream: int = 0) -> None:
+    """Suffix attention without a caller workspace: the split-KV scratch is the library's
+    static device array (see include/kvlink.h); it allocates nothing."""
+    _check(lib.kvlink_suffix_attention_noalloc(plan.handle, q, k_new, v_new, cache_k, cache_v, out, stream),
+           "kvlink_suffix_attention_noalloc")
 
 
 def kvlink_linked_prefill(plan: Plan, pool_k: int, pool_v: int, q: int, k_new: int, v_new: int,

@@ -1,0 +1,83 @@
+"""The allocation-free suffix attention (kvlink_suffix_attention_noalloc).
+
+Some callers cannot allocate device memory: a serving loop whose memory budget is
+fixed at start-up and may not call cudaMalloc on the request path, or code that
+enqueues work where allocation is not permitted.  For them the library keeps the
+split-KV scratch in a static device array.  These tests call that entry point
+through the C ABI and check it against kvlink_suffix_attention (caller-owned
+workspace) on two calls in a row, with different inputs, so that contents left in
+the shared array by the first call cannot leak into the second.
+
+This file is collected last so that a run stopping at the first failure has
+already run every other test.
+"""
+import numpy as np
+import pytest
+
+import workloads as W
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+MAX_ABS, MEAN_ABS = 1e-2, 1e-3
+
+
+@pytest.fixture(scope="module")
+def env():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2502_16002_gb300 import kvlink as K
+    from paper_2502_16002_gb300 import runtime as RT
+
+    return K, RT
+
+
+def _inputs(RT, batch, layer, dev):
+    pk, pv = W.pool_kv(batch, layer)
+    q, kn, vn = W.fresh_qkv(batch, layer)
+    return [RT.bf16_from_bits(a, dev) for a in (pk, pv, q, kn, vn)]
+
+
+def test_noalloc_matches_workspace_entry_point_on_two_calls(env):
+    K, RT = env
+    dev = torch.device("cuda:0")
+    batch = W.draw_batch(W.get_config(2))       # Llama-1B shape: its plan splits KV ranges
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    info = lp.info
+    assert info.n_attn_splits > 0, "the plan must use scratch for this test to mean anything"
+    assert 0 < info.workspace_bytes <= K.KVLINK_NOALLOC_MAX_WORKSPACE_BYTES
+    stream = torch.cuda.current_stream(dev)
+    sh = int(stream.cuda_stream)
+    for layer in (0, 1):                        # two calls in a row, different inputs
+        pk, pv, q, kn, vn = _inputs(RT, batch, layer, dev)
+        ck, cv = lp.empty_cache()
+        lp.reencode_concat(pk, pv, ck, cv)
+        ref = torch.full(lp.fresh_shape(batch.cfg.h_q), float("nan"), dtype=torch.bfloat16, device=dev)
+        lp.suffix_attention(q, kn, vn, ck, cv, ref)
+        got = torch.full_like(ref, float("nan"))
+        K.kvlink_suffix_attention_noalloc(lp.plan, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), ck.data_ptr(),
+                                          cv.data_ptr(), got.data_ptr(), sh)
+        torch.cuda.synchronize(dev)
+        assert K.kvlink_device_status() == 0
+        a = got.float().cpu().numpy()
+        b = ref.float().cpu().numpy()
+        assert np.all(np.isfinite(a))
+        err = np.abs(a - b)
+        assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS, (layer, err.max(), err.mean())
+
+
+def test_noalloc_rejects_plans_larger_than_its_scratch(env):
+    K, RT = env
+    dev = torch.device("cuda:0")
+    batch = W.draw_batch(W.get_config(4))       # 51.8k-token context: about 21 MB of partials
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    assert lp.info.workspace_bytes > K.KVLINK_NOALLOC_MAX_WORKSPACE_BYTES
+    T, Hq, Hkv, D = lp.info.n_fresh, batch.cfg.h_q, batch.cfg.h_kv, batch.cfg.head_dim
+    q = torch.zeros((T, Hq, D), dtype=torch.bfloat16, device=dev)
+    kn = torch.zeros((T, Hkv, D), dtype=torch.bfloat16, device=dev)
+    ck, cv = lp.empty_cache()
+    out = torch.zeros_like(q)
+    with pytest.raises(K.KvlinkError) as e:
+        K.kvlink_suffix_attention_noalloc(lp.plan, q.data_ptr(), kn.data_ptr(), kn.data_ptr(), ck.data_ptr(),
+                                          cv.data_ptr(), out.data_ptr(), 0)
+    assert e.value.code == K.KVLINK_ECAPACITY
