@@ -110,6 +110,31 @@ __device__ __forceinline__ uint32_t pack2_bf16(float a, float b) {
     return *reinterpret_cast<const uint32_t*>(&h);
 }
 
+// 2^x for a pair of floats on the FMA pipe: x = n + f with n = rint(x) (taken from the
+// mantissa of x + 1.5*2^23) and f in [-1/2, 1/2]; 2^f from a degree-3 minimax polynomial
+// (Remez exchange on relative error, max relative error 7.5e-5, far below the bf16
+// quantum of P); 2^n added into the exponent field.  Inputs are clamped at -127, which
+// yields 0 or a value below 2^-126, i.e. nothing against any unmasked term.
+__device__ __forceinline__ uint64_t exp2_poly2(uint64_t x2) {
+    constexpr float kC0 = 0.99992806f, kC1 = 0.69326097f, kC2 = 0.24261113f, kC3 = 0.05517167f;
+    constexpr float kRound = 12582912.0f;  // 1.5 * 2^23
+    float a, b;
+    f2_unpack(x2, a, b);
+    const uint64_t x = f2_pack(fmaxf(a, -127.f), fmaxf(b, -127.f));
+    const uint64_t t = fadd2(x, f2_pack(kRound, kRound));
+    const uint64_t n = fadd2(t, f2_pack(-kRound, -kRound));
+    const uint64_t f = ffma2(n, f2_pack(-1.f, -1.f), x);
+    uint64_t p = ffma2(f, f2_pack(kC3, kC3), f2_pack(kC2, kC2));
+    p = ffma2(p, f, f2_pack(kC1, kC1));
+    p = ffma2(p, f, f2_pack(kC0, kC0));
+    float pa, pb, ta, tb;
+    f2_unpack(p, pa, pb);
+    f2_unpack(t, ta, tb);
+    const float ra = __int_as_float(__float_as_int(pa) + (int)((uint32_t)__float_as_int(ta) << 23));
+    const float rb = __int_as_float(__float_as_int(pb) + (int)((uint32_t)__float_as_int(tb) << 23));
+    return f2_pack(ra, rb);
+}
+
 // TMA producer loop for one ring (K or V): tiles j = 0..n-1 of the item's key range.
 template <int STAGES, int ATOMS>
 __device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes, const CUtensorMap* map,
@@ -267,19 +292,24 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             tmem_ld32(s_col + 96, *reinterpret_cast<uint32_t(*)[32]>(s + 96));
             tmem_ld_wait();
 
-            // raw row max (scale > 0 commutes with max); masked slots become -inf
+            // raw row max (scale > 0 commutes with max); masked slots become -inf.  Eight
+            // independent running maxima keep the dependency chain short.
             const int key0 = (it.kv_tile0 + j) * kAttnBN;
-            float mx = -INFINITY;
+            float mx8[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
             if (key0 + kAttnBN - 1 > it.min_pos) {
 #pragma unroll
                 for (int c = 0; c < 128; ++c) {
                     if (key0 + c > pos) s[c] = __float_as_uint(-INFINITY);
-                    mx = fmaxf(mx, __uint_as_float(s[c]));
+                    mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
                 }
             } else {
 #pragma unroll
-                for (int c = 0; c < 128; ++c) mx = fmaxf(mx, __uint_as_float(s[c]));
+                for (int c = 0; c < 128; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
             }
+            const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
             const float m_new = fmaxf(m, mx * scale_log2);
             const bool resc = m_new > m + kRescaleThreshold;
             float alpha = 1.f;
@@ -303,16 +333,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     tmem_st32(o_col, o);
                 }
             }
+            // p = exp2(s * scale - m) on column pairs (packed f32x2 arithmetic); three pairs
+            // in eight go to the FMA pipe (exp2_poly2), the rest to MUFU, to balance the two
             const float mu = (m == -INFINITY) ? 0.f : m;
-            float rs = 0.f;
+            const uint64_t sc2 = f2_pack(scale_log2, scale_log2);
+            const uint64_t nmu2 = f2_pack(-mu, -mu);
+            uint64_t acc[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) acc[e] = f2_pack(0.f, 0.f);
             uint32_t pk[64];
 #pragma unroll
             for (int c = 0; c < 64; ++c) {
-                const float p0 = ex2_approx(fmaf(__uint_as_float(s[2 * c]), scale_log2, -mu));
-                const float p1 = ex2_approx(fmaf(__uint_as_float(s[2 * c + 1]), scale_log2, -mu));
-                rs += p0 + p1;
+                const uint64_t x2 = ffma2(f2_pack(__uint_as_float(s[2 * c]), __uint_as_float(s[2 * c + 1])), sc2, nmu2);
+                uint64_t p2;
+                if ((c & 7) >= 5) {
+                    p2 = exp2_poly2(x2);
+                } else {
+                    float a, b;
+                    f2_unpack(x2, a, b);
+                    p2 = f2_pack(ex2_approx(a), ex2_approx(b));
+                }
+                acc[c & 3] = fadd2(acc[c & 3], p2);
+                float p0, p1;
+                f2_unpack(p2, p0, p1);
                 pk[c] = pack2_bf16(p0, p1);
             }
+            float rs0, rs1;
+            f2_unpack(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), rs0, rs1);
+            const float rs = rs0 + rs1;
             l += rs;
             // P_j (bf16) over the first 64 columns of its S buffer, read there by the PV MMA
             tmem_st32(s_col + 0, *reinterpret_cast<uint32_t(*)[32]>(pk + 0));

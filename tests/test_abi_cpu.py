@@ -158,3 +158,22 @@ def test_plan_is_deterministic(K):
     a = K.kvlink_plan_get_segments(_plan(K, batch))
     b = K.kvlink_plan_get_segments(_plan(K, batch))
     assert a.tobytes() == b.tobytes()
+
+
+def test_attention_exp2_polynomial_accuracy():
+    """The FMA-pipe 2^x used for part of the softmax: evaluate the kernel's own constants
+    and range reduction in float32 and check them against 2^x in float64."""
+    src = open(os.path.join(ROOT, "paper_2502_16002_gb300", "csrc", "kvlink_attention_tc.cu")).read()
+    c = {k: np.float32(v) for k, v in re.findall(r"\b(kC[0-3]) = ([0-9.]+)f", src)}
+    assert set(c) == {"kC0", "kC1", "kC2", "kC3"}
+    x = np.concatenate([np.linspace(-126, 8, 2_000_001), np.arange(-126, 9) + 0.5]).astype(np.float32)
+    rnd = np.float32(12582912.0)
+    t = (x + rnd).astype(np.float32)
+    n = (t - rnd).astype(np.float32)
+    f = (x - n).astype(np.float32)
+    assert np.all(np.abs(f) <= 0.5)
+    p = ((c["kC3"] * f + c["kC2"]) * f + c["kC1"]) * f + c["kC0"]
+    bits = p.astype(np.float32).view(np.int32) + (t.view(np.uint32) << np.uint32(23)).view(np.int32)
+    got = bits.view(np.float32).astype(np.float64)
+    want = np.exp2(x.astype(np.float64))
+    assert np.max(np.abs(got / want - 1)) < 1e-4
