@@ -113,14 +113,17 @@ __device__ __forceinline__ uint32_t pack2_bf16(float a, float b) {
 // 2^x for a pair of floats on the FMA pipe: x = n + f with n = rint(x) (taken from the
 // mantissa of x + 1.5*2^23) and f in [-1/2, 1/2]; 2^f from a degree-3 minimax polynomial
 // (Remez exchange on relative error, max relative error 7.5e-5, far below the bf16
-// quantum of P); 2^n added into the exponent field.  Inputs are clamped at -127, which
-// yields 0 or a value below 2^-126, i.e. nothing against any unmasked term.
+// quantum of P); 2^n added into the exponent field.  Inputs are clamped at kExpFloor =
+// -126 so that the exponent field never wraps (p >= 2^-1/2 keeps it >= 0): anything at
+// or below the floor comes out as a non-negative value under 2^-125, i.e. nothing
+// against any unmasked term.
 __device__ __forceinline__ uint64_t exp2_poly2(uint64_t x2) {
     constexpr float kC0 = 0.99992806f, kC1 = 0.69326097f, kC2 = 0.24261113f, kC3 = 0.05517167f;
     constexpr float kRound = 12582912.0f;  // 1.5 * 2^23
+    constexpr float kExpFloor = -126.0f;
     float a, b;
     f2_unpack(x2, a, b);
-    const uint64_t x = f2_pack(fmaxf(a, -127.f), fmaxf(b, -127.f));
+    const uint64_t x = f2_pack(fmaxf(a, kExpFloor), fmaxf(b, kExpFloor));
     const uint64_t t = fadd2(x, f2_pack(kRound, kRound));
     const uint64_t n = fadd2(t, f2_pack(-kRound, -kRound));
     const uint64_t f = ffma2(n, f2_pack(-1.f, -1.f), x);

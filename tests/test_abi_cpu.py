@@ -161,19 +161,26 @@ def test_plan_is_deterministic(K):
 
 
 def test_attention_exp2_polynomial_accuracy():
-    """The FMA-pipe 2^x used for part of the softmax: evaluate the kernel's own constants
-    and range reduction in float32 and check them against 2^x in float64."""
+    """The FMA-pipe 2^x used for part of the softmax: evaluate the kernel's own constants,
+    clamp and range reduction in float32 and check them against 2^x in float64, including
+    inputs far below the clamp (masked scores are -inf)."""
     src = open(os.path.join(ROOT, "paper_2502_16002_gb300", "csrc", "kvlink_attention_tc.cu")).read()
     c = {k: np.float32(v) for k, v in re.findall(r"\b(kC[0-3]) = ([0-9.]+)f", src)}
     assert set(c) == {"kC0", "kC1", "kC2", "kC3"}
-    x = np.concatenate([np.linspace(-126, 8, 2_000_001), np.arange(-126, 9) + 0.5]).astype(np.float32)
+    floor = np.float32(re.search(r"kExpFloor = (-?[0-9.]+)f", src).group(1))
+    x = np.concatenate([np.linspace(-140, 8, 3_000_001), np.arange(-140, 9) + 0.5,
+                        [-1e30, -np.inf]]).astype(np.float32)
+    xc = np.maximum(x, floor)
     rnd = np.float32(12582912.0)
-    t = (x + rnd).astype(np.float32)
+    t = (xc + rnd).astype(np.float32)
     n = (t - rnd).astype(np.float32)
-    f = (x - n).astype(np.float32)
+    f = (xc - n).astype(np.float32)
     assert np.all(np.abs(f) <= 0.5)
     p = ((c["kC3"] * f + c["kC2"]) * f + c["kC1"]) * f + c["kC0"]
     bits = p.astype(np.float32).view(np.int32) + (t.view(np.uint32) << np.uint32(23)).view(np.int32)
     got = bits.view(np.float32).astype(np.float64)
-    want = np.exp2(x.astype(np.float64))
-    assert np.max(np.abs(got / want - 1)) < 1e-4
+    assert np.all(np.isfinite(got)) and np.all(got >= 0)
+    normal = x >= floor + 1          # results in the normal float range
+    want = np.exp2(x[normal].astype(np.float64))
+    assert np.max(np.abs(got[normal] / want - 1)) < 1e-4
+    assert np.all(got[~normal] < 2.0 ** -124)   # at or near the clamp: negligible, never negative
