@@ -49,6 +49,12 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 constexpr int32_t kAttnStatusWaitTimeout = 0x41;
 constexpr float kRescaleThreshold = 8.0f;         // log2 units: rescale O when the max grows by > 2^8
+#ifndef KVLINK_EXP_POLY_FROM
+#define KVLINK_EXP_POLY_FROM 5                     // column pairs c with (c % 8) >= this use exp2_poly2
+#endif
+#ifndef KVLINK_PRODUCER_BACKOFF_NS
+#define KVLINK_PRODUCER_BACKOFF_NS 0               // sleep between polls of the TMA producers' waits
+#endif
 
 template <int D>
 struct TcCfg {
@@ -78,6 +84,23 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatil
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            *abort_flag = 1;
+            atomicCAS(&g_attn_status, 0, kAttnStatusWaitTimeout);
+            return false;
+        }
+    }
+}
+
+// wait_bar with a short sleep between polls, for roles off the critical path
+__device__ __forceinline__ bool wait_bar_backoff(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
+    if (KVLINK_PRODUCER_BACKOFF_NS == 0) return wait_bar(bar, parity, abort_flag);
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        __nanosleep(KVLINK_PRODUCER_BACKOFF_NS);
         if (mbar_try_wait(bar, parity)) return true;
         if (*abort_flag) return false;
         if (globaltimer_ns() - t0 > kWaitLimitNs) {
@@ -146,7 +169,7 @@ __device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes
     int issued = 0;
     for (int j = 0; j < n; ++j) {
         const int st = j % STAGES;
-        if (!wait_bar(empty + st, ((j / STAGES) & 1) ^ 1, abort_flag)) break;
+        if (!wait_bar_backoff(empty + st, ((j / STAGES) & 1) ^ 1, abort_flag)) break;
         mbar_arrive_expect_tx(full + st, stage_bytes);
 #pragma unroll
         for (int a = 0; a < ATOMS; ++a)
@@ -349,7 +372,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             for (int c = 0; c < 64; ++c) {
                 const uint64_t x2 = ffma2(f2_pack(__uint_as_float(s[2 * c]), __uint_as_float(s[2 * c + 1])), sc2, nmu2);
                 uint64_t p2;
-                if ((c & 7) >= 5) {
+                if ((c & 7) >= KVLINK_EXP_POLY_FROM) {
                     p2 = exp2_poly2(x2);
                 } else {
                     float a, b;

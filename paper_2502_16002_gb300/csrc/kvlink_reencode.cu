@@ -103,21 +103,18 @@ __device__ __forceinline__ void rotate8(uint4& lo, uint4& hi, const float4 (&cs)
 // --------------------------------------------------------------------------
 // A3 + A4: persistent re-encode/copy through a shared-memory ring.
 // --------------------------------------------------------------------------
-constexpr int kCopyConsumerWarps = 8;                               // rotate keys in shared memory
-constexpr int kCopyConsumers = 32 * kCopyConsumerWarps;
-constexpr int kCopyThreads = 32 + kCopyConsumers + 32;             // + producer warp + store warp
+constexpr int kCopyConsumers = 128;                  // 4 warps rotate keys in shared memory
+constexpr int kCopyThreads = 32 + kCopyConsumers;    // + 1 producer warp
 constexpr int kCopyStages = 3;
-constexpr uint32_t kCopyHeader = 2048;                              // unit record + RoPE row
 constexpr uint64_t kCopyWaitLimitNs = 2000000000ull;
 constexpr int32_t kCopyStatusWaitTimeout = 0x21;
 
 static __device__ int32_t g_copy_status;
 
 struct CopySmem {
-    static constexpr uint32_t STAGE = kCopyHeader + 2 * kCopyStageBytes;   // header, K, V
+    static constexpr uint32_t STAGE = 2 * kCopyStageBytes;   // K then V
     static constexpr uint32_t OFF_BAR = kCopyStages * STAGE;
-    // full[S], rotated[S], empty[S]
-    static constexpr uint32_t BYTES = OFF_BAR + 3 * kCopyStages * 8 + 16 + 128;
+    static constexpr uint32_t BYTES = OFF_BAR + 2 * kCopyStages * 8 + 16 + 128;
 };
 
 __device__ __forceinline__ bool copy_wait(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
@@ -144,14 +141,11 @@ __device__ __forceinline__ void copy_drain(uint64_t* bar, uint32_t parity) {
 }
 
 // CTA b handles the contiguous range of work units [n*b/grid, n*(b+1)/grid).
-//   warp 0       producer: writes the unit record into the stage header and bulk-loads the
-//                unit's K rows, V rows and (documents) RoPE row into the stage
-//   warps 1-8    consumers: rotate a document unit's keys in place; each thread keeps a
-//                fixed (head, j0) slot and reads its eight double-float cos/sin pairs from
-//                the header; every warp then signals the stage as ready
-//   warp 9       store: bulk-stores K and V to the linked cache and frees a stage once its
-//                stores have read it
-// V is never touched by the threads.
+// Producer (warp 0, one thread): bulk-loads a unit's K rows and V rows into a stage.
+// Consumers (warps 1-4): rotate the unit's keys in place when it is a document (each
+// thread keeps a fixed (head, j0) slot and its eight double-float cos/sin pairs), then
+// one thread bulk-stores K and V to the linked cache and frees the stage once the
+// stores have read it.  V is never touched by the threads.
 template <int D>
 __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     const CopyChunk* __restrict__ chunks, int n_chunks, const float4* __restrict__ rope, int h_kv,
@@ -163,20 +157,17 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     const uint32_t raw_addr = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + ((128u - (raw_addr & 127u)) & 127u);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + CopySmem::OFF_BAR);
-    uint64_t* rotated = full + kCopyStages;
-    uint64_t* empty = rotated + kCopyStages;
+    uint64_t* empty = full + kCopyStages;
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(empty + kCopyStages);
 
     const int c_begin = (int)((int64_t)n_chunks * blockIdx.x / gridDim.x);
     const int c_end = (int)((int64_t)n_chunks * (blockIdx.x + 1) / gridDim.x);
     const int64_t row_elems = (int64_t)h_kv * D;
     const uint32_t row_bytes = (uint32_t)(row_elems * 2);
-    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kCopyStages; ++i) {
             mbar_init(full + i, 1);
-            mbar_init(rotated + i, kCopyConsumerWarps);
             mbar_init(empty + i, 1);
         }
         *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_copy_status) != 0 ? 1 : 0;
@@ -185,86 +176,78 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     __syncthreads();
     if (*abort_flag) return;  // uniform: written before the barrier
 
-    if (warp == 0) {
+    if (threadIdx.x < 32) {
         // ------------------------------------------------------------ producer
-        if (lane == 0) {
+        if (threadIdx.x == 0) {
             int issued = 0;
             for (int c = c_begin, i = 0; c < c_end; ++c, ++i) {
                 const int st = i % kCopyStages;
                 if (!copy_wait(empty + st, ((i / kCopyStages) & 1) ^ 1, abort_flag)) break;
                 const CopyChunk ch = chunks[c];
-                uint8_t* stage = smem + st * CopySmem::STAGE;
-                *reinterpret_cast<CopyChunk*>(stage) = ch;  // published by the arrive below
                 const bool fresh = ch.kind == KVLINK_SEG_LINK || ch.kind == KVLINK_SEG_QUESTION;
-                const bool doc = ch.kind == KVLINK_SEG_DOC;
                 const __nv_bfloat16* sk = (fresh ? k_new : pool_k) + ch.src_row * row_elems;
                 const __nv_bfloat16* sv = (fresh ? v_new : pool_v) + ch.src_row * row_elems;
                 const uint32_t bytes = (uint32_t)ch.n * row_bytes;
-                const uint32_t rope_bytes = doc ? (uint32_t)(D / 2) * 16u : 0u;
-                mbar_arrive_expect_tx(full + st, 2 * bytes + rope_bytes);
-                if (doc) bulk_load(stage + 1024, rope + (int64_t)ch.table * (D / 2), rope_bytes, full + st);
-                bulk_load(stage + kCopyHeader, sk, bytes, full + st);
-                bulk_load(stage + kCopyHeader + kCopyStageBytes, sv, bytes, full + st);
+                uint8_t* stage = smem + st * CopySmem::STAGE;
+                mbar_arrive_expect_tx(full + st, 2 * bytes);
+                bulk_load(stage, sk, bytes, full + st);
+                bulk_load(stage + kCopyStageBytes, sv, bytes, full + st);
                 issued = i + 1;
             }
             // no load may still be in flight when the CTA leaves
             for (int i = issued - kCopyStages > 0 ? issued - kCopyStages : 0; i < issued; ++i)
                 copy_drain(full + i % kCopyStages, (i / kCopyStages) & 1);
         }
-    } else if (warp == 1 + kCopyConsumerWarps) {
-        // ------------------------------------------------------------ store
-        if (lane == 0) {
-            for (int c = c_begin, i = 0; c < c_end; ++c, ++i) {
-                const int st = i % kCopyStages;
-                if (!copy_wait(rotated + st, (i / kCopyStages) & 1, abort_flag)) break;
-                uint8_t* stage = smem + st * CopySmem::STAGE;
-                const CopyChunk ch = *reinterpret_cast<const CopyChunk*>(stage);
-                const uint32_t bytes = (uint32_t)ch.n * row_bytes;
-                bulk_store(cache_k + ch.dst_row * row_elems, stage + kCopyHeader, bytes);
-                bulk_store(cache_v + ch.dst_row * row_elems, stage + kCopyHeader + kCopyStageBytes, bytes);
-                bulk_commit();
-                bulk_wait_read<1>();  // the previous unit's stores have read their stage
-                if (i > 0) mbar_arrive(empty + (i - 1) % kCopyStages);
-            }
-            bulk_wait<0>();
-        }
-    } else {
-        // ------------------------------------------------------------ consumers
-        const int tc = threadIdx.x - 32;
-        constexpr int UPH = D / 16;              // (lo, hi) chunk pairs per head
-        const int U = h_kv * UPH;                // pairs per token, a power of two <= 128
-        const int TPP = kCopyConsumers / U;      // tokens per pass
-        const int unit = tc % U;
-        const int tok0 = tc / U;
-        const int head = unit / UPH;
-        const int j0 = (unit % UPH) * 8;
-        const uint32_t lo_off = (uint32_t)(head * D + j0) * 2;
-        for (int c = c_begin, i = 0; c < c_end; ++c, ++i) {
-            const int st = i % kCopyStages;
-            const bool ok = copy_wait(full + st, (i / kCopyStages) & 1, abort_flag);
-            if (!__all_sync(0xffffffffu, ok)) break;
-            uint8_t* stage = smem + st * CopySmem::STAGE;
-            const CopyChunk ch = *reinterpret_cast<const CopyChunk*>(stage);
-            if (ch.kind == KVLINK_SEG_DOC) {
-                float4 cs[8];
-                const float4* t = reinterpret_cast<const float4*>(stage + 1024) + j0;
+        return;
+    }
+
+    // ---------------------------------------------------------------- consumers
+    const int tc = threadIdx.x - 32;
+    constexpr int UPH = D / 16;                // (lo, hi) chunk pairs per head
+    const int U = h_kv * UPH;                  // pairs per token, a power of two <= 128
+    const int TPP = kCopyConsumers / U;        // tokens per pass
+    const int unit = tc % U;
+    const int tok0 = tc / U;
+    const int head = unit / UPH;
+    const int j0 = (unit % UPH) * 8;
+    const uint32_t lo_off = (uint32_t)(head * D + j0) * 2;
+    int cur_table = -1;
+    float4 cs[8];
+    for (int c = c_begin, i = 0; c < c_end; ++c, ++i) {
+        const int st = i % kCopyStages;
+        copy_wait(full + st, (i / kCopyStages) & 1, abort_flag);
+        named_bar_sync(1, kCopyConsumers);
+        if (*abort_flag) break;  // uniform: every consumer passed the barrier first
+        const CopyChunk ch = chunks[c];
+        uint8_t* stage = smem + st * CopySmem::STAGE;
+        if (ch.kind == KVLINK_SEG_DOC) {
+            if (ch.table != cur_table) {
+                const float4* t = rope + (int64_t)ch.table * (D / 2) + j0;
 #pragma unroll
-                for (int q = 0; q < 8; ++q) cs[q] = t[q];
-                uint8_t* kb = stage + kCopyHeader;
-                for (int tt = tok0; tt < ch.n; tt += TPP) {
-                    uint4* lo = reinterpret_cast<uint4*>(kb + (uint32_t)tt * row_bytes + lo_off);
-                    uint4* hi = reinterpret_cast<uint4*>(kb + (uint32_t)tt * row_bytes + lo_off + D);
-                    uint4 a = *lo, b = *hi;
-                    rotate8(a, b, cs);
-                    *lo = a;
-                    *hi = b;
-                }
-                fence_proxy_async_smem();  // the bulk store reads these writes through the async proxy
+                for (int q = 0; q < 8; ++q) cs[q] = __ldg(t + q);
+                cur_table = ch.table;
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(rotated + st);
+            for (int t = tok0; t < ch.n; t += TPP) {
+                uint4* lo = reinterpret_cast<uint4*>(stage + (uint32_t)t * row_bytes + lo_off);
+                uint4* hi = reinterpret_cast<uint4*>(stage + (uint32_t)t * row_bytes + lo_off + D);
+                uint4 a = *lo, b = *hi;
+                rotate8(a, b, cs);
+                *lo = a;
+                *hi = b;
+            }
+            fence_proxy_async_smem();  // the bulk store reads these writes through the async proxy
+        }
+        named_bar_sync(1, kCopyConsumers);
+        if (tc == 0) {
+            const uint32_t bytes = (uint32_t)ch.n * row_bytes;
+            bulk_store(cache_k + ch.dst_row * row_elems, stage, bytes);
+            bulk_store(cache_v + ch.dst_row * row_elems, stage + kCopyStageBytes, bytes);
+            bulk_commit();
+            bulk_wait_read<1>();  // the previous unit's stores have read their stage
+            if (i > 0) mbar_arrive(empty + (i - 1) % kCopyStages);
         }
     }
+    if (tc == 0) bulk_wait<0>();
 }
 
 void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv, int num_sms,

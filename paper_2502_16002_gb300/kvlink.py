@@ -13,7 +13,9 @@ import os
 
 import numpy as np
 
-_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libkvlink.so")
+# the in-tree build; KVLINK_LIBRARY may name another build of the same library
+_LIB_PATH = os.environ.get("KVLINK_LIBRARY") or os.path.join(os.path.dirname(os.path.abspath(__file__)),
+                                                              "libkvlink.so")
 
 KVLINK_OK = 0
 KVLINK_EINVAL = -1
