@@ -40,17 +40,17 @@ using namespace sm100;
 
 static __device__ int32_t g_attn_status;
 
-constexpr int kTcThreads = 224;
-constexpr int kSoftmaxWarps = 4;
-constexpr int kTmaKWarp = 4;
-constexpr int kMmaWarp = 5;
-constexpr int kTmaVWarp = 6;
+constexpr int kSoftmaxWarps = 8;
+constexpr int kTmaKWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr int kTmaVWarp = 10;
+constexpr int kTcThreads = 32 * 11;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 constexpr int32_t kAttnStatusWaitTimeout = 0x41;
 constexpr float kRescaleThreshold = 8.0f;         // log2 units: rescale O when the max grows by > 2^8
 #ifndef KVLINK_EXP_POLY_FROM
-#define KVLINK_EXP_POLY_FROM 5                     // column pairs c with (c % 8) >= this use exp2_poly2
+#define KVLINK_EXP_POLY_FROM 8                     // column pairs c with (c % 8) >= this use exp2_poly2
 #endif
 #ifndef KVLINK_PRODUCER_BACKOFF_NS
 #define KVLINK_PRODUCER_BACKOFF_NS 0               // sleep between polls of the TMA producers' waits
@@ -61,7 +61,6 @@ struct TcCfg {
     static constexpr int ATOMS = D / 64;                 // 128-byte swizzle atoms along head_dim
     static constexpr int NK = (D == 128) ? 3 : 5;        // K ring stages
     static constexpr int NV = (D == 128) ? 3 : 5;        // V ring stages
-    static constexpr int NB = 3;                         // S/P buffers in TMEM
     static constexpr uint32_t ATOM_BYTES = 128 * 128;    // [128 rows][64 bf16]
     static constexpr uint32_t Q_BYTES = ATOMS * ATOM_BYTES;
     static constexpr uint32_t KV_BYTES = ATOMS * ATOM_BYTES;
@@ -69,12 +68,14 @@ struct TcCfg {
     static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
     static constexpr uint32_t OFF_V = OFF_K + NK * KV_BYTES;
     static constexpr uint32_t OFF_BAR = OFF_V + NV * KV_BYTES;
-    // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB], p_full[NB], o_done[NB], drain
-    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 3 * NB + 1;
+    // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV],
+    // s_full[2], s_free[2], p_full[2], o_done[2], drain
+    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 4 * 2 + 1;
     static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
-    // TMEM columns: S/P buffers then the O accumulator
-    static constexpr uint32_t TMEM_S = 0;                // buffer b at b * 128
-    static constexpr uint32_t TMEM_O = NB * kAttnBN;
+    // TMEM columns: S0, S1 (fp32 scores), P0, P1 (bf16 pairs), O (fp32 accumulator)
+    static constexpr uint32_t TMEM_S = 0;                // S buffer b at b * 128
+    static constexpr uint32_t TMEM_P = 2 * kAttnBN;      // P buffer b at TMEM_P + b * 64
+    static constexpr uint32_t TMEM_O = TMEM_P + kAttnBN;
     static_assert(TMEM_O + D <= kTmemCols, "TMEM budget");
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
 };
@@ -186,7 +187,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                    const __grid_constant__ CUtensorMap tm_v, DevicePlan P, __nv_bfloat16* __restrict__ out,
                    float* __restrict__ ws, int h_q, float scale_log2) {
     using C = TcCfg<D>;
-    constexpr int NK = C::NK, NV = C::NV, NB = C::NB;
+    constexpr int NK = C::NK, NV = C::NV;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
@@ -198,9 +199,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     uint64_t* bar_v_full = bar_k_empty + NK;
     uint64_t* bar_v_empty = bar_v_full + NV;
     uint64_t* bar_s_full = bar_v_empty + NV;
-    uint64_t* bar_p_full = bar_s_full + NB;
-    uint64_t* bar_o_done = bar_p_full + NB;
-    uint64_t* bar_drain = bar_o_done + NB;
+    uint64_t* bar_s_free = bar_s_full + 2;
+    uint64_t* bar_p_full = bar_s_free + 2;
+    uint64_t* bar_o_done = bar_p_full + 2;
+    uint64_t* bar_drain = bar_o_done + 2;
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + C::N_BARS);
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(tmem_holder + 1);
 
@@ -210,8 +212,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < C::N_BARS; ++i) {
-            const bool p_full = bars + i >= bar_p_full && bars + i < bar_p_full + NB;
-            mbar_init(bars + i, p_full ? kSoftmaxWarps : 1);
+            const bool softmax_arrivals = (bars + i >= bar_s_free && bars + i < bar_s_free + 2) ||
+                                          (bars + i >= bar_p_full && bars + i < bar_p_full + 2);
+            mbar_init(bars + i, softmax_arrivals ? kSoftmaxWarps : 1);
         }
         // after a recorded failure, later launches skip their work instead of waiting out their bounds
         *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_attn_status) != 0 ? 1 : 0;
@@ -259,14 +262,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
             const uint32_t sQ = smem_u32(smem + C::OFF_Q);
             bool ok = wait_bar(bar_q_full, 0, abort_flag);
-            // O += P_i V_i, P_i (bf16) read from its S buffer in TMEM
+            // O += P_i V_i, P_i (bf16 pairs) read from TMEM
             auto issue_pv = [&](int i) -> bool {
-                const int b = i % NB, sv = i % NV;
-                if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag)) return false;
+                const int b = i & 1, sv = i % NV;
+                if (!wait_bar(bar_p_full + b, (i >> 1) & 1, abort_flag)) return false;
                 if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag)) return false;
                 tc_fence_after();
                 const uint32_t sV = smem_u32(smem + C::OFF_V + sv * C::KV_BYTES);
-                const uint32_t pcol = tmem + C::TMEM_S + b * kAttnBN;
+                const uint32_t pcol = tmem + C::TMEM_P + b * (kAttnBN / 2);
 #pragma unroll
                 for (int kk = 0; kk < kAttnBN / 16; ++kk)
                     mma_bf16_ts(tmem + C::TMEM_O, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, C::ATOM_BYTES, 1024),
@@ -276,10 +279,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 return true;
             };
             for (int j = 0; ok && j < n_tiles; ++j) {
-                const int sk = j % NK, b = j % NB;
+                const int sk = j % NK, b = j & 1;
                 if (!(ok = wait_bar(bar_k_full + sk, (j / NK) & 1, abort_flag))) break;
-                // buffer b last held P_{j-NB}: its PV must have finished reading it
-                if (j >= NB && !(ok = wait_bar(bar_o_done + b, ((j - NB) / NB) & 1, abort_flag))) break;
+                // S buffer b last held S_{j-2}: every softmax warp must have read it
+                if (!(ok = wait_bar(bar_s_free + b, ((j >> 1) & 1) ^ 1, abort_flag))) break;
                 tc_fence_after();
                 const uint32_t sK = smem_u32(smem + C::OFF_K + sk * C::KV_BYTES);
 #pragma unroll
@@ -297,43 +300,61 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             drain_bar(bar_drain, 0);
         }
     } else {
-        // ------------------------------------------------------------ softmax + epilogue (warps 0-3)
-        const int r = threadIdx.x;  // tile row == TMEM lane
+        // ------------------------------------------------------------ softmax + epilogue (warps 0-7)
+        // Warp w reads TMEM lane quadrant w % 4 (rows 32 (w % 4) ..) and owns the column half
+        // h = w / 4: keys [64 h, 64 h + 64) of every tile, and O columns [D/2 h, D/2 h + D/2).
+        // Both warps of a row compute the full-row maximum themselves (the other half is
+        // streamed through scratch registers), so they agree on m without synchronising.
+        const int quad = warp & 3, half = warp >> 2;
+        const int r = quad * 32 + lane;  // tile row == TMEM lane
         const int tok = it.tok0 + r / G;
         const bool valid = tok < it.tok1;
         const int frow = P.cu_fresh[it.query] + tok;
         const int pos = valid ? P.fresh_pos[frow] : 0x7fffffff;
-        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+        const int own0 = half * 64, other0 = 64 - own0;
+        constexpr int DH = D / 2;
         float m = -INFINITY, l = 0.f;
         bool ok = true;
         for (int j = 0; j < n_tiles; ++j) {
-            const int b = j % NB;
-            if (!(ok = warp_wait(bar_s_full + b, (j / NB) & 1, abort_flag))) break;
+            const int b = j & 1;
+            if (!(ok = warp_wait(bar_s_full + b, (j >> 1) & 1, abort_flag))) break;
             tc_fence_after();
-            uint32_t s[128];
             const uint32_t s_col = tmem + lane_base + C::TMEM_S + b * kAttnBN;
-            tmem_ld32(s_col + 0, *reinterpret_cast<uint32_t(*)[32]>(s + 0));
-            tmem_ld32(s_col + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
-            tmem_ld32(s_col + 64, *reinterpret_cast<uint32_t(*)[32]>(s + 64));
-            tmem_ld32(s_col + 96, *reinterpret_cast<uint32_t(*)[32]>(s + 96));
-            tmem_ld_wait();
-
-            // raw row max (scale > 0 commutes with max); masked slots become -inf.  Eight
-            // independent running maxima keep the dependency chain short.
             const int key0 = (it.kv_tile0 + j) * kAttnBN;
+            const bool masked = key0 + kAttnBN - 1 > it.min_pos;
+            uint32_t s[64];
             float mx8[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
-            if (key0 + kAttnBN - 1 > it.min_pos) {
+            {
+                uint32_t t[32];
 #pragma unroll
-                for (int c = 0; c < 128; ++c) {
-                    if (key0 + c > pos) s[c] = __float_as_uint(-INFINITY);
-                    mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
+                for (int part = 0; part < 2; ++part) {
+                    tmem_ld32(s_col + other0 + part * 32, t);
+                    tmem_ld_wait();
+                    const int kb = key0 + other0 + part * 32;
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) {
+                        const float v = (masked && kb + c > pos) ? -INFINITY : __uint_as_float(t[c]);
+                        mx8[c & 7] = fmaxf(mx8[c & 7], v);
+                    }
                 }
-            } else {
-#pragma unroll
-                for (int c = 0; c < 128; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
+                tmem_ld32(s_col + own0, *reinterpret_cast<uint32_t(*)[32]>(s + 0));
+                tmem_ld32(s_col + own0 + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
+                tmem_ld_wait();
             }
+            // this warp is done with S buffer b
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_s_free + b);
+            if (masked) {
+#pragma unroll
+                for (int c = 0; c < 64; ++c)
+                    if (key0 + own0 + c > pos) s[c] = __float_as_uint(-INFINITY);
+            }
+#pragma unroll
+            for (int c = 0; c < 64; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
             const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                                    fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
             const float m_new = fmaxf(m, mx * scale_log2);
@@ -346,12 +367,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             if (j > 0 && __any_sync(0xffffffffu, resc)) {
                 // O is touched only while no PV is in flight: PV_{j-1} done, PV_j not yet issued
-                if (!(ok = warp_wait(bar_o_done + (j - 1) % NB, ((j - 1) / NB) & 1, abort_flag))) break;
+                if (!(ok = warp_wait(bar_o_done + ((j - 1) & 1), ((j - 1) >> 1) & 1, abort_flag))) break;
                 tc_fence_after();
 #pragma unroll
-                for (int c4 = 0; c4 < D / 32; ++c4) {
+                for (int c4 = 0; c4 < DH / 32; ++c4) {
                     uint32_t o[32];
-                    const uint32_t o_col = tmem + lane_base + C::TMEM_O + c4 * 32;
+                    const uint32_t o_col = tmem + lane_base + C::TMEM_O + half * DH + c4 * 32;
                     tmem_ld32(o_col, o);
                     tmem_ld_wait();
 #pragma unroll
@@ -359,25 +380,24 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     tmem_st32(o_col, o);
                 }
             }
-            // p = exp2(s * scale - m) on column pairs (packed f32x2 arithmetic); three pairs
-            // in eight go to the FMA pipe (exp2_poly2), the rest to MUFU, to balance the two
+            // p = exp2(s * scale - m) on column pairs with packed f32x2 arithmetic
             const float mu = (m == -INFINITY) ? 0.f : m;
             const uint64_t sc2 = f2_pack(scale_log2, scale_log2);
             const uint64_t nmu2 = f2_pack(-mu, -mu);
             uint64_t acc[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) acc[e] = f2_pack(0.f, 0.f);
-            uint32_t pk[64];
+            uint32_t pk[32];
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
+            for (int c = 0; c < 32; ++c) {
                 const uint64_t x2 = ffma2(f2_pack(__uint_as_float(s[2 * c]), __uint_as_float(s[2 * c + 1])), sc2, nmu2);
                 uint64_t p2;
                 if ((c & 7) >= KVLINK_EXP_POLY_FROM) {
                     p2 = exp2_poly2(x2);
                 } else {
-                    float a, b;
-                    f2_unpack(x2, a, b);
-                    p2 = f2_pack(ex2_approx(a), ex2_approx(b));
+                    float a, bb;
+                    f2_unpack(x2, a, bb);
+                    p2 = f2_pack(ex2_approx(a), ex2_approx(bb));
                 }
                 acc[c & 3] = fadd2(acc[c & 3], p2);
                 float p0, p1;
@@ -386,26 +406,32 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             float rs0, rs1;
             f2_unpack(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), rs0, rs1);
-            const float rs = rs0 + rs1;
-            l += rs;
-            // P_j (bf16) over the first 64 columns of its S buffer, read there by the PV MMA
-            tmem_st32(s_col + 0, *reinterpret_cast<uint32_t(*)[32]>(pk + 0));
-            tmem_st32(s_col + 32, *reinterpret_cast<uint32_t(*)[32]>(pk + 32));
+            l += rs0 + rs1;
+            // P buffer b last held P_{j-2}: its PV must have finished reading it
+            if (j >= 2 && !(ok = warp_wait(bar_o_done + b, ((j - 2) >> 1) & 1, abort_flag))) break;
+            tc_fence_after();
+            tmem_st32(tmem + lane_base + C::TMEM_P + b * (kAttnBN / 2) + half * 32, pk);
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_p_full + b);
         }
-        if (ok && n_tiles > 0) ok = warp_wait(bar_o_done + (n_tiles - 1) % NB, ((n_tiles - 1) / NB) & 1, abort_flag);
+        if (ok && n_tiles > 0)
+            ok = warp_wait(bar_o_done + ((n_tiles - 1) & 1), ((n_tiles - 1) >> 1) & 1, abort_flag);
+        // combine the two halves' row sums (the K ring is idle by now: reuse its first KB)
+        float* lsum = reinterpret_cast<float*>(smem + C::OFF_K);
+        lsum[half * kAttnBM + r] = l;
+        named_bar_sync(1 + quad, 64);
+        const float l_all = l + lsum[(1 - half) * kAttnBM + r];
         if (ok) {
             tc_fence_after();
             if (it.slot < 0) {
-                const float inv = 1.f / l;
-                __nv_bfloat16* orow = out + ((int64_t)frow * h_q + it.kv_head * G + (r % G)) * D;
+                const float inv = 1.f / l_all;
+                __nv_bfloat16* orow = out + ((int64_t)frow * h_q + it.kv_head * G + (r % G)) * D + half * DH;
 #pragma unroll
-                for (int c4 = 0; c4 < D / 32; ++c4) {
+                for (int c4 = 0; c4 < DH / 32; ++c4) {
                     uint32_t o[32];
-                    tmem_ld32(tmem + lane_base + C::TMEM_O + c4 * 32, o);
+                    tmem_ld32(tmem + lane_base + C::TMEM_O + half * DH + c4 * 32, o);
                     tmem_ld_wait();
                     if (valid) {
 #pragma unroll
@@ -422,17 +448,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             } else {
                 float* wo = ws + (int64_t)it.slot * kAttnBM * (D + 2);
 #pragma unroll
-                for (int c4 = 0; c4 < D / 32; ++c4) {
+                for (int c4 = 0; c4 < DH / 32; ++c4) {
                     uint32_t o[32];
-                    tmem_ld32(tmem + lane_base + C::TMEM_O + c4 * 32, o);
+                    tmem_ld32(tmem + lane_base + C::TMEM_O + half * DH + c4 * 32, o);
                     tmem_ld_wait();
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
-                        *reinterpret_cast<uint4*>(wo + r * D + c4 * 32 + 4 * q) =
+                        *reinterpret_cast<uint4*>(wo + r * D + half * DH + c4 * 32 + 4 * q) =
                             make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
                 }
-                wo[kAttnBM * D + r] = m;
-                wo[kAttnBM * D + kAttnBM + r] = l;
+                if (half == 0) {
+                    wo[kAttnBM * D + r] = m;
+                    wo[kAttnBM * D + kAttnBM + r] = l_all;
+                }
             }
         }
     }
