@@ -5,19 +5,19 @@
 // tiles of that query's linked cache.  Rows are (token, head) pairs, so the G
 // heads of a GQA group share every K/V tile load.
 //
-// Warp roles (224 threads, one CTA per SM, 512 TMEM columns):
-//   warps 0-3  softmax + epilogue; thread r owns row r = TMEM lane r
-//   warp 4     TMA: Q once, then K tiles into an NK-stage ring
-//   warp 5     TMEM allocation and the single MMA-issuing thread
-//   warp 6     TMA: V tiles into an NV-stage ring
-// Per KV tile j (TMEM: three S/P buffers of 128 columns, then O):
-//   S_j = Q K_j^T           tcgen05.mma SMEM x SMEM -> S buffer j%3
-//   P_j = exp2(S_j c - m)   softmax warps: TMEM -> registers -> bf16 P written back
-//                           over the first 64 columns of the same buffer
+// Warp roles (384 threads, one CTA per SM, 512 TMEM columns):
+//   warps 0-7  softmax + epilogue; warp w owns TMEM lane quadrant w % 4 (rows
+//              32 (w % 4) ..) and column half w / 4 of every tile and of O
+//   warp 8     TMA: Q once, then K tiles into an NK-stage ring
+//   warp 9     TMA: V tiles into an NV-stage ring
+//   warp 11    TMEM allocation and the single MMA-issuing thread
+// Per KV tile j (TMEM: S0, S1 fp32 scores, P0, P1 bf16 pairs, O):
+//   S_j = Q K_j^T           tcgen05.mma SMEM x SMEM -> S buffer j%2
+//   P_j = exp2(S_j c - m)   softmax warps: TMEM -> registers -> bf16 P buffer j%2
 //   O  += P_j V_j           tcgen05.mma TMEM x SMEM (P from TMEM, V read MN-major)
-// S_j is issued only after PV_{j-3} has finished reading the buffer, so up to
-// three tiles are in flight and the softmax never waits on a PV except to
-// rescale O.  The running max m is raised only when it grows by more than 2^8,
+// A softmax warp frees its S buffer as soon as it has loaded it, so S_{j+1} and
+// PV_{j-1} run on the tensor cores while the softmax of tile j runs; the softmax
+// waits on a PV only to reuse a P buffer (PV_{j-2}) or to rescale O.  The running max m is raised only when it grows by more than 2^8,
 // so that rescale is rare.  The mask keeps key slot j for a row at global
 // position p iff j <= p, and is evaluated only on tiles that reach past the
 // tile's smallest row position.  Items whose KV range was split write
@@ -41,13 +41,15 @@ using namespace sm100;
 static __device__ int32_t g_attn_status;
 
 constexpr int kSoftmaxWarps = 8;
-constexpr int kTmaKWarp = 8;
-constexpr int kMmaWarp = 9;
-constexpr int kTmaVWarp = 10;
-constexpr int kTcThreads = 32 * 11;
+constexpr int kTmaKWarp = 8;    // SMSP 0
+constexpr int kTmaVWarp = 9;    // SMSP 1
+constexpr int kMmaWarp = 11;    // SMSP 3, which carries only two softmax warps (warp 10 idles)
+constexpr int kTcThreads = 32 * 12;
+constexpr uint32_t kSmemSlack = 128;  // room to align the dynamic shared memory base to 1024
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 constexpr int32_t kAttnStatusWaitTimeout = 0x41;
+constexpr int32_t kAttnStatusSmemAlign = 0x42;
 constexpr float kRescaleThreshold = 8.0f;         // log2 units: rescale O when the max grows by > 2^8
 #ifndef KVLINK_EXP_POLY_FROM
 #define KVLINK_EXP_POLY_FROM 8                     // column pairs c with (c % 8) >= this use exp2_poly2
@@ -67,11 +69,12 @@ struct TcCfg {
     static constexpr uint32_t OFF_Q = 0;
     static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
     static constexpr uint32_t OFF_V = OFF_K + NK * KV_BYTES;
-    static constexpr uint32_t OFF_BAR = OFF_V + NV * KV_BYTES;
+    static constexpr uint32_t OFF_RED = OFF_V + NV * KV_BYTES;   // row-max exchange [2][2][128] f32
+    static constexpr uint32_t OFF_BAR = OFF_RED + 2 * 2 * kAttnBM * 4;
     // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV],
     // s_full[2], s_free[2], p_full[2], o_done[2], drain
     static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 4 * 2 + 1;
-    static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
+    static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + kSmemSlack;
     // TMEM columns: S0, S1 (fp32 scores), P0, P1 (bf16 pairs), O (fp32 accumulator)
     static constexpr uint32_t TMEM_S = 0;                // S buffer b at b * 128
     static constexpr uint32_t TMEM_P = 2 * kAttnBN;      // P buffer b at TMEM_P + b * 64
@@ -188,9 +191,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                    float* __restrict__ ws, int h_q, float scale_log2) {
     using C = TcCfg<D>;
     constexpr int NK = C::NK, NV = C::NV;
-    extern __shared__ uint8_t smem_raw[];
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
-    uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
+    const uint32_t pad = (1024u - (raw_addr & 1023u)) & 1023u;
+    if (pad > kSmemSlack) {  // uniform: the same base for every thread of the CTA
+        if (threadIdx.x == 0) atomicCAS(&g_attn_status, 0, kAttnStatusSmemAlign);
+        return;
+    }
+    uint8_t* smem = smem_raw + pad;
 
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
     uint64_t* bar_q_full = bars;
@@ -260,7 +268,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (lane == 0) {
             constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
             constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
-            const uint32_t sQ = smem_u32(smem + C::OFF_Q);
+            // descriptors of every operand tile, built once; a K step only moves the start address
+            const uint64_t dQ = sdesc_sw128(smem_u32(smem + C::OFF_Q), 16, 1024);
+            const uint64_t dK0 = sdesc_sw128(smem_u32(smem + C::OFF_K), 16, 1024);
+            const uint64_t dV0 = sdesc_sw128(smem_u32(smem + C::OFF_V), C::ATOM_BYTES, 1024);
+            constexpr uint64_t kStageStep = C::KV_BYTES >> 4;  // start-address units per ring stage
             bool ok = wait_bar(bar_q_full, 0, abort_flag);
             // O += P_i V_i, P_i (bf16 pairs) read from TMEM
             auto issue_pv = [&](int i) -> bool {
@@ -268,12 +280,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 if (!wait_bar(bar_p_full + b, (i >> 1) & 1, abort_flag)) return false;
                 if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag)) return false;
                 tc_fence_after();
-                const uint32_t sV = smem_u32(smem + C::OFF_V + sv * C::KV_BYTES);
                 const uint32_t pcol = tmem + C::TMEM_P + b * (kAttnBN / 2);
+                const uint64_t dv = dV0 + (uint64_t)sv * kStageStep;
 #pragma unroll
                 for (int kk = 0; kk < kAttnBN / 16; ++kk)
-                    mma_bf16_ts(tmem + C::TMEM_O, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, C::ATOM_BYTES, 1024),
-                                idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
+                    mma_bf16_ts(tmem + C::TMEM_O, pcol + kk * 8, dv + (uint64_t)((kk * 16 * 128) >> 4), idesc_pv,
+                                (i > 0 || kk > 0) ? 1u : 0u);
                 mma_commit(bar_o_done + b);
                 mma_commit(bar_v_empty + sv);
                 return true;
@@ -284,12 +296,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 // S buffer b last held S_{j-2}: every softmax warp must have read it
                 if (!(ok = wait_bar(bar_s_free + b, ((j >> 1) & 1) ^ 1, abort_flag))) break;
                 tc_fence_after();
-                const uint32_t sK = smem_u32(smem + C::OFF_K + sk * C::KV_BYTES);
+                const uint64_t dk = dK0 + (uint64_t)sk * kStageStep;
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint32_t koff = (kk >> 2) * C::ATOM_BYTES + (kk & 3) * 32;
-                    mma_bf16_ss(tmem + C::TMEM_S + b * kAttnBN, sdesc_sw128(sQ + koff, 16, 1024),
-                                sdesc_sw128(sK + koff, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
+                    const uint64_t koff = (uint64_t)((((kk >> 2) * C::ATOM_BYTES) + (kk & 3) * 32) >> 4);
+                    mma_bf16_ss(tmem + C::TMEM_S + b * kAttnBN, dQ + koff, dk + koff, idesc_qk, kk > 0 ? 1u : 0u);
                 }
                 mma_commit(bar_s_full + b);
                 mma_commit(bar_k_empty + sk);
@@ -303,8 +314,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // ------------------------------------------------------------ softmax + epilogue (warps 0-7)
         // Warp w reads TMEM lane quadrant w % 4 (rows 32 (w % 4) ..) and owns the column half
         // h = w / 4: keys [64 h, 64 h + 64) of every tile, and O columns [D/2 h, D/2 h + D/2).
-        // Both warps of a row compute the full-row maximum themselves (the other half is
-        // streamed through scratch registers), so they agree on m without synchronising.
+        // The two warps of a row combine their half-row maxima through shared memory, so
+        // they agree on m; each keeps the running sum of its own half.
         const int quad = warp & 3, half = warp >> 2;
         const int r = quad * 32 + lane;  // tile row == TMEM lane
         const int tok = it.tok0 + r / G;
@@ -312,7 +323,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int frow = P.cu_fresh[it.query] + tok;
         const int pos = valid ? P.fresh_pos[frow] : 0x7fffffff;
         const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-        const int own0 = half * 64, other0 = 64 - own0;
+        const int own0 = half * 64;
+        volatile float* red = reinterpret_cast<volatile float*>(smem + C::OFF_RED);
         constexpr int DH = D / 2;
         float m = -INFINITY, l = 0.f;
         bool ok = true;
@@ -324,26 +336,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int key0 = (it.kv_tile0 + j) * kAttnBN;
             const bool masked = key0 + kAttnBN - 1 > it.min_pos;
             uint32_t s[64];
-            float mx8[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
-            {
-                uint32_t t[32];
-#pragma unroll
-                for (int part = 0; part < 2; ++part) {
-                    tmem_ld32(s_col + other0 + part * 32, t);
-                    tmem_ld_wait();
-                    const int kb = key0 + other0 + part * 32;
-#pragma unroll
-                    for (int c = 0; c < 32; ++c) {
-                        const float v = (masked && kb + c > pos) ? -INFINITY : __uint_as_float(t[c]);
-                        mx8[c & 7] = fmaxf(mx8[c & 7], v);
-                    }
-                }
-                tmem_ld32(s_col + own0, *reinterpret_cast<uint32_t(*)[32]>(s + 0));
-                tmem_ld32(s_col + own0 + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
-                tmem_ld_wait();
-            }
+            tmem_ld32(s_col + own0, *reinterpret_cast<uint32_t(*)[32]>(s + 0));
+            tmem_ld32(s_col + own0 + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
+            tmem_ld_wait();
             // this warp is done with S buffer b
             tc_fence_before();
             __syncwarp();
@@ -353,10 +348,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 for (int c = 0; c < 64; ++c)
                     if (key0 + own0 + c > pos) s[c] = __float_as_uint(-INFINITY);
             }
+            float mx8[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
 #pragma unroll
             for (int c = 0; c < 64; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
-            const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+            const float pmx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                    fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+            // the two warps of this row exchange their half-row maxima (buffer b: the partner
+            // read of tile j-2 happened before it reached the barrier of tile j-1)
+            red[(b * 2 + half) * kAttnBM + r] = pmx;
+            named_bar_sync(1 + quad, 64);
+            const float mx = fmaxf(pmx, red[(b * 2 + (1 - half)) * kAttnBM + r]);
             const float m_new = fmaxf(m, mx * scale_log2);
             const bool resc = m_new > m + kRescaleThreshold;
             float alpha = 1.f;
