@@ -72,8 +72,8 @@ struct TcCfg {
     static constexpr uint32_t OFF_RED = OFF_V + NV * KV_BYTES;   // row-max exchange [2][2][128] f32
     static constexpr uint32_t OFF_BAR = OFF_RED + 2 * 2 * kAttnBM * 4;
     // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV],
-    // s_full[2], s_free[2], p_full[2], o_done[2], drain
-    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 4 * 2 + 1;
+    // s_full[2], s_free[2], p_full[2], o_done[2], drain, pair_max[4][2], pair_sum[4]
+    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 4 * 2 + 1 + 8 + 4;
     static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + kSmemSlack;
     // TMEM columns: S0, S1 (fp32 scores), P0, P1 (bf16 pairs), O (fp32 accumulator)
     static constexpr uint32_t TMEM_S = 0;                // S buffer b at b * 128
@@ -211,6 +211,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     uint64_t* bar_p_full = bar_s_free + 2;
     uint64_t* bar_o_done = bar_p_full + 2;
     uint64_t* bar_drain = bar_o_done + 2;
+    uint64_t* bar_pair_max = bar_drain + 1;   // [quad][b]: both warps of a row wrote their half max
+    uint64_t* bar_pair_sum = bar_pair_max + 8;  // [quad]: both warps of a row wrote their half sum
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + C::N_BARS);
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(tmem_holder + 1);
 
@@ -222,7 +224,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int i = 0; i < C::N_BARS; ++i) {
             const bool softmax_arrivals = (bars + i >= bar_s_free && bars + i < bar_s_free + 2) ||
                                           (bars + i >= bar_p_full && bars + i < bar_p_full + 2);
-            mbar_init(bars + i, softmax_arrivals ? kSoftmaxWarps : 1);
+            const bool pair = bars + i >= bar_pair_max;
+            mbar_init(bars + i, softmax_arrivals ? kSoftmaxWarps : (pair ? 2 : 1));
         }
         // after a recorded failure, later launches skip their work instead of waiting out their bounds
         *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_attn_status) != 0 ? 1 : 0;
@@ -310,12 +313,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             mma_commit(bar_drain);  // arrives once every MMA issued above has completed
             drain_bar(bar_drain, 0);
         }
-    } else {
+    } else if (warp < kSoftmaxWarps) {
         // ------------------------------------------------------------ softmax + epilogue (warps 0-7)
         // Warp w reads TMEM lane quadrant w % 4 (rows 32 (w % 4) ..) and owns the column half
         // h = w / 4: keys [64 h, 64 h + 64) of every tile, and O columns [D/2 h, D/2 h + D/2).
-        // The two warps of a row combine their half-row maxima through shared memory, so
-        // they agree on m; each keeps the running sum of its own half.
+        // The two warps of a row combine their half-row maxima through shared memory (with
+        // an mbarrier per row quadrant and S buffer), so they agree on m; each keeps the
+        // running sum of its own half, and the halves are added once at the end.
         const int quad = warp & 3, half = warp >> 2;
         const int r = quad * 32 + lane;  // tile row == TMEM lane
         const int tok = it.tok0 + r / G;
@@ -355,10 +359,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             for (int c = 0; c < 64; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
             const float pmx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                                     fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-            // the two warps of this row exchange their half-row maxima (buffer b: the partner
-            // read of tile j-2 happened before it reached the barrier of tile j-1)
+            // the two warps of this row exchange their half-row maxima (slot b: the partner
+            // read the tile j-2 value before it arrived for tile j-1)
             red[(b * 2 + half) * kAttnBM + r] = pmx;
-            named_bar_sync(1 + quad, 64);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_pair_max + quad * 2 + b);
+            if (!(ok = warp_wait(bar_pair_max + quad * 2 + b, (j >> 1) & 1, abort_flag))) break;
             const float mx = fmaxf(pmx, red[(b * 2 + (1 - half)) * kAttnBM + r]);
             const float m_new = fmaxf(m, mx * scale_log2);
             const bool resc = m_new > m + kRescaleThreshold;
@@ -422,10 +428,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (ok && n_tiles > 0)
             ok = warp_wait(bar_o_done + ((n_tiles - 1) & 1), ((n_tiles - 1) >> 1) & 1, abort_flag);
         // combine the two halves' row sums (the K ring is idle by now: reuse its first KB)
-        float* lsum = reinterpret_cast<float*>(smem + C::OFF_K);
-        lsum[half * kAttnBM + r] = l;
-        named_bar_sync(1 + quad, 64);
-        const float l_all = l + lsum[(1 - half) * kAttnBM + r];
+        volatile float* lsum = reinterpret_cast<volatile float*>(smem + C::OFF_K);
+        if (ok) {
+            lsum[half * kAttnBM + r] = l;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_pair_sum + quad);
+            ok = warp_wait(bar_pair_sum + quad, 0, abort_flag);
+        }
+        const float l_all = ok ? l + lsum[(1 - half) * kAttnBM + r] : 0.f;
         if (ok) {
             tc_fence_after();
             if (it.slot < 0) {
