@@ -5,19 +5,19 @@
 // tiles of that query's linked cache.  Rows are (token, head) pairs, so the G
 // heads of a GQA group share every K/V tile load.
 //
-// Warp roles (384 threads, one CTA per SM, 512 TMEM columns):
-//   warps 0-7  softmax + epilogue; warp w owns TMEM lane quadrant w % 4 (rows
-//              32 (w % 4) ..) and column half w / 4 of every tile and of O
-//   warp 8     TMA: Q once, then K tiles into an NK-stage ring
-//   warp 9     TMA: V tiles into an NV-stage ring
-//   warp 11    TMEM allocation and the single MMA-issuing thread
-// Per KV tile j (TMEM: S0, S1 fp32 scores, P0, P1 bf16 pairs, O):
-//   S_j = Q K_j^T           tcgen05.mma SMEM x SMEM -> S buffer j%2
-//   P_j = exp2(S_j c - m)   softmax warps: TMEM -> registers -> bf16 P buffer j%2
+// Warp roles (224 threads, one CTA per SM, 512 TMEM columns):
+//   warps 0-3  softmax + epilogue; thread r owns row r = TMEM lane r
+//   warp 4     TMA: Q once, then K tiles into an NK-stage ring
+//   warp 5     TMEM allocation and the single MMA-issuing thread
+//   warp 6     TMA: V tiles into an NV-stage ring
+// Per KV tile j (TMEM: three S/P buffers of 128 columns, then O):
+//   S_j = Q K_j^T           tcgen05.mma SMEM x SMEM -> S buffer j%3
+//   P_j = exp2(S_j c - m)   softmax warps: TMEM -> registers -> bf16 P written back
+//                           over the first 64 columns of the same buffer
 //   O  += P_j V_j           tcgen05.mma TMEM x SMEM (P from TMEM, V read MN-major)
-// A softmax warp frees its S buffer as soon as it has loaded it, so S_{j+1} and
-// PV_{j-1} run on the tensor cores while the softmax of tile j runs; the softmax
-// waits on a PV only to reuse a P buffer (PV_{j-2}) or to rescale O.  The running max m is raised only when it grows by more than 2^8,
+// S_j is issued only after PV_{j-3} has finished reading the buffer, so up to
+// three tiles are in flight and the softmax never waits on a PV except to
+// rescale O.  The running max m is raised only when it grows by more than 2^8,
 // so that rescale is rare.  The mask keeps key slot j for a row at global
 // position p iff j <= p, and is evaluated only on tiles that reach past the
 // tile's smallest row position.  Items whose KV range was split write
@@ -40,16 +40,14 @@ using namespace sm100;
 
 static __device__ int32_t g_attn_status;
 
-constexpr int kSoftmaxWarpsPerTile = 4;  // one warp per TMEM lane quadrant, per M-tile
-constexpr int kTmaKWarp = 8;    // SMSP 0
-constexpr int kTmaVWarp = 9;    // SMSP 1
-constexpr int kMmaWarp = 11;    // SMSP 3, the one without a TMA warp (warp 10 idles)
-constexpr int kTcThreads = 32 * 12;
-constexpr uint32_t kSmemSlack = 128;  // room to align the dynamic shared memory base to 1024
+constexpr int kTcThreads = 224;
+constexpr int kSoftmaxWarps = 4;
+constexpr int kTmaKWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kTmaVWarp = 6;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 constexpr int32_t kAttnStatusWaitTimeout = 0x41;
-constexpr int32_t kAttnStatusSmemAlign = 0x42;
 constexpr float kRescaleThreshold = 8.0f;         // log2 units: rescale O when the max grows by > 2^8
 #ifndef KVLINK_EXP_POLY_FROM
 #define KVLINK_EXP_POLY_FROM 8                     // column pairs c with (c % 8) >= this use exp2_poly2
@@ -61,22 +59,23 @@ constexpr float kRescaleThreshold = 8.0f;         // log2 units: rescale O when 
 template <int D>
 struct TcCfg {
     static constexpr int ATOMS = D / 64;                 // 128-byte swizzle atoms along head_dim
-    static constexpr int NK = (D == 128) ? 3 : 6;        // K ring stages
-    static constexpr int NV = (D == 128) ? 2 : 6;        // V ring stages
+    static constexpr int NK = (D == 128) ? 3 : 5;        // K ring stages
+    static constexpr int NV = (D == 128) ? 3 : 5;        // V ring stages
+    static constexpr int NB = 3;                         // S/P buffers in TMEM
     static constexpr uint32_t ATOM_BYTES = 128 * 128;    // [128 rows][64 bf16]
-    static constexpr uint32_t Q_BYTES = ATOMS * ATOM_BYTES;   // one M-tile of Q
+    static constexpr uint32_t Q_BYTES = ATOMS * ATOM_BYTES;
     static constexpr uint32_t KV_BYTES = ATOMS * ATOM_BYTES;
-    static constexpr uint32_t OFF_Q = 0;                 // M-tile t at OFF_Q + t * Q_BYTES
-    static constexpr uint32_t OFF_K = 2 * Q_BYTES;
+    static constexpr uint32_t OFF_Q = 0;
+    static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
     static constexpr uint32_t OFF_V = OFF_K + NK * KV_BYTES;
     static constexpr uint32_t OFF_BAR = OFF_V + NV * KV_BYTES;
-    // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[2], p_full[2], o_done[2], drain
-    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 6 + 1;
-    static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + kSmemSlack;
-    // TMEM: M-tile t owns columns [t * 256, t * 256 + 256): S (P in bf16 pairs over its
-    // first 64 columns), then the O accumulator
-    static constexpr uint32_t TMEM_TILE = 256, TMEM_S = 0, TMEM_O = 128;
-    static_assert(TMEM_TILE + TMEM_O + D <= kTmemCols, "TMEM budget");
+    // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB], p_full[NB], o_done[NB], drain
+    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 3 * NB + 1;
+    static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
+    // TMEM columns: S/P buffers then the O accumulator
+    static constexpr uint32_t TMEM_S = 0;                // buffer b at b * 128
+    static constexpr uint32_t TMEM_O = NB * kAttnBN;
+    static_assert(TMEM_O + D <= kTmemCols, "TMEM budget");
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
 };
 
@@ -187,15 +186,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                    const __grid_constant__ CUtensorMap tm_v, DevicePlan P, __nv_bfloat16* __restrict__ out,
                    float* __restrict__ ws, int h_q, float scale_log2) {
     using C = TcCfg<D>;
-    constexpr int NK = C::NK, NV = C::NV;
-    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    constexpr int NK = C::NK, NV = C::NV, NB = C::NB;
+    extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
-    const uint32_t pad = (1024u - (raw_addr & 1023u)) & 1023u;
-    if (pad > kSmemSlack) {  // uniform: the same base for every thread of the CTA
-        if (threadIdx.x == 0) atomicCAS(&g_attn_status, 0, kAttnStatusSmemAlign);
-        return;
-    }
-    uint8_t* smem = smem_raw + pad;
+    uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
 
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
     uint64_t* bar_q_full = bars;
@@ -203,25 +197,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     uint64_t* bar_k_empty = bar_k_full + NK;
     uint64_t* bar_v_full = bar_k_empty + NK;
     uint64_t* bar_v_empty = bar_v_full + NV;
-    uint64_t* bar_s_full = bar_v_empty + NV;   // [M-tile]
-    uint64_t* bar_p_full = bar_s_full + 2;     // [M-tile], one arrival per softmax warp
-    uint64_t* bar_o_done = bar_p_full + 2;     // [M-tile]: the M-tile's latest PV has completed
-    uint64_t* bar_drain = bar_o_done + 2;
+    uint64_t* bar_s_full = bar_v_empty + NV;
+    uint64_t* bar_p_full = bar_s_full + NB;
+    uint64_t* bar_o_done = bar_p_full + NB;
+    uint64_t* bar_drain = bar_o_done + NB;
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + C::N_BARS);
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(tmem_holder + 1);
 
     const AttnItem it = P.items[blockIdx.x];
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    // key tiles of this item that each M-tile processes (M-tile 0 may stop early)
-    const int n_all = it.kv_tile1 - it.kv_tile0;
-    const bool has1 = it.tok1 > it.tok_mid;
-    const int n0 = max(0, min(it.kv_tile1, it.kv_end0) - it.kv_tile0);
-    const int n1 = has1 ? n_all : 0;
+    const int n_tiles = it.kv_tile1 - it.kv_tile0;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < C::N_BARS; ++i) {
-            const bool softmax_arrivals = bars + i >= bar_p_full && bars + i < bar_p_full + 2;
-            mbar_init(bars + i, softmax_arrivals ? kSoftmaxWarpsPerTile : 1);
+            const bool p_full = bars + i >= bar_p_full && bars + i < bar_p_full + NB;
+            mbar_init(bars + i, p_full ? kSoftmaxWarps : 1);
         }
         // after a recorded failure, later launches skip their work instead of waiting out their bounds
         *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_attn_status) != 0 ? 1 : 0;
@@ -246,130 +236,106 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (skip) {
         // nothing issued: fall through to the teardown
     } else if (warp == kTmaKWarp) {
-        // ------------------------------------------------------------ Q (both M-tiles), then the K ring
+        // ------------------------------------------------------------ Q, then the K ring
         if (lane == 0) {
-            const int f0 = P.cu_fresh[it.query];
-            mbar_arrive_expect_tx(bar_q_full, 2 * C::Q_BYTES);
+            const int q_row0 = P.cu_fresh[it.query] + it.tok0;
+            mbar_arrive_expect_tx(bar_q_full, C::Q_BYTES);
 #pragma unroll
-            for (int t = 0; t < 2; ++t)
-#pragma unroll
-                for (int a = 0; a < C::ATOMS; ++a)
-                    tma_load_3d(smem + C::OFF_Q + t * C::Q_BYTES + a * C::ATOM_BYTES, &tm_q, a * 64, it.kv_head * G,
-                                f0 + (t == 0 ? it.tok0 : it.tok_mid), bar_q_full);
-            produce_ring<NK, C::ATOMS>(smem + C::OFF_K, C::KV_BYTES, &tm_k, bar_k_full, bar_k_empty, n_all,
+            for (int a = 0; a < C::ATOMS; ++a)
+                tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &tm_q, a * 64, it.kv_head * G, q_row0, bar_q_full);
+            produce_ring<NK, C::ATOMS>(smem + C::OFF_K, C::KV_BYTES, &tm_k, bar_k_full, bar_k_empty, n_tiles,
                                        it.kv_head, key_row0, abort_flag);
             drain_bar(bar_q_full, 0);
         }
     } else if (warp == kTmaVWarp) {
         // ------------------------------------------------------------ the V ring
         if (lane == 0)
-            produce_ring<NV, C::ATOMS>(smem + C::OFF_V, C::KV_BYTES, &tm_v, bar_v_full, bar_v_empty, n_all,
+            produce_ring<NV, C::ATOMS>(smem + C::OFF_V, C::KV_BYTES, &tm_v, bar_v_full, bar_v_empty, n_tiles,
                                        it.kv_head, key_row0, abort_flag);
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
-        // Order: S0(0) S1(0) | PV0(j) S0(j+1) PV1(j) S1(j+1) | ...  so that the S of one M-tile
-        // runs on the tensor cores while the other M-tile's softmax is still producing P.
         if (lane == 0) {
             constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
             constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
-            constexpr uint64_t kStageStep = C::KV_BYTES >> 4;  // start-address units per ring stage
-            const uint64_t dQ0 = sdesc_sw128(smem_u32(smem + C::OFF_Q), 16, 1024);
-            const uint64_t dK0 = sdesc_sw128(smem_u32(smem + C::OFF_K), 16, 1024);
-            const uint64_t dV0 = sdesc_sw128(smem_u32(smem + C::OFF_V), C::ATOM_BYTES, 1024);
+            const uint32_t sQ = smem_u32(smem + C::OFF_Q);
             bool ok = wait_bar(bar_q_full, 0, abort_flag);
-            // S_t(j) = Q_t K_j^T into M-tile t's S columns
-            auto issue_s = [&](int t, int j) -> bool {
-                const int sk = j % NK;
-                if (!wait_bar(bar_k_full + sk, (j / NK) & 1, abort_flag)) return false;
-                // the S columns hold P_t(j-1) until PV_t(j-1) has read them
-                if (j >= 1 && !wait_bar(bar_o_done + t, (j - 1) & 1, abort_flag)) return false;
+            // O += P_i V_i, P_i (bf16) read from its S buffer in TMEM
+            auto issue_pv = [&](int i) -> bool {
+                const int b = i % NB, sv = i % NV;
+                if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag)) return false;
+                if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag)) return false;
                 tc_fence_after();
-                const uint64_t dq = dQ0 + (uint64_t)t * (C::Q_BYTES >> 4);
-                const uint64_t dk = dK0 + (uint64_t)sk * kStageStep;
-                const uint32_t d_tmem = tmem + t * C::TMEM_TILE + C::TMEM_S;
-#pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint64_t koff = (uint64_t)((((kk >> 2) * C::ATOM_BYTES) + (kk & 3) * 32) >> 4);
-                    mma_bf16_ss(d_tmem, dq + koff, dk + koff, idesc_qk, kk > 0 ? 1u : 0u);
-                }
-                mma_commit(bar_s_full + t);
-                if (t == 1 || j >= n1) mma_commit(bar_k_empty + sk);  // last reader of K_j
-                return true;
-            };
-            // O_t += P_t(j) V_j, P_t(j) (bf16 pairs) read from TMEM
-            auto issue_pv = [&](int t, int j) -> bool {
-                const int sv = j % NV;
-                if (!wait_bar(bar_p_full + t, j & 1, abort_flag)) return false;
-                if (!wait_bar(bar_v_full + sv, (j / NV) & 1, abort_flag)) return false;
-                tc_fence_after();
-                const uint64_t dv = dV0 + (uint64_t)sv * kStageStep;
-                const uint32_t pcol = tmem + t * C::TMEM_TILE + C::TMEM_S;
-                const uint32_t d_tmem = tmem + t * C::TMEM_TILE + C::TMEM_O;
+                const uint32_t sV = smem_u32(smem + C::OFF_V + sv * C::KV_BYTES);
+                const uint32_t pcol = tmem + C::TMEM_S + b * kAttnBN;
 #pragma unroll
                 for (int kk = 0; kk < kAttnBN / 16; ++kk)
-                    mma_bf16_ts(d_tmem, pcol + kk * 8, dv + (uint64_t)((kk * 16 * 128) >> 4), idesc_pv,
-                                (j > 0 || kk > 0) ? 1u : 0u);
-                mma_commit(bar_o_done + t);
-                if (t == 1 || j >= n1) mma_commit(bar_v_empty + sv);  // last reader of V_j
+                    mma_bf16_ts(tmem + C::TMEM_O, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, C::ATOM_BYTES, 1024),
+                                idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
+                mma_commit(bar_o_done + b);
+                mma_commit(bar_v_empty + sv);
                 return true;
             };
-            if (ok && n0 > 0) ok = issue_s(0, 0);
-            if (ok && n1 > 0) ok = issue_s(1, 0);
-            for (int j = 0; ok && j < n_all; ++j) {
-                if (ok && j < n0) ok = issue_pv(0, j);
-                if (ok && j + 1 < n0) ok = issue_s(0, j + 1);
-                if (ok && j < n1) ok = issue_pv(1, j);
-                if (ok && j + 1 < n1) ok = issue_s(1, j + 1);
+            for (int j = 0; ok && j < n_tiles; ++j) {
+                const int sk = j % NK, b = j % NB;
+                if (!(ok = wait_bar(bar_k_full + sk, (j / NK) & 1, abort_flag))) break;
+                // buffer b last held P_{j-NB}: its PV must have finished reading it
+                if (j >= NB && !(ok = wait_bar(bar_o_done + b, ((j - NB) / NB) & 1, abort_flag))) break;
+                tc_fence_after();
+                const uint32_t sK = smem_u32(smem + C::OFF_K + sk * C::KV_BYTES);
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t koff = (kk >> 2) * C::ATOM_BYTES + (kk & 3) * 32;
+                    mma_bf16_ss(tmem + C::TMEM_S + b * kAttnBN, sdesc_sw128(sQ + koff, 16, 1024),
+                                sdesc_sw128(sK + koff, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
+                }
+                mma_commit(bar_s_full + b);
+                mma_commit(bar_k_empty + sk);
+                if (j >= 1) ok = issue_pv(j - 1);
             }
+            if (ok && n_tiles > 0) ok = issue_pv(n_tiles - 1);
             mma_commit(bar_drain);  // arrives once every MMA issued above has completed
             drain_bar(bar_drain, 0);
         }
-    } else if (warp < 2 * kSoftmaxWarpsPerTile) {
-        // ------------------------------------------------------------ softmax + epilogue (warps 0-7)
-        // Warp w serves M-tile t = w / 4 and reads TMEM lane quadrant w % 4: thread r owns
-        // row r of that M-tile (one (token, head) row), over all 128 keys of every tile.
-        const int t = warp / kSoftmaxWarpsPerTile, quad = warp & 3;
-        const int r = quad * 32 + lane;
-        const int t_begin = t == 0 ? it.tok0 : it.tok_mid, t_end = t == 0 ? it.tok_mid : it.tok1;
-        const int tok = t_begin + r / G;
-        const bool valid = tok < t_end;
+    } else {
+        // ------------------------------------------------------------ softmax + epilogue (warps 0-3)
+        const int r = threadIdx.x;  // tile row == TMEM lane
+        const int tok = it.tok0 + r / G;
+        const bool valid = tok < it.tok1;
         const int frow = P.cu_fresh[it.query] + tok;
         const int pos = valid ? P.fresh_pos[frow] : 0x7fffffff;
-        const int min_pos = t == 0 ? it.min_pos0 : it.min_pos1;
-        const int n_t = t == 0 ? n0 : n1;
-        const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-        const uint32_t s_col = tmem + lane_base + t * C::TMEM_TILE + C::TMEM_S;
-        const uint32_t o_col = tmem + lane_base + t * C::TMEM_TILE + C::TMEM_O;
+        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
         float m = -INFINITY, l = 0.f;
         bool ok = true;
-        for (int j = 0; j < n_t; ++j) {
-            if (!(ok = warp_wait(bar_s_full + t, j & 1, abort_flag))) break;
+        for (int j = 0; j < n_tiles; ++j) {
+            const int b = j % NB;
+            if (!(ok = warp_wait(bar_s_full + b, (j / NB) & 1, abort_flag))) break;
             tc_fence_after();
+            uint32_t s[128];
+            const uint32_t s_col = tmem + lane_base + C::TMEM_S + b * kAttnBN;
+            tmem_ld32(s_col + 0, *reinterpret_cast<uint32_t(*)[32]>(s + 0));
+            tmem_ld32(s_col + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
+            tmem_ld32(s_col + 64, *reinterpret_cast<uint32_t(*)[32]>(s + 64));
+            tmem_ld32(s_col + 96, *reinterpret_cast<uint32_t(*)[32]>(s + 96));
+            tmem_ld_wait();
+
+            // raw row max (scale > 0 commutes with max); masked slots become -inf.  Eight
+            // independent running maxima keep the dependency chain short.
             const int key0 = (it.kv_tile0 + j) * kAttnBN;
-            const bool masked = key0 + kAttnBN - 1 > min_pos;
-            float mx;
-            {
-                // pass 1: raw row max over the 128 scores (scale > 0 commutes with max), read in
-                // two halves of 64 columns
-                float mx8[8];
+            float mx8[8];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
+            for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
+            if (key0 + kAttnBN - 1 > it.min_pos) {
 #pragma unroll
-                for (int h2 = 0; h2 < 2; ++h2) {
-                    uint32_t s[64];
-                    tmem_ld32(s_col + h2 * 64, *reinterpret_cast<uint32_t(*)[32]>(s + 0));
-                    tmem_ld32(s_col + h2 * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int c = 0; c < 64; ++c) {
-                        const float v =
-                            (masked && key0 + h2 * 64 + c > pos) ? -INFINITY : __uint_as_float(s[c]);
-                        mx8[c & 7] = fmaxf(mx8[c & 7], v);
-                    }
+                for (int c = 0; c < 128; ++c) {
+                    if (key0 + c > pos) s[c] = __float_as_uint(-INFINITY);
+                    mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
                 }
-                mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                           fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+            } else {
+#pragma unroll
+                for (int c = 0; c < 128; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
             }
+            const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
             const float m_new = fmaxf(m, mx * scale_log2);
             const bool resc = m_new > m + kRescaleThreshold;
             float alpha = 1.f;
@@ -379,74 +345,59 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 m = m_new;
             }
             if (j > 0 && __any_sync(0xffffffffu, resc)) {
-                // O is touched only while no PV is in flight: PV_t(j-1) done, PV_t(j) not yet issued
-                if (!(ok = warp_wait(bar_o_done + t, (j - 1) & 1, abort_flag))) break;
+                // O is touched only while no PV is in flight: PV_{j-1} done, PV_j not yet issued
+                if (!(ok = warp_wait(bar_o_done + (j - 1) % NB, ((j - 1) / NB) & 1, abort_flag))) break;
                 tc_fence_after();
 #pragma unroll
                 for (int c4 = 0; c4 < D / 32; ++c4) {
                     uint32_t o[32];
-                    tmem_ld32(o_col + c4 * 32, o);
+                    const uint32_t o_col = tmem + lane_base + C::TMEM_O + c4 * 32;
+                    tmem_ld32(o_col, o);
                     tmem_ld_wait();
 #pragma unroll
                     for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                    tmem_st32(o_col + c4 * 32, o);
+                    tmem_st32(o_col, o);
                 }
             }
-            // pass 2: p = exp2(s * scale - m) on column pairs (packed f32x2); P_t(j) as bf16 pairs
-            // over the first 64 S columns.  Keys are re-read in two halves; each half is read
-            // before any P column that overlaps it is written.
+            // p = exp2(s * scale - m) on column pairs (packed f32x2 arithmetic); three pairs
+            // in eight go to the FMA pipe (exp2_poly2), the rest to MUFU, to balance the two
             const float mu = (m == -INFINITY) ? 0.f : m;
             const uint64_t sc2 = f2_pack(scale_log2, scale_log2);
             const uint64_t nmu2 = f2_pack(-mu, -mu);
             uint64_t acc[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) acc[e] = f2_pack(0.f, 0.f);
+            uint32_t pk[64];
 #pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-                uint32_t s[64];
-                tmem_ld32(s_col + h2 * 64, *reinterpret_cast<uint32_t(*)[32]>(s + 0));
-                tmem_ld32(s_col + h2 * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
-                tmem_ld_wait();
-                if (masked) {
-#pragma unroll
-                    for (int c = 0; c < 64; ++c)
-                        if (key0 + h2 * 64 + c > pos) s[c] = __float_as_uint(-INFINITY);
+            for (int c = 0; c < 64; ++c) {
+                const uint64_t x2 = ffma2(f2_pack(__uint_as_float(s[2 * c]), __uint_as_float(s[2 * c + 1])), sc2, nmu2);
+                uint64_t p2;
+                if ((c & 7) >= KVLINK_EXP_POLY_FROM) {
+                    p2 = exp2_poly2(x2);
+                } else {
+                    float a, b;
+                    f2_unpack(x2, a, b);
+                    p2 = f2_pack(ex2_approx(a), ex2_approx(b));
                 }
-#pragma unroll
-                for (int q2 = 0; q2 < 2; ++q2) {
-                    uint32_t pk[16];
-#pragma unroll
-                    for (int c = 0; c < 16; ++c) {
-                        const int cc = q2 * 16 + c;  // column pair within this half
-                        const uint64_t x2 =
-                            ffma2(f2_pack(__uint_as_float(s[2 * cc]), __uint_as_float(s[2 * cc + 1])), sc2, nmu2);
-                        uint64_t p2;
-                        if ((cc & 7) >= KVLINK_EXP_POLY_FROM) {
-                            p2 = exp2_poly2(x2);
-                        } else {
-                            float a, b;
-                            f2_unpack(x2, a, b);
-                            p2 = f2_pack(ex2_approx(a), ex2_approx(b));
-                        }
-                        acc[c & 3] = fadd2(acc[c & 3], p2);
-                        float p0, p1;
-                        f2_unpack(p2, p0, p1);
-                        pk[c] = pack2_bf16(p0, p1);
-                    }
-                    tmem_st16(s_col + h2 * 32 + q2 * 16, pk);
-                }
+                acc[c & 3] = fadd2(acc[c & 3], p2);
+                float p0, p1;
+                f2_unpack(p2, p0, p1);
+                pk[c] = pack2_bf16(p0, p1);
             }
             float rs0, rs1;
             f2_unpack(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), rs0, rs1);
-            l += rs0 + rs1;
+            const float rs = rs0 + rs1;
+            l += rs;
+            // P_j (bf16) over the first 64 columns of its S buffer, read there by the PV MMA
+            tmem_st32(s_col + 0, *reinterpret_cast<uint32_t(*)[32]>(pk + 0));
+            tmem_st32(s_col + 32, *reinterpret_cast<uint32_t(*)[32]>(pk + 32));
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar_p_full + t);
+            if (lane == 0) mbar_arrive(bar_p_full + b);
         }
-        if (ok && n_t > 0) ok = warp_wait(bar_o_done + t, (n_t - 1) & 1, abort_flag);
-        const bool exists = t == 0 || has1;
-        if (ok && exists) {
+        if (ok && n_tiles > 0) ok = warp_wait(bar_o_done + (n_tiles - 1) % NB, ((n_tiles - 1) / NB) & 1, abort_flag);
+        if (ok) {
             tc_fence_after();
             if (it.slot < 0) {
                 const float inv = 1.f / l;
@@ -454,7 +405,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
                 for (int c4 = 0; c4 < D / 32; ++c4) {
                     uint32_t o[32];
-                    tmem_ld32(o_col + c4 * 32, o);
+                    tmem_ld32(tmem + lane_base + C::TMEM_O + c4 * 32, o);
                     tmem_ld_wait();
                     if (valid) {
 #pragma unroll
@@ -469,19 +420,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                 }
             } else {
-                // partial result of this key range; an M-tile with no key tile here writes an
-                // empty partial (O = 0, m = -inf, l = 0) that the merge weighs with zero
-                float* wo = ws + (int64_t)(it.slot + t) * kAttnBM * (D + 2);
+                float* wo = ws + (int64_t)it.slot * kAttnBM * (D + 2);
 #pragma unroll
                 for (int c4 = 0; c4 < D / 32; ++c4) {
                     uint32_t o[32];
-                    if (n_t > 0) {
-                        tmem_ld32(o_col + c4 * 32, o);
-                        tmem_ld_wait();
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < 32; ++e) o[e] = 0u;
-                    }
+                    tmem_ld32(tmem + lane_base + C::TMEM_O + c4 * 32, o);
+                    tmem_ld_wait();
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
                         *reinterpret_cast<uint4*>(wo + r * D + c4 * 32 + 4 * q) =
@@ -512,11 +456,10 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(DevicePlan P, const flo
     for (int idx = threadIdx.x; idx < n_rows * D; idx += blockDim.x) {
         const int r = idx / D, d = idx % D;
         float M = -INFINITY;
-        for (int s = 0; s < mg.n_split; ++s)
-            M = fmaxf(M, ws[(int64_t)(mg.slot0 + s * mg.slot_stride) * slot_floats + kAttnBM * D + r]);
+        for (int s = 0; s < mg.n_split; ++s) M = fmaxf(M, ws[(mg.slot0 + s) * slot_floats + kAttnBM * D + r]);
         float L = 0.f, O = 0.f;
         for (int s = 0; s < mg.n_split; ++s) {
-            const float* w = ws + (int64_t)(mg.slot0 + s * mg.slot_stride) * slot_floats;
+            const float* w = ws + (mg.slot0 + s) * slot_floats;
             const float ms = w[kAttnBM * D + r];
             const float f = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
             L += w[kAttnBM * D + kAttnBM + r] * f;

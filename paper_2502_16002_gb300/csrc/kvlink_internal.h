@@ -34,33 +34,27 @@ struct CopyChunk {
 };
 static_assert(sizeof(CopyChunk) == 32, "CopyChunk layout");
 
-// One attention work item: two M-tiles of up to 128 rows each ((token, query head) rows
-// of one query and one KV head) that share every key/value tile, over a range of key
-// tiles.  M-tile 0 holds the earlier tokens, so its key range ends no later than tile 1's.
+// One attention work item: an M-tile of (token, head) rows of one query and KV head,
+// over KV tiles [kv_tile0, kv_tile1).
 struct AttnItem {
     int32_t query;
     int32_t kv_head;
-    int32_t tok0, tok_mid, tok1;  // M-tile 0 = tokens [tok0, tok_mid), M-tile 1 = [tok_mid, tok1)
-                                  // (query-relative; M-tile 1 may be empty)
-    int32_t kv_tile0, kv_tile1;   // key tiles of kAttnBN keys handled by this item
-    int32_t kv_end0;              // M-tile 0 needs key tiles < kv_end0 only
-    int32_t slot;                 // partial-result slots slot (M-tile 0) and slot + 1 (M-tile 1),
-                                  // or -1: write the output directly
-    int32_t min_pos0, min_pos1;   // smallest row position of each M-tile: keys <= min_pos are
-                                  // visible to every row of that tile
-    int32_t pad;
+    int32_t tok0, tok1;          // fresh tokens [tok0, tok1) of the query (query-relative)
+    int32_t kv_tile0, kv_tile1;  // key tiles of kAttnBN keys
+    int32_t slot;                // partial-result slot, or -1: write the output directly
+    int32_t min_pos;             // smallest position of the tile's rows: keys <= min_pos
+                                 // are visible to every row of the tile
 };
-static_assert(sizeof(AttnItem) == 48, "AttnItem layout");
+static_assert(sizeof(AttnItem) == 32, "AttnItem layout");
 
 // Rows of one (query, KV head, M-tile) whose KV range was split over several items.
 struct MergeGroup {
     int32_t query;
     int32_t kv_head;
     int32_t tok0, tok1;
-    int32_t slot0;               // partial slot of the first split
+    int32_t slot0;               // first partial slot; the group's slots are consecutive
     int32_t n_split;
-    int32_t slot_stride;         // slot distance between consecutive splits
-    int32_t pad;
+    int32_t pad0, pad1;
 };
 static_assert(sizeof(MergeGroup) == 32, "MergeGroup layout");
 

@@ -174,53 +174,47 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     }
 
     // ---- attention work items
-    // M-tiles of one (query, KV head) split the query's fresh tokens into near-equal runs
-    // of at most kAttnBM / G tokens; a tile's key range ends at its last token.  Consecutive
-    // M-tiles are paired into one item so that they share every K/V tile load.
+    // M-tiles of one (query, KV head) split the query's fresh tokens into near-equal
+    // runs of at most kAttnBM / G tokens; a tile's key range ends at its last token.
     const int G = d->h_q / d->h_kv;
     const int tok_per_tile = kAttnBM / G;
-    struct Pair { int32_t b, g, t0, tm, t1, end0, end1, min0, min1; };
-    std::vector<Pair> pairs;
+    struct Tile { int32_t b, g, t0, t1, n_tiles, min_pos; };
+    std::vector<Tile> tiles;
     int64_t work = 0;
     p->attn_pairs = 0;
     for (int b = 0; b < B; ++b) {
         const int32_t f0 = p->cu_fresh[b], T = p->cu_fresh[b + 1] - f0;
         for (int r = 0; r < T; ++r) p->attn_pairs += (int64_t)p->fresh_pos[f0 + r] + 1;
         const int n_mt = (T + tok_per_tile - 1) / tok_per_tile;
-        auto bound = [&](int mt) { return (int)((int64_t)T * mt / n_mt); };
-        auto kv_end = [&](int t1) { return (p->fresh_pos[f0 + t1 - 1] + kAttnBN) / kAttnBN; };
         for (int g = 0; g < d->h_kv; ++g) {
-            for (int mt = 0; mt < n_mt; mt += 2) {
-                const int t0 = bound(mt), tm = bound(mt + 1);
-                const int t1 = mt + 1 < n_mt ? bound(mt + 2) : tm;
-                const int end0 = kv_end(tm);
-                const int end1 = t1 > tm ? kv_end(t1) : end0;
-                pairs.push_back({b, g, t0, tm, t1, end0, end1, p->fresh_pos[f0 + t0],
-                                 t1 > tm ? p->fresh_pos[f0 + tm] : 0});
-                work += end1;
+            for (int mt = 0; mt < n_mt; ++mt) {
+                const int t0 = (int)((int64_t)T * mt / n_mt), t1 = (int)((int64_t)T * (mt + 1) / n_mt);
+                const int32_t kv_len = p->fresh_pos[f0 + t1 - 1] + 1;  // positions increase within a query
+                const int32_t nt = (kv_len + kAttnBN - 1) / kAttnBN;
+                tiles.push_back({b, g, t0, t1, nt, p->fresh_pos[f0 + t0]});
+                work += nt;
             }
         }
     }
-    // split long key ranges so that the items spread evenly over the SMs
+    // split long KV ranges so that the items spread evenly over the SMs
     const int64_t per_sm = (work + 2 * (int64_t)num_sms - 1) / (2 * (int64_t)num_sms);
     const int32_t max_tiles = (int32_t)std::max<int64_t>(8, per_sm);
     p->items.clear();
     p->merges.clear();
     p->n_slots = 0;
-    for (const Pair& q : pairs) {
-        const int32_t n_split = (q.end1 + max_tiles - 1) / max_tiles;
+    for (const Tile& t : tiles) {
+        const int32_t n_split = (t.n_tiles + max_tiles - 1) / max_tiles;
         if (n_split <= 1) {
-            p->items.push_back({q.b, q.g, q.t0, q.tm, q.t1, 0, q.end1, q.end0, -1, q.min0, q.min1, 0});
+            p->items.push_back({t.b, t.g, t.t0, t.t1, 0, t.n_tiles, -1, t.min_pos});
             continue;
         }
-        p->merges.push_back({q.b, q.g, q.t0, q.tm, p->n_slots, n_split, 2, 0});
-        if (q.t1 > q.tm) p->merges.push_back({q.b, q.g, q.tm, q.t1, p->n_slots + 1, n_split, 2, 0});
+        p->merges.push_back({t.b, t.g, t.t0, t.t1, p->n_slots, n_split, 0, 0});
         for (int s = 0; s < n_split; ++s) {
-            const int32_t a = (int32_t)((int64_t)q.end1 * s / n_split);
-            const int32_t e = (int32_t)((int64_t)q.end1 * (s + 1) / n_split);
-            p->items.push_back({q.b, q.g, q.t0, q.tm, q.t1, a, e, q.end0, p->n_slots + 2 * s, q.min0, q.min1, 0});
+            const int32_t a = (int32_t)((int64_t)t.n_tiles * s / n_split);
+            const int32_t e = (int32_t)((int64_t)t.n_tiles * (s + 1) / n_split);
+            p->items.push_back({t.b, t.g, t.t0, t.t1, a, e, p->n_slots + s, t.min_pos});
         }
-        p->n_slots += 2 * n_split;
+        p->n_slots += n_split;
     }
     // Launch order: the items of one (query, KV head) stay adjacent, so that CTAs running
     // at the same time read the same K/V tiles (served from L2 after the first); groups
