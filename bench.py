@@ -40,7 +40,10 @@ UNIT = "us/query"
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from the committed ncu
 # summaries under profiles/, keyed by (kernel, workload); None until captured for
 # the current kernel version.
-NCU_TRAFFIC = {}
+NCU_TRAFFIC = {
+    ("attention", 3): 193690880,   # profiles/attention_tc_llama8b_b8_zipf.md
+    ("reencode", 3): 228842496,    # profiles/reencode_llama8b_b8_zipf.md
+}
 
 
 def _peaks():
