@@ -95,3 +95,37 @@ class LinkedPrefill:
                                 k_new.data_ptr(), v_new.data_ptr(), cache_k.data_ptr(),
                                 cache_v.data_ptr(), out.data_ptr(), self.workspace.data_ptr(),
                                 self.workspace.numel(), _stream_handle(stream))
+
+    def linked_prefill_layers_from_host(self, pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new,
+                                        cache_k, cache_v, out, h_out, streams=None):
+        """Every layer of the linked prefill with the fresh rows in host memory.
+
+        Per layer l: h_q[l], h_k_new[l], h_v_new[l] (pinned host tensors) are copied to
+        q[l], k_new[l], v_new[l] on an input stream, kvlink_linked_prefill runs on the
+        compute stream once they have landed, and out[l] is copied to h_out[l] (pinned) on
+        an output stream once it is written.  The copies of one layer thus overlap the
+        kernels of the layers around it.  Returns after the last output has arrived.
+
+        streams: optional (input, compute, output) torch.cuda.Stream triple.
+        """
+        if streams is None:
+            streams = (torch.cuda.Stream(self.device), torch.cuda.current_stream(self.device),
+                       torch.cuda.Stream(self.device))
+        s_in, s_c, s_out = streams
+        n = len(pool_k)
+        for l in range(n):
+            ev_in = torch.cuda.Event()
+            with torch.cuda.stream(s_in):
+                q[l].copy_(h_q[l], non_blocking=True)
+                k_new[l].copy_(h_k_new[l], non_blocking=True)
+                v_new[l].copy_(h_v_new[l], non_blocking=True)
+                ev_in.record(s_in)
+            s_c.wait_event(ev_in)
+            self.linked_prefill(pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l],
+                                out[l], stream=s_c)
+            ev_out = torch.cuda.Event()
+            ev_out.record(s_c)
+            s_out.wait_event(ev_out)
+            with torch.cuda.stream(s_out):
+                h_out[l].copy_(out[l], non_blocking=True)
+        s_out.synchronize()

@@ -208,3 +208,36 @@ def test_llama8b_paged_serving_sampled(RT):
         check_query(batch, b, lp, gk, gv, gout, inp)
     for b in (1, 17, 40):
         check_query(batch, b, lp, gk, gv, gout, inp, attention=False)
+
+
+def test_layers_from_host_pipeline_matches_per_layer_calls(RT):
+    """The host-to-host pipelined helper gives the same bytes as per-layer device calls."""
+    batch = W.draw_batch(W.get_config(2))
+    dev = torch.device("cuda:0")
+    L = 2
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    pk, pv, qh, kh, vh = [], [], [], [], []
+    for layer in range(L):
+        a, b = W.pool_kv(batch, layer)
+        q, k, v = W.fresh_qkv(batch, layer)
+        pk.append(RT.bf16_from_bits(a, dev))
+        pv.append(RT.bf16_from_bits(b, dev))
+        qh.append(RT.bf16_from_bits(q).pin_memory())
+        kh.append(RT.bf16_from_bits(k).pin_memory())
+        vh.append(RT.bf16_from_bits(v).pin_memory())
+    shape_q, shape_k = qh[0].shape, kh[0].shape
+    dq = [torch.empty(shape_q, dtype=torch.bfloat16, device=dev) for _ in range(L)]
+    dk = [torch.empty(shape_k, dtype=torch.bfloat16, device=dev) for _ in range(L)]
+    dv = [torch.empty(shape_k, dtype=torch.bfloat16, device=dev) for _ in range(L)]
+    caches = [lp.empty_cache() for _ in range(L)]
+    dout = [torch.empty(shape_q, dtype=torch.bfloat16, device=dev) for _ in range(L)]
+    hout = [torch.empty(shape_q, dtype=torch.bfloat16).pin_memory() for _ in range(L)]
+    lp.linked_prefill_layers_from_host(pk, pv, qh, kh, vh, dq, dk, dv, [c[0] for c in caches],
+                                       [c[1] for c in caches], dout, hout)
+    for layer in range(L):
+        ck, cv = lp.empty_cache()
+        ref = torch.empty(shape_q, dtype=torch.bfloat16, device=dev)
+        lp.linked_prefill(pk[layer], pv[layer], qh[layer].to(dev), kh[layer].to(dev), vh[layer].to(dev),
+                          ck, cv, ref)
+        torch.cuda.synchronize()
+        assert torch.equal(hout[layer].view(torch.int16), ref.cpu().view(torch.int16))
