@@ -166,6 +166,30 @@ def algorithmic_counts(batch, info):
                 attn_flops=attn_flops, attn_bytes=attn_bytes, unique_pool_tokens=unique_tokens)
 
 
+# ------------------------------------------------------------------ multi-rank bookkeeping
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """The largest value of x over all ranks (timing only: no data-path collective)."""
+    if world == 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_us_per_query(ms_per_step: float, batch_per_rank: int, world: int) -> float:
+    """Every rank serves its own batch in parallel: queries of all ranks over the slowest rank's time."""
+    return ms_per_step * 1e3 / (batch_per_rank * world)
+
+
+def rank_batch_seed(rank: int) -> int:
+    """Each rank draws an independent batch (weak scaling: fixed work per GPU)."""
+    return rank
+
+
 # ------------------------------------------------------------------ our arm
 
 def run_ours(args, rank, world, local_rank):
@@ -177,7 +201,7 @@ def run_ours(args, rank, world, local_rank):
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
     cfg = W.get_config(args.config)
-    batch = W.draw_batch(cfg, seed=rank)           # every rank serves its own batch
+    batch = W.draw_batch(cfg, seed=rank_batch_seed(rank))   # every rank serves its own batch
     L = args.layers or cfg.layers
     lp = LinkedPrefill.from_batch(batch, device=dev)
     info = lp.info
@@ -210,14 +234,6 @@ def run_ours(args, rank, world, local_rank):
             import torch.distributed as dist
             dist.barrier()
 
-    def max_over_ranks(x):
-        if world == 1:
-            return x
-        import torch.distributed as dist
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
-
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize(dev)
@@ -236,10 +252,10 @@ def run_ours(args, rank, world, local_rank):
         torch.cuda.synchronize(dev)
         clk.stop()
         barrier()
-    ms_total = max_over_ranks(e0.elapsed_time(e1))
+    ms_total = max_over_ranks(e0.elapsed_time(e1), world, dev)
     ms_per_step = ms_total / args.steps
     us_per_query = ms_per_step * 1e3 / cfg.batch      # per rank; ranks run in parallel
-    value = ms_per_step * 1e3 / (cfg.batch * world)   # whole job: all ranks' queries / time
+    value = whole_job_us_per_query(ms_per_step, cfg.batch, world)
     assert K.kvlink_device_status() == 0
 
     # ---- per-kernel pass: same work through the separate calls, events around each
@@ -292,9 +308,9 @@ def run_ours(args, rank, world, local_rank):
             e2e_step()
         t1 = time.perf_counter()
         barrier()
-        e2e_ms = max_over_ranks((t1 - t0) * 1e3) / e2e_steps
+        e2e_ms = max_over_ranks((t1 - t0) * 1e3, world, dev) / e2e_steps
         h2d = (h_q.numel() + h_kn.numel() + h_vn.numel()) * 2 + int(info.device_bytes)
-        e2e = {"value": round(e2e_ms * 1e3 / (cfg.batch * world), 3), "unit": UNIT,
+        e2e = {"value": round(whole_job_us_per_query(e2e_ms, cfg.batch, world), 3), "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(h_out.numel() * 2),
                "steps": e2e_steps,
                "note": "per step: host plan build + table upload; per layer, fresh q/k/v H2D from pinned "
