@@ -195,6 +195,18 @@ int kvlink_suffix_attention_simt(const kvlink_plan_t* plan, const void* d_q, con
                                  const void* d_v_new, void* d_cache_k, void* d_cache_v, void* d_out,
                                  kvlink_stream_t stream);
 
+/* RoPE of the fresh rows at their global positions, in place (Sec. 2.2: the token at
+ * position i carries R_i; Sec. 2.3: link and question tokens are encoded at their
+ * positions in the linked sequence):
+ *   q[r][h]     = R_{p_r}(q[r][h])      for every query head h,
+ *   k_new[r][g] = R_{p_r}(k_new[r][g])  for every KV head g,
+ * p_r the global position of fresh row r, theta the plan's (kvlink_plan_upload), pairs
+ * (j, j + D/2).  For producers that project fresh rows without RoPE:
+ * kvlink_suffix_attention and kvlink_linked_prefill take q and k_new already rotated.
+ * d_q: [n_fresh][h_q][D], d_k_new: [n_fresh][h_kv][D], bf16; each result within one bf16
+ * ulp of the fp64 rotation.  Errors: EINVAL, ECUDA. */
+int kvlink_rope_fresh(const kvlink_plan_t* plan, void* d_q, void* d_k_new, kvlink_stream_t stream);
+
 /* One layer of the linked prefill: kvlink_reencode_concat with the fresh-row
  * placement fused into the same launch, then the suffix attention.  Same arguments
  * and errors as the two calls it chains. */

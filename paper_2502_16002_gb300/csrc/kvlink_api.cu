@@ -16,6 +16,8 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
                      const void* pool_k, const void* pool_v, const void* k_new, const void* v_new, void* cache_k,
                      void* cache_v, cudaStream_t stream);
 int read_copy_status(int32_t* status);
+void launch_rope_fresh(const int32_t* d_fresh_pos, int n_fresh, int head_dim, double theta, void* q, int h_q,
+                       void* k, int h_kv, cudaStream_t stream);
 int clear_copy_status();
 void launch_attention_simt(const DevicePlan& P, int n_fresh, int head_dim, int h_q, int h_kv,
                            const void* q, const void* cache_k, const void* cache_v, void* out,
@@ -277,6 +279,15 @@ int kvlink_linked_prefill(const kvlink_plan_t* p, const void* pool_k, const void
     rc = check_launch("reencode_kernel (fused)");
     if (rc) return rc;
     return attention_common(p, q, cache_k, cache_v, out, ws, ws_bytes, s);
+}
+
+int kvlink_rope_fresh(const kvlink_plan_t* p, void* q, void* k_new, kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (!q || !k_new) return KVLINK_EINVAL;
+    launch_rope_fresh(p->dev.fresh_pos, p->cu_fresh.back(), p->head_dim, p->theta, q, p->h_q, k_new, p->h_kv,
+                      (cudaStream_t)stream);
+    return check_launch("rope_fresh_kernel");
 }
 
 int kvlink_device_status(int32_t* status) {

@@ -280,6 +280,41 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
     }
 }
 
+// --------------------------------------------------------------------------
+// RoPE of the fresh rows at their global positions (Sec. 2.2: a token at position i
+// carries R_i).  One thread per (fresh row, j < D/2): the angle pos * theta^(-2j/D) is
+// formed in float64, cos/sin are split into float pairs, and pair (j, j + D/2) of every
+// query head and KV head of the row is rotated in place with the compensated products
+// of the re-encode, so each output is within one bf16 ulp of the fp64 rotation.
+// --------------------------------------------------------------------------
+__global__ void rope_fresh_kernel(const int32_t* __restrict__ fresh_pos, int n_fresh, int head_dim, double theta,
+                                  __nv_bfloat16* __restrict__ q, int h_q, __nv_bfloat16* __restrict__ k, int h_kv) {
+    const int half = head_dim / 2;
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (int64_t)n_fresh * half) return;
+    const int r = (int)(i / half), j = (int)(i % half);
+    const double angle = (double)fresh_pos[r] * pow(theta, -2.0 * (double)j / (double)head_dim);
+    double sn, cs;
+    sincos(angle, &sn, &cs);
+    const float ch = (float)cs, cl = (float)(cs - (double)ch), sh = (float)sn, sl = (float)(sn - (double)sh);
+    auto rot = [&](__nv_bfloat16* row) {
+        const float x = __bfloat162float(row[j]), y = __bfloat162float(row[j + half]);
+        row[j] = __float2bfloat16_rn(rot_first(x, y, ch, cl, sh, sl));
+        row[j + half] = __float2bfloat16_rn(rot_second(x, y, ch, cl, sh, sl));
+    };
+    for (int h = 0; h < h_q; ++h) rot(q + ((int64_t)r * h_q + h) * head_dim);
+    for (int h = 0; h < h_kv; ++h) rot(k + ((int64_t)r * h_kv + h) * head_dim);
+}
+
+void launch_rope_fresh(const int32_t* d_fresh_pos, int n_fresh, int head_dim, double theta, void* q, int h_q,
+                       void* k, int h_kv, cudaStream_t stream) {
+    const int64_t n = (int64_t)n_fresh * (head_dim / 2);
+    if (n == 0) return;
+    const int threads = 256;
+    rope_fresh_kernel<<<(unsigned)((n + threads - 1) / threads), threads, 0, stream>>>(
+        d_fresh_pos, n_fresh, head_dim, theta, (__nv_bfloat16*)q, h_q, (__nv_bfloat16*)k, h_kv);
+}
+
 int read_copy_status(int32_t* status) {
     return cudaMemcpyFromSymbol(status, g_copy_status, sizeof(int32_t)) == cudaSuccess ? KVLINK_OK : KVLINK_ECUDA;
 }

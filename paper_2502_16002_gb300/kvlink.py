@@ -92,6 +92,7 @@ def _load():
         "kvlink_suffix_attention": (C.c_int, [P, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_suffix_attention_simt": (C.c_int, [P, V, V, V, V, V, V, V]),
         "kvlink_suffix_attention_noalloc": (C.c_int, [P, V, V, V, V, V, V, V]),
+        "kvlink_rope_fresh": (C.c_int, [P, V, V, V]),
         "kvlink_linked_prefill": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
@@ -111,7 +112,7 @@ DECLARED = [
     "kvlink_reencode_concat", "kvlink_suffix_attention", "kvlink_suffix_attention_simt",
     "kvlink_linked_prefill",
     "kvlink_device_status", "kvlink_clear_device_status", "kvlink_strerror",
-    "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc",
+    "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc", "kvlink_rope_fresh",
 ]
 
 # size of the static scratch used by kvlink_suffix_attention_noalloc (include/kvlink.h)
@@ -243,6 +244,10 @@ def kvlink_suffix_attention_noalloc(plan: Plan, q: int, k_new, v_new, cache_k: i
     static device array (see include/kvlink.h); it allocates nothing."""
     _check(lib.kvlink_suffix_attention_noalloc(plan.handle, q, k_new, v_new, cache_k, cache_v, out, stream),
            "kvlink_suffix_attention_noalloc")
+
+
+def kvlink_rope_fresh(plan: Plan, q: int, k_new: int, stream: int = 0) -> None:
+    _check(lib.kvlink_rope_fresh(plan.handle, q, k_new, stream), "kvlink_rope_fresh")
 
 
 def kvlink_linked_prefill(plan: Plan, pool_k: int, pool_v: int, q: int, k_new: int, v_new: int,

@@ -83,6 +83,9 @@ class LinkedPrefill:
                                   self.workspace.data_ptr(), self.workspace.numel(),
                                   _stream_handle(stream))
 
+    def rope_fresh(self, q, k_new, stream=None):
+        K.kvlink_rope_fresh(self.plan, q.data_ptr(), k_new.data_ptr(), _stream_handle(stream))
+
     def suffix_attention_simt(self, q, k_new, v_new, cache_k, cache_v, out, stream=None):
         K.kvlink_suffix_attention_simt(self.plan, q.data_ptr(),
                                        k_new.data_ptr() if k_new is not None else None,

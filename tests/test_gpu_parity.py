@@ -241,3 +241,31 @@ def test_layers_from_host_pipeline_matches_per_layer_calls(RT):
                           ck, cv, ref)
         torch.cuda.synchronize()
         assert torch.equal(hout[layer].view(torch.int16), ref.cpu().view(torch.int16))
+
+
+@pytest.mark.parametrize("cfg_index", [2, 4])
+def test_rope_fresh_within_one_ulp(RT, cfg_index):
+    """Fresh q/k rotated at their global positions (positions up to 51.8k for workload 4)."""
+    from paper_2502_16002_gb300 import kvlink as K
+    batch = W.draw_batch(W.get_config(cfg_index))
+    dev = torch.device("cuda:0")
+    q, kn, _ = W.fresh_qkv(batch, 0)
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    dq, dk = RT.bf16_from_bits(q, dev), RT.bf16_from_bits(kn, dev)
+    lp.rope_fresh(dq, dk)
+    torch.cuda.synchronize()
+    pos = K.kvlink_plan_get_fresh_positions(lp.plan).astype(np.int64)
+    theta = batch.cfg.theta
+    for got, src in ((RT.bits_from_bf16(dq), q), (RT.bits_from_bf16(dk), kn)):
+        want = O.f64_to_bf16_bits(O.rope_rotate(O.bf16_bits_to_f64(src), pos[:, None], theta))
+        assert ulp_distance(got, want).max() <= 1
+
+
+def test_ttft_comparison_harness_runs(RT):
+    """The standard-vs-linked TTFT harness on a small case, with the caches in host memory."""
+    from paper_2502_16002_gb300 import ttft
+    dev = torch.device("cuda:0")
+    layer = ttft.Layer(dev)
+    t_std, t_lnk, n_ctx, T = ttft.measure(64, 3, 5, 16, True, dev, layer)
+    assert n_ctx == 3 * 64 + 16 and T == 3 * 5 + 16
+    assert t_std > 0 and t_lnk > 0
