@@ -17,7 +17,9 @@ scales by the layer count (every layer costs the same):
 
 Both arms use the same weights, the same cuBLAS GEMMs (torch.matmul) and the same
 elementwise glue (RMSNorm, SiLU, residual adds in torch); RoPE of the fresh rows and all
-attention run in this library's kernels.  No accuracy is claimed: the weights are random.
+attention run in this library's kernels.  Each arm's layer is captured in a CUDA graph, so
+host launch overhead is out of both measurements.  No accuracy is claimed: the weights are
+random.
 
     python -m paper_2502_16002_gb300.ttft [--lengths 100 200 300 400 500] [--links 1 5]
 """
@@ -84,6 +86,21 @@ def _plan(doc_lens, n_link, q_len, device, prefix=0):
                          q_len=[q_len], device=device)
 
 
+def _graphed(fn):
+    """fn captured in a CUDA graph (launch overhead out of the measurement, for both arms)."""
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):  # warm-up outside capture: kernel attributes, cuBLAS handles
+        fn()
+        fn()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        fn()
+    return g.replay
+
+
 def _time(fn, warmup=10, iters=40):
     for _ in range(warmup):
         fn()
@@ -134,8 +151,8 @@ def measure(doc_len, n_docs, n_link, q_len, host_caches, device, layer):
         lp.linked_prefill(pool_k, pool_v, q, k, v, ck, cv, out)
         return _finish(layer, x_new, out)
 
-    t_std = _time(standard)
-    t_lnk = _time(linked)
+    t_std = _time(_graphed(standard))
+    t_lnk = _time(_graphed(linked))
     assert K.kvlink_device_status() == 0
     return t_std, t_lnk, n_ctx, T
 
