@@ -157,6 +157,68 @@ def measure(doc_len, n_docs, n_link, q_len, host_caches, device, layer):
     return t_std, t_lnk, n_ctx, T
 
 
+def measure_pipelined(doc_len, n_docs, n_link, q_len, device, layer, layers=LAYERS):
+    """Whole-model TTFT (ms) of both arms with the linked arm's document caches in pinned host
+    memory: every layer's caches are copied to the GPU on a copy stream into one of two device
+    slots while the previous layer computes (Sec. 3.3: caches in CPU memory, loading counted
+    in TTFT).  Each arm's `layers` layers run as one CUDA graph."""
+    n_ctx = n_docs * doc_len + q_len
+    std = _plan([], 0, n_ctx, device)
+    x_std = torch.randn(n_ctx, HIDDEN, device=device, dtype=torch.bfloat16)
+    ck_s, cv_s = std.empty_cache()
+    out_s = torch.empty(n_ctx, H_Q, HEAD_DIM, device=device, dtype=torch.bfloat16)
+
+    def standard():
+        x = x_std
+        for _ in range(layers):
+            q, k, v = _qkv(layer, x)
+            std.rope_fresh(q, k)
+            std.suffix_attention(q, k, v, ck_s, cv_s, out_s)
+            x = _finish(layer, x, out_s)
+        return x
+
+    lp = _plan([doc_len] * n_docs, n_link, q_len, device)
+    rows = n_docs * doc_len
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(1)
+    h_k = [torch.randn(rows, H_KV, HEAD_DIM, generator=gen).to(torch.bfloat16).pin_memory() for _ in range(layers)]
+    h_v = [torch.randn(rows, H_KV, HEAD_DIM, generator=gen).to(torch.bfloat16).pin_memory() for _ in range(layers)]
+    slot_k = [torch.empty(rows, H_KV, HEAD_DIM, device=device, dtype=torch.bfloat16) for _ in range(2)]
+    slot_v = [torch.empty(rows, H_KV, HEAD_DIM, device=device, dtype=torch.bfloat16) for _ in range(2)]
+    T = int(lp.info.n_fresh)
+    x_new = torch.randn(T, HIDDEN, device=device, dtype=torch.bfloat16)
+    ck, cv = lp.empty_cache()
+    out = torch.empty(T, H_Q, HEAD_DIM, device=device, dtype=torch.bfloat16)
+    copy_stream = torch.cuda.Stream(device)
+
+    def linked():
+        compute = torch.cuda.current_stream(device)
+        done = [None, None]
+        x = x_new
+        for l in range(layers):
+            b = l % 2
+            copy_stream.wait_stream(compute) if done[b] is None else copy_stream.wait_event(done[b])
+            with torch.cuda.stream(copy_stream):
+                slot_k[b].copy_(h_k[l], non_blocking=True)
+                slot_v[b].copy_(h_v[l], non_blocking=True)
+                loaded = torch.cuda.Event()
+                loaded.record(copy_stream)
+            q, k, v = _qkv(layer, x)
+            lp.rope_fresh(q, k)
+            compute.wait_event(loaded)
+            lp.linked_prefill(slot_k[b], slot_v[b], q, k, v, ck, cv, out)
+            x = _finish(layer, x, out)
+            done[b] = torch.cuda.Event()
+            done[b].record(compute)
+        compute.wait_stream(copy_stream)
+        return x
+
+    t_std = _time(_graphed(standard), warmup=3, iters=10)
+    t_lnk = _time(_graphed(linked), warmup=3, iters=10)
+    assert K.kvlink_device_status() == 0
+    return t_std, t_lnk, n_ctx, T
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--lengths", type=int, nargs="+", default=[100, 200, 300, 400, 500])
@@ -164,9 +226,23 @@ def main():
     ap.add_argument("--docs", type=int, default=10)
     ap.add_argument("--question", type=int, default=32)
     ap.add_argument("--host-caches", action="store_true")
+    ap.add_argument("--pipelined", action="store_true",
+                    help="whole model, caches in host memory, per-layer loading overlapped with compute")
     args = ap.parse_args()
     dev = torch.device("cuda:0")
     layer = Layer(dev)
+    if args.pipelined:
+        for n_link in args.links:
+            for L in args.lengths:
+                t_std, t_lnk, n_ctx, T = measure_pipelined(L, args.docs, n_link, args.question, dev, layer)
+                print(json.dumps({
+                    "workload": f"{args.docs} docs x {L} tokens, question {args.question}, KVLink{n_link}",
+                    "context_tokens": n_ctx, "fresh_tokens": T, "ttft_standard_ms": round(t_std, 3),
+                    "ttft_linked_ms": round(t_lnk, 3), "reduction_pct": round(100 * (1 - t_lnk / t_std), 1),
+                    "caches": "pinned host memory, per-layer copies overlapped with the previous layer",
+                    "layers": LAYERS, "shape": "Llama-3.1-8B, random bf16 weights, whole model in one graph"}),
+                    flush=True)
+        return
     for n_link in args.links:
         for L in args.lengths:
             t_std, t_lnk, n_ctx, T = measure(L, args.docs, n_link, args.question, args.host_caches, dev, layer)
