@@ -31,7 +31,9 @@
  * Sequence layout of one query b (Sec. 2.3: link tokens follow every document):
  *   [prefix (P tokens), doc_1 (l_1), link_1 (K), doc_2, link_2, ..., doc_N, link_N,
  *    question (Q_b)]
- *   A position's slot in the query's linked cache equals its global position.
+ *   In the default (interleaved) layout a position's row in the query's linked
+ *   cache equals its global position; the links-at-end layout (KVLINK_LAYOUT_*)
+ *   stores the same positions in another order.
  *   The prefix is an optional cached pool entry (e.g. a system prompt) at
  *   positions 0..P-1.  Cached document i starts at s_i and its keys, stored rotated
  *   at local positions 0..l_i-1, are rotated by delta_i = s_i (Sec. 2.2).
@@ -90,7 +92,18 @@ typedef struct {
 
     int32_t num_sms;           /* SMs the attention work is balanced over (0 = query the
                                   current device; 152 if none is visible)                 */
+    int32_t layout;            /* physical order of the linked cache, KVLINK_LAYOUT_*     */
 } kvlink_batch_desc_t;
+
+/* Physical order of a query's rows in the linked cache.  Positions (and so RoPE and
+ * the mask) are the same in both; only the cache row of a position differs.
+ *   INTERLEAVED   row = global position: [prefix, doc_1, link_1, ..., doc_N, link_N,
+ *                 question]
+ *   LINKS_AT_END  the cached entries concatenated first, then the fresh rows in fresh
+ *                 order: [prefix, doc_1, ..., doc_N, link_1, ..., link_N, question]
+ *                 (Sec. 2.3, inference: the caches are loaded and concatenated and the
+ *                 link tokens are appended at the end of the reordered sequence).  */
+enum { KVLINK_LAYOUT_INTERLEAVED = 0, KVLINK_LAYOUT_LINKS_AT_END = 1 };
 
 /* One contiguous run of the linked sequence (Sec. 2.3 layout). */
 typedef struct {
@@ -99,7 +112,7 @@ typedef struct {
     int32_t src;     /* cached: pool entry id; fresh: first fresh row (global index) */
     int32_t len;     /* tokens                                                       */
     int64_t dst;     /* first row in the batch's contiguous linked cache
-                        (= cu_ctx[b] + pos)                                          */
+                        (= cu_ctx[b] + pos in the interleaved layout)                */
     int32_t pos;     /* global position of the first token within query b; for a
                         cached document this is also its RoPE delta (Sec. 2.2)       */
     int32_t table;   /* row of the RoPE delta table (cached documents), else -1      */
@@ -111,6 +124,19 @@ enum {
     KVLINK_SEG_LINK = 2,     /* fresh link-token rows (Sec. 2.3)             */
     KVLINK_SEG_QUESTION = 3  /* fresh question rows                          */
 };
+
+/* Where the key and value of one position of the linked sequence come from, and the
+ * linked-cache row they occupy.  The plan holds one per position, indexed by
+ * cu_ctx[b] + position. */
+typedef struct {
+    int32_t kind;    /* KVLINK_SRC_POOL or KVLINK_SRC_FRESH                              */
+    int32_t row;     /* POOL: row of the pool tensor (paged pool: physical block *
+                        pool_block_size + offset); FRESH: row of k_new / v_new            */
+    int32_t slot;    /* row of the batch's linked cache that holds this position         */
+    int32_t table;   /* RoPE delta table row when the key is re-encoded (documents), else -1 */
+} kvlink_source_t;
+
+enum { KVLINK_SRC_POOL = 0, KVLINK_SRC_FRESH = 1 };
 
 typedef struct kvlink_plan kvlink_plan_t; /* opaque */
 
@@ -130,9 +156,9 @@ typedef struct {
     int64_t attn_pairs;       /* unmasked (fresh row, key) pairs, per KV head group   */
 } kvlink_plan_info_t;
 
-/* Build the host tables of a batch: the interleaved layout of every query
- * (Sec. 2.3), the segment table, the re-encode work units and the attention work
- * items.  Validates every id and length against the pool.  Integer only; the
+/* Build the host tables of a batch: the layout of every query (Sec. 2.3), the
+ * segment table, the per-position sources, the re-encode work units and the attention
+ * work items.  Validates every id and length against the pool.  Integer only; the
  * result is deterministic.  On success *out owns host memory until
  * kvlink_plan_destroy.  Errors: EINVAL, EBOUNDS, EUNSUPPORTED. */
 int kvlink_plan_create(const kvlink_batch_desc_t* desc, kvlink_plan_t** out);
@@ -146,6 +172,11 @@ int kvlink_plan_get_info(const kvlink_plan_t* plan, kvlink_plan_info_t* info);
 int kvlink_plan_get_segments(const kvlink_plan_t* plan, kvlink_segment_t* seg, int32_t cap);
 int kvlink_plan_get_offsets(const kvlink_plan_t* plan, int64_t* cu_ctx, int32_t* cu_fresh);
 int kvlink_plan_get_fresh_positions(const kvlink_plan_t* plan, int32_t* fresh_pos, int32_t cap);
+/* src: [cap] sources, one per position of every query (ctx_rows of them), at
+ * cu_ctx[b] + position.  With a zero-copy value cache (kvlink_linked_prefill_fused with
+ * d_cache_v NULL) this is where each position's value row lives.
+ * Errors: EINVAL, ECAPACITY. */
+int kvlink_plan_get_sources(const kvlink_plan_t* plan, kvlink_source_t* src, int64_t cap);
 
 /* Copy the plan's tables to the caller's device buffer d_buf (>= device_bytes,
  * 256-byte aligned) and build the RoPE delta table there: cos and sin of
@@ -214,6 +245,26 @@ int kvlink_linked_prefill(const kvlink_plan_t* plan, const void* d_pool_k, const
                           const void* d_q, const void* d_k_new, const void* d_v_new,
                           void* d_cache_k, void* d_cache_v, void* d_out,
                           void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream);
+
+/* One layer of the linked prefill in a single attention kernel (Sec. 2.2 + Sec. 2.3):
+ * the same result as kvlink_linked_prefill, but the attention reads every key and
+ * value where it already is (pool rows for the prefix and documents, k_new / v_new
+ * for the fresh rows), rotates document keys by their delta in shared memory on the
+ * way to the tensor cores, and writes the linked cache as a side output, so the cache
+ * is written once and never read back.
+ *   - d_cache_k / d_cache_v receive the linked cache exactly as kvlink_linked_prefill
+ *     writes it (same bits), in the plan's layout.  Either may be NULL: that half is
+ *     then not written.  With d_cache_v NULL the values stay in the pool and in v_new
+ *     (zero-copy values: kvlink_plan_get_sources says where each position's value row
+ *     is), halving the cache bytes written.
+ *   - d_q, d_k_new, d_v_new: as for kvlink_suffix_attention (q and k_new rotated at
+ *     their positions).  d_workspace: >= workspace_bytes.
+ * The output equals kvlink_linked_prefill's bit for bit (same tiles, same order of
+ * operations).  Errors: EINVAL, ECAPACITY, EUNSUPPORTED, ECUDA. */
+int kvlink_linked_prefill_fused(const kvlink_plan_t* plan, const void* d_pool_k, const void* d_pool_v,
+                                const void* d_q, const void* d_k_new, const void* d_v_new,
+                                void* d_cache_k, void* d_cache_v, void* d_out,
+                                void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream);
 
 /* Allocation-free variant of kvlink_suffix_attention.  The paper has no counterpart:
  * this entry point serves callers that may not allocate device memory at all, such as

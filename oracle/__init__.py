@@ -7,6 +7,6 @@ from .kvlink_oracle import *  # noqa: F401,F403
 from .kvlink_oracle import (  # noqa: F401
     Layout, LinkedCache, bf16_bits_to_f64, f64_to_bf16_bits, rope_inv_freq, rope_rotate,
     linked_layout, training_mask, inference_mask, pool_doc_rows, reencode_concat,
-    suffix_attention, linked_prefill_query,
+    suffix_attention, linked_prefill_query, links_at_end_rows,
 )
 from .run import oracle_query_layer  # noqa: F401

@@ -170,6 +170,23 @@ def linked_layout(prefix_len: int, doc_lens: Sequence[int], n_link: int, q_len: 
                   owner=np.asarray(owner, dtype=np.int64))
 
 
+def links_at_end_rows(layout: Layout) -> np.ndarray:
+    """Cache row of every position in the physical order of Sec. 2.3 ("Inference"): the
+    precomputed caches are loaded and concatenated, and the new link tokens are appended
+    at the end of the reordered sequence (for Fig. 2: tokens 1, 2, 4, 5, 7, then links 3,
+    6, 8); the question, also run in the forward pass, follows the links.  Positions, and
+    so RoPE and the mask, are unchanged; only the row that holds a position moves.
+    Returns rows[pos] (int64 [C]).  Built by listing the positions in physical order.
+    """
+    order = [p for p in range(layout.total) if layout.kind[p] in (PREFIX, DOC)]
+    order += [p for p in range(layout.total) if layout.kind[p] == LINK]
+    order += [p for p in range(layout.total) if layout.kind[p] == QUESTION]
+    rows = np.empty(layout.total, dtype=np.int64)
+    for r, p in enumerate(order):
+        rows[p] = r
+    return rows
+
+
 # ---------------------------------------------------------------------------
 # Masks (Sec. 2.3, Fig. 2)
 # ---------------------------------------------------------------------------
@@ -279,15 +296,21 @@ def reencode_concat(pool_k: np.ndarray, pool_v: np.ndarray, pool_start, pool_len
 
 
 def suffix_attention(q: np.ndarray, cache_k: np.ndarray, cache_v: np.ndarray,
-                     fresh_pos: np.ndarray) -> np.ndarray:
-    """out[r, h] = softmax_j( q[r,h] . K[j,g] / sqrt(D), j <= pos(r) ) . V[:, g], g = h // G.
+                     fresh_pos: np.ndarray, key_pos: Optional[np.ndarray] = None) -> np.ndarray:
+    """out[r, h] = softmax_j( q[r,h] . K[j,g] / sqrt(D), pos(j) <= pos(r) ) . V[:, g], g = h // G.
 
-    All arguments float64: q [T, H_q, D], cache_k/cache_v [C, H_kv, D].
+    All arguments float64: q [T, H_q, D], cache_k/cache_v [C, H_kv, D].  key_pos[j] is
+    the position held by cache row j (default: row j holds position j, the interleaved
+    layout); the mask compares positions, so any physical order of the rows gives the
+    same result.
     """
     T, Hq, D = q.shape
     C, Hkv, _ = cache_k.shape
     G = Hq // Hkv
-    allowed = inference_mask(fresh_pos, C)
+    if key_pos is None:
+        allowed = inference_mask(fresh_pos, C)
+    else:
+        allowed = np.asarray(key_pos, dtype=np.int64)[None, :] <= np.asarray(fresh_pos, dtype=np.int64)[:, None]
     out = np.zeros((T, Hq, D), dtype=np.float64)
     for h in range(Hq):
         g = h // G

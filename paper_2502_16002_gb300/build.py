@@ -29,6 +29,7 @@ SOURCES = [
     "kvlink_reencode.cu",
     "kvlink_attention_simt.cu",
     "kvlink_attention_tc.cu",
+    "kvlink_attention_fused.cu",
     "kvlink_noalloc.cu",
 ]
 

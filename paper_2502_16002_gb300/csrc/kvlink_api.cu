@@ -27,6 +27,12 @@ int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fr
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err);
 int read_attention_status(int32_t* status);
 int clear_attention_status();
+int launch_attention_fused(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t pool_rows,
+                           int64_t ctx_rows, int head_dim, int h_q, int h_kv, const void* q, const void* pool_k,
+                           const void* pool_v, const void* k_new, const void* v_new, void* cache_k, void* cache_v,
+                           void* out, void* ws, bool from_cache, cudaStream_t stream, cudaError_t* err);
+int read_fused_status(int32_t* status);
+int clear_fused_status();
 }  // namespace kvlink
 
 using namespace kvlink;
@@ -150,6 +156,13 @@ int kvlink_plan_get_fresh_positions(const kvlink_plan_t* p, int32_t* pos, int32_
     return KVLINK_OK;
 }
 
+int kvlink_plan_get_sources(const kvlink_plan_t* p, kvlink_source_t* src, int64_t cap) {
+    if (!p || !src) return KVLINK_EINVAL;
+    if (cap < (int64_t)p->src.size()) return KVLINK_ECAPACITY;
+    std::memcpy(src, p->src.data(), p->src.size() * sizeof(kvlink_source_t));
+    return KVLINK_OK;
+}
+
 int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes, kvlink_stream_t stream) {
     if (!p || !d_buf) return KVLINK_EINVAL;
     if (!(theta > 1.0)) return KVLINK_EINVAL;
@@ -169,6 +182,10 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     put(p->off_fresh_query, p->fresh_query.data(), p->fresh_query.size() * sizeof(int32_t));
     put(p->off_items, p->items.data(), p->items.size() * sizeof(AttnItem));
     put(p->off_merges, p->merges.data(), p->merges.size() * sizeof(MergeGroup));
+    put(p->off_src, p->src.data(), p->src.size() * sizeof(kvlink_source_t));
+    put(p->off_cu_grp, p->cu_grp.data(), p->cu_grp.size() * sizeof(int32_t));
+    put(p->off_grp_src, p->grp_src.data(), p->grp_src.size() * sizeof(int32_t));
+    put(p->off_grp_slot, p->grp_slot.data(), p->grp_slot.size() * sizeof(int32_t));
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = cudaMemcpyAsync(d_buf, host.data(), p->device_bytes, cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload copy");
@@ -188,6 +205,10 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     d.fresh_query = (const int32_t*)(b + p->off_fresh_query);
     d.items = (const AttnItem*)(b + p->off_items);
     d.merges = (const MergeGroup*)(b + p->off_merges);
+    d.src = (const kvlink_source_t*)(b + p->off_src);
+    d.cu_grp = (const int32_t*)(b + p->off_cu_grp);
+    d.grp_src = (const int32_t*)(b + p->off_grp_src);
+    d.grp_slot = (const int32_t*)(b + p->off_grp_slot);
     launch_rope_table(d.seg, (int)p->seg.size(), (float4*)(b + p->off_rope), p->head_dim, theta, s);
     int rc = check_launch("rope_table_kernel");
     if (rc != KVLINK_OK) return rc;
@@ -225,9 +246,15 @@ static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k
     if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
     if (ws && !aligned16(ws)) return KVLINK_EINVAL;
     cudaError_t err = cudaSuccess;
-    const int rc = launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
-                                       p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out,
-                                       ws, s, &err);
+    int rc;
+    if (p->layout == KVLINK_LAYOUT_INTERLEAVED)  // cache row = position: K/V tiles by TMA
+        rc = launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
+                                 p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, ws, s,
+                                 &err);
+    else  // rows gathered in position order through the source table
+        rc = launch_attention_fused(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
+                                    p->pool_rows, p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, nullptr, nullptr, nullptr, nullptr, cache_k,
+                                    cache_v, out, ws, true, s, &err);
     if (rc == KVLINK_ECUDA) return cuda_fail(err, "suffix attention launch");
     return rc;
 }
@@ -281,6 +308,26 @@ int kvlink_linked_prefill(const kvlink_plan_t* p, const void* pool_k, const void
     return attention_common(p, q, cache_k, cache_v, out, ws, ws_bytes, s);
 }
 
+int kvlink_linked_prefill_fused(const kvlink_plan_t* p, const void* pool_k, const void* pool_v, const void* q,
+                                const void* k_new, const void* v_new, void* cache_k, void* cache_v, void* out,
+                                void* ws, size_t ws_bytes, kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (!pool_k || !pool_v || !q || !k_new || !v_new || !out) return KVLINK_EINVAL;
+    if (!aligned16(pool_k) || !aligned16(pool_v) || !aligned16(q) || !aligned16(k_new) || !aligned16(v_new) ||
+        !aligned16(out))
+        return KVLINK_EINVAL;
+    if ((cache_k && !aligned16(cache_k)) || (cache_v && !aligned16(cache_v))) return KVLINK_EINVAL;
+    if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
+    if (ws && !aligned16(ws)) return KVLINK_EINVAL;
+    cudaError_t err = cudaSuccess;
+    rc = launch_attention_fused(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
+                                p->pool_rows, p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, pool_k, pool_v, k_new, v_new, cache_k, cache_v, out,
+                                ws, false, (cudaStream_t)stream, &err);
+    if (rc == KVLINK_ECUDA) return cuda_fail(err, "fused linked prefill launch");
+    return rc;
+}
+
 int kvlink_rope_fresh(const kvlink_plan_t* p, void* q, void* k_new, kvlink_stream_t stream) {
     int rc = check_plan(p);
     if (rc) return rc;
@@ -292,16 +339,18 @@ int kvlink_rope_fresh(const kvlink_plan_t* p, void* q, void* k_new, kvlink_strea
 
 int kvlink_device_status(int32_t* status) {
     if (!status) return KVLINK_EINVAL;
-    int32_t a = 0, c = 0;
+    int32_t a = 0, c = 0, f = 0;
     int rc = read_attention_status(&a);
     if (rc == KVLINK_OK) rc = read_copy_status(&c);
-    *status = a != 0 ? a : c;
+    if (rc == KVLINK_OK) rc = read_fused_status(&f);
+    *status = a != 0 ? a : (c != 0 ? c : f);
     return rc;
 }
 
 int kvlink_clear_device_status(void) {
-    const int rc = clear_attention_status();
-    return rc != KVLINK_OK ? rc : clear_copy_status();
+    int rc = clear_attention_status();
+    if (rc == KVLINK_OK) rc = clear_copy_status();
+    return rc != KVLINK_OK ? rc : clear_fused_status();
 }
 
 }  // extern "C"

@@ -1,6 +1,7 @@
 // Suffix attention on the CUDA cores (Sec. 2.3, "inference"): one CTA per
 // (fresh row, KV head) computes the G query heads that share the KV head, over
-// the row's visible slots 0..pos.  Each of the four warps streams every fourth
+// the row's visible positions 0..pos (cache rows from the plan's source table, so
+// any physical layout of the cache works).  Each of the four warps streams every fourth
 // key with an online softmax; the warps' partial results are merged at the end.
 // This is the plain, unblocked form of the computation: it reads every visible
 // key once per fresh row and uses no tensor cores.  It serves head dims and
@@ -43,7 +44,7 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(DevicePlan P, const __nv
         l[h] = 0.f;
     }
     for (int j = warp; j <= pos; j += NW) {
-        const int64_t off = ((base + j) * h_kv + g) * D + lane * DPL;
+        const int64_t off = ((int64_t)P.src[base + j].slot * h_kv + g) * D + lane * DPL;  // position j's row
         float kk[DPL], vv[DPL];
 #pragma unroll
         for (int e = 0; e < DPL; ++e) {

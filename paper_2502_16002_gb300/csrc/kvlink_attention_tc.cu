@@ -32,6 +32,7 @@
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 
+#include "kvlink_attention_common.cuh"
 #include "kvlink_internal.h"
 #include "kvlink_sm100.cuh"
 
@@ -46,15 +47,6 @@ constexpr int kTmaKWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kTmaVWarp = 6;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
-constexpr int32_t kAttnStatusWaitTimeout = 0x41;
-constexpr float kRescaleThreshold = 8.0f;         // log2 units: rescale O when the max grows by > 2^8
-#ifndef KVLINK_EXP_POLY_FROM
-#define KVLINK_EXP_POLY_FROM 8                     // column pairs c with (c % 8) >= this use exp2_poly2
-#endif
-#ifndef KVLINK_PRODUCER_BACKOFF_NS
-#define KVLINK_PRODUCER_BACKOFF_NS 0               // sleep between polls of the TMA producers' waits
-#endif
 
 template <int D>
 struct TcCfg {
@@ -79,88 +71,6 @@ struct TcCfg {
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
 };
 
-// Wait for phase `parity` of `bar`; false if another role aborted or the time limit passed.
-__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (*abort_flag) return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
-            *abort_flag = 1;
-            atomicCAS(&g_attn_status, 0, kAttnStatusWaitTimeout);
-            return false;
-        }
-    }
-}
-
-// wait_bar with a short sleep between polls, for roles off the critical path
-__device__ __forceinline__ bool wait_bar_backoff(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
-    if (KVLINK_PRODUCER_BACKOFF_NS == 0) return wait_bar(bar, parity, abort_flag);
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    while (true) {
-        __nanosleep(KVLINK_PRODUCER_BACKOFF_NS);
-        if (mbar_try_wait(bar, parity)) return true;
-        if (*abort_flag) return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
-            *abort_flag = 1;
-            atomicCAS(&g_attn_status, 0, kAttnStatusWaitTimeout);
-            return false;
-        }
-    }
-}
-
-// Same, but ignores the abort flag: used to drain this thread's own async work.
-__device__ __forceinline__ void drain_bar(uint64_t* bar, uint32_t parity) {
-    const uint64_t t0 = globaltimer_ns();
-    while (!mbar_try_wait(bar, parity)) {
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
-            atomicCAS(&g_attn_status, 0, kAttnStatusWaitTimeout);
-            return;
-        }
-    }
-}
-
-// All lanes wait; the warp proceeds only if every lane saw the phase complete.
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
-    const bool ok = wait_bar(bar, parity, abort_flag);
-    return __all_sync(0xffffffffu, ok);
-}
-
-__device__ __forceinline__ uint32_t pack2_bf16(float a, float b) {
-    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-    return *reinterpret_cast<const uint32_t*>(&h);
-}
-
-// 2^x for a pair of floats on the FMA pipe: x = n + f with n = rint(x) (taken from the
-// mantissa of x + 1.5*2^23) and f in [-1/2, 1/2]; 2^f from a degree-3 minimax polynomial
-// (Remez exchange on relative error, max relative error 7.5e-5, far below the bf16
-// quantum of P); 2^n added into the exponent field.  Inputs are clamped at kExpFloor =
-// -126 so that the exponent field never wraps (p >= 2^-1/2 keeps it >= 0): anything at
-// or below the floor comes out as a non-negative value under 2^-125, i.e. nothing
-// against any unmasked term.
-__device__ __forceinline__ uint64_t exp2_poly2(uint64_t x2) {
-    constexpr float kC0 = 0.99992806f, kC1 = 0.69326097f, kC2 = 0.24261113f, kC3 = 0.05517167f;
-    constexpr float kRound = 12582912.0f;  // 1.5 * 2^23
-    constexpr float kExpFloor = -126.0f;
-    float a, b;
-    f2_unpack(x2, a, b);
-    const uint64_t x = f2_pack(fmaxf(a, kExpFloor), fmaxf(b, kExpFloor));
-    const uint64_t t = fadd2(x, f2_pack(kRound, kRound));
-    const uint64_t n = fadd2(t, f2_pack(-kRound, -kRound));
-    const uint64_t f = ffma2(n, f2_pack(-1.f, -1.f), x);
-    uint64_t p = ffma2(f, f2_pack(kC3, kC3), f2_pack(kC2, kC2));
-    p = ffma2(p, f, f2_pack(kC1, kC1));
-    p = ffma2(p, f, f2_pack(kC0, kC0));
-    float pa, pb, ta, tb;
-    f2_unpack(p, pa, pb);
-    f2_unpack(t, ta, tb);
-    const float ra = __int_as_float(__float_as_int(pa) + (int)((uint32_t)__float_as_int(ta) << 23));
-    const float rb = __int_as_float(__float_as_int(pb) + (int)((uint32_t)__float_as_int(tb) << 23));
-    return f2_pack(ra, rb);
-}
-
 // TMA producer loop for one ring (K or V): tiles j = 0..n-1 of the item's key range.
 template <int STAGES, int ATOMS>
 __device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes, const CUtensorMap* map,
@@ -169,7 +79,7 @@ __device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes
     int issued = 0;
     for (int j = 0; j < n; ++j) {
         const int st = j % STAGES;
-        if (!wait_bar_backoff(empty + st, ((j / STAGES) & 1) ^ 1, abort_flag)) break;
+        if (!wait_bar(empty + st, ((j / STAGES) & 1) ^ 1, abort_flag, &g_attn_status)) break;
         mbar_arrive_expect_tx(full + st, stage_bytes);
 #pragma unroll
         for (int a = 0; a < ATOMS; ++a)
@@ -177,7 +87,8 @@ __device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes
         issued = j + 1;
     }
     // no copy may still be in flight when the CTA leaves
-    for (int j = issued - STAGES > 0 ? issued - STAGES : 0; j < issued; ++j) drain_bar(full + j % STAGES, (j / STAGES) & 1);
+    for (int j = issued - STAGES > 0 ? issued - STAGES : 0; j < issued; ++j)
+        drain_bar(full + j % STAGES, (j / STAGES) & 1, &g_attn_status);
 }
 
 template <int D, int G>
@@ -245,7 +156,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &tm_q, a * 64, it.kv_head * G, q_row0, bar_q_full);
             produce_ring<NK, C::ATOMS>(smem + C::OFF_K, C::KV_BYTES, &tm_k, bar_k_full, bar_k_empty, n_tiles,
                                        it.kv_head, key_row0, abort_flag);
-            drain_bar(bar_q_full, 0);
+            drain_bar(bar_q_full, 0, &g_attn_status);
         }
     } else if (warp == kTmaVWarp) {
         // ------------------------------------------------------------ the V ring
@@ -258,12 +169,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
             constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
             const uint32_t sQ = smem_u32(smem + C::OFF_Q);
-            bool ok = wait_bar(bar_q_full, 0, abort_flag);
+            bool ok = wait_bar(bar_q_full, 0, abort_flag, &g_attn_status);
             // O += P_i V_i, P_i (bf16) read from its S buffer in TMEM
             auto issue_pv = [&](int i) -> bool {
                 const int b = i % NB, sv = i % NV;
-                if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag)) return false;
-                if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag)) return false;
+                if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag, &g_attn_status)) return false;
+                if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag, &g_attn_status)) return false;
                 tc_fence_after();
                 const uint32_t sV = smem_u32(smem + C::OFF_V + sv * C::KV_BYTES);
                 const uint32_t pcol = tmem + C::TMEM_S + b * kAttnBN;
@@ -277,9 +188,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             };
             for (int j = 0; ok && j < n_tiles; ++j) {
                 const int sk = j % NK, b = j % NB;
-                if (!(ok = wait_bar(bar_k_full + sk, (j / NK) & 1, abort_flag))) break;
+                if (!(ok = wait_bar(bar_k_full + sk, (j / NK) & 1, abort_flag, &g_attn_status))) break;
                 // buffer b last held P_{j-NB}: its PV must have finished reading it
-                if (j >= NB && !(ok = wait_bar(bar_o_done + b, ((j - NB) / NB) & 1, abort_flag))) break;
+                if (j >= NB && !(ok = wait_bar(bar_o_done + b, ((j - NB) / NB) & 1, abort_flag, &g_attn_status))) break;
                 tc_fence_after();
                 const uint32_t sK = smem_u32(smem + C::OFF_K + sk * C::KV_BYTES);
 #pragma unroll
@@ -294,147 +205,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             if (ok && n_tiles > 0) ok = issue_pv(n_tiles - 1);
             mma_commit(bar_drain);  // arrives once every MMA issued above has completed
-            drain_bar(bar_drain, 0);
+            drain_bar(bar_drain, 0, &g_attn_status);
         }
     } else {
         // ------------------------------------------------------------ softmax + epilogue (warps 0-3)
-        const int r = threadIdx.x;  // tile row == TMEM lane
-        const int tok = it.tok0 + r / G;
-        const bool valid = tok < it.tok1;
-        const int frow = P.cu_fresh[it.query] + tok;
-        const int pos = valid ? P.fresh_pos[frow] : 0x7fffffff;
-        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-        float m = -INFINITY, l = 0.f;
-        bool ok = true;
-        for (int j = 0; j < n_tiles; ++j) {
-            const int b = j % NB;
-            if (!(ok = warp_wait(bar_s_full + b, (j / NB) & 1, abort_flag))) break;
-            tc_fence_after();
-            uint32_t s[128];
-            const uint32_t s_col = tmem + lane_base + C::TMEM_S + b * kAttnBN;
-            tmem_ld32(s_col + 0, *reinterpret_cast<uint32_t(*)[32]>(s + 0));
-            tmem_ld32(s_col + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
-            tmem_ld32(s_col + 64, *reinterpret_cast<uint32_t(*)[32]>(s + 64));
-            tmem_ld32(s_col + 96, *reinterpret_cast<uint32_t(*)[32]>(s + 96));
-            tmem_ld_wait();
-
-            // raw row max (scale > 0 commutes with max); masked slots become -inf.  Eight
-            // independent running maxima keep the dependency chain short.
-            const int key0 = (it.kv_tile0 + j) * kAttnBN;
-            float mx8[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
-            if (key0 + kAttnBN - 1 > it.min_pos) {
-#pragma unroll
-                for (int c = 0; c < 128; ++c) {
-                    if (key0 + c > pos) s[c] = __float_as_uint(-INFINITY);
-                    mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
-                }
-            } else {
-#pragma unroll
-                for (int c = 0; c < 128; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
-            }
-            const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-            const float m_new = fmaxf(m, mx * scale_log2);
-            const bool resc = m_new > m + kRescaleThreshold;
-            float alpha = 1.f;
-            if (resc) {
-                alpha = ex2_approx(m - m_new);
-                l *= alpha;
-                m = m_new;
-            }
-            if (j > 0 && __any_sync(0xffffffffu, resc)) {
-                // O is touched only while no PV is in flight: PV_{j-1} done, PV_j not yet issued
-                if (!(ok = warp_wait(bar_o_done + (j - 1) % NB, ((j - 1) / NB) & 1, abort_flag))) break;
-                tc_fence_after();
-#pragma unroll
-                for (int c4 = 0; c4 < D / 32; ++c4) {
-                    uint32_t o[32];
-                    const uint32_t o_col = tmem + lane_base + C::TMEM_O + c4 * 32;
-                    tmem_ld32(o_col, o);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                    tmem_st32(o_col, o);
-                }
-            }
-            // p = exp2(s * scale - m) on column pairs (packed f32x2 arithmetic); three pairs
-            // in eight go to the FMA pipe (exp2_poly2), the rest to MUFU, to balance the two
-            const float mu = (m == -INFINITY) ? 0.f : m;
-            const uint64_t sc2 = f2_pack(scale_log2, scale_log2);
-            const uint64_t nmu2 = f2_pack(-mu, -mu);
-            uint64_t acc[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) acc[e] = f2_pack(0.f, 0.f);
-            uint32_t pk[64];
-#pragma unroll
-            for (int c = 0; c < 64; ++c) {
-                const uint64_t x2 = ffma2(f2_pack(__uint_as_float(s[2 * c]), __uint_as_float(s[2 * c + 1])), sc2, nmu2);
-                uint64_t p2;
-                if ((c & 7) >= KVLINK_EXP_POLY_FROM) {
-                    p2 = exp2_poly2(x2);
-                } else {
-                    float a, b;
-                    f2_unpack(x2, a, b);
-                    p2 = f2_pack(ex2_approx(a), ex2_approx(b));
-                }
-                acc[c & 3] = fadd2(acc[c & 3], p2);
-                float p0, p1;
-                f2_unpack(p2, p0, p1);
-                pk[c] = pack2_bf16(p0, p1);
-            }
-            float rs0, rs1;
-            f2_unpack(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), rs0, rs1);
-            const float rs = rs0 + rs1;
-            l += rs;
-            // P_j (bf16) over the first 64 columns of its S buffer, read there by the PV MMA
-            tmem_st32(s_col + 0, *reinterpret_cast<uint32_t(*)[32]>(pk + 0));
-            tmem_st32(s_col + 32, *reinterpret_cast<uint32_t(*)[32]>(pk + 32));
-            tmem_st_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar_p_full + b);
-        }
-        if (ok && n_tiles > 0) ok = warp_wait(bar_o_done + (n_tiles - 1) % NB, ((n_tiles - 1) / NB) & 1, abort_flag);
-        if (ok) {
-            tc_fence_after();
-            if (it.slot < 0) {
-                const float inv = 1.f / l;
-                __nv_bfloat16* orow = out + ((int64_t)frow * h_q + it.kv_head * G + (r % G)) * D;
-#pragma unroll
-                for (int c4 = 0; c4 < D / 32; ++c4) {
-                    uint32_t o[32];
-                    tmem_ld32(tmem + lane_base + C::TMEM_O + c4 * 32, o);
-                    tmem_ld_wait();
-                    if (valid) {
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            uint4 w;
-                            w.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * inv, __uint_as_float(o[8 * q + 1]) * inv);
-                            w.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv);
-                            w.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv);
-                            w.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv);
-                            *reinterpret_cast<uint4*>(orow + c4 * 32 + 8 * q) = w;
-                        }
-                    }
-                }
-            } else {
-                float* wo = ws + (int64_t)it.slot * kAttnBM * (D + 2);
-#pragma unroll
-                for (int c4 = 0; c4 < D / 32; ++c4) {
-                    uint32_t o[32];
-                    tmem_ld32(tmem + lane_base + C::TMEM_O + c4 * 32, o);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        *reinterpret_cast<uint4*>(wo + r * D + c4 * 32 + 4 * q) =
-                            make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
-                }
-                wo[kAttnBM * D + r] = m;
-                wo[kAttnBM * D + kAttnBM + r] = l;
-            }
-        }
+        softmax_role<D, G, NB>(it, P, tmem + C::TMEM_S, tmem + C::TMEM_O, n_tiles, bar_s_full, bar_p_full,
+                               bar_o_done, abort_flag, &g_attn_status, out, ws, h_q, scale_log2);
     }
 
     tc_fence_before();
@@ -486,7 +262,7 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 // bf16 tensor [d2][d1][d0] (d0 contiguous), box {b0, b1, b2}, 128-byte swizzle
-static bool make_map_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint32_t b0,
+bool make_map_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint32_t b0,
                         uint32_t b1, uint32_t b2) {
     auto fn = encode_fn();
     if (!fn) return false;
@@ -517,6 +293,17 @@ static cudaError_t launch_tc_dg(const CUtensorMap& mq, const CUtensorMap& mk, co
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (n_merges > 0) attn_merge_kernel<D><<<n_merges, 256, 0, stream>>>(P, ws, (__nv_bfloat16*)out, h_q, G);
+    return cudaGetLastError();
+}
+
+// Merge launch shared with the fused kernel: one CTA per merge group.
+cudaError_t launch_attn_merge(const DevicePlan& P, int n_merges, const float* ws, void* out, int h_q, int G,
+                              int head_dim, cudaStream_t stream) {
+    if (n_merges <= 0) return cudaSuccess;
+    if (head_dim == 128)
+        attn_merge_kernel<128><<<n_merges, 256, 0, stream>>>(P, ws, (__nv_bfloat16*)out, h_q, G);
+    else
+        attn_merge_kernel<64><<<n_merges, 256, 0, stream>>>(P, ws, (__nv_bfloat16*)out, h_q, G);
     return cudaGetLastError();
 }
 

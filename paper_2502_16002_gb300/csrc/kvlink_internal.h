@@ -44,8 +44,11 @@ struct AttnItem {
     int32_t slot;                // partial-result slot, or -1: write the output directly
     int32_t min_pos;             // smallest position of the tile's rows: keys <= min_pos
                                  // are visible to every row of the tile
+    int32_t owner;               // 1: the item's key range is written to the linked cache
+                                 // by the fused kernel (the last M-tile of each (query,
+                                 // KV head) covers every position exactly once)
 };
-static_assert(sizeof(AttnItem) == 32, "AttnItem layout");
+static_assert(sizeof(AttnItem) == 36, "AttnItem layout");
 
 // Rows of one (query, KV head, M-tile) whose KV range was split over several items.
 struct MergeGroup {
@@ -71,7 +74,16 @@ struct DevicePlan {
     const int32_t* fresh_query;  // [n_fresh]
     const AttnItem* items;       // [n_items]
     const MergeGroup* merges;    // [n_merges]
+    const kvlink_source_t* src;  // [ctx_rows] by cu_ctx[b] + position
+    // Groups of 8 positions (8m .. 8m+7 of a query), at cu_grp[b] + m: the first row of
+    // the group when its 8 rows are consecutive in one tensor (one 8-row TMA copy), else
+    // -1 (rows copied one by one; also the query's last, partial group).
+    const int32_t* cu_grp;       // [B+1]
+    const int32_t* grp_src;      // pool row, or kGrpFresh | fresh row
+    const int32_t* grp_slot;     // linked-cache row
 };
+constexpr int32_t kGrpFresh = 1 << 30;
+constexpr int32_t kGrpRowMask = kGrpFresh - 1;
 
 }  // namespace kvlink
 
@@ -81,6 +93,7 @@ struct kvlink_plan {
     int32_t pool_docs = 0, pool_block_size = 0;
     int64_t pool_rows = 0;
     int32_t num_sms = 0;
+    int32_t layout = KVLINK_LAYOUT_INTERLEAVED;
 
     // host tables
     std::vector<int64_t> pool_start;
@@ -94,6 +107,8 @@ struct kvlink_plan {
     std::vector<int32_t> cu_fresh;
     std::vector<int32_t> fresh_pos;
     std::vector<int32_t> fresh_query;
+    std::vector<kvlink_source_t> src;
+    std::vector<int32_t> cu_grp, grp_src, grp_slot;
     std::vector<kvlink::AttnItem> items;
     std::vector<kvlink::MergeGroup> merges;
     int32_t n_slots = 0;
@@ -103,7 +118,8 @@ struct kvlink_plan {
     // layout of the device buffer (byte offsets) and its total size
     size_t off_seg = 0, off_chunks = 0, off_rope = 0, off_pool_start = 0, off_pool_bt = 0,
            off_cu_ctx = 0, off_cu_fresh = 0, off_fresh_pos = 0, off_fresh_query = 0,
-           off_items = 0, off_merges = 0, device_bytes = 0;
+           off_items = 0, off_merges = 0, off_src = 0, off_cu_grp = 0, off_grp_src = 0, off_grp_slot = 0,
+           device_bytes = 0;
     size_t workspace_bytes = 0;
 
     // set by kvlink_plan_upload

@@ -43,6 +43,9 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     if (bs > 0 && d->pool_rows % bs != 0)
         return fail(why, KVLINK_EINVAL, "paged pool_rows must be a multiple of pool_block_size");
     if (num_sms <= 0) return fail(why, KVLINK_EINVAL, "num_sms must be resolved");
+    if (d->layout != KVLINK_LAYOUT_INTERLEAVED && d->layout != KVLINK_LAYOUT_LINKS_AT_END)
+        return fail(why, KVLINK_EINVAL, "unknown layout");
+    if (d->pool_rows > kGrpRowMask) return fail(why, KVLINK_EUNSUPPORTED, "pool_rows above 2^30 - 1");
 
     p->batch = d->batch;
     p->n_link = d->n_link;
@@ -53,6 +56,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     p->pool_block_size = bs;
     p->pool_rows = d->pool_rows;
     p->num_sms = num_sms;
+    p->layout = d->layout;
     p->pool_len.assign(d->pool_len, d->pool_len + d->pool_docs);
     p->pool_start.assign(d->pool_start, d->pool_start + d->pool_docs);
 
@@ -78,14 +82,19 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         }
     }
 
-    // ---- layout of every query: [prefix, doc_1, link_1, ..., doc_N, link_N, question]
+    // ---- layout of every query.  Positions: [prefix, doc_1, link_1, ..., doc_N, link_N,
+    // question].  Cache rows: the same (interleaved), or the cached entries first and the
+    // fresh rows after them in fresh order (links at the end).
     const int B = d->batch, K = d->n_link;
+    const bool at_end = d->layout == KVLINK_LAYOUT_LINKS_AT_END;
     int64_t total_docs = 0;
     for (int b = 0; b < B; ++b) {
         if (d->n_docs[b] < 0 || d->q_len[b] < 0) return fail(why, KVLINK_EINVAL, "negative count");
         total_docs += d->n_docs[b];
     }
     if (total_docs > 0 && !d->doc_ids) return fail(why, KVLINK_EINVAL, "doc_ids is null");
+    for (int64_t i = 0; i < total_docs; ++i)
+        if (d->doc_ids[i] < 0 || d->doc_ids[i] >= d->pool_docs) return fail(why, KVLINK_EBOUNDS, "doc id out of range");
 
     p->seg.clear();
     p->cu_ctx.assign(B + 1, 0);
@@ -102,23 +111,33 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         int64_t pos = 0;
         const int pre = d->prefix_doc[b];
         if (pre >= d->pool_docs || pre < -1) return fail(why, KVLINK_EBOUNDS, "prefix_doc out of range");
+        // cache rows: cached entries from row 0, fresh rows from n_cached (links at the end)
+        int64_t n_cached = pre >= 0 ? p->pool_len[pre] : 0;
+        for (int i = 0; i < d->n_docs[b]; ++i) n_cached += p->pool_len[d->doc_ids[doc_off + i]];
+        int64_t cached_row = 0, fresh_row = n_cached;
+        auto row_of = [&](bool cached, int32_t len) -> int64_t {
+            if (!at_end) return ctx + pos;
+            int64_t& r = cached ? cached_row : fresh_row;
+            const int64_t out = ctx + r;
+            r += len;
+            return out;
+        };
         if (pre >= 0 && p->pool_len[pre] > 0) {
             const int32_t P = p->pool_len[pre];
-            p->seg.push_back({b, KVLINK_SEG_PREFIX, pre, P, ctx + pos, (int32_t)pos, -1});
+            p->seg.push_back({b, KVLINK_SEG_PREFIX, pre, P, row_of(true, P), (int32_t)pos, -1});
             pos += P;
             p->cached_tokens += P;
         }
         for (int i = 0; i < d->n_docs[b]; ++i) {
             const int doc = d->doc_ids[doc_off + i];
-            if (doc < 0 || doc >= d->pool_docs) return fail(why, KVLINK_EBOUNDS, "doc id out of range");
             const int32_t L = p->pool_len[doc];
             if (L > 0) {
-                p->seg.push_back({b, KVLINK_SEG_DOC, doc, L, ctx + pos, (int32_t)pos, p->n_rope_rows++});
+                p->seg.push_back({b, KVLINK_SEG_DOC, doc, L, row_of(true, L), (int32_t)pos, p->n_rope_rows++});
                 pos += L;
                 p->cached_tokens += L;
             }
             if (K > 0) {
-                p->seg.push_back({b, KVLINK_SEG_LINK, (int32_t)fresh, K, ctx + pos, (int32_t)pos, -1});
+                p->seg.push_back({b, KVLINK_SEG_LINK, (int32_t)fresh, K, row_of(false, K), (int32_t)pos, -1});
                 for (int k = 0; k < K; ++k) {
                     p->fresh_pos.push_back((int32_t)(pos + k));
                     p->fresh_query.push_back(b);
@@ -130,7 +149,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         doc_off += d->n_docs[b];
         const int Q = d->q_len[b];
         if (Q > 0) {
-            p->seg.push_back({b, KVLINK_SEG_QUESTION, (int32_t)fresh, Q, ctx + pos, (int32_t)pos, -1});
+            p->seg.push_back({b, KVLINK_SEG_QUESTION, (int32_t)fresh, Q, row_of(false, Q), (int32_t)pos, -1});
             for (int k = 0; k < Q; ++k) {
                 p->fresh_pos.push_back((int32_t)(pos + k));
                 p->fresh_query.push_back(b);
@@ -145,6 +164,52 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     p->cu_ctx[B] = ctx;
     p->cu_fresh[B] = (int32_t)fresh;
     if (fresh > INT32_MAX / 64) return fail(why, KVLINK_EUNSUPPORTED, "too many fresh rows");
+    if (ctx > kGrpRowMask) return fail(why, KVLINK_EUNSUPPORTED, "linked cache above 2^30 - 1 rows");
+
+    // ---- per-position sources: where each position's K/V row is read from, and its cache row
+    p->src.assign((size_t)ctx, kvlink_source_t{0, 0, 0, -1});
+    for (const kvlink_segment_t& sg : p->seg) {
+        const bool cached = sg.kind == KVLINK_SEG_PREFIX || sg.kind == KVLINK_SEG_DOC;
+        for (int t = 0; t < sg.len; ++t) {
+            kvlink_source_t& e = p->src[(size_t)(p->cu_ctx[sg.query] + sg.pos + t)];
+            if (!cached) {
+                e.kind = KVLINK_SRC_FRESH;
+                e.row = sg.src + t;
+            } else {
+                e.kind = KVLINK_SRC_POOL;
+                e.row = (int32_t)(bs == 0 ? p->pool_start[sg.src] + t
+                                          : (int64_t)p->pool_block_table[p->pool_start[sg.src] + t / bs] * bs + t % bs);
+            }
+            e.slot = (int32_t)(sg.dst + t);
+            e.table = sg.table;
+        }
+    }
+
+    // ---- groups of 8 positions whose rows are consecutive in their source (and, apart,
+    // in the linked cache): each is one 8-row TMA copy in the gathering attention kernel
+    p->cu_grp.assign(B + 1, 0);
+    p->grp_src.clear();
+    p->grp_slot.clear();
+    for (int b = 0; b < B; ++b) {
+        const int64_t c0 = p->cu_ctx[b], C = p->cu_ctx[b + 1] - c0;
+        p->cu_grp[b] = (int32_t)p->grp_src.size();
+        for (int64_t m = 0; m * 8 < C; ++m) {
+            int32_t gs = -1, gc = -1;
+            if (m * 8 + 8 <= C) {
+                const kvlink_source_t* e = &p->src[(size_t)(c0 + m * 8)];
+                bool run_src = true, run_slot = true;
+                for (int i = 1; i < 8; ++i) {
+                    run_src = run_src && e[i].kind == e[0].kind && e[i].row == e[0].row + i;
+                    run_slot = run_slot && e[i].slot == e[0].slot + i;
+                }
+                if (run_src) gs = e[0].row | (e[0].kind == KVLINK_SRC_FRESH ? kGrpFresh : 0);
+                if (run_slot) gc = e[0].slot;
+            }
+            p->grp_src.push_back(gs);
+            p->grp_slot.push_back(gc);
+        }
+    }
+    p->cu_grp[B] = (int32_t)p->grp_src.size();
 
     // ---- re-encode work units: cached segments first, then fresh segments.  A unit never
     // crosses a pool block, so its source rows, like its cache rows, are contiguous.
@@ -178,7 +243,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     // runs of at most kAttnBM / G tokens; a tile's key range ends at its last token.
     const int G = d->h_q / d->h_kv;
     const int tok_per_tile = kAttnBM / G;
-    struct Tile { int32_t b, g, t0, t1, n_tiles, min_pos; };
+    struct Tile { int32_t b, g, t0, t1, n_tiles, min_pos, owner; };
     std::vector<Tile> tiles;
     int64_t work = 0;
     p->attn_pairs = 0;
@@ -191,7 +256,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
                 const int t0 = (int)((int64_t)T * mt / n_mt), t1 = (int)((int64_t)T * (mt + 1) / n_mt);
                 const int32_t kv_len = p->fresh_pos[f0 + t1 - 1] + 1;  // positions increase within a query
                 const int32_t nt = (kv_len + kAttnBN - 1) / kAttnBN;
-                tiles.push_back({b, g, t0, t1, nt, p->fresh_pos[f0 + t0]});
+                tiles.push_back({b, g, t0, t1, nt, p->fresh_pos[f0 + t0], mt == n_mt - 1 ? 1 : 0});
                 work += nt;
             }
         }
@@ -205,14 +270,14 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     for (const Tile& t : tiles) {
         const int32_t n_split = (t.n_tiles + max_tiles - 1) / max_tiles;
         if (n_split <= 1) {
-            p->items.push_back({t.b, t.g, t.t0, t.t1, 0, t.n_tiles, -1, t.min_pos});
+            p->items.push_back({t.b, t.g, t.t0, t.t1, 0, t.n_tiles, -1, t.min_pos, t.owner});
             continue;
         }
         p->merges.push_back({t.b, t.g, t.t0, t.t1, p->n_slots, n_split, 0, 0});
         for (int s = 0; s < n_split; ++s) {
             const int32_t a = (int32_t)((int64_t)t.n_tiles * s / n_split);
             const int32_t e = (int32_t)((int64_t)t.n_tiles * (s + 1) / n_split);
-            p->items.push_back({t.b, t.g, t.t0, t.t1, a, e, p->n_slots + s, t.min_pos});
+            p->items.push_back({t.b, t.g, t.t0, t.t1, a, e, p->n_slots + s, t.min_pos, t.owner});
         }
         p->n_slots += n_split;
     }
@@ -249,6 +314,10 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     p->off_fresh_query = take(p->fresh_query.size() * sizeof(int32_t));
     p->off_items = take(p->items.size() * sizeof(AttnItem));
     p->off_merges = take(p->merges.size() * sizeof(MergeGroup));
+    p->off_src = take(p->src.size() * sizeof(kvlink_source_t));
+    p->off_cu_grp = take(p->cu_grp.size() * sizeof(int32_t));
+    p->off_grp_src = take(p->grp_src.size() * sizeof(int32_t));
+    p->off_grp_slot = take(p->grp_slot.size() * sizeof(int32_t));
     p->device_bytes = off;
     p->uploaded = false;
     return KVLINK_OK;

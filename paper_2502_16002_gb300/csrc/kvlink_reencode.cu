@@ -7,17 +7,13 @@
 // through a 3-stage shared-memory ring with bulk (TMA) copies: global -> shared
 // loads, an in-place rotation of the document keys, shared -> global stores.
 //
-// Precision: a rotated component x cos a - y sin a can cancel to far below |x|,
-// where the bf16 quantum is tiny; an fp32 cos/sin (relative error 2^-24) would
-// then be off by many bf16 ulps.  The table therefore holds cos and sin as
-// unevaluated float pairs hi + lo (about 48 significant bits, split from the
-// fp64 values) and the kernel forms the products with their exact FMA rounding
-// errors, so the fp32 result carries an absolute error near 2^-47 |x| and rounds
-// to within one bf16 ulp of the correctly rounded fp64 rotation.
+// The rotation itself (double-float cos/sin, compensated products) is in
+// kvlink_rope.cuh, shared with the fused linked-prefill kernel.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "kvlink_internal.h"
+#include "kvlink_rope.cuh"
 #include "kvlink_sm100.cuh"
 
 namespace kvlink {
@@ -50,54 +46,6 @@ void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float4* d_rope,
     const int threads = 256;
     rope_table_kernel<<<(unsigned)((n + threads - 1) / threads), threads, 0, stream>>>(
         d_seg, n_seg, d_rope, half, theta, head_dim);
-}
-
-// --------------------------------------------------------------------------
-// Rotation of one (lo, hi) pair of 16-byte key chunks: 8 RoPE pairs (j, j + D/2).
-// --------------------------------------------------------------------------
-__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-
-__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
-    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);  // round to nearest even
-    return *reinterpret_cast<const uint32_t*>(&h);
-}
-
-// x c - y s and y c + x s with c = ch + cl, s = sh + sl (double-float), x, y exact.
-// The leading products are rounded explicitly (no contraction) and their exact
-// rounding errors recovered with FMA; the small terms are added once at the end.
-__device__ __forceinline__ float rot_first(float x, float y, float ch, float cl, float sh, float sl) {
-    const float p1 = __fmul_rn(x, ch), p2 = __fmul_rn(y, sh);
-    const float e1 = fmaf(x, ch, -p1), e2 = fmaf(y, sh, -p2);
-    const float t = __fsub_rn(p1, p2);
-    const float corr = (e1 - e2) + fmaf(x, cl, -(y * sl));
-    return __fadd_rn(t, corr);
-}
-
-__device__ __forceinline__ float rot_second(float x, float y, float ch, float cl, float sh, float sl) {
-    const float p1 = __fmul_rn(y, ch), p2 = __fmul_rn(x, sh);
-    const float e1 = fmaf(y, ch, -p1), e2 = fmaf(x, sh, -p2);
-    const float t = __fadd_rn(p1, p2);
-    const float corr = (e1 + e2) + fmaf(y, cl, x * sl);
-    return __fadd_rn(t, corr);
-}
-
-// lo' = lo cos - hi sin ; hi' = hi cos + lo sin, for the 8 pairs of one (lo, hi) chunk pair
-__device__ __forceinline__ void rotate8(uint4& lo, uint4& hi, const float4 (&cs)[8]) {
-    uint32_t* a = reinterpret_cast<uint32_t*>(&lo);
-    uint32_t* b = reinterpret_cast<uint32_t*>(&hi);
-#pragma unroll
-    for (int w = 0; w < 4; ++w) {
-        const float x0 = bf16lo(a[w]), x1 = bf16hi(a[w]);
-        const float y0 = bf16lo(b[w]), y1 = bf16hi(b[w]);
-        const float4 c0 = cs[2 * w], c1 = cs[2 * w + 1];
-        const float r0 = rot_first(x0, y0, c0.x, c0.y, c0.z, c0.w);
-        const float r1 = rot_first(x1, y1, c1.x, c1.y, c1.z, c1.w);
-        const float t0 = rot_second(x0, y0, c0.x, c0.y, c0.z, c0.w);
-        const float t1 = rot_second(x1, y1, c1.x, c1.y, c1.z, c1.w);
-        a[w] = pack_bf16(r0, r1);
-        b[w] = pack_bf16(t0, t1);
-    }
 }
 
 // --------------------------------------------------------------------------

@@ -26,6 +26,8 @@ KVLINK_ECUDA = -5
 KVLINK_EDEVICE = -6
 
 KVLINK_SEG_PREFIX, KVLINK_SEG_DOC, KVLINK_SEG_LINK, KVLINK_SEG_QUESTION = 0, 1, 2, 3
+KVLINK_LAYOUT_INTERLEAVED, KVLINK_LAYOUT_LINKS_AT_END = 0, 1
+KVLINK_SRC_POOL, KVLINK_SRC_FRESH = 0, 1
 
 
 class kvlink_batch_desc_t(C.Structure):
@@ -44,6 +46,7 @@ class kvlink_batch_desc_t(C.Structure):
         ("doc_ids", C.POINTER(C.c_int32)),
         ("q_len", C.POINTER(C.c_int32)),
         ("num_sms", C.c_int32),
+        ("layout", C.c_int32),
     ]
 
 
@@ -56,6 +59,7 @@ class kvlink_segment_t(C.Structure):
 
 SEGMENT_DTYPE = np.dtype([("query", "<i4"), ("kind", "<i4"), ("src", "<i4"), ("len", "<i4"),
                           ("dst", "<i8"), ("pos", "<i4"), ("table", "<i4")])
+SOURCE_DTYPE = np.dtype([("kind", "<i4"), ("row", "<i4"), ("slot", "<i4"), ("table", "<i4")])
 
 
 class kvlink_plan_info_t(C.Structure):
@@ -87,6 +91,7 @@ def _load():
         "kvlink_plan_get_segments": (C.c_int, [P, V, C.c_int32]),
         "kvlink_plan_get_offsets": (C.c_int, [P, V, V]),
         "kvlink_plan_get_fresh_positions": (C.c_int, [P, V, C.c_int32]),
+        "kvlink_plan_get_sources": (C.c_int, [P, V, C.c_int64]),
         "kvlink_plan_upload": (C.c_int, [P, C.c_double, V, C.c_size_t, V]),
         "kvlink_reencode_concat": (C.c_int, [P, V, V, V, V, V]),
         "kvlink_suffix_attention": (C.c_int, [P, V, V, V, V, V, V, V, C.c_size_t, V]),
@@ -94,6 +99,7 @@ def _load():
         "kvlink_suffix_attention_noalloc": (C.c_int, [P, V, V, V, V, V, V, V]),
         "kvlink_rope_fresh": (C.c_int, [P, V, V, V]),
         "kvlink_linked_prefill": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
+        "kvlink_linked_prefill_fused": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
     }
@@ -113,6 +119,7 @@ DECLARED = [
     "kvlink_linked_prefill",
     "kvlink_device_status", "kvlink_clear_device_status", "kvlink_strerror",
     "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc", "kvlink_rope_fresh",
+    "kvlink_plan_get_sources", "kvlink_linked_prefill_fused",
 ]
 
 # size of the static scratch used by kvlink_suffix_attention_noalloc (include/kvlink.h)
@@ -162,7 +169,7 @@ class Plan:
 
 def kvlink_plan_create(*, n_link, h_q, h_kv, head_dim, pool_len, pool_start, pool_rows,
                        prefix_doc, n_docs, doc_ids, q_len, pool_block_size=0,
-                       pool_block_table=None, num_sms=0) -> Plan:
+                       pool_block_table=None, num_sms=0, layout=KVLINK_LAYOUT_INTERLEAVED) -> Plan:
     arrs = dict(pool_len=_i32(pool_len), pool_start=_i64(pool_start), prefix_doc=_i32(prefix_doc),
                 n_docs=_i32(n_docs), doc_ids=_i32(doc_ids), q_len=_i32(q_len))
     bt = _i32(pool_block_table) if pool_block_table is not None else None
@@ -181,6 +188,7 @@ def kvlink_plan_create(*, n_link, h_q, h_kv, head_dim, pool_len, pool_start, poo
     d.doc_ids = _ptr(arrs["doc_ids"], C.c_int32) if len(arrs["doc_ids"]) else None
     d.q_len = _ptr(arrs["q_len"], C.c_int32)
     d.num_sms = int(num_sms)
+    d.layout = int(layout)
     h = C.c_void_p()
     _check(lib.kvlink_plan_create(C.byref(d), C.byref(h)), "kvlink_plan_create")
     return Plan(h)
@@ -213,6 +221,13 @@ def kvlink_plan_get_fresh_positions(plan: Plan) -> np.ndarray:
     out = np.zeros(n, np.int32)
     _check(lib.kvlink_plan_get_fresh_positions(plan.handle, out.ctypes.data, n),
            "kvlink_plan_get_fresh_positions")
+    return out
+
+
+def kvlink_plan_get_sources(plan: Plan) -> np.ndarray:
+    n = kvlink_plan_get_info(plan).ctx_rows
+    out = np.zeros(n, dtype=SOURCE_DTYPE)
+    _check(lib.kvlink_plan_get_sources(plan.handle, out.ctypes.data, n), "kvlink_plan_get_sources")
     return out
 
 
@@ -255,6 +270,13 @@ def kvlink_linked_prefill(plan: Plan, pool_k: int, pool_v: int, q: int, k_new: i
                           stream: int = 0) -> None:
     _check(lib.kvlink_linked_prefill(plan.handle, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out,
                                      workspace, workspace_bytes, stream), "kvlink_linked_prefill")
+
+
+def kvlink_linked_prefill_fused(plan: Plan, pool_k: int, pool_v: int, q: int, k_new: int, v_new: int,
+                                cache_k, cache_v, out: int, workspace, workspace_bytes: int,
+                                stream: int = 0) -> None:
+    _check(lib.kvlink_linked_prefill_fused(plan.handle, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out,
+                                           workspace, workspace_bytes, stream), "kvlink_linked_prefill_fused")
 
 
 def kvlink_device_status() -> int:

@@ -32,13 +32,13 @@ class LinkedPrefill:
 
     def __init__(self, *, n_link, h_q, h_kv, head_dim, theta, pool_len, pool_start, pool_rows,
                  prefix_doc, n_docs, doc_ids, q_len, pool_block_size=0, pool_block_table=None,
-                 num_sms=0, device="cuda", stream=None):
+                 num_sms=0, layout=K.KVLINK_LAYOUT_INTERLEAVED, device="cuda", stream=None):
         self.device = torch.device(device)
         self.plan = K.kvlink_plan_create(
             n_link=n_link, h_q=h_q, h_kv=h_kv, head_dim=head_dim, pool_len=pool_len,
             pool_start=pool_start, pool_rows=pool_rows, prefix_doc=prefix_doc, n_docs=n_docs,
             doc_ids=doc_ids, q_len=q_len, pool_block_size=pool_block_size,
-            pool_block_table=pool_block_table, num_sms=num_sms)
+            pool_block_table=pool_block_table, num_sms=num_sms, layout=layout)
         self.info = K.kvlink_plan_get_info(self.plan)
         self.theta = float(theta)
         self.plan_buf = torch.empty(max(int(self.info.device_bytes), 256), dtype=torch.uint8,
@@ -49,15 +49,19 @@ class LinkedPrefill:
                              _stream_handle(stream))
 
     @classmethod
-    def from_batch(cls, batch, device="cuda", num_sms=0, stream=None):
+    def from_batch(cls, batch, device="cuda", num_sms=0, stream=None, layout=K.KVLINK_LAYOUT_INTERLEAVED):
         """From a workloads.Batch-like object (pool metadata and per-query tables)."""
         cfg = batch.cfg
         return cls(n_link=cfg.n_link, h_q=cfg.h_q, h_kv=cfg.h_kv, head_dim=cfg.head_dim,
                    theta=cfg.theta, pool_len=batch.pool_len, pool_start=batch.pool_start,
                    pool_rows=batch.pool_rows, prefix_doc=batch.prefix_doc, n_docs=batch.n_docs,
                    doc_ids=batch.doc_ids, q_len=batch.q_len, pool_block_size=cfg.pool_block_size,
-                   pool_block_table=batch.pool_block_table, num_sms=num_sms, device=device,
-                   stream=stream)
+                   pool_block_table=batch.pool_block_table, num_sms=num_sms, layout=layout,
+                   device=device, stream=stream)
+
+    def sources(self) -> np.ndarray:
+        """Per-position sources (kvlink_source_t records) of the plan."""
+        return K.kvlink_plan_get_sources(self.plan)
 
     # shapes of the per-layer tensors
     def cache_shape(self):
@@ -98,6 +102,15 @@ class LinkedPrefill:
                                 k_new.data_ptr(), v_new.data_ptr(), cache_k.data_ptr(),
                                 cache_v.data_ptr(), out.data_ptr(), self.workspace.data_ptr(),
                                 self.workspace.numel(), _stream_handle(stream))
+
+    def linked_prefill_fused(self, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out, stream=None):
+        """One kernel: attention over pool/fresh rows, linked cache written as a side output
+        (cache_k / cache_v may be None: that half is not written)."""
+        K.kvlink_linked_prefill_fused(self.plan, pool_k.data_ptr(), pool_v.data_ptr(), q.data_ptr(),
+                                      k_new.data_ptr(), v_new.data_ptr(),
+                                      cache_k.data_ptr() if cache_k is not None else None,
+                                      cache_v.data_ptr() if cache_v is not None else None, out.data_ptr(),
+                                      self.workspace.data_ptr(), self.workspace.numel(), _stream_handle(stream))
 
     def linked_prefill_layers_from_host(self, pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new,
                                         cache_k, cache_v, out, h_out, streams=None):

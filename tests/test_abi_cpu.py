@@ -95,6 +95,49 @@ def test_segment_table_matches_oracle_layout(K, cfg_index):
     assert info.attn_pairs == int(np.sum(fpos.astype(np.int64) + 1))
 
 
+@pytest.mark.parametrize("cfg_index", [1, 2, 3, 4, 5])
+@pytest.mark.parametrize("layout", [0, 1])
+def test_sources_and_rows_match_oracle(K, cfg_index, layout):
+    """Per-position sources: the cache row of every position (interleaved: the position;
+    links at the end: the oracle's Sec. 2.3 order), and the pool or fresh row it is read
+    from, checked by fetching row ids through the oracle's pool addressing."""
+    batch = W.draw_batch(W.get_config(cfg_index))
+    cfg = batch.cfg
+    plan = _plan(K, batch, layout=layout)
+    src = K.kvlink_plan_get_sources(plan)
+    seg = K.kvlink_plan_get_segments(plan)
+    cu_ctx, cu_fresh = K.kvlink_plan_get_offsets(plan)
+    assert len(src) == cu_ctx[-1]
+    bs = cfg.pool_block_size
+    ids = np.arange(batch.pool_rows, dtype=np.int64)
+    pool_ids = ids.reshape(-1, bs) if bs else ids
+    for b in range(cfg.batch):
+        lay = _oracle_layout(batch, b)
+        rows = O.links_at_end_rows(lay) if layout else np.arange(lay.total)
+        c0 = int(cu_ctx[b])
+        mine = src[c0: c0 + lay.total]
+        assert np.array_equal(mine["slot"], c0 + rows)
+        fresh = (lay.kind == O.LINK) | (lay.kind == O.QUESTION)
+        assert np.all(mine["kind"][fresh] == K.KVLINK_SRC_FRESH)
+        assert np.array_equal(mine["row"][fresh], cu_fresh[b] + np.arange(int(fresh.sum())))
+        assert np.all(mine["kind"][~fresh] == K.KVLINK_SRC_POOL)
+        assert np.all(mine["table"][lay.kind != O.DOC] == -1)
+        def entry_rows(e):
+            return O.pool_doc_rows(pool_ids, int(e), batch.pool_start, batch.pool_len,
+                                   batch.pool_block_table, bs)
+        if lay.prefix_len:
+            assert np.array_equal(mine["row"][: lay.prefix_len], entry_rows(batch.prefix_doc[b]))
+        qseg = seg[(seg["query"] == b) & (seg["kind"] == K.KVLINK_SEG_DOC)]
+        for i, d in enumerate(batch.docs_of(b)):
+            s0, L = int(lay.doc_start[i]), int(lay.doc_len[i])
+            assert np.array_equal(mine["row"][s0: s0 + L], entry_rows(d))
+            assert np.all(mine["table"][s0: s0 + L] == qseg["table"][i])
+        # every segment is one contiguous run of cache rows starting at its dst
+        for sg in seg[seg["query"] == b]:
+            p0, n = int(sg["pos"]), int(sg["len"])
+            assert np.array_equal(rows[p0: p0 + n], int(sg["dst"]) - c0 + np.arange(n))
+
+
 def _items(K, plan):
     """Attention items and merge groups, read back from the plan's device-buffer image."""
     import paper_2502_16002_gb300.kvlink as KK
@@ -134,6 +177,9 @@ def test_invalid_arguments_are_rejected_before_launch(K):
     with pytest.raises(K.KvlinkError) as e:
         _plan(K, batch, q_len=np.asarray([0], np.int32), n_link=0)   # no fresh rows
     assert e.value.code == K.KVLINK_EINVAL
+    with pytest.raises(K.KvlinkError) as e:
+        _plan(K, batch, layout=2)
+    assert e.value.code == K.KVLINK_EINVAL
     plan = _plan(K, batch)
     info = K.kvlink_plan_get_info(plan)
     with pytest.raises(K.KvlinkError) as e:       # too small: rejected before any CUDA call
@@ -141,6 +187,9 @@ def test_invalid_arguments_are_rejected_before_launch(K):
     assert e.value.code == K.KVLINK_ECAPACITY
     with pytest.raises(K.KvlinkError) as e:       # not uploaded yet
         K.kvlink_reencode_concat(plan, 256, 256, 256, 256, 0)
+    assert e.value.code == K.KVLINK_EINVAL
+    with pytest.raises(K.KvlinkError) as e:       # not uploaded yet
+        K.kvlink_linked_prefill_fused(plan, 256, 256, 256, 256, 256, None, None, 256, 256, 1 << 20, 0)
     assert e.value.code == K.KVLINK_EINVAL
 
 
@@ -164,7 +213,7 @@ def test_attention_exp2_polynomial_accuracy():
     """The FMA-pipe 2^x used for part of the softmax: evaluate the kernel's own constants,
     clamp and range reduction in float32 and check them against 2^x in float64, including
     inputs far below the clamp (masked scores are -inf)."""
-    src = open(os.path.join(ROOT, "paper_2502_16002_gb300", "csrc", "kvlink_attention_tc.cu")).read()
+    src = open(os.path.join(ROOT, "paper_2502_16002_gb300", "csrc", "kvlink_attention_common.cuh")).read()
     c = {k: np.float32(v) for k, v in re.findall(r"\b(kC[0-3]) = ([0-9.]+)f", src)}
     assert set(c) == {"kC0", "kC1", "kC2", "kC3"}
     floor = np.float32(re.search(r"kExpFloor = (-?[0-9.]+)f", src).group(1))

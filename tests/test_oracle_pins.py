@@ -150,6 +150,58 @@ def test_figure2_inference_map_equals_training_map():
     assert np.array_equal(O.inference_mask(fp, 9), _golden_mask()[fp])
 
 
+def test_figure2_links_appended_at_end():
+    """Sec. 2.3 (inference): the caches of the documents (tokens 1, 2, 4, 5, 7) are loaded
+    and concatenated, and the new link tokens 3, 6 and 8 are appended at the end of the
+    reordered sequence; the question token 9 follows them."""
+    lay = O.linked_layout(0, [2, 2, 1], 1, 1)
+    rows = O.links_at_end_rows(lay)
+    held = np.empty(9, np.int64)
+    held[rows] = np.arange(9)
+    assert list(held + 1) == [1, 2, 4, 5, 7, 3, 6, 8, 9]
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_links_at_end_rows_invariants(seed):
+    rng = np.random.default_rng(300 + seed)
+    P = int(rng.integers(0, 5))
+    lens = rng.integers(1, 9, size=int(rng.integers(1, 6))).tolist()
+    K, Q = int(rng.choice([0, 1, 3])), int(rng.integers(1, 5))
+    lay = O.linked_layout(P, lens, K, Q)
+    rows = O.links_at_end_rows(lay)
+    assert sorted(rows.tolist()) == list(range(lay.total))          # a permutation
+    n_cached = P + sum(lens)
+    cached = (lay.kind == O.PREFIX) | (lay.kind == O.DOC)
+    assert np.array_equal(np.sort(rows[cached]), np.arange(n_cached))  # caches first
+    assert np.all(np.diff(rows[cached]) > 0) and np.all(np.diff(rows[lay.fresh_pos]) > 0)
+    assert np.array_equal(rows[lay.fresh_pos], np.arange(n_cached, lay.total))
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_links_at_end_cache_gives_the_interleaved_attention(seed):
+    """The same keys and values stored links-at-end and masked by position give the output
+    of the interleaved cache (itself pinned to the brute-force training map); masking by row
+    index instead of position would not."""
+    rng = np.random.default_rng(400 + seed)
+    lens = rng.integers(2, 7, size=3).tolist()
+    lay = O.linked_layout(int(rng.integers(0, 3)), lens, 2, 3)
+    C, Hq, Hkv, D = lay.total, 4, 2, 8
+    q = rng.standard_normal((C, Hq, D))
+    k = rng.standard_normal((C, Hkv, D))
+    v = rng.standard_normal((C, Hkv, D))
+    fp = lay.fresh_pos
+    want = O.suffix_attention(q[fp], k, v, fp)
+    rows = O.links_at_end_rows(lay)
+    k_phys, v_phys = np.empty_like(k), np.empty_like(v)
+    k_phys[rows], v_phys[rows] = k, v
+    key_pos = np.empty(C, np.int64)
+    key_pos[rows] = np.arange(C)
+    got = O.suffix_attention(q[fp], k_phys, v_phys, fp, key_pos=key_pos)
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
+    wrong = O.suffix_attention(q[fp], k_phys, v_phys, fp)
+    assert not np.allclose(wrong, want)
+
+
 def test_second_token_of_second_document_position():
     # Sec. 2.2: with no link tokens, the second token of Doc_b sits at |Doc_a| + 2 (1-based)
     for la in [1, 5, 37]:
