@@ -12,6 +12,12 @@ tokens per query).  Inputs are synthetic N(0,1) bf16, resident in HBM; every lay
 has its own pool, cache and fresh tensors, so each step streams well over L2.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config 3] [--impl ours|reference]
+                  [--path two-kernel|one-kernel|one-kernel-k-only] [--layout interleaved|links_at_end]
+
+--path selects the library entry point the step calls per layer: kvlink_linked_prefill
+(re-encode kernel, then the suffix-attention kernel; the default), or
+kvlink_linked_prefill_fused (one kernel; -k-only leaves the values in the pool).
+--layout selects the physical order of the linked cache.
 
 Prints one JSON line (rank 0).  --impl reference times the fp64 CPU oracle on the
 host cores on a bounded sample of the same workload.
@@ -41,8 +47,8 @@ UNIT = "us/query"
 # summaries under profiles/, keyed by (kernel, workload); None until captured for
 # the current kernel version.
 NCU_TRAFFIC = {
-    ("attention", 3): 193690880,   # profiles/attention_tc_llama8b_b8_zipf.md
-    ("reencode", 3): 228842496,    # profiles/reencode_llama8b_b8_zipf.md
+    ("attention", 3): 315316224,   # profiles/attention_tc_llama8b_b8_zipf.md
+    ("reencode", 3): 228032000,    # profiles/reencode_llama8b_b8_zipf.md
 }
 
 
@@ -203,7 +209,8 @@ def run_ours(args, rank, world, local_rank):
     cfg = W.get_config(args.config)
     batch = W.draw_batch(cfg, seed=rank_batch_seed(rank))   # every rank serves its own batch
     L = args.layers or cfg.layers
-    lp = LinkedPrefill.from_batch(batch, device=dev)
+    layout = {"interleaved": K.KVLINK_LAYOUT_INTERLEAVED, "links_at_end": K.KVLINK_LAYOUT_LINKS_AT_END}[args.layout]
+    lp = LinkedPrefill.from_batch(batch, device=dev, layout=layout)
     info = lp.info
     ctx, T = int(info.ctx_rows), int(info.n_fresh)
     H, Hq, D = cfg.h_kv, cfg.h_q, cfg.head_dim
@@ -223,11 +230,22 @@ def run_ours(args, rank, world, local_rank):
     ws, wsb = lp.workspace.data_ptr(), lp.workspace.numel()
     plan = lp.plan
 
-    def step():
-        for l in range(L):
+    one_kernel = args.path != "two-kernel"
+
+    def layer_call(l):
+        if one_kernel:
+            K.kvlink_linked_prefill_fused(plan, pool_k[l].data_ptr(), pool_v[l].data_ptr(), q[l].data_ptr(),
+                                          kn[l].data_ptr(), vn[l].data_ptr(), ck[l].data_ptr(),
+                                          None if args.path == "one-kernel-k-only" else cv[l].data_ptr(),
+                                          out[l].data_ptr(), ws, wsb, sh)
+        else:
             K.kvlink_linked_prefill(plan, pool_k[l].data_ptr(), pool_v[l].data_ptr(), q[l].data_ptr(),
                                     kn[l].data_ptr(), vn[l].data_ptr(), ck[l].data_ptr(), cv[l].data_ptr(),
                                     out[l].data_ptr(), ws, wsb, sh)
+
+    def step():
+        for l in range(L):
+            layer_call(l)
 
     def barrier():
         if world > 1:
@@ -267,20 +285,29 @@ def run_ours(args, rank, world, local_rank):
         for l in range(L):
             a, b_, c = ev[i]
             a.record(stream)
+            if one_kernel:      # the whole layer is one kernel: timed as the "attention" launch
+                b_.record(stream)
+                layer_call(l)
+                c.record(stream)
+                i += 1
+                continue
             K.kvlink_reencode_concat(plan, pool_k[l].data_ptr(), pool_v[l].data_ptr(), ck[l].data_ptr(),
                                      cv[l].data_ptr(), sh)
             b_.record(stream)
-            K.kvlink_suffix_attention(plan, q[l].data_ptr(), kn[l].data_ptr(), vn[l].data_ptr(),
+            # the attention kernel alone: the fresh rows are already in the cache (timed step)
+            K.kvlink_suffix_attention(plan, q[l].data_ptr(), None, None,
                                       ck[l].data_ptr(), cv[l].data_ptr(), out[l].data_ptr(), ws, wsb, sh)
             c.record(stream)
             i += 1
     torch.cuda.synchronize(dev)
     t_re = float(np.mean([a.elapsed_time(b_) for a, b_, _ in ev])) * 1e-3   # s per launch
     t_at = float(np.mean([b_.elapsed_time(c) for _, b_, c in ev])) * 1e-3
+    if one_kernel:
+        t_re = float("nan")
 
     # ---- end to end through the public API with host buffers
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not one_kernel and args.layout == "interleaved":
         h_q = torch.empty(q.shape, dtype=q.dtype, pin_memory=True)
         h_kn = torch.empty(kn.shape, dtype=kn.dtype, pin_memory=True)
         h_vn = torch.empty(vn.shape, dtype=vn.dtype, pin_memory=True)
@@ -323,18 +350,35 @@ def run_ours(args, rank, world, local_rank):
     at_tfs = cnt["attn_flops"] / t_at / 1e12
     re_frac = re_gbs / peaks["hbm_gbs"]
     at_frac = at_tfs / peaks["bf16_tflops_sustained"]
-    dominant = "attention" if t_at >= t_re else "reencode"
+    dominant = "attention" if one_kernel or t_at >= t_re else "reencode"
+    default_path = not one_kernel and args.layout == "interleaved"
     if dominant == "attention":
-        roof = {"kernel": "kvlink suffix attention", "bound": "tensor", "achieved": round(at_tfs, 2),
+        name = ("kvlink linked_prefill_fused (one kernel)" if one_kernel else
+                "kvlink suffix attention" + ("" if args.layout == "interleaved" else " (rows gathered)"))
+        roof = {"kernel": name, "bound": "tensor", "achieved": round(at_tfs, 2),
                 "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s", "frac": round(at_frac, 4),
-                "traffic": NCU_TRAFFIC.get(("attention", cfg.index)),
+                "traffic": NCU_TRAFFIC.get(("attention", cfg.index)) if default_path else None,
                 "peak_kind": f"bf16 sustained, {peaks['source']}"}
     else:
         roof = {"kernel": "kvlink reencode_concat", "bound": "hbm", "achieved": round(re_gbs, 1),
                 "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(re_frac, 4),
-                "traffic": NCU_TRAFFIC.get(("reencode", cfg.index)),
+                "traffic": NCU_TRAFFIC.get(("reencode", cfg.index)) if default_path else None,
                 "peak_kind": f"HBM copy, {peaks['source']}"}
-    n_kernels_per_layer = 2 + (1 if info.n_attn_splits > 0 else 0)
+    n_kernels_per_layer = (1 if one_kernel else 2) + (1 if info.n_attn_splits > 0 else 0)
+    attn_entry = {"us_per_launch": round(t_at * 1e6, 2), "TFLOP_per_s": round(at_tfs, 2),
+                  "frac_bf16_sustained": round(at_frac, 4),
+                  "frac_bf16_burst": round(at_tfs / peaks["bf16_tflops"], 4),
+                  "algorithmic_flops": cnt["attn_flops"],
+                  "hbm_bound_us": round(cnt["attn_bytes"] / peaks["hbm_gbs"] / 1e3, 2)}
+    if one_kernel:
+        kernels = {"linked_prefill_fused": attn_entry}
+    else:
+        kernels = {"reencode_concat": {"us_per_launch": round(t_re * 1e6, 2), "GB_per_s": round(re_gbs, 1),
+                                       "frac_hbm": round(re_frac, 4),
+                                       "frac_8TBs": round(re_gbs / 8000.0, 4),
+                                       "algorithmic_bytes": cnt["reencode_bytes"],
+                                       "bytes_per_query_doc_count": cnt["reencode_bytes_naive"]},
+                   "suffix_attention": attn_entry}
     res = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
@@ -344,22 +388,12 @@ def run_ours(args, rank, world, local_rank):
                    "head_dim": D, "docs_per_query": cfg.docs_per_query, "n_link": cfg.n_link,
                    "ctx_tokens_per_query": ctx // cfg.batch, "fresh_rows": T,
                    "parallelism": f"replicas x{world} (independent batches)",
+                   "path": args.path, "layout": args.layout,
                    "l2": "inputs larger than L2: each layer has its own pool "
                          f"({pool_k[0].numel() * 4 / 1e6:.0f} MB K+V) and cache "
                          f"({ck[0].numel() * 4 / 1e6:.0f} MB K+V)"},
         "roofline": roof,
-        "kernels": {
-            "reencode_concat": {"us_per_launch": round(t_re * 1e6, 2), "GB_per_s": round(re_gbs, 1),
-                                "frac_hbm": round(re_frac, 4),
-                                "frac_8TBs": round(re_gbs / 8000.0, 4),
-                                "algorithmic_bytes": cnt["reencode_bytes"],
-                                "bytes_per_query_doc_count": cnt["reencode_bytes_naive"]},
-            "suffix_attention": {"us_per_launch": round(t_at * 1e6, 2), "TFLOP_per_s": round(at_tfs, 2),
-                                 "frac_bf16_sustained": round(at_frac, 4),
-                                 "frac_bf16_burst": round(at_tfs / peaks["bf16_tflops"], 4),
-                                 "algorithmic_flops": cnt["attn_flops"],
-                                 "hbm_bound_us": round(cnt["attn_bytes"] / peaks["hbm_gbs"] / 1e3, 2)},
-        },
+        "kernels": kernels,
         "per_rank_us_per_query": round(us_per_query, 3),
         "gpu_launches": int(args.steps * L * n_kernels_per_layer),
         "clocks": clk.summary(),
@@ -437,6 +471,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--path", choices=["two-kernel", "one-kernel", "one-kernel-k-only"], default="two-kernel")
+    ap.add_argument("--layout", choices=["interleaved", "links_at_end"], default="interleaved")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)

@@ -266,6 +266,18 @@ int kvlink_linked_prefill_fused(const kvlink_plan_t* plan, const void* d_pool_k,
                                 void* d_cache_k, void* d_cache_v, void* d_out,
                                 void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream);
 
+/* The linked prefill of n_layers layers (the attention side of one whole prefill) in
+ * one call: for every layer l, in order, kvlink_linked_prefill(plan, pool_k[l],
+ * pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l], out[l], ...).  Each
+ * argument is a HOST array of n_layers device pointers.  One workspace serves all layers
+ * (they run in stream order).  Errors: as kvlink_linked_prefill; a failing layer stops
+ * the sequence (layers before it have been enqueued). */
+int kvlink_linked_prefill_layers(const kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
+                                 const void* const* d_pool_v, const void* const* d_q,
+                                 const void* const* d_k_new, const void* const* d_v_new, void* const* d_cache_k,
+                                 void* const* d_cache_v, void* const* d_out, void* d_workspace,
+                                 size_t workspace_bytes, kvlink_stream_t stream);
+
 /* Allocation-free variant of kvlink_suffix_attention.  The paper has no counterpart:
  * this entry point serves callers that may not allocate device memory at all, such as
  * a serving loop whose memory budget is fixed at start-up (cudaMalloc can synchronise

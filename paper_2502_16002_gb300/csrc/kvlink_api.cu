@@ -328,6 +328,22 @@ int kvlink_linked_prefill_fused(const kvlink_plan_t* p, const void* pool_k, cons
     return rc;
 }
 
+int kvlink_linked_prefill_layers(const kvlink_plan_t* p, int32_t n_layers, const void* const* pool_k,
+                                 const void* const* pool_v, const void* const* q, const void* const* k_new,
+                                 const void* const* v_new, void* const* cache_k, void* const* cache_v,
+                                 void* const* out, void* ws, size_t ws_bytes, kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (n_layers <= 0 || !pool_k || !pool_v || !q || !k_new || !v_new || !cache_k || !cache_v || !out)
+        return KVLINK_EINVAL;
+    for (int l = 0; l < n_layers; ++l) {
+        rc = kvlink_linked_prefill(p, pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l],
+                                   out[l], ws, ws_bytes, stream);
+        if (rc) return rc;
+    }
+    return KVLINK_OK;
+}
+
 int kvlink_rope_fresh(const kvlink_plan_t* p, void* q, void* k_new, kvlink_stream_t stream) {
     int rc = check_plan(p);
     if (rc) return rc;

@@ -46,50 +46,7 @@ constexpr int kSoftmaxWarps = 4;
 constexpr int kTmaKWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kTmaVWarp = 6;
-constexpr uint32_t kTmemCols = 512;
 
-template <int D>
-struct TcCfg {
-    static constexpr int ATOMS = D / 64;                 // 128-byte swizzle atoms along head_dim
-    static constexpr int NK = (D == 128) ? 3 : 5;        // K ring stages
-    static constexpr int NV = (D == 128) ? 3 : 5;        // V ring stages
-    static constexpr int NB = 3;                         // S/P buffers in TMEM
-    static constexpr uint32_t ATOM_BYTES = 128 * 128;    // [128 rows][64 bf16]
-    static constexpr uint32_t Q_BYTES = ATOMS * ATOM_BYTES;
-    static constexpr uint32_t KV_BYTES = ATOMS * ATOM_BYTES;
-    static constexpr uint32_t OFF_Q = 0;
-    static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
-    static constexpr uint32_t OFF_V = OFF_K + NK * KV_BYTES;
-    static constexpr uint32_t OFF_BAR = OFF_V + NV * KV_BYTES;
-    // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB], p_full[NB], o_done[NB], drain
-    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 3 * NB + 1;
-    static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
-    // TMEM columns: S/P buffers then the O accumulator
-    static constexpr uint32_t TMEM_S = 0;                // buffer b at b * 128
-    static constexpr uint32_t TMEM_O = NB * kAttnBN;
-    static_assert(TMEM_O + D <= kTmemCols, "TMEM budget");
-    static_assert(SMEM_BYTES <= 232448, "shared memory budget");
-};
-
-// TMA producer loop for one ring (K or V): tiles j = 0..n-1 of the item's key range.
-template <int STAGES, int ATOMS>
-__device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes, const CUtensorMap* map,
-                                             uint64_t* full, uint64_t* empty, int n, int g, int key_row0,
-                                             volatile int32_t* abort_flag) {
-    int issued = 0;
-    for (int j = 0; j < n; ++j) {
-        const int st = j % STAGES;
-        if (!wait_bar(empty + st, ((j / STAGES) & 1) ^ 1, abort_flag, &g_attn_status)) break;
-        mbar_arrive_expect_tx(full + st, stage_bytes);
-#pragma unroll
-        for (int a = 0; a < ATOMS; ++a)
-            tma_load_3d(ring + st * stage_bytes + a * (128 * 128), map, a * 64, g, key_row0 + j * kAttnBN, full + st);
-        issued = j + 1;
-    }
-    // no copy may still be in flight when the CTA leaves
-    for (int j = issued - STAGES > 0 ? issued - STAGES : 0; j < issued; ++j)
-        drain_bar(full + j % STAGES, (j / STAGES) & 1, &g_attn_status);
-}
 
 template <int D, int G>
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -155,58 +112,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             for (int a = 0; a < C::ATOMS; ++a)
                 tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &tm_q, a * 64, it.kv_head * G, q_row0, bar_q_full);
             produce_ring<NK, C::ATOMS>(smem + C::OFF_K, C::KV_BYTES, &tm_k, bar_k_full, bar_k_empty, n_tiles,
-                                       it.kv_head, key_row0, abort_flag);
+                                       it.kv_head, key_row0, abort_flag, &g_attn_status);
             drain_bar(bar_q_full, 0, &g_attn_status);
         }
     } else if (warp == kTmaVWarp) {
         // ------------------------------------------------------------ the V ring
         if (lane == 0)
             produce_ring<NV, C::ATOMS>(smem + C::OFF_V, C::KV_BYTES, &tm_v, bar_v_full, bar_v_empty, n_tiles,
-                                       it.kv_head, key_row0, abort_flag);
+                                       it.kv_head, key_row0, abort_flag, &g_attn_status);
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
-            constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
-            const uint32_t sQ = smem_u32(smem + C::OFF_Q);
-            bool ok = wait_bar(bar_q_full, 0, abort_flag, &g_attn_status);
-            // O += P_i V_i, P_i (bf16) read from its S buffer in TMEM
-            auto issue_pv = [&](int i) -> bool {
-                const int b = i % NB, sv = i % NV;
-                if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag, &g_attn_status)) return false;
-                if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag, &g_attn_status)) return false;
-                tc_fence_after();
-                const uint32_t sV = smem_u32(smem + C::OFF_V + sv * C::KV_BYTES);
-                const uint32_t pcol = tmem + C::TMEM_S + b * kAttnBN;
-#pragma unroll
-                for (int kk = 0; kk < kAttnBN / 16; ++kk)
-                    mma_bf16_ts(tmem + C::TMEM_O, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, C::ATOM_BYTES, 1024),
-                                idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
-                mma_commit(bar_o_done + b);
-                mma_commit(bar_v_empty + sv);
-                return true;
-            };
-            for (int j = 0; ok && j < n_tiles; ++j) {
-                const int sk = j % NK, b = j % NB;
-                if (!(ok = wait_bar(bar_k_full + sk, (j / NK) & 1, abort_flag, &g_attn_status))) break;
-                // buffer b last held P_{j-NB}: its PV must have finished reading it
-                if (j >= NB && !(ok = wait_bar(bar_o_done + b, ((j - NB) / NB) & 1, abort_flag, &g_attn_status))) break;
-                tc_fence_after();
-                const uint32_t sK = smem_u32(smem + C::OFF_K + sk * C::KV_BYTES);
-#pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint32_t koff = (kk >> 2) * C::ATOM_BYTES + (kk & 3) * 32;
-                    mma_bf16_ss(tmem + C::TMEM_S + b * kAttnBN, sdesc_sw128(sQ + koff, 16, 1024),
-                                sdesc_sw128(sK + koff, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
-                }
-                mma_commit(bar_s_full + b);
-                mma_commit(bar_k_empty + sk);
-                if (j >= 1) ok = issue_pv(j - 1);
-            }
-            if (ok && n_tiles > 0) ok = issue_pv(n_tiles - 1);
-            mma_commit(bar_drain);  // arrives once every MMA issued above has completed
-            drain_bar(bar_drain, 0, &g_attn_status);
-        }
+        if (lane == 0)
+            mma_role_tma<D, NK, NV, NB>(smem, C::OFF_Q, C::OFF_K, C::OFF_V, C::KV_BYTES, C::ATOM_BYTES, tmem + C::TMEM_S,
+                                       tmem + C::TMEM_O, n_tiles, bar_q_full, bar_k_full, bar_k_empty, bar_v_full,
+                                       bar_v_empty, bar_s_full, bar_p_full, bar_o_done, bar_drain, abort_flag,
+                                       &g_attn_status);
     } else {
         // ------------------------------------------------------------ softmax + epilogue (warps 0-3)
         softmax_role<D, G, NB>(it, P, tmem + C::TMEM_S, tmem + C::TMEM_O, n_tiles, bar_s_full, bar_p_full,

@@ -281,21 +281,36 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         }
         p->n_slots += n_split;
     }
-    // Launch order: the items of one (query, KV head) stay adjacent, so that CTAs running
-    // at the same time read the same K/V tiles (served from L2 after the first); groups
-    // go longest first, and so do the items inside a group.
+    // Launch order.  The items of one (query, KV head) stay adjacent, so that CTAs running
+    // at the same time read the same K/V tiles (served from L2 after the first); groups go
+    // longest first, and so do the items inside a group.  Items of at most 55% of the
+    // longest item's key tiles are held back to the end, longest first: run inside their
+    // groups they leave the long items of the last groups to start late and run alone at
+    // the end of the grid, while at the end they fill the gaps of the last wave (their K/V
+    // tiles, a prefix of their group's, are read once more).
     {
         std::vector<int64_t> group_cost((size_t)B * d->h_kv, 0);
-        for (const AttnItem& it : p->items)
-            group_cost[(size_t)it.query * d->h_kv + it.kv_head] =
-                std::max<int64_t>(group_cost[(size_t)it.query * d->h_kv + it.kv_head], it.kv_tile1 - it.kv_tile0);
+        int64_t longest = 0;
+        for (const AttnItem& it : p->items) {
+            const int64_t c = it.kv_tile1 - it.kv_tile0;
+            int64_t& g = group_cost[(size_t)it.query * d->h_kv + it.kv_head];
+            g = std::max(g, c);
+            longest = std::max(longest, c);
+        }
         std::stable_sort(p->items.begin(), p->items.end(), [&](const AttnItem& x, const AttnItem& y) {
-            const int64_t gx = group_cost[(size_t)x.query * d->h_kv + x.kv_head];
-            const int64_t gy = group_cost[(size_t)y.query * d->h_kv + y.kv_head];
-            if (gx != gy) return gx > gy;
+            const int64_t cx = x.kv_tile1 - x.kv_tile0, cy = y.kv_tile1 - y.kv_tile0;
+            const bool late_x = cx * 100 <= longest * 55, late_y = cy * 100 <= longest * 55;
+            if (late_x != late_y) return late_y;
+            if (!late_x) {
+                const int64_t gx = group_cost[(size_t)x.query * d->h_kv + x.kv_head];
+                const int64_t gy = group_cost[(size_t)y.query * d->h_kv + y.kv_head];
+                if (gx != gy) return gx > gy;
+            } else if (cx != cy) {
+                return cx > cy;
+            }
             if (x.query != y.query) return x.query < y.query;
             if (x.kv_head != y.kv_head) return x.kv_head < y.kv_head;
-            return (x.kv_tile1 - x.kv_tile0) > (y.kv_tile1 - y.kv_tile0);
+            return cx > cy;
         });
     }
     p->workspace_bytes = (size_t)p->n_slots * (size_t)kAttnBM * ((size_t)d->head_dim + 2) * sizeof(float);

@@ -100,6 +100,7 @@ def _load():
         "kvlink_rope_fresh": (C.c_int, [P, V, V, V]),
         "kvlink_linked_prefill": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_linked_prefill_fused": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
+        "kvlink_linked_prefill_layers": (C.c_int, [P, C.c_int32, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
     }
@@ -119,7 +120,7 @@ DECLARED = [
     "kvlink_linked_prefill",
     "kvlink_device_status", "kvlink_clear_device_status", "kvlink_strerror",
     "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc", "kvlink_rope_fresh",
-    "kvlink_plan_get_sources", "kvlink_linked_prefill_fused",
+    "kvlink_plan_get_sources", "kvlink_linked_prefill_fused", "kvlink_linked_prefill_layers",
 ]
 
 # size of the static scratch used by kvlink_suffix_attention_noalloc (include/kvlink.h)
@@ -277,6 +278,22 @@ def kvlink_linked_prefill_fused(plan: Plan, pool_k: int, pool_v: int, q: int, k_
                                 stream: int = 0) -> None:
     _check(lib.kvlink_linked_prefill_fused(plan.handle, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out,
                                            workspace, workspace_bytes, stream), "kvlink_linked_prefill_fused")
+
+
+def _ptr_array(ptrs):
+    arr = (C.c_void_p * len(ptrs))(*[int(x) for x in ptrs])
+    return arr
+
+
+def kvlink_linked_prefill_layers(plan: Plan, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out,
+                                 workspace, workspace_bytes: int, stream: int = 0) -> None:
+    """Every argument but the plan, workspace and stream: a sequence of per-layer device pointers."""
+    n = len(pool_k)
+    arrs = [_ptr_array(x) for x in (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out)]
+    if any(len(a) != n for a in arrs):
+        raise ValueError("every per-layer pointer list needs one entry per layer")
+    _check(lib.kvlink_linked_prefill_layers(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs], workspace,
+                                            workspace_bytes, stream), "kvlink_linked_prefill_layers")
 
 
 def kvlink_device_status() -> int:

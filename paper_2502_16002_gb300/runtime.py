@@ -112,6 +112,12 @@ class LinkedPrefill:
                                       cache_v.data_ptr() if cache_v is not None else None, out.data_ptr(),
                                       self.workspace.data_ptr(), self.workspace.numel(), _stream_handle(stream))
 
+    def linked_prefill_layers(self, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out, stream=None):
+        """All layers in one ABI call (sequences of per-layer tensors)."""
+        ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out)]
+        K.kvlink_linked_prefill_layers(self.plan, *ptrs, self.workspace.data_ptr(), self.workspace.numel(),
+                                       _stream_handle(stream))
+
     def linked_prefill_layers_from_host(self, pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new,
                                         cache_k, cache_v, out, h_out, streams=None):
         """Every layer of the linked prefill with the fresh rows in host memory.

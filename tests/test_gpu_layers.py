@@ -1,0 +1,60 @@
+"""GPU check of the all-layers call: for every layer it must give exactly (bit for bit)
+what the per-layer kvlink_linked_prefill gives; one query of the last layer is also
+checked against the fp64 oracle.
+"""
+import numpy as np
+import pytest
+
+import workloads as W
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from _gpu_common import check_query  # noqa: E402
+
+
+@pytest.fixture(scope="module")
+def RT():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2502_16002_gb300 import runtime
+
+    return runtime
+
+
+def _sentinel_cache(lp):
+    ck, cv = lp.empty_cache()
+    ck.view(torch.int16).fill_(-1)
+    cv.view(torch.int16).fill_(-1)
+    return ck, cv
+
+
+@pytest.mark.parametrize("cfg_index,n_layers", [(2, 3), (5, 2)])
+def test_all_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers):
+    from paper_2502_16002_gb300 import kvlink as K
+    dev = torch.device("cuda:0")
+    batch = W.draw_batch(W.get_config(cfg_index))
+    pk, pv, q, kn, vn, raw = [], [], [], [], [], []
+    for layer in range(n_layers):
+        a, b = W.pool_kv(batch, layer)
+        x, y, z = W.fresh_qkv(batch, layer)
+        raw.append((a, b, x, y, z))
+        for lst, arr in zip((pk, pv, q, kn, vn), (a, b, x, y, z)):
+            lst.append(RT.bf16_from_bits(arr, dev))
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    caches = [_sentinel_cache(lp) for _ in range(n_layers)]
+    outs = [torch.full_like(x, float("nan")) for x in q]
+    lp.linked_prefill_layers(pk, pv, q, kn, vn, [c[0] for c in caches], [c[1] for c in caches], outs)
+    for layer in range(n_layers):
+        ck, cv = _sentinel_cache(lp)
+        ref = torch.full_like(q[layer], float("nan"))
+        lp.linked_prefill(pk[layer], pv[layer], q[layer], kn[layer], vn[layer], ck, cv, ref)
+        torch.cuda.synchronize()
+        assert torch.equal(outs[layer].view(torch.int16), ref.view(torch.int16)), layer
+        assert torch.equal(caches[layer][0].view(torch.int16), ck.view(torch.int16)), layer
+        assert torch.equal(caches[layer][1].view(torch.int16), cv.view(torch.int16)), layer
+    assert K.kvlink_device_status() == 0
+    last = n_layers - 1
+    gk, gv = RT.bits_from_bf16(caches[last][0]), RT.bits_from_bf16(caches[last][1])
+    gout = outs[last].float().cpu().numpy().astype(np.float64)
+    check_query(batch, 0, lp, gk, gv, gout, raw[last])
