@@ -239,8 +239,10 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     }
 
     // ---- attention work items
-    // M-tiles of one (query, KV head) split the query's fresh tokens into near-equal
-    // runs of at most kAttnBM / G tokens; a tile's key range ends at its last token.
+    // M-tiles of one (query, KV head) cut the query's fresh tokens into runs of kAttnBM / G
+    // tokens counted back from the last one, the remainder going to the first run: a tile's
+    // key range ends at its last token, so the padding rows of a partial tile cost least in
+    // the tile with the shortest range (the earliest link tokens).
     const int G = d->h_q / d->h_kv;
     const int tok_per_tile = kAttnBM / G;
     struct Tile { int32_t b, g, t0, t1, n_tiles, min_pos, owner; };
@@ -253,7 +255,8 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         const int n_mt = (T + tok_per_tile - 1) / tok_per_tile;
         for (int g = 0; g < d->h_kv; ++g) {
             for (int mt = 0; mt < n_mt; ++mt) {
-                const int t0 = (int)((int64_t)T * mt / n_mt), t1 = (int)((int64_t)T * (mt + 1) / n_mt);
+                const int t0 = mt == 0 ? 0 : T - (n_mt - mt) * tok_per_tile;
+                const int t1 = T - (n_mt - 1 - mt) * tok_per_tile;
                 const int32_t kv_len = p->fresh_pos[f0 + t1 - 1] + 1;  // positions increase within a query
                 const int32_t nt = (kv_len + kAttnBN - 1) / kAttnBN;
                 tiles.push_back({b, g, t0, t1, nt, p->fresh_pos[f0 + t0], mt == n_mt - 1 ? 1 : 0});
@@ -261,9 +264,12 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
             }
         }
     }
-    // split long KV ranges so that the items spread evenly over the SMs
-    const int64_t per_sm = (work + 2 * (int64_t)num_sms - 1) / (2 * (int64_t)num_sms);
-    const int32_t max_tiles = (int32_t)std::max<int64_t>(8, per_sm);
+    // Split long KV ranges (into partials merged afterwards) only when there are fewer
+    // items than SMs: with at least one item per SM the merges and the extra prologues
+    // cost more than the balance they buy (measured on the 8B-shape workloads).
+    int32_t max_tiles = INT32_MAX;
+    if ((int64_t)tiles.size() < (int64_t)num_sms)
+        max_tiles = (int32_t)std::max<int64_t>(8, (work + num_sms - 1) / num_sms);
     p->items.clear();
     p->merges.clear();
     p->n_slots = 0;

@@ -11,6 +11,8 @@ the shared array by the first call cannot leak into the second.
 This file is collected last so that a run stopping at the first failure has
 already run every other test.
 """
+import dataclasses
+
 import numpy as np
 import pytest
 
@@ -69,8 +71,12 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(env):
 def test_noalloc_rejects_plans_larger_than_its_scratch(env):
     K, RT = env
     dev = torch.device("cuda:0")
-    batch = W.draw_batch(W.get_config(4))       # 51.8k-token context: about 21 MB of partials
-    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    # 100 documents x 512 tokens and one 32-token question, no link tokens: 8 items for 152
+    # SMs, so every KV range is split, into about 10 MB of partials
+    base = W.draw_batch(W.get_config(4))
+    batch = dataclasses.replace(base, cfg=dataclasses.replace(base.cfg, n_link=0),
+                                q_len=np.asarray([32], np.int32))
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev, num_sms=152)
     assert lp.info.workspace_bytes > K.KVLINK_NOALLOC_MAX_WORKSPACE_BYTES
     T, Hq, Hkv, D = lp.info.n_fresh, batch.cfg.h_q, batch.cfg.h_kv, batch.cfg.head_dim
     q = torch.zeros((T, Hq, D), dtype=torch.bfloat16, device=dev)
