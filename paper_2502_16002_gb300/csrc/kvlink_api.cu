@@ -28,9 +28,9 @@ int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fr
 int read_attention_status(int32_t* status);
 int clear_attention_status();
 int launch_attention_fused(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t pool_rows,
-                           int64_t ctx_rows, int head_dim, int h_q, int h_kv, const void* q, const void* pool_k,
-                           const void* pool_v, const void* k_new, const void* v_new, void* cache_k, void* cache_v,
-                           void* out, void* ws, bool from_cache, cudaStream_t stream, cudaError_t* err);
+                           int head_dim, int h_q, int h_kv, const void* q, const void* pool_k, const void* pool_v,
+                           const void* k_new, const void* v_new, void* cache_k, void* cache_v, void* out, void* ws,
+                           cudaStream_t stream, cudaError_t* err);
 int read_fused_status(int32_t* status);
 int clear_fused_status();
 }  // namespace kvlink
@@ -185,7 +185,9 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     put(p->off_src, p->src.data(), p->src.size() * sizeof(kvlink_source_t));
     put(p->off_cu_grp, p->cu_grp.data(), p->cu_grp.size() * sizeof(int32_t));
     put(p->off_grp_src, p->grp_src.data(), p->grp_src.size() * sizeof(int32_t));
-    put(p->off_grp_slot, p->grp_slot.data(), p->grp_slot.size() * sizeof(int32_t));
+    put(p->off_src_row, p->src_row.data(), p->src_row.size() * sizeof(kvlink_source_t));
+    put(p->off_fresh_vis, p->fresh_vis.data(), p->fresh_vis.size() * sizeof(int32_t));
+    put(p->off_fresh_row0, p->fresh_row0.data(), p->fresh_row0.size() * sizeof(int32_t));
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = cudaMemcpyAsync(d_buf, host.data(), p->device_bytes, cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload copy");
@@ -208,7 +210,9 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     d.src = (const kvlink_source_t*)(b + p->off_src);
     d.cu_grp = (const int32_t*)(b + p->off_cu_grp);
     d.grp_src = (const int32_t*)(b + p->off_grp_src);
-    d.grp_slot = (const int32_t*)(b + p->off_grp_slot);
+    d.src_row = (const kvlink_source_t*)(b + p->off_src_row);
+    d.fresh_vis = (const int32_t*)(b + p->off_fresh_vis);
+    d.fresh_row0 = (const int32_t*)(b + p->off_fresh_row0);
     launch_rope_table(d.seg, (int)p->seg.size(), (float4*)(b + p->off_rope), p->head_dim, theta, s);
     int rc = check_launch("rope_table_kernel");
     if (rc != KVLINK_OK) return rc;
@@ -246,15 +250,9 @@ static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k
     if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
     if (ws && !aligned16(ws)) return KVLINK_EINVAL;
     cudaError_t err = cudaSuccess;
-    int rc;
-    if (p->layout == KVLINK_LAYOUT_INTERLEAVED)  // cache row = position: K/V tiles by TMA
-        rc = launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
-                                 p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, ws, s,
-                                 &err);
-    else  // rows gathered in position order through the source table
-        rc = launch_attention_fused(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
-                                    p->pool_rows, p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, nullptr, nullptr, nullptr, nullptr, cache_k,
-                                    cache_v, out, ws, true, s, &err);
+    const int rc = launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
+                                       p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out,
+                                       ws, s, &err);
     if (rc == KVLINK_ECUDA) return cuda_fail(err, "suffix attention launch");
     return rc;
 }
@@ -322,8 +320,8 @@ int kvlink_linked_prefill_fused(const kvlink_plan_t* p, const void* pool_k, cons
     if (ws && !aligned16(ws)) return KVLINK_EINVAL;
     cudaError_t err = cudaSuccess;
     rc = launch_attention_fused(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
-                                p->pool_rows, p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, pool_k, pool_v, k_new, v_new, cache_k, cache_v, out,
-                                ws, false, (cudaStream_t)stream, &err);
+                                p->pool_rows, p->head_dim, p->h_q, p->h_kv, q, pool_k, pool_v, k_new, v_new, cache_k,
+                                cache_v, out, ws, (cudaStream_t)stream, &err);
     if (rc == KVLINK_ECUDA) return cuda_fail(err, "fused linked prefill launch");
     return rc;
 }

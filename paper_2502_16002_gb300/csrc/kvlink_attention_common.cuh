@@ -7,8 +7,7 @@
 // reads S_j from TMEM buffer j % NB, masks keys whose position is above the row's
 // position, raises the running max (rescaling O in TMEM only when the max grew by
 // more than 2^8), writes P_j = exp2(S_j c - m) as bf16 over the first half of the
-// same buffer and signals the MMA thread.  Keys are visited in position order, so
-// key index = position.  At the end it normalises O and stores the output rows, or
+// same buffer and signals the MMA thread.  Keys are visited in cache-row order.  At the end it normalises O and stores the output rows, or
 // stores the unnormalised partial (O, m, l) when the item's KV range was split.
 #pragma once
 
@@ -123,21 +122,22 @@ __device__ __forceinline__ uint64_t exp2_poly2(uint64_t x2) {
     return f2_pack(ra, rb);
 }
 
-// TMA producer loop for one ring (K or V) of a materialised linked cache: key tiles
-// j = 0..n-1 of the item's range, rows key_row0 + 128 j .. of KV head g.
+// TMA producer loop for one ring (K or V) of a materialised linked cache: the n key tiles
+// of the item's list, rows ctx0 + 128 * item_tile(it, kv_tile0 + j) .. of its KV head.
 template <int STAGES, int ATOMS>
 __device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes, const CUtensorMap* map,
-                                             uint64_t* full, uint64_t* empty, int n, int g, int key_row0,
-                                             volatile int32_t* abort_flag, int32_t* status) {
+                                             uint64_t* full, uint64_t* empty, int n, const AttnItem& it,
+                                             int ctx0, volatile int32_t* abort_flag, int32_t* status) {
     using namespace sm100;
     int issued = 0;
     for (int j = 0; j < n; ++j) {
         const int st = j % STAGES;
         if (!wait_bar(empty + st, ((j / STAGES) & 1) ^ 1, abort_flag, status)) break;
+        const int row = ctx0 + item_tile(it, it.kv_tile0 + j) * kAttnBN;
         mbar_arrive_expect_tx(full + st, stage_bytes);
 #pragma unroll
         for (int a = 0; a < ATOMS; ++a)
-            tma_load_3d(ring + st * stage_bytes + a * (128 * 128), map, a * 64, g, key_row0 + j * kAttnBN, full + st);
+            tma_load_3d(ring + st * stage_bytes + a * (128 * 128), map, a * 64, it.kv_head, row, full + st);
         issued = j + 1;
     }
     // no copy may still be in flight when the CTA leaves
@@ -214,7 +214,10 @@ __device__ __forceinline__ void softmax_role(const AttnItem& it, const DevicePla
     const int tok = it.tok0 + r / G;
     const bool valid = tok < it.tok1;
     const int frow = P.cu_fresh[it.query] + tok;
-    const int pos = valid ? P.fresh_pos[frow] : 0x7fffffff;
+    // visible cache rows (query-relative): [0, vis_a) and [F, F + vis_b)
+    const int vis_a = valid ? P.fresh_vis[frow] : 0x7fffffff;
+    const int F = P.fresh_row0[it.query];
+    const uint32_t vis_b = valid ? (uint32_t)(tok + 1) : 0u;
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
     float m = -INFINITY, l = 0.f;
     bool ok = true;
@@ -231,16 +234,29 @@ __device__ __forceinline__ void softmax_role(const AttnItem& it, const DevicePla
         tmem_ld_wait();
 
         // raw row max (scale > 0 commutes with max); masked keys become -inf.  Eight
-        // independent running maxima keep the dependency chain short.
-        const int key0 = (it.kv_tile0 + j) * kAttnBN;
+        // independent running maxima keep the dependency chain short.  A tile lies in one
+        // run of rows (cached rows, or the fresh rows at the end), where the visible keys
+        // are those below one limit; only a tile holding the end of the cached rows and the
+        // start of the fresh rows needs both comparisons.
+        const int key0 = item_tile(it, it.kv_tile0 + j) * kAttnBN;
         float mx8[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
-        if (key0 + kAttnBN - 1 > it.min_pos) {
+        if (key0 + kAttnBN > it.min_vis) {  // some row of the tile may not see every key
+            if (key0 + kAttnBN <= F || key0 >= F) {
+                const int lim = key0 >= F ? F + (int)vis_b : vis_a;
 #pragma unroll
-            for (int c = 0; c < 128; ++c) {
-                if (key0 + c > pos) s[c] = __float_as_uint(-INFINITY);
-                mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
+                for (int c = 0; c < 128; ++c) {
+                    if (key0 + c >= lim) s[c] = __float_as_uint(-INFINITY);
+                    mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
+                }
+            } else {
+#pragma unroll
+                for (int c = 0; c < 128; ++c) {
+                    const int kr = key0 + c;
+                    if (!(kr < vis_a || (uint32_t)(kr - F) < vis_b)) s[c] = __float_as_uint(-INFINITY);
+                    mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
+                }
             }
         } else {
 #pragma unroll

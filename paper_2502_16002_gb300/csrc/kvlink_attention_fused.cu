@@ -12,12 +12,10 @@
 // (kvlink_attention_common.cuh, same tiles, same MMA order), so the cache and the
 // output equal the two-kernel path's bit for bit.
 //
-// Keys are visited in position order: key tile j of an item holds positions
-// [128 j, 128 j + 128) of its query, gathered row by row through the plan's source
-// table.  The mask therefore compares positions whatever the physical order of the
-// cache (interleaved, or links at the end), and the same kernel also runs the suffix
-// attention over a cache in the links-at-end order (from_cache: rows read from the
-// cache through the table, nothing written).
+// Keys are visited in linked-cache row order, as in the suffix-attention kernel: key
+// tile t of an item stands for cache rows [128 t, 128 t + 128) of its query, whose
+// sources come from the plan's per-row source table, and the same per-row visibility
+// mask applies, in either physical layout (interleaved, or links at the end).
 //
 // Warp roles (384 threads = 3 warpgroups, one CTA per SM, 512 TMEM columns):
 //   warps 0-3  softmax + epilogue, thread r owns tile row r = TMEM lane r
@@ -100,8 +98,8 @@ struct FusedCfg {
     static_assert(RG * RPT == kAttnBN, "gather split");
 };
 
-// Source tensors of the 8-row TMA copies: A = pool (or the linked cache when reading
-// from it), F = fresh rows; [rows][h_kv][D] bf16, box {64, 1, 8}.
+// Source tensors of the 8-row TMA copies: A = pool, F = fresh rows; [rows][h_kv][D]
+// bf16, box {64, 1, 8}.
 struct FusedMaps {
     CUtensorMap q, ak, av, fk, fv;
 };
@@ -111,13 +109,12 @@ struct FusedArgs {
     const __nv_bfloat16* pool_v;
     const __nv_bfloat16* k_new;
     const __nv_bfloat16* v_new;
-    __nv_bfloat16* cache_k;  // side output of owner items (NULL: not written); the source when from_cache
+    __nv_bfloat16* cache_k;  // side output of owner items (NULL: not written)
     __nv_bfloat16* cache_v;
     __nv_bfloat16* out;
     float* ws;
     int h_q, h_kv;
     float scale_log2;
-    int from_cache;
 };
 
 // Byte offset of 16-byte chunk `ch` (dims 8ch..8ch+7) of tile row r in a 128-byte
@@ -134,17 +131,17 @@ __device__ __forceinline__ kvlink_source_t load_source(const kvlink_source_t* sr
 // TMA role (one thread): the 8-row group copies of every key tile of the item.
 template <int D>
 __device__ __forceinline__ void tma_role(const AttnItem& it, const DevicePlan& P, const FusedMaps& M,
-                                         bool from_cache, uint8_t* smem, uint64_t* raw_full, uint64_t* kv_empty,
-                                         int n_tiles, volatile int32_t* abort_flag) {
+                                         uint8_t* smem, uint64_t* raw_full, uint64_t* kv_empty, int n_tiles,
+                                         volatile int32_t* abort_flag) {
     using C = FusedCfg<D>;
-    const int32_t* grp = from_cache ? P.grp_slot : P.grp_src;
+    const int32_t* grp = P.grp_src;
     const int gbase = P.cu_grp[it.query];
     const int n_grp = P.cu_grp[it.query + 1] - gbase;
     int issued = 0;
     for (int j = 0; j < n_tiles; ++j) {
         const int st = j % C::NS;
         if (!wait_bar(kv_empty + st, ((j / C::NS) & 1) ^ 1, abort_flag, &g_fused_status)) break;
-        const int m0 = (it.kv_tile0 + j) * (kAttnBN / 8);
+        const int m0 = item_tile(it, it.kv_tile0 + j) * (kAttnBN / 8);
         int32_t gw[kAttnBN / 8];
         uint32_t n = 0;
 #pragma unroll
@@ -185,10 +182,10 @@ __device__ __forceinline__ void gather_role(const AttnItem& it, const DevicePlan
     const int n_pos = (int)(P.cu_ctx[it.query + 1] - ctx0);
     const int64_t row_elems = (int64_t)A.h_kv * D;
     const int64_t col0 = (int64_t)it.kv_head * D + 8 * c;  // lo chunk of this thread within a row
-    const bool own_k = it.owner && !A.from_cache && A.cache_k != nullptr;
-    const bool own_v = it.owner && !A.from_cache && A.cache_v != nullptr;
+    const bool own_k = it.owner && A.cache_k != nullptr;
+    const bool own_v = it.owner && A.cache_v != nullptr;
     const uint32_t kv_base = smem_u32(smem + C::OFF_KV);
-    const int32_t* grp = A.from_cache ? P.grp_slot : P.grp_src;
+    const int32_t* grp = P.grp_src;
     const int gbase = P.cu_grp[it.query];
 
     // rows of key tile j outside the TMA groups: copied row by row, or zero-filled past
@@ -198,7 +195,7 @@ __device__ __forceinline__ void gather_role(const AttnItem& it, const DevicePlan
         if (!warp_wait(kv_empty + st, ((j / C::NS) & 1) ^ 1, abort_flag, &g_fused_status)) return false;
         const uint32_t sk = kv_base + st * C::STAGE_BYTES, sv = sk + C::HALF_BYTES;
         uint8_t* gk = smem + C::OFF_KV + st * C::STAGE_BYTES;
-        const int key0 = (it.kv_tile0 + j) * kAttnBN;
+        const int key0 = item_tile(it, it.kv_tile0 + j) * kAttnBN;
         // all of the tile's records first: one load latency, not one per row (the copies
         // below are compiler barriers for memory accesses)
         bool by_row[C::RPT];
@@ -211,7 +208,7 @@ __device__ __forceinline__ void gather_role(const AttnItem& it, const DevicePlan
 #pragma unroll
         for (int k = 0; k < C::RPT; ++k) {
             const int pos = key0 + g + C::RG * k;
-            es[k] = by_row[k] ? load_source(P.src, ctx0 + pos) : kvlink_source_t{0, 0, 0, -1};
+            es[k] = by_row[k] ? load_source(P.src_row, ctx0 + pos) : kvlink_source_t{0, 0, 0, -1};
         }
 #pragma unroll
         for (int k = 0; k < C::RPT; ++k) {
@@ -221,9 +218,7 @@ __device__ __forceinline__ void gather_role(const AttnItem& it, const DevicePlan
                 const kvlink_source_t& e = es[k];
                 const __nv_bfloat16 *kb, *vb;
                 int64_t row;
-                if (A.from_cache) {
-                    kb = A.cache_k, vb = A.cache_v, row = e.slot;
-                } else if (e.kind == KVLINK_SRC_FRESH) {
+                if (e.kind == KVLINK_SRC_FRESH) {
                     kb = A.k_new, vb = A.v_new, row = e.row;
                 } else {
                     kb = A.pool_k, vb = A.pool_v, row = e.row;
@@ -254,19 +249,19 @@ __device__ __forceinline__ void gather_role(const AttnItem& it, const DevicePlan
         if (!warp_wait(raw_full + st, (j / C::NS) & 1, abort_flag, &g_fused_status)) return false;
         uint8_t* sk = smem + C::OFF_KV + st * C::STAGE_BYTES;
         uint8_t* sv = sk + C::HALF_BYTES;
-        const int key0 = (it.kv_tile0 + j) * kAttnBN;
+        const int key0 = item_tile(it, it.kv_tile0 + j) * kAttnBN;
         kvlink_source_t es[C::RPT];
 #pragma unroll
         for (int k = 0; k < C::RPT; ++k) {
             const int pos = key0 + g + C::RG * k;
-            es[k] = pos < n_pos ? load_source(P.src, ctx0 + pos) : kvlink_source_t{0, 0, 0, -1};
+            es[k] = pos < n_pos ? load_source(P.src_row, ctx0 + pos) : kvlink_source_t{0, 0, 0, -1};
         }
 #pragma unroll
         for (int k = 0; k < C::RPT; ++k) {
             const int r = g + C::RG * k, pos = key0 + r;
             if (pos >= n_pos) continue;
             const kvlink_source_t& e = es[k];
-            const bool rot = !A.from_cache && e.table >= 0;
+            const bool rot = e.table >= 0;
             const uint32_t o_lo = swz(c, r), o_hi = swz(c + C::CP, r);
             if (rot || own_k) {
                 uint4 a = *reinterpret_cast<const uint4*>(sk + o_lo);
@@ -419,7 +414,7 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
             mma_commit(bar_drain);  // arrives once every MMA issued above has completed
             drain_bar(bar_drain, 0, &g_fused_status);
         } else if (warp == kFusedTmaWarp && lane == 0) {
-            tma_role<D>(it, P, M, A.from_cache != 0, smem, bar_raw_full, bar_kv_empty, n_tiles, abort_flag);
+            tma_role<D>(it, P, M, smem, bar_raw_full, bar_kv_empty, n_tiles, abort_flag);
         }
     } else {
         setmaxnreg_inc<kSoftmaxRegs>();
@@ -450,32 +445,24 @@ static cudaError_t launch_fused_dg(const FusedMaps& M, const DevicePlan& P, cons
     return cudaGetLastError();
 }
 
-// Fused linked prefill (from_cache = false: sources are the pool and the fresh rows,
-// owner items write cache_k / cache_v where non-NULL), or the suffix attention over a
-// materialised cache in any layout (from_cache = true).  Returns 0, KVLINK_ECUDA or
-// KVLINK_EUNSUPPORTED.
+// Fused linked prefill: sources are the pool and the fresh rows; owner items write
+// cache_k / cache_v where non-NULL.  Returns 0, KVLINK_ECUDA or KVLINK_EUNSUPPORTED.
 int launch_attention_fused(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t pool_rows,
-                           int64_t ctx_rows, int head_dim, int h_q, int h_kv, const void* q, const void* pool_k,
-                           const void* pool_v, const void* k_new, const void* v_new, void* cache_k, void* cache_v,
-                           void* out, void* ws, bool from_cache, cudaStream_t stream, cudaError_t* err) {
+                           int head_dim, int h_q, int h_kv, const void* q, const void* pool_k, const void* pool_v,
+                           const void* k_new, const void* v_new, void* cache_k, void* cache_v, void* out, void* ws,
+                           cudaStream_t stream, cudaError_t* err) {
     const int G = h_q / h_kv;
     FusedMaps M;
     const uint64_t D = (uint64_t)head_dim, H = (uint64_t)h_kv;
-    const void* a_k = from_cache ? cache_k : pool_k;
-    const void* a_v = from_cache ? cache_v : pool_v;
-    const uint64_t a_rows = from_cache ? (uint64_t)ctx_rows : (uint64_t)pool_rows;
-    // from the linked cache no fresh-row copies are issued: the F maps then point at it too
-    const void* f_k = from_cache ? cache_k : k_new;
-    const void* f_v = from_cache ? cache_v : v_new;
-    const uint64_t f_rows = from_cache ? (uint64_t)ctx_rows : (uint64_t)n_fresh;
     if (!make_map_3d(&M.q, q, D, (uint64_t)h_q, (uint64_t)n_fresh, 64, (uint32_t)G, (uint32_t)(kAttnBM / G)) ||
-        !make_map_3d(&M.ak, a_k, D, H, a_rows, 64, 1, 8) || !make_map_3d(&M.av, a_v, D, H, a_rows, 64, 1, 8) ||
-        !make_map_3d(&M.fk, f_k, D, H, f_rows, 64, 1, 8) || !make_map_3d(&M.fv, f_v, D, H, f_rows, 64, 1, 8))
+        !make_map_3d(&M.ak, pool_k, D, H, (uint64_t)pool_rows, 64, 1, 8) ||
+        !make_map_3d(&M.av, pool_v, D, H, (uint64_t)pool_rows, 64, 1, 8) ||
+        !make_map_3d(&M.fk, k_new, D, H, (uint64_t)n_fresh, 64, 1, 8) ||
+        !make_map_3d(&M.fv, v_new, D, H, (uint64_t)n_fresh, 64, 1, 8))
         return KVLINK_EUNSUPPORTED;
     using bf = __nv_bfloat16;
     FusedArgs A{(const bf*)pool_k, (const bf*)pool_v, (const bf*)k_new, (const bf*)v_new, (bf*)cache_k,
-                (bf*)cache_v, (bf*)out, (float*)ws, h_q, h_kv, 1.4426950408889634f / sqrtf((float)head_dim),
-                from_cache ? 1 : 0};
+                (bf*)cache_v, (bf*)out, (float*)ws, h_q, h_kv, 1.4426950408889634f / sqrtf((float)head_dim)};
     cudaError_t e = cudaErrorInvalidValue;
 #define KVLINK_FUSED_CASE(DD, GG) \
     if (head_dim == DD && G == GG) e = launch_fused_dg<DD, GG>(M, P, A, n_items, stream);

@@ -2,8 +2,9 @@
 //
 // Work item = one M-tile of up to 128 rows (up to 128/G fresh tokens x the G
 // query heads that share one KV head) of one query, over a range of 128-key
-// tiles of that query's linked cache.  Rows are (token, head) pairs, so the G
-// heads of a GQA group share every K/V tile load.
+// tiles of that query's linked cache (cache-row order; in the links-at-end layout the
+// cached rows and the fresh rows at the end form two runs).  Rows are (token, head)
+// pairs, so the G heads of a GQA group share every K/V tile load.
 //
 // Warp roles (224 threads, one CTA per SM, 512 TMEM columns):
 //   warps 0-3  softmax + epilogue; thread r owns row r = TMEM lane r
@@ -18,9 +19,9 @@
 // S_j is issued only after PV_{j-3} has finished reading the buffer, so up to
 // three tiles are in flight and the softmax never waits on a PV except to
 // rescale O.  The running max m is raised only when it grows by more than 2^8,
-// so that rescale is rare.  The mask keeps key slot j for a row at global
-// position p iff j <= p, and is evaluated only on tiles that reach past the
-// tile's smallest row position.  Items whose KV range was split write
+// so that rescale is rare.  The mask keeps the cache rows holding positions up to
+// the row's own (a threshold pair per row, see softmax_role) and is evaluated only on
+// tiles that reach past the rows every row of the tile sees.  Items whose KV range was split write
 // unnormalised partials (O, m, l) to the workspace; attn_merge_kernel combines them.
 //
 // Every mbarrier wait is bounded in time.  On expiry the kernel records
@@ -99,7 +100,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
     const bool skip = *abort_flag != 0;  // written before the barrier: uniform across the CTA
-    const int key_row0 = (int)P.cu_ctx[it.query] + it.kv_tile0 * kAttnBN;
+    const int ctx0 = (int)P.cu_ctx[it.query];
 
     if (skip) {
         // nothing issued: fall through to the teardown
@@ -111,15 +112,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
             for (int a = 0; a < C::ATOMS; ++a)
                 tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &tm_q, a * 64, it.kv_head * G, q_row0, bar_q_full);
-            produce_ring<NK, C::ATOMS>(smem + C::OFF_K, C::KV_BYTES, &tm_k, bar_k_full, bar_k_empty, n_tiles,
-                                       it.kv_head, key_row0, abort_flag, &g_attn_status);
+            produce_ring<NK, C::ATOMS>(smem + C::OFF_K, C::KV_BYTES, &tm_k, bar_k_full, bar_k_empty, n_tiles, it,
+                                       ctx0, abort_flag, &g_attn_status);
             drain_bar(bar_q_full, 0, &g_attn_status);
         }
     } else if (warp == kTmaVWarp) {
         // ------------------------------------------------------------ the V ring
         if (lane == 0)
-            produce_ring<NV, C::ATOMS>(smem + C::OFF_V, C::KV_BYTES, &tm_v, bar_v_full, bar_v_empty, n_tiles,
-                                       it.kv_head, key_row0, abort_flag, &g_attn_status);
+            produce_ring<NV, C::ATOMS>(smem + C::OFF_V, C::KV_BYTES, &tm_v, bar_v_full, bar_v_empty, n_tiles, it,
+                                       ctx0, abort_flag, &g_attn_status);
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0)

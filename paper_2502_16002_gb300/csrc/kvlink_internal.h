@@ -2,6 +2,7 @@
 #pragma once
 
 #include <stdint.h>
+#include <cuda_runtime.h>
 #include <vector_types.h>
 
 #include <string>
@@ -35,20 +36,33 @@ struct CopyChunk {
 static_assert(sizeof(CopyChunk) == 32, "CopyChunk layout");
 
 // One attention work item: an M-tile of (token, head) rows of one query and KV head,
-// over KV tiles [kv_tile0, kv_tile1).
+// over a range of the query's key tiles (kAttnBN cache rows each, in cache-row order).
+// The tiles an M-tile needs form at most two runs: rows [0, a) holding the cached
+// entries (every layout), and, in the links-at-end layout, the fresh rows at the end.
+// Tile v of that list is v itself for v < a_tiles, else b_tile0 + (v - a_tiles); the
+// item covers list entries [kv_tile0, kv_tile1).
 struct AttnItem {
     int32_t query;
     int32_t kv_head;
     int32_t tok0, tok1;          // fresh tokens [tok0, tok1) of the query (query-relative)
-    int32_t kv_tile0, kv_tile1;  // key tiles of kAttnBN keys
+    int32_t kv_tile0, kv_tile1;  // entries of the tile list
     int32_t slot;                // partial-result slot, or -1: write the output directly
-    int32_t min_pos;             // smallest position of the tile's rows: keys <= min_pos
-                                 // are visible to every row of the tile
+    int32_t min_vis;             // cache rows below min_vis are visible to every row
     int32_t owner;               // 1: the item's key range is written to the linked cache
-                                 // by the fused kernel (the last M-tile of each (query,
-                                 // KV head) covers every position exactly once)
+                                 // by the one-kernel path (the last M-tile of each (query,
+                                 // KV head) covers every cache row exactly once)
+    int32_t a_tiles;             // tiles of the first run (rows from 0)
+    int32_t b_tile0;             // first tile of the second run
 };
-static_assert(sizeof(AttnItem) == 36, "AttnItem layout");
+static_assert(sizeof(AttnItem) == 44, "AttnItem layout");
+
+// Key tile (kAttnBN rows from the query's first cache row) of entry v of an item's list.
+__host__ __device__ inline int32_t item_tile(const AttnItem& it, int32_t v) {
+    return v < it.a_tiles ? v : it.b_tile0 + (v - it.a_tiles);
+}
+
+// fresh_row0 of a query without a fresh region at the end (interleaved layout)
+constexpr int32_t kNoFreshRegion = 0x3fffffff;
 
 // Rows of one (query, KV head, M-tile) whose KV range was split over several items.
 struct MergeGroup {
@@ -75,12 +89,17 @@ struct DevicePlan {
     const AttnItem* items;       // [n_items]
     const MergeGroup* merges;    // [n_merges]
     const kvlink_source_t* src;  // [ctx_rows] by cu_ctx[b] + position
-    // Groups of 8 positions (8m .. 8m+7 of a query), at cu_grp[b] + m: the first row of
-    // the group when its 8 rows are consecutive in one tensor (one 8-row TMA copy), else
+    const kvlink_source_t* src_row;  // [ctx_rows] the same records by linked-cache row
+    // Visibility of fresh row r (query b): cache rows [0, fresh_vis[r]) and, when the query
+    // keeps its fresh rows at the end, [fresh_row0[b], fresh_row0[b] + f + 1) with f the row's
+    // index among the query's fresh rows (interleaved: fresh_row0 = kNoFreshRegion).
+    const int32_t* fresh_vis;    // [n_fresh]
+    const int32_t* fresh_row0;   // [B], query-relative
+    // Groups of 8 cache rows (8m .. 8m+7 of a query), at cu_grp[b] + m: the first source
+    // row when the group's 8 rows are consecutive in one tensor (one 8-row TMA copy), else
     // -1 (rows copied one by one; also the query's last, partial group).
     const int32_t* cu_grp;       // [B+1]
     const int32_t* grp_src;      // pool row, or kGrpFresh | fresh row
-    const int32_t* grp_slot;     // linked-cache row
 };
 constexpr int32_t kGrpFresh = 1 << 30;
 constexpr int32_t kGrpRowMask = kGrpFresh - 1;
@@ -107,8 +126,9 @@ struct kvlink_plan {
     std::vector<int32_t> cu_fresh;
     std::vector<int32_t> fresh_pos;
     std::vector<int32_t> fresh_query;
-    std::vector<kvlink_source_t> src;
-    std::vector<int32_t> cu_grp, grp_src, grp_slot;
+    std::vector<kvlink_source_t> src, src_row;
+    std::vector<int32_t> fresh_vis, fresh_row0;
+    std::vector<int32_t> cu_grp, grp_src;
     std::vector<kvlink::AttnItem> items;
     std::vector<kvlink::MergeGroup> merges;
     int32_t n_slots = 0;
@@ -118,7 +138,8 @@ struct kvlink_plan {
     // layout of the device buffer (byte offsets) and its total size
     size_t off_seg = 0, off_chunks = 0, off_rope = 0, off_pool_start = 0, off_pool_bt = 0,
            off_cu_ctx = 0, off_cu_fresh = 0, off_fresh_pos = 0, off_fresh_query = 0,
-           off_items = 0, off_merges = 0, off_src = 0, off_cu_grp = 0, off_grp_src = 0, off_grp_slot = 0,
+           off_items = 0, off_merges = 0, off_src = 0, off_cu_grp = 0, off_grp_src = 0, off_src_row = 0,
+           off_fresh_vis = 0, off_fresh_row0 = 0,
            device_bytes = 0;
     size_t workspace_bytes = 0;
 

@@ -29,10 +29,6 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
 int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t ctx_rows,
                         int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err);
-int launch_attention_fused(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t pool_rows,
-                           int64_t ctx_rows, int head_dim, int h_q, int h_kv, const void* q, const void* pool_k,
-                           const void* pool_v, const void* k_new, const void* v_new, void* cache_k, void* cache_v,
-                           void* out, void* ws, bool from_cache, cudaStream_t stream, cudaError_t* err);
 }  // namespace kvlink
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[KVLINK_NOALLOC_MAX_WORKSPACE_BYTES];
@@ -82,11 +78,7 @@ extern "C" int kvlink_suffix_attention_noalloc(const kvlink_plan_t* p, const voi
         if (cudaGetLastError() != cudaSuccess) return KVLINK_ECUDA;
     }
     cudaError_t err = cudaSuccess;
-    if (p->layout == KVLINK_LAYOUT_INTERLEAVED)
-        return kvlink::launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(),
-                                           p->cu_fresh.back(), p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q,
-                                           cache_k, cache_v, out, ws, s, &err);
-    return kvlink::launch_attention_fused(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
-                                          p->pool_rows, p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, nullptr, nullptr, nullptr, nullptr,
-                                          cache_k, cache_v, out, ws, true, s, &err);
+    return kvlink::launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
+                                       p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, ws,
+                                       s, &err);
 }

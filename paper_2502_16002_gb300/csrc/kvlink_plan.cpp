@@ -185,28 +185,39 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         }
     }
 
-    // ---- groups of 8 positions whose rows are consecutive in their source (and, apart,
-    // in the linked cache): each is one 8-row TMA copy in the gathering attention kernel
+    // ---- the same records in cache-row order, and the visibility of every fresh row
+    p->src_row.assign((size_t)ctx, kvlink_source_t{0, 0, 0, -1});
+    for (const kvlink_source_t& e : p->src) p->src_row[(size_t)e.slot] = e;
+    p->fresh_vis.assign(p->fresh_pos.size(), 0);
+    p->fresh_row0.assign(B, kNoFreshRegion);
+    for (int b = 0; b < B; ++b) {
+        const int32_t f0 = p->cu_fresh[b], T = p->cu_fresh[b + 1] - f0;
+        const int64_t C = p->cu_ctx[b + 1] - p->cu_ctx[b];
+        if (at_end) p->fresh_row0[b] = (int32_t)(C - T);
+        for (int32_t f = 0; f < T; ++f) {
+            const int32_t pos = p->fresh_pos[f0 + f];
+            // links at the end: the cached rows before the position (f of the pos earlier
+            // positions are fresh); interleaved: every row up to the position
+            p->fresh_vis[f0 + f] = at_end ? pos - f : pos + 1;
+        }
+    }
+
+    // ---- groups of 8 cache rows whose sources are consecutive in one tensor: each is one
+    // 8-row TMA copy in the one-kernel path
     p->cu_grp.assign(B + 1, 0);
     p->grp_src.clear();
-    p->grp_slot.clear();
     for (int b = 0; b < B; ++b) {
         const int64_t c0 = p->cu_ctx[b], C = p->cu_ctx[b + 1] - c0;
         p->cu_grp[b] = (int32_t)p->grp_src.size();
         for (int64_t m = 0; m * 8 < C; ++m) {
-            int32_t gs = -1, gc = -1;
+            int32_t gs = -1;
             if (m * 8 + 8 <= C) {
-                const kvlink_source_t* e = &p->src[(size_t)(c0 + m * 8)];
-                bool run_src = true, run_slot = true;
-                for (int i = 1; i < 8; ++i) {
-                    run_src = run_src && e[i].kind == e[0].kind && e[i].row == e[0].row + i;
-                    run_slot = run_slot && e[i].slot == e[0].slot + i;
-                }
-                if (run_src) gs = e[0].row | (e[0].kind == KVLINK_SRC_FRESH ? kGrpFresh : 0);
-                if (run_slot) gc = e[0].slot;
+                const kvlink_source_t* e = &p->src_row[(size_t)(c0 + m * 8)];
+                bool run = true;
+                for (int i = 1; i < 8; ++i) run = run && e[i].kind == e[0].kind && e[i].row == e[0].row + i;
+                if (run) gs = e[0].row | (e[0].kind == KVLINK_SRC_FRESH ? kGrpFresh : 0);
             }
             p->grp_src.push_back(gs);
-            p->grp_slot.push_back(gc);
         }
     }
     p->cu_grp[B] = (int32_t)p->grp_src.size();
@@ -245,7 +256,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     // the tile with the shortest range (the earliest link tokens).
     const int G = d->h_q / d->h_kv;
     const int tok_per_tile = kAttnBM / G;
-    struct Tile { int32_t b, g, t0, t1, n_tiles, min_pos, owner; };
+    struct Tile { int32_t b, g, t0, t1, n_tiles, min_vis, owner, a_tiles, b_tile0; };
     std::vector<Tile> tiles;
     int64_t work = 0;
     p->attn_pairs = 0;
@@ -257,9 +268,21 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
             for (int mt = 0; mt < n_mt; ++mt) {
                 const int t0 = mt == 0 ? 0 : T - (n_mt - mt) * tok_per_tile;
                 const int t1 = T - (n_mt - 1 - mt) * tok_per_tile;
-                const int32_t kv_len = p->fresh_pos[f0 + t1 - 1] + 1;  // positions increase within a query
-                const int32_t nt = (kv_len + kAttnBN - 1) / kAttnBN;
-                tiles.push_back({b, g, t0, t1, nt, p->fresh_pos[f0 + t0], mt == n_mt - 1 ? 1 : 0});
+                // visibility grows with position, so the tile's last row sees the most
+                int32_t a_tiles = (p->fresh_vis[f0 + t1 - 1] + kAttnBN - 1) / kAttnBN;
+                int32_t b_tile0 = 0, b_tiles = 0;
+                if (p->fresh_row0[b] != kNoFreshRegion) {
+                    const int32_t F = p->fresh_row0[b];
+                    b_tile0 = F / kAttnBN;
+                    const int32_t b_end = (F + t1 + kAttnBN - 1) / kAttnBN;
+                    if (b_tile0 <= a_tiles) {  // the runs touch: one run from row 0
+                        a_tiles = std::max(a_tiles, b_end);
+                    } else {
+                        b_tiles = b_end - b_tile0;
+                    }
+                }
+                const int32_t nt = a_tiles + b_tiles;
+                tiles.push_back({b, g, t0, t1, nt, p->fresh_vis[f0 + t0], mt == n_mt - 1 ? 1 : 0, a_tiles, b_tile0});
                 work += nt;
             }
         }
@@ -276,14 +299,14 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     for (const Tile& t : tiles) {
         const int32_t n_split = (t.n_tiles + max_tiles - 1) / max_tiles;
         if (n_split <= 1) {
-            p->items.push_back({t.b, t.g, t.t0, t.t1, 0, t.n_tiles, -1, t.min_pos, t.owner});
+            p->items.push_back({t.b, t.g, t.t0, t.t1, 0, t.n_tiles, -1, t.min_vis, t.owner, t.a_tiles, t.b_tile0});
             continue;
         }
         p->merges.push_back({t.b, t.g, t.t0, t.t1, p->n_slots, n_split, 0, 0});
         for (int s = 0; s < n_split; ++s) {
             const int32_t a = (int32_t)((int64_t)t.n_tiles * s / n_split);
             const int32_t e = (int32_t)((int64_t)t.n_tiles * (s + 1) / n_split);
-            p->items.push_back({t.b, t.g, t.t0, t.t1, a, e, p->n_slots + s, t.min_pos, t.owner});
+            p->items.push_back({t.b, t.g, t.t0, t.t1, a, e, p->n_slots + s, t.min_vis, t.owner, t.a_tiles, t.b_tile0});
         }
         p->n_slots += n_split;
     }
@@ -338,7 +361,9 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     p->off_src = take(p->src.size() * sizeof(kvlink_source_t));
     p->off_cu_grp = take(p->cu_grp.size() * sizeof(int32_t));
     p->off_grp_src = take(p->grp_src.size() * sizeof(int32_t));
-    p->off_grp_slot = take(p->grp_slot.size() * sizeof(int32_t));
+    p->off_src_row = take(p->src_row.size() * sizeof(kvlink_source_t));
+    p->off_fresh_vis = take(p->fresh_vis.size() * sizeof(int32_t));
+    p->off_fresh_row0 = take(p->fresh_row0.size() * sizeof(int32_t));
     p->device_bytes = off;
     p->uploaded = false;
     return KVLINK_OK;

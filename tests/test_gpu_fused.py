@@ -7,7 +7,7 @@ against the fp64 oracle (same tolerances as the two-kernel path) and, bit for bi
 against the two-kernel path, which it must reproduce exactly: the same rotation code,
 the same tiles and the same order of MMAs.  The links-at-end layout stores the same
 positions in another row order; the attention masks by position, so its output must
-equal the interleaved layout's bit for bit as well.
+equal the interleaved layout's up to the rounding of a different summation order.
 """
 import numpy as np
 import pytest
@@ -51,9 +51,12 @@ def test_one_kernel_equals_two_kernel_path_bitwise(RT, cfg_index, layer, layout)
     assert np.array_equal(gk, rk) and np.array_equal(gv, rv), "linked cache differs from the two-kernel path"
     assert _same_bits(gout, rout), "output differs from the two-kernel path"
     if lo:
-        # the same attention in the interleaved layout: identical bits
+        # the same attention in the interleaved layout: the keys come in another order (the
+        # cached rows, then the fresh rows), so the sums round differently, within the
+        # attention tolerance of each other
         _, _, _, iout, _ = run_layer(RT, batch, layer, "fused", layout=0)
-        assert _same_bits(gout, iout), "links-at-end output differs from the interleaved one"
+        d = np.abs(gout - iout)
+        assert d.max() <= 1e-2 and d.mean() <= 1e-4, (d.max(), d.mean())
     for b in sorted({0, batch.cfg.batch - 1}):
         check_query(batch, b, lp, gk, gv, gout, inp, layout=lo)
 
