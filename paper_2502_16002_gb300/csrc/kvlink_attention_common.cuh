@@ -44,8 +44,8 @@ struct TcCfg {
     static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
     static constexpr uint32_t OFF_V = OFF_K + NK * KV_BYTES;
     static constexpr uint32_t OFF_BAR = OFF_V + NV * KV_BYTES;
-    // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB], p_full[NB], o_done[NB], drain
-    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 3 * NB + 1;
+    // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB], p_full[NB], o_done[NB], drain x2
+    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 3 * NB + 2;
     static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
     // TMEM columns: S/P buffers then the O accumulator
     static constexpr uint32_t TMEM_S = 0;                // buffer b at b * 128
@@ -145,42 +145,25 @@ __device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes
         drain_bar(full + j % STAGES, (j / STAGES) & 1, status);
 }
 
-// The single MMA-issuing thread with K and V in separate TMA rings (NK, NV stages):
-//   S_j = Q K_j^T into S buffer j % NB (after PV_{j-NB} has read that buffer), then
-//   O += P_{j-1} V_{j-1} with P read from TMEM, V MN-major from shared memory.
-template <int D, int NK, int NV, int NB>
-__device__ __forceinline__ void mma_role_tma(uint8_t* smem, uint32_t off_q, uint32_t off_k, uint32_t off_v,
-                                             uint32_t kv_bytes, uint32_t atom_bytes, uint32_t tmem_s,
-                                             uint32_t tmem_o, int n_tiles, uint64_t* bar_q_full,
-                                             uint64_t* bar_k_full, uint64_t* bar_k_empty, uint64_t* bar_v_full,
-                                             uint64_t* bar_v_empty, uint64_t* bar_s_full, uint64_t* bar_p_full,
-                                             uint64_t* bar_o_done, uint64_t* bar_drain,
-                                             volatile int32_t* abort_flag, int32_t* status) {
+// Two MMA-issuing threads, one for S_j = Q K_j^T and one for O += P_i V_i.  A thread that
+// waits on an mbarrier right after its own tcgen05.commit was seen to stall until its MMAs
+// had drained (~400 cycles per tile with one issuer doing both); with two issuers each
+// waits only on its own work while the other keeps the tensor pipe fed.  S_j goes into S
+// buffer j % NB once PV_{j-NB} has read that buffer; PV_i reads P_i from TMEM and V_i
+// MN-major from shared memory.
+template <int D, int NK, int NB>
+__device__ __forceinline__ void mma_s_role(uint8_t* smem, uint32_t off_q, uint32_t off_k, uint32_t kv_bytes,
+                                           uint32_t atom_bytes, uint32_t tmem_s, int n_tiles, uint64_t* bar_q_full,
+                                           uint64_t* bar_k_full, uint64_t* bar_k_empty, uint64_t* bar_s_full,
+                                           uint64_t* bar_o_done, uint64_t* bar_drain, volatile int32_t* abort_flag,
+                                           int32_t* status) {
     using namespace sm100;
     constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
-    constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
     const uint32_t sQ = smem_u32(smem + off_q);
     bool ok = wait_bar(bar_q_full, 0, abort_flag, status);
-    // O += P_i V_i, P_i (bf16) read from its S buffer in TMEM
-    auto issue_pv = [&](int i) -> bool {
-        const int b = i % NB, sv = i % NV;
-        if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag, status)) return false;
-        if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag, status)) return false;
-        tc_fence_after();
-        const uint32_t sV = smem_u32(smem + off_v + sv * kv_bytes);
-        const uint32_t pcol = tmem_s + b * kAttnBN;
-#pragma unroll
-        for (int kk = 0; kk < kAttnBN / 16; ++kk)
-            mma_bf16_ts(tmem_o, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, atom_bytes, 1024), idesc_pv,
-                        (i > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(bar_o_done + b);
-        mma_commit(bar_v_empty + sv);
-        return true;
-    };
     for (int j = 0; ok && j < n_tiles; ++j) {
         const int sk = j % NK, b = j % NB;
         if (!(ok = wait_bar(bar_k_full + sk, (j / NK) & 1, abort_flag, status))) break;
-        // buffer b last held P_{j-NB}: its PV must have finished reading it
         if (j >= NB && !(ok = wait_bar(bar_o_done + b, ((j - NB) / NB) & 1, abort_flag, status))) break;
         tc_fence_after();
         const uint32_t sK = smem_u32(smem + off_k + sk * kv_bytes);
@@ -192,10 +175,33 @@ __device__ __forceinline__ void mma_role_tma(uint8_t* smem, uint32_t off_q, uint
         }
         mma_commit(bar_s_full + b);
         mma_commit(bar_k_empty + sk);
-        if (j >= 1) ok = issue_pv(j - 1);
     }
-    if (ok && n_tiles > 0) ok = issue_pv(n_tiles - 1);
-    mma_commit(bar_drain);  // arrives once every MMA issued above has completed
+    mma_commit(bar_drain);
+    drain_bar(bar_drain, 0, status);
+}
+
+template <int D, int NV, int NB>
+__device__ __forceinline__ void mma_pv_role(uint8_t* smem, uint32_t off_v, uint32_t kv_bytes, uint32_t atom_bytes,
+                                            uint32_t tmem_s, uint32_t tmem_o, int n_tiles, uint64_t* bar_v_full,
+                                            uint64_t* bar_v_empty, uint64_t* bar_p_full, uint64_t* bar_o_done,
+                                            uint64_t* bar_drain, volatile int32_t* abort_flag, int32_t* status) {
+    using namespace sm100;
+    constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
+    for (int i = 0; i < n_tiles; ++i) {
+        const int b = i % NB, sv = i % NV;
+        if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag, status)) break;
+        if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag, status)) break;
+        tc_fence_after();
+        const uint32_t sV = smem_u32(smem + off_v + sv * kv_bytes);
+        const uint32_t pcol = tmem_s + b * kAttnBN;
+#pragma unroll
+        for (int kk = 0; kk < kAttnBN / 16; ++kk)
+            mma_bf16_ts(tmem_o, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, atom_bytes, 1024), idesc_pv,
+                        (i > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(bar_o_done + b);
+        mma_commit(bar_v_empty + sv);
+    }
+    mma_commit(bar_drain);
     drain_bar(bar_drain, 0, status);
 }
 

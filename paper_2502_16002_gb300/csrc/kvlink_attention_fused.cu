@@ -31,8 +31,8 @@
 //              keys in place (the eight double-float cos/sin of its pairs stay in
 //              registers while the segment does not change), stores owned rows to the
 //              linked cache, and publishes.
-//   warp 8     TMEM allocation, Q by TMA, the single MMA-issuing thread; warps 10-11
-//              idle (they complete the third warpgroup)
+//   warp 8     TMEM allocation, Q by TMA, the thread issuing S = Q K^T; warp 10: the
+//              thread issuing O += P V; warp 11 idle (completes the third warpgroup)
 // Registers: launched at 168 per thread (384 x 168 <= 64K); the third warpgroup drops
 // to 56 and the softmax warpgroup rises to 232, so that on each SM sub-partition
 // (one warp of each warpgroup, 512 registers per thread in all) 232 + 168 + 56 fit.
@@ -68,8 +68,9 @@ static_assert(128 * (kSoftmaxRegs - kLaunchRegs) <= 128 * (kLaunchRegs - kIdleRe
 static_assert(kSoftmaxRegs + kLaunchRegs + kIdleRegs <= 512, "sub-partition register budget");
 constexpr int kGatherWarp0 = 4;  // warps 4-7
 constexpr int kGatherThreads = 128;
-constexpr int kFusedMmaWarp = 8;
+constexpr int kFusedMmaWarp = 8;   // S = Q K^T issuer (and TMEM, Q)
 constexpr int kFusedTmaWarp = 9;
+constexpr int kFusedPvWarp = 10;   // O += P V issuer
 constexpr uint32_t kFusedTmemCols = 512;
 
 template <int D>
@@ -84,8 +85,8 @@ struct FusedCfg {
     static constexpr uint32_t OFF_Q = 0;
     static constexpr uint32_t OFF_KV = Q_BYTES;
     static constexpr uint32_t OFF_BAR = OFF_KV + NS * STAGE_BYTES;
-    // q_full, raw_full[NS], kv_full[NS], kv_empty[NS], s_full[NB], p_full[NB], o_done[NB], drain
-    static constexpr int N_BARS = 2 + 3 * NS + 3 * NB;
+    // q_full, raw_full[NS], kv_full[NS], kv_empty[NS], s_full[NB], p_full[NB], o_done[NB], drain x2
+    static constexpr int N_BARS = 3 + 3 * NS + 3 * NB;
     static constexpr uint32_t GROUP_TX = 8 * 128 * ATOMS * 2;  // K and V bytes of one 8-row group
     static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
     static constexpr uint32_t TMEM_S = 0;                  // buffer b at b * 128
@@ -369,7 +370,6 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
         setmaxnreg_dec<kIdleRegs>();
         if (warp == kFusedMmaWarp && lane == 0) {
             constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
-            constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
             const uint32_t sQ = smem_u32(smem + C::OFF_Q);
             const int q_row0 = P.cu_fresh[it.query] + it.tok0;
             mbar_arrive_expect_tx(bar_q_full, C::Q_BYTES);
@@ -378,21 +378,6 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
                 tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &M.q, a * 64, it.kv_head * G, q_row0, bar_q_full);
             bool ok = wait_bar(bar_q_full, 0, abort_flag, &g_fused_status);
             if (!ok) drain_bar(bar_q_full, 0, &g_fused_status);  // the Q copy lands before the CTA leaves
-            // O += P_i V_i, P_i (bf16) read from its S buffer in TMEM; frees stage i % NS
-            auto issue_pv = [&](int i) -> bool {
-                const int b = i % NB, st = i % NS;
-                if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag, &g_fused_status)) return false;
-                tc_fence_after();
-                const uint32_t sV = smem_u32(smem + C::OFF_KV + st * C::STAGE_BYTES + C::HALF_BYTES);
-                const uint32_t pcol = tmem + C::TMEM_S + b * kAttnBN;
-#pragma unroll
-                for (int kk = 0; kk < kAttnBN / 16; ++kk)
-                    mma_bf16_ts(tmem + C::TMEM_O, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, C::ATOM_BYTES, 1024),
-                                idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
-                mma_commit(bar_o_done + b);
-                mma_commit(bar_kv_empty + st);
-                return true;
-            };
             for (int j = 0; ok && j < n_tiles; ++j) {
                 const int st = j % NS, b = j % NB;
                 if (!(ok = wait_bar(bar_kv_full + st, (j / NS) & 1, abort_flag, &g_fused_status))) break;
@@ -408,11 +393,28 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
                                 sdesc_sw128(sK + koff, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
                 }
                 mma_commit(bar_s_full + b);
-                if (j >= 1) ok = issue_pv(j - 1);
             }
-            if (ok && n_tiles > 0) ok = issue_pv(n_tiles - 1);
             mma_commit(bar_drain);  // arrives once every MMA issued above has completed
             drain_bar(bar_drain, 0, &g_fused_status);
+        } else if (warp == kFusedPvWarp && lane == 0) {
+            constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
+            // O += P_i V_i, P_i (bf16) read from its S buffer in TMEM; frees stage i % NS
+            for (int i = 0; i < n_tiles; ++i) {
+                const int b = i % NB, st = i % NS;
+                if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag, &g_fused_status)) break;
+                if (!wait_bar(bar_kv_full + st, (i / NS) & 1, abort_flag, &g_fused_status)) break;
+                tc_fence_after();
+                const uint32_t sV = smem_u32(smem + C::OFF_KV + st * C::STAGE_BYTES + C::HALF_BYTES);
+                const uint32_t pcol = tmem + C::TMEM_S + b * kAttnBN;
+#pragma unroll
+                for (int kk = 0; kk < kAttnBN / 16; ++kk)
+                    mma_bf16_ts(tmem + C::TMEM_O, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, C::ATOM_BYTES, 1024),
+                                idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
+                mma_commit(bar_o_done + b);
+                mma_commit(bar_kv_empty + st);
+            }
+            mma_commit(bar_drain + 1);
+            drain_bar(bar_drain + 1, 0, &g_fused_status);
         } else if (warp == kFusedTmaWarp && lane == 0) {
             tma_role<D>(it, P, M, smem, bar_raw_full, bar_kv_empty, n_tiles, abort_flag);
         }

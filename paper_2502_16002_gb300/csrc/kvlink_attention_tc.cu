@@ -6,11 +6,12 @@
 // cached rows and the fresh rows at the end form two runs).  Rows are (token, head)
 // pairs, so the G heads of a GQA group share every K/V tile load.
 //
-// Warp roles (224 threads, one CTA per SM, 512 TMEM columns):
+// Warp roles (256 threads, one CTA per SM, 512 TMEM columns):
 //   warps 0-3  softmax + epilogue; thread r owns row r = TMEM lane r
 //   warp 4     TMA: Q once, then K tiles into an NK-stage ring
-//   warp 5     TMEM allocation and the single MMA-issuing thread
+//   warp 5     TMEM allocation and the thread issuing the S = Q K^T MMAs
 //   warp 6     TMA: V tiles into an NV-stage ring
+//   warp 7     the thread issuing the O += P V MMAs
 // Per KV tile j (TMEM: three S/P buffers of 128 columns, then O):
 //   S_j = Q K_j^T           tcgen05.mma SMEM x SMEM -> S buffer j%3
 //   P_j = exp2(S_j c - m)   softmax warps: TMEM -> registers -> bf16 P written back
@@ -18,7 +19,7 @@
 //   O  += P_j V_j           tcgen05.mma TMEM x SMEM (P from TMEM, V read MN-major)
 // S_j is issued only after PV_{j-3} has finished reading the buffer, so up to
 // three tiles are in flight and the softmax never waits on a PV except to
-// rescale O.  The running max m is raised only when it grows by more than 2^8,
+// rescale O.  S and PV come from two issuing threads (see mma_s_role).  The running max m is raised only when it grows by more than 2^8,
 // so that rescale is rare.  The mask keeps the cache rows holding positions up to
 // the row's own (a threshold pair per row, see softmax_role) and is evaluated only on
 // tiles that reach past the rows every row of the tile sees.  Items whose KV range was split write
@@ -42,7 +43,8 @@ using namespace sm100;
 
 static __device__ int32_t g_attn_status;
 
-constexpr int kTcThreads = 224;
+constexpr int kTcThreads = 256;
+constexpr int kPvWarp = 7;
 constexpr int kSoftmaxWarps = 4;
 constexpr int kTmaKWarp = 4;
 constexpr int kMmaWarp = 5;
@@ -122,12 +124,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             produce_ring<NV, C::ATOMS>(smem + C::OFF_V, C::KV_BYTES, &tm_v, bar_v_full, bar_v_empty, n_tiles, it,
                                        ctx0, abort_flag, &g_attn_status);
     } else if (warp == kMmaWarp) {
-        // ------------------------------------------------------------ MMA issuer
         if (lane == 0)
-            mma_role_tma<D, NK, NV, NB>(smem, C::OFF_Q, C::OFF_K, C::OFF_V, C::KV_BYTES, C::ATOM_BYTES, tmem + C::TMEM_S,
-                                       tmem + C::TMEM_O, n_tiles, bar_q_full, bar_k_full, bar_k_empty, bar_v_full,
-                                       bar_v_empty, bar_s_full, bar_p_full, bar_o_done, bar_drain, abort_flag,
-                                       &g_attn_status);
+            mma_s_role<D, NK, NB>(smem, C::OFF_Q, C::OFF_K, C::KV_BYTES, C::ATOM_BYTES, tmem + C::TMEM_S, n_tiles,
+                                  bar_q_full, bar_k_full, bar_k_empty, bar_s_full, bar_o_done, bar_drain, abort_flag,
+                                  &g_attn_status);
+    } else if (warp == kPvWarp) {
+        if (lane == 0)
+            mma_pv_role<D, NV, NB>(smem, C::OFF_V, C::KV_BYTES, C::ATOM_BYTES, tmem + C::TMEM_S, tmem + C::TMEM_O,
+                                   n_tiles, bar_v_full, bar_v_empty, bar_p_full, bar_o_done, bar_drain + 1,
+                                   abort_flag, &g_attn_status);
     } else {
         // ------------------------------------------------------------ softmax + epilogue (warps 0-3)
         softmax_role<D, G, NB>(it, P, tmem + C::TMEM_S, tmem + C::TMEM_O, n_tiles, bar_s_full, bar_p_full,
