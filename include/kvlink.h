@@ -266,12 +266,27 @@ int kvlink_linked_prefill_fused(const kvlink_plan_t* plan, const void* d_pool_k,
                                 void* d_cache_k, void* d_cache_v, void* d_out,
                                 void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream);
 
+/* Re-encode + concat (Sec. 2.2, Sec. 2.1) of the document caches of n_layers layers in
+ * one launch: the same result as kvlink_reencode_concat(plan, pool_k[l], pool_v[l],
+ * cache_k[l], cache_v[l]) for every layer l, bit for bit.  The precomputed document
+ * caches do not depend on the forward pass of the fresh rows, so a prefill can rotate
+ * every layer's caches before its first layer runs, in one launch instead of one per
+ * layer (the fresh rows are then placed per layer by kvlink_suffix_attention with
+ * k_new / v_new).  Each argument is a HOST array
+ * of n_layers device pointers (each 16-byte aligned; per layer, the shapes of
+ * kvlink_reencode_concat).  Errors: EINVAL (a NULL or misaligned pointer, n_layers <= 0),
+ * the plan errors of kvlink_reencode_concat, ECUDA. */
+int kvlink_reencode_concat_layers(const kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
+                                  const void* const* d_pool_v, void* const* d_cache_k, void* const* d_cache_v,
+                                  kvlink_stream_t stream);
+
 /* The linked prefill of n_layers layers (the attention side of one whole prefill) in
- * one call: for every layer l, in order, kvlink_linked_prefill(plan, pool_k[l],
- * pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l], out[l], ...).  Each
- * argument is a HOST array of n_layers device pointers.  One workspace serves all layers
- * (they run in stream order).  Errors: as kvlink_linked_prefill; a failing layer stops
- * the sequence (layers before it have been enqueued). */
+ * one call, with the same results, bit for bit, as kvlink_linked_prefill(plan,
+ * pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l], out[l], ...)
+ * for every layer l in order, which is what it enqueues.  Each argument is a HOST array
+ * of n_layers device pointers.  One workspace serves all layers (they run in stream
+ * order).  Every pointer is checked before the first launch.  Errors: as
+ * kvlink_linked_prefill. */
 int kvlink_linked_prefill_layers(const kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
                                  const void* const* d_pool_v, const void* const* d_q,
                                  const void* const* d_k_new, const void* const* d_v_new, void* const* d_cache_k,
@@ -299,10 +314,23 @@ int kvlink_suffix_attention_noalloc(const kvlink_plan_t* plan, const void* d_q, 
                                     const void* d_v_new, void* d_cache_k, void* d_cache_v, void* d_out,
                                     kvlink_stream_t stream);
 
-/* Device status word: 0 when no kernel reported an error since the last clear.
- * Reading synchronises with the current device.  Errors: ECUDA. */
+/* Device status word: 0 when no kernel reported an error since the last clear, else the
+ * first code recorded: KVLINK_STATUS_WAIT_TIMEOUT (an attention pipeline wait ran out)
+ * or KVLINK_STATUS_COPY_TIMEOUT (a re-encode pipeline wait ran out).  While it is set,
+ * later launches skip their work (outputs undefined) instead of waiting out their
+ * bounds; kvlink_clear_device_status() re-arms them.  Reading synchronises with the
+ * current device.  Errors: ECUDA. */
+#define KVLINK_STATUS_WAIT_TIMEOUT 0x41
+#define KVLINK_STATUS_COPY_TIMEOUT 0x21
 int kvlink_device_status(int32_t* status);
 int kvlink_clear_device_status(void);
+
+/* Failure-path self-test: one GPU thread waits, through the same bounded mbarrier wait
+ * the attention kernels use, on a barrier that nothing arrives at, with a limit of
+ * limit_ms (1..2000).  The wait runs out and records KVLINK_STATUS_WAIT_TIMEOUT in the
+ * status word, as a stalled pipeline would; nothing traps and the context stays usable.
+ * Errors: EINVAL (limit out of range), ECUDA. */
+int kvlink_selftest_wait_timeout(uint32_t limit_ms, kvlink_stream_t stream);
 
 const char* kvlink_strerror(int code);
 /* Text of the last CUDA error seen by this thread (empty if none). */

@@ -15,6 +15,9 @@ void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float4* d_rope,
 void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv, int num_sms,
                      const void* pool_k, const void* pool_v, const void* k_new, const void* v_new, void* cache_k,
                      void* cache_v, cudaStream_t stream);
+void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int h_kv, int num_sms, int n_layers,
+                            const void* const* pool_k, const void* const* pool_v, void* const* cache_k,
+                            void* const* cache_v, cudaStream_t stream);
 int read_copy_status(int32_t* status);
 void launch_rope_fresh(const int32_t* d_fresh_pos, int n_fresh, int head_dim, double theta, void* q, int h_q,
                        void* k, int h_kv, cudaStream_t stream);
@@ -33,6 +36,7 @@ int launch_attention_fused(const DevicePlan& P, int n_items, int n_merges, int n
                            cudaStream_t stream, cudaError_t* err);
 int read_fused_status(int32_t* status);
 int clear_fused_status();
+int launch_wait_selftest(uint32_t limit_ms, cudaStream_t stream);
 }  // namespace kvlink
 
 using namespace kvlink;
@@ -234,6 +238,26 @@ int kvlink_reencode_concat(const kvlink_plan_t* p, const void* pool_k, const voi
     return check_launch("reencode_kernel");
 }
 
+static bool all_aligned(int32_t n, const void* const* a) {
+    for (int32_t l = 0; l < n; ++l)
+        if (!a[l] || !aligned16(a[l])) return false;
+    return true;
+}
+
+int kvlink_reencode_concat_layers(const kvlink_plan_t* p, int32_t n_layers, const void* const* pool_k,
+                                  const void* const* pool_v, void* const* cache_k, void* const* cache_v,
+                                  kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (n_layers <= 0 || !pool_k || !pool_v || !cache_k || !cache_v) return KVLINK_EINVAL;
+    if (!all_aligned(n_layers, pool_k) || !all_aligned(n_layers, pool_v) ||
+        !all_aligned(n_layers, (const void* const*)cache_k) || !all_aligned(n_layers, (const void* const*)cache_v))
+        return KVLINK_EINVAL;
+    launch_reencode_layers(p->dev, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, n_layers, pool_k, pool_v,
+                           cache_k, cache_v, (cudaStream_t)stream);
+    return check_launch("reencode_kernel (layers)");
+}
+
 static int place_fresh(const kvlink_plan_t* p, const void* k_new, const void* v_new, void* cache_k,
                        void* cache_v, cudaStream_t s) {
     const int n_all = (int)p->chunks.size();
@@ -334,6 +358,18 @@ int kvlink_linked_prefill_layers(const kvlink_plan_t* p, int32_t n_layers, const
     if (rc) return rc;
     if (n_layers <= 0 || !pool_k || !pool_v || !q || !k_new || !v_new || !cache_k || !cache_v || !out)
         return KVLINK_EINVAL;
+    // every argument is checked before the first launch
+    if (!all_aligned(n_layers, q) || !all_aligned(n_layers, k_new) || !all_aligned(n_layers, v_new) ||
+        !all_aligned(n_layers, (const void* const*)out))
+        return KVLINK_EINVAL;
+    if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
+    if (ws && !aligned16(ws)) return KVLINK_EINVAL;
+    if (!all_aligned(n_layers, pool_k) || !all_aligned(n_layers, pool_v) ||
+        !all_aligned(n_layers, (const void* const*)cache_k) || !all_aligned(n_layers, (const void* const*)cache_v))
+        return KVLINK_EINVAL;
+    // per layer, one re-encode launch that also places the fresh rows, then the suffix
+    // attention.  (Re-encoding every layer's documents in one launch first streams at the
+    // same rate and then needs a separate fresh-row launch per layer: slower.)
     for (int l = 0; l < n_layers; ++l) {
         rc = kvlink_linked_prefill(p, pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l],
                                    out[l], ws, ws_bytes, stream);
@@ -349,6 +385,12 @@ int kvlink_rope_fresh(const kvlink_plan_t* p, void* q, void* k_new, kvlink_strea
     launch_rope_fresh(p->dev.fresh_pos, p->cu_fresh.back(), p->head_dim, p->theta, q, p->h_q, k_new, p->h_kv,
                       (cudaStream_t)stream);
     return check_launch("rope_fresh_kernel");
+}
+
+int kvlink_selftest_wait_timeout(uint32_t limit_ms, kvlink_stream_t stream) {
+    if (limit_ms < 1 || limit_ms > 2000) return KVLINK_EINVAL;
+    const int rc = launch_wait_selftest(limit_ms, (cudaStream_t)stream);
+    return rc == KVLINK_OK ? KVLINK_OK : check_launch("wait_selftest_kernel");
 }
 
 int kvlink_device_status(int32_t* status) {

@@ -56,13 +56,13 @@ struct TcCfg {
 
 // Wait for phase `parity` of `bar`; false if another role aborted or the time limit passed.
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag,
-                                         int32_t* status) {
+                                         int32_t* status, uint64_t limit_ns = kWaitLimitNs) {
     if (sm100::mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = sm100::globaltimer_ns();
     while (true) {
         if (sm100::mbar_try_wait(bar, parity)) return true;
         if (*abort_flag) return false;
-        if (sm100::globaltimer_ns() - t0 > kWaitLimitNs) {
+        if (sm100::globaltimer_ns() - t0 > limit_ns) {
             *abort_flag = 1;
             atomicCAS(status, 0, kAttnStatusWaitTimeout);
             return false;

@@ -261,6 +261,24 @@ int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fr
     return KVLINK_OK;
 }
 
+// Failure-path self-test: one thread waits, through the kernels' bounded wait, on an
+// mbarrier that nothing arrives at.  The wait runs out after limit_ns and records
+// kAttnStatusWaitTimeout in the attention status word, exactly as a stalled pipeline would.
+__global__ void wait_selftest_kernel(uint64_t limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int32_t abort_flag;
+    if (threadIdx.x != 0) return;
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+    wait_bar(&bar, 0, &abort_flag, &g_attn_status, limit_ns);
+}
+
+int launch_wait_selftest(uint32_t limit_ms, cudaStream_t stream) {
+    wait_selftest_kernel<<<1, 32, 0, stream>>>((uint64_t)limit_ms * 1000000ull);
+    return cudaGetLastError() == cudaSuccess ? KVLINK_OK : KVLINK_ECUDA;
+}
+
 int read_attention_status(int32_t* status) {
     return cudaMemcpyFromSymbol(status, g_attn_status, sizeof(int32_t)) == cudaSuccess ? KVLINK_OK : KVLINK_ECUDA;
 }

@@ -12,6 +12,9 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
+#include <cstdint>
+
 #include "kvlink_internal.h"
 #include "kvlink_rope.cuh"
 #include "kvlink_sm100.cuh"
@@ -88,18 +91,30 @@ __device__ __forceinline__ void copy_drain(uint64_t* bar, uint32_t parity) {
         }
 }
 
-// CTA b handles the contiguous range of work units [n*b/grid, n*(b+1)/grid).
+// Pool and linked-cache tensors of up to MAXL layers, passed by value.  Layer l's
+// units are the plan's n_chunks units applied to pool_k[l], pool_v[l] -> cache_k[l],
+// cache_v[l]; the document caches of every layer are inputs, so all layers can be
+// re-encoded in one launch ahead of the per-layer attention.
+template <int MAXL>
+struct LayerPtrs {
+    const __nv_bfloat16* pool_k[MAXL];
+    const __nv_bfloat16* pool_v[MAXL];
+    __nv_bfloat16* cache_k[MAXL];
+    __nv_bfloat16* cache_v[MAXL];
+};
+constexpr int kMaxLayersPerLaunch = 64;     // 2 KB of kernel parameters
+
+// Work unit u = layer * n_chunks + c.  CTA b handles the contiguous range of units
+// [n*b/grid, n*(b+1)/grid), n = n_layers * n_chunks.
 // Producer (warp 0, one thread): bulk-loads a unit's K rows and V rows into a stage.
 // Consumers (warps 1-4): rotate the unit's keys in place when it is a document (each
 // thread keeps a fixed (head, j0) slot and its eight double-float cos/sin pairs), then
 // one thread bulk-stores K and V to the linked cache and frees the stage once the
 // stores have read it.  V is never touched by the threads.
-template <int D>
+template <int D, int MAXL>
 __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
-    const CopyChunk* __restrict__ chunks, int n_chunks, const float4* __restrict__ rope, int h_kv,
-    const __nv_bfloat16* __restrict__ pool_k, const __nv_bfloat16* __restrict__ pool_v,
-    const __nv_bfloat16* __restrict__ k_new, const __nv_bfloat16* __restrict__ v_new,
-    __nv_bfloat16* __restrict__ cache_k, __nv_bfloat16* __restrict__ cache_v) {
+    const CopyChunk* __restrict__ chunks, int n_chunks, int n_layers, const float4* __restrict__ rope, int h_kv,
+    const LayerPtrs<MAXL> L, const __nv_bfloat16* __restrict__ k_new, const __nv_bfloat16* __restrict__ v_new) {
     using namespace sm100;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
@@ -108,8 +123,9 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     uint64_t* empty = full + kCopyStages;
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(empty + kCopyStages);
 
-    const int c_begin = (int)((int64_t)n_chunks * blockIdx.x / gridDim.x);
-    const int c_end = (int)((int64_t)n_chunks * (blockIdx.x + 1) / gridDim.x);
+    const int64_t n_units = (int64_t)n_chunks * n_layers;
+    const int c_begin = (int)(n_units * blockIdx.x / gridDim.x);
+    const int c_end = (int)(n_units * (blockIdx.x + 1) / gridDim.x);
     const int64_t row_elems = (int64_t)h_kv * D;
     const uint32_t row_bytes = (uint32_t)(row_elems * 2);
 
@@ -131,10 +147,11 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
             for (int c = c_begin, i = 0; c < c_end; ++c, ++i) {
                 const int st = i % kCopyStages;
                 if (!copy_wait(empty + st, ((i / kCopyStages) & 1) ^ 1, abort_flag)) break;
-                const CopyChunk ch = chunks[c];
+                const int layer = MAXL == 1 ? 0 : c / n_chunks;
+                const CopyChunk ch = chunks[c - layer * n_chunks];
                 const bool fresh = ch.kind == KVLINK_SEG_LINK || ch.kind == KVLINK_SEG_QUESTION;
-                const __nv_bfloat16* sk = (fresh ? k_new : pool_k) + ch.src_row * row_elems;
-                const __nv_bfloat16* sv = (fresh ? v_new : pool_v) + ch.src_row * row_elems;
+                const __nv_bfloat16* sk = (fresh ? k_new : L.pool_k[layer]) + ch.src_row * row_elems;
+                const __nv_bfloat16* sv = (fresh ? v_new : L.pool_v[layer]) + ch.src_row * row_elems;
                 const uint32_t bytes = (uint32_t)ch.n * row_bytes;
                 uint8_t* stage = smem + st * CopySmem::STAGE;
                 mbar_arrive_expect_tx(full + st, 2 * bytes);
@@ -166,7 +183,8 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
         copy_wait(full + st, (i / kCopyStages) & 1, abort_flag);
         named_bar_sync(1, kCopyConsumers);
         if (*abort_flag) break;  // uniform: every consumer passed the barrier first
-        const CopyChunk ch = chunks[c];
+        const int layer = MAXL == 1 ? 0 : c / n_chunks;
+        const CopyChunk ch = chunks[c - layer * n_chunks];
         uint8_t* stage = smem + st * CopySmem::STAGE;
         if (ch.kind == KVLINK_SEG_DOC) {
             if (ch.table != cur_table) {
@@ -188,8 +206,8 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
         named_bar_sync(1, kCopyConsumers);
         if (tc == 0) {
             const uint32_t bytes = (uint32_t)ch.n * row_bytes;
-            bulk_store(cache_k + ch.dst_row * row_elems, stage, bytes);
-            bulk_store(cache_v + ch.dst_row * row_elems, stage + kCopyStageBytes, bytes);
+            bulk_store(L.cache_k[layer] + ch.dst_row * row_elems, stage, bytes);
+            bulk_store(L.cache_v[layer] + ch.dst_row * row_elems, stage + kCopyStageBytes, bytes);
             bulk_commit();
             bulk_wait_read<1>();  // the previous unit's stores have read their stage
             if (i > 0) mbar_arrive(empty + (i - 1) % kCopyStages);
@@ -198,33 +216,58 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     if (tc == 0) bulk_wait<0>();
 }
 
+template <int D, int MAXL>
+static void launch_reencode_t(const CopyChunk* ch, int n_chunks, int n_layers, const float4* rope, int h_kv,
+                              int num_sms, const LayerPtrs<MAXL>& L, const void* k_new, const void* v_new,
+                              cudaStream_t stream) {
+    static bool attr = false;
+    if (!attr) {
+        cudaFuncSetAttribute(reencode_kernel<D, MAXL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)CopySmem::BYTES);
+        attr = true;
+    }
+    const int64_t n_units = (int64_t)n_chunks * n_layers;
+    const int grid = n_units < num_sms ? (int)n_units : num_sms;
+    reencode_kernel<D, MAXL><<<grid, kCopyThreads, CopySmem::BYTES, stream>>>(
+        ch, n_chunks, n_layers, rope, h_kv, L, (const __nv_bfloat16*)k_new, (const __nv_bfloat16*)v_new);
+}
+
 void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv, int num_sms,
                      const void* pool_k, const void* pool_v, const void* k_new, const void* v_new, void* cache_k,
                      void* cache_v, cudaStream_t stream) {
     if (n_chunks <= 0) return;
     using bf = __nv_bfloat16;
-    const int grid = n_chunks < num_sms ? n_chunks : num_sms;
+    LayerPtrs<1> L{{(const bf*)pool_k}, {(const bf*)pool_v}, {(bf*)cache_k}, {(bf*)cache_v}};
     const CopyChunk* ch = P.chunks + chunk_base;
-    if (head_dim == 128) {
-        static bool attr = false;
-        if (!attr) {
-            cudaFuncSetAttribute(reencode_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)CopySmem::BYTES);
-            attr = true;
+    if (head_dim == 128)
+        launch_reencode_t<128, 1>(ch, n_chunks, 1, P.rope, h_kv, num_sms, L, k_new, v_new, stream);
+    else
+        launch_reencode_t<64, 1>(ch, n_chunks, 1, P.rope, h_kv, num_sms, L, k_new, v_new, stream);
+}
+
+// The document chunks [0, n_chunks) of n_layers layers, kMaxLayersPerLaunch layers per launch.
+void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int h_kv, int num_sms, int n_layers,
+                            const void* const* pool_k, const void* const* pool_v, void* const* cache_k,
+                            void* const* cache_v, cudaStream_t stream) {
+    if (n_chunks <= 0) return;
+    using bf = __nv_bfloat16;
+    // unit indices stay below 2^31
+    const int per_launch = (int)std::min<int64_t>(kMaxLayersPerLaunch, INT32_MAX / n_chunks);
+    for (int l0 = 0; l0 < n_layers; l0 += per_launch) {
+        const int nl = std::min(n_layers - l0, per_launch);
+        LayerPtrs<kMaxLayersPerLaunch> L{};
+        for (int l = 0; l < nl; ++l) {
+            L.pool_k[l] = (const bf*)pool_k[l0 + l];
+            L.pool_v[l] = (const bf*)pool_v[l0 + l];
+            L.cache_k[l] = (bf*)cache_k[l0 + l];
+            L.cache_v[l] = (bf*)cache_v[l0 + l];
         }
-        reencode_kernel<128><<<grid, kCopyThreads, CopySmem::BYTES, stream>>>(
-            ch, n_chunks, P.rope, h_kv, (const bf*)pool_k, (const bf*)pool_v, (const bf*)k_new, (const bf*)v_new,
-            (bf*)cache_k, (bf*)cache_v);
-    } else {
-        static bool attr = false;
-        if (!attr) {
-            cudaFuncSetAttribute(reencode_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)CopySmem::BYTES);
-            attr = true;
-        }
-        reencode_kernel<64><<<grid, kCopyThreads, CopySmem::BYTES, stream>>>(
-            ch, n_chunks, P.rope, h_kv, (const bf*)pool_k, (const bf*)pool_v, (const bf*)k_new, (const bf*)v_new,
-            (bf*)cache_k, (bf*)cache_v);
+        if (head_dim == 128)
+            launch_reencode_t<128, kMaxLayersPerLaunch>(P.chunks, n_chunks, nl, P.rope, h_kv, num_sms, L, nullptr,
+                                                        nullptr, stream);
+        else
+            launch_reencode_t<64, kMaxLayersPerLaunch>(P.chunks, n_chunks, nl, P.rope, h_kv, num_sms, L, nullptr,
+                                                       nullptr, stream);
     }
 }
 

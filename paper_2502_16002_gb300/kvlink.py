@@ -28,6 +28,7 @@ KVLINK_EDEVICE = -6
 KVLINK_SEG_PREFIX, KVLINK_SEG_DOC, KVLINK_SEG_LINK, KVLINK_SEG_QUESTION = 0, 1, 2, 3
 KVLINK_LAYOUT_INTERLEAVED, KVLINK_LAYOUT_LINKS_AT_END = 0, 1
 KVLINK_SRC_POOL, KVLINK_SRC_FRESH = 0, 1
+KVLINK_STATUS_WAIT_TIMEOUT, KVLINK_STATUS_COPY_TIMEOUT = 0x41, 0x21
 
 
 class kvlink_batch_desc_t(C.Structure):
@@ -101,8 +102,10 @@ def _load():
         "kvlink_linked_prefill": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_linked_prefill_fused": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_linked_prefill_layers": (C.c_int, [P, C.c_int32, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
+        "kvlink_reencode_concat_layers": (C.c_int, [P, C.c_int32, V, V, V, V, V]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
+        "kvlink_selftest_wait_timeout": (C.c_int, [C.c_uint32, V]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -121,6 +124,8 @@ DECLARED = [
     "kvlink_device_status", "kvlink_clear_device_status", "kvlink_strerror",
     "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc", "kvlink_rope_fresh",
     "kvlink_plan_get_sources", "kvlink_linked_prefill_fused", "kvlink_linked_prefill_layers",
+    "kvlink_reencode_concat_layers",
+    "kvlink_selftest_wait_timeout",
 ]
 
 # size of the static scratch used by kvlink_suffix_attention_noalloc (include/kvlink.h)
@@ -296,6 +301,16 @@ def kvlink_linked_prefill_layers(plan: Plan, pool_k, pool_v, q, k_new, v_new, ca
                                             workspace_bytes, stream), "kvlink_linked_prefill_layers")
 
 
+def kvlink_reencode_concat_layers(plan: Plan, pool_k, pool_v, cache_k, cache_v, stream: int = 0) -> None:
+    """Every argument but the plan and stream: a sequence of per-layer device pointers."""
+    n = len(pool_k)
+    arrs = [_ptr_array(x) for x in (pool_k, pool_v, cache_k, cache_v)]
+    if any(len(a) != n for a in arrs):
+        raise ValueError("every per-layer pointer list needs one entry per layer")
+    _check(lib.kvlink_reencode_concat_layers(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs], stream),
+           "kvlink_reencode_concat_layers")
+
+
 def kvlink_device_status() -> int:
     s = C.c_int32(0)
     _check(lib.kvlink_device_status(C.byref(s)), "kvlink_device_status")
@@ -304,3 +319,7 @@ def kvlink_device_status() -> int:
 
 def kvlink_clear_device_status() -> None:
     _check(lib.kvlink_clear_device_status(), "kvlink_clear_device_status")
+
+
+def kvlink_selftest_wait_timeout(limit_ms: int, stream: int = 0) -> None:
+    _check(lib.kvlink_selftest_wait_timeout(int(limit_ms), stream), "kvlink_selftest_wait_timeout")

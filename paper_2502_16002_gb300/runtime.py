@@ -118,6 +118,11 @@ class LinkedPrefill:
         K.kvlink_linked_prefill_layers(self.plan, *ptrs, self.workspace.data_ptr(), self.workspace.numel(),
                                        _stream_handle(stream))
 
+    def reencode_concat_layers(self, pool_k, pool_v, cache_k, cache_v, stream=None):
+        """The document caches of all layers in one launch (sequences of per-layer tensors)."""
+        ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, cache_k, cache_v)]
+        K.kvlink_reencode_concat_layers(self.plan, *ptrs, _stream_handle(stream))
+
     def linked_prefill_layers_from_host(self, pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new,
                                         cache_k, cache_v, out, h_out, streams=None):
         """Every layer of the linked prefill with the fresh rows in host memory.

@@ -1,6 +1,8 @@
-"""GPU check of the all-layers call: for every layer it must give exactly (bit for bit)
-what the per-layer kvlink_linked_prefill gives; one query of the last layer is also
-checked against the fp64 oracle.
+"""GPU check of the all-layers calls.  kvlink_linked_prefill_layers must give, for every
+layer, exactly (bit for bit) what the per-layer kvlink_linked_prefill gives, and
+kvlink_reencode_concat_layers exactly what kvlink_reencode_concat gives per layer,
+including across the kernel's per-launch layer limit; one query of the last layer is
+also checked against the fp64 oracle.
 """
 import numpy as np
 import pytest
@@ -29,8 +31,8 @@ def _sentinel_cache(lp):
     return ck, cv
 
 
-@pytest.mark.parametrize("cfg_index,n_layers", [(2, 3), (5, 2)])
-def test_all_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers):
+@pytest.mark.parametrize("cfg_index,n_layers,layout", [(2, 3, 0), (5, 2, 0), (3, 2, 1)])
+def test_all_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers, layout):
     from paper_2502_16002_gb300 import kvlink as K
     dev = torch.device("cuda:0")
     batch = W.draw_batch(W.get_config(cfg_index))
@@ -41,7 +43,7 @@ def test_all_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers):
         raw.append((a, b, x, y, z))
         for lst, arr in zip((pk, pv, q, kn, vn), (a, b, x, y, z)):
             lst.append(RT.bf16_from_bits(arr, dev))
-    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev, layout=layout)
     caches = [_sentinel_cache(lp) for _ in range(n_layers)]
     outs = [torch.full_like(x, float("nan")) for x in q]
     lp.linked_prefill_layers(pk, pv, q, kn, vn, [c[0] for c in caches], [c[1] for c in caches], outs)
@@ -57,4 +59,29 @@ def test_all_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers):
     last = n_layers - 1
     gk, gv = RT.bits_from_bf16(caches[last][0]), RT.bits_from_bf16(caches[last][1])
     gout = outs[last].float().cpu().numpy().astype(np.float64)
-    check_query(batch, 0, lp, gk, gv, gout, raw[last])
+    check_query(batch, 0, lp, gk, gv, gout, raw[last], layout=layout)
+
+
+@pytest.mark.parametrize("cfg_index,n_layers", [(1, 70), (2, 5), (5, 3)])
+def test_reencode_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers):
+    """70 layers of the two-document workload cross the 64-layers-per-launch limit; the
+    paged pool (workload 5) resolves its block tables per unit."""
+    from paper_2502_16002_gb300 import kvlink as K
+    dev = torch.device("cuda:0")
+    batch = W.draw_batch(W.get_config(cfg_index))
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    c = batch.cfg
+    shape = ((batch.pool_rows // c.pool_block_size, c.pool_block_size, c.h_kv, c.head_dim) if c.pool_block_size
+             else (batch.pool_rows, c.h_kv, c.head_dim))
+    pk = [W.normal_bf16_torch(shape, 7000 + 2 * l, dev) for l in range(n_layers)]
+    pv = [W.normal_bf16_torch(shape, 7001 + 2 * l, dev) for l in range(n_layers)]
+    caches = [_sentinel_cache(lp) for _ in range(n_layers)]
+    lp.reencode_concat_layers(pk, pv, [c[0] for c in caches], [c[1] for c in caches])
+    torch.cuda.synchronize()
+    for layer in range(n_layers):
+        ck, cv = _sentinel_cache(lp)
+        lp.reencode_concat(pk[layer], pv[layer], ck, cv)
+        torch.cuda.synchronize()
+        assert torch.equal(caches[layer][0].view(torch.int16), ck.view(torch.int16)), layer
+        assert torch.equal(caches[layer][1].view(torch.int16), cv.view(torch.int16)), layer
+    assert K.kvlink_device_status() == 0
