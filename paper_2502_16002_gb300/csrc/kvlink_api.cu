@@ -178,6 +178,7 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     };
     put(p->off_seg, p->seg.data(), p->seg.size() * sizeof(kvlink_segment_t));
     put(p->off_chunks, p->chunks.data(), p->chunks.size() * sizeof(CopyChunk));
+    put(p->off_chunks_sorted, p->chunks_sorted.data(), p->chunks_sorted.size() * sizeof(CopyChunk));
     put(p->off_pool_start, p->pool_start.data(), p->pool_start.size() * sizeof(int64_t));
     put(p->off_pool_bt, p->pool_block_table.data(), p->pool_block_table.size() * sizeof(int32_t));
     put(p->off_cu_ctx, p->cu_ctx.data(), p->cu_ctx.size() * sizeof(int64_t));
@@ -202,6 +203,7 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     DevicePlan& d = p->dev;
     d.seg = (const kvlink_segment_t*)(b + p->off_seg);
     d.chunks = (const CopyChunk*)(b + p->off_chunks);
+    d.chunks_sorted = (const CopyChunk*)(b + p->off_chunks_sorted);
     d.rope = (const float4*)(b + p->off_rope);
     d.pool_start = (const int64_t*)(b + p->off_pool_start);
     d.pool_block_table = (const int32_t*)(b + p->off_pool_bt);
@@ -261,8 +263,8 @@ int kvlink_reencode_concat_layers(const kvlink_plan_t* p, int32_t n_layers, cons
 static int place_fresh(const kvlink_plan_t* p, const void* k_new, const void* v_new, void* cache_k,
                        void* cache_v, cudaStream_t s) {
     const int n_all = (int)p->chunks.size();
-    launch_reencode(p->dev, p->n_chunks_cached, n_all - p->n_chunks_cached, p->head_dim, p->h_kv,
-                    p->num_sms, nullptr, nullptr, k_new, v_new, cache_k, cache_v, s);
+    launch_reencode(p->dev, p->n_chunks_cached, n_all - p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms,
+                    nullptr, nullptr, k_new, v_new, cache_k, cache_v, s);
     return check_launch("fresh placement");
 }
 

@@ -79,6 +79,7 @@ static_assert(sizeof(MergeGroup) == 32, "MergeGroup layout");
 struct DevicePlan {
     const kvlink_segment_t* seg;
     const CopyChunk* chunks;     // cached-segment chunks first, then fresh-segment chunks
+    const CopyChunk* chunks_sorted;  // the cached chunks by source row (all-layer re-encode)
     const float4* rope;          // [n_rope_rows][D/2] (cos hi, cos lo, sin hi, sin lo)
     const int64_t* pool_start;   // [pool_docs]
     const int32_t* pool_block_table;
@@ -121,6 +122,7 @@ struct kvlink_plan {
     std::vector<kvlink_segment_t> seg;
     std::vector<kvlink::CopyChunk> chunks;
     int32_t n_chunks_cached = 0;
+    std::vector<kvlink::CopyChunk> chunks_sorted;   // the cached chunks by source row
     int32_t n_rope_rows = 0;
     std::vector<int64_t> cu_ctx;
     std::vector<int32_t> cu_fresh;
@@ -136,6 +138,7 @@ struct kvlink_plan {
     int64_t attn_pairs = 0;
 
     // layout of the device buffer (byte offsets) and its total size
+    size_t off_chunks_sorted = 0;
     size_t off_seg = 0, off_chunks = 0, off_rope = 0, off_pool_start = 0, off_pool_bt = 0,
            off_cu_ctx = 0, off_cu_fresh = 0, off_fresh_pos = 0, off_fresh_query = 0,
            off_items = 0, off_merges = 0, off_src = 0, off_cu_grp = 0, off_grp_src = 0, off_src_row = 0,

@@ -248,7 +248,13 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         }
         if (pass == 0) p->n_chunks_cached = (int32_t)p->chunks.size();
     }
-
+    // the cached chunks ordered by source row, for the all-layer re-encode: the chunks of a
+    // document that several queries retrieved become adjacent, and the kernel loads their
+    // rows once for all destinations
+    p->chunks_sorted.assign(p->chunks.begin(), p->chunks.begin() + p->n_chunks_cached);
+    std::stable_sort(p->chunks_sorted.begin(), p->chunks_sorted.end(), [](const CopyChunk& a, const CopyChunk& b) {
+        return a.src_row != b.src_row ? a.src_row < b.src_row : a.n < b.n;
+    });
     // ---- attention work items
     // M-tiles of one (query, KV head) cut the query's fresh tokens into runs of kAttnBM / G
     // tokens counted back from the last one, the remainder going to the first run: a tile's
@@ -349,6 +355,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
     p->off_seg = take(p->seg.size() * sizeof(kvlink_segment_t));
     p->off_chunks = take(p->chunks.size() * sizeof(CopyChunk));
+    p->off_chunks_sorted = take(p->chunks_sorted.size() * sizeof(CopyChunk));
     p->off_rope = take((size_t)p->n_rope_rows * (d->head_dim / 2) * sizeof(float4));
     p->off_pool_start = take(p->pool_start.size() * sizeof(int64_t));
     p->off_pool_bt = take(p->pool_block_table.size() * sizeof(int32_t));

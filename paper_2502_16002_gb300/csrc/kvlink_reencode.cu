@@ -3,9 +3,11 @@
 //
 // The re-encode kernel is a streaming copy bound by HBM bandwidth.  Work units are
 // runs of tokens whose K/V rows are contiguous in the source and in the linked
-// cache (resolved on the host).  A persistent CTA per SM pipelines its units
-// through a 3-stage shared-memory ring with bulk (TMA) copies: global -> shared
-// loads, an in-place rotation of the document keys, shared -> global stores.
+// cache (resolved on the host).  A persistent CTA per SM pipelines a contiguous range
+// of units through a 3-stage shared-memory ring: one bulk (TMA) global -> shared load
+// per group of consecutive units that read the same rows, document keys rotated on
+// their way from shared memory to global memory, values and unrotated keys
+// bulk-stored from shared memory.
 //
 // The rotation itself (double-float cos/sin, compensated products) is in
 // kvlink_rope.cuh, shared with the fused linked-prefill kernel.
@@ -104,13 +106,29 @@ struct LayerPtrs {
 };
 constexpr int kMaxLayersPerLaunch = 64;     // 2 KB of kernel parameters
 
-// Work unit u = layer * n_chunks + c.  CTA b handles the contiguous range of units
-// [n*b/grid, n*(b+1)/grid), n = n_layers * n_chunks.
-// Producer (warp 0, one thread): bulk-loads a unit's K rows and V rows into a stage.
-// Consumers (warps 1-4): rotate the unit's keys in place when it is a document (each
-// thread keeps a fixed (head, j0) slot and its eight double-float cos/sin pairs), then
-// one thread bulk-stores K and V to the linked cache and frees the stage once the
-// stores have read it.  V is never touched by the threads.
+// Chunk u = layer * n_chunks + c of the flattened range.  CTA b handles the contiguous
+// range [n*b/grid, n*(b+1)/grid), n = n_layers * n_chunks, in groups of consecutive
+// chunks that read the same source rows (same layer, same tensor, same first row and
+// length), loading each group's rows once.  The one-layer launches take the chunks in
+// linked-cache order (consecutive chunks never share rows); the all-layer launch takes
+// the document chunks sorted by pool row, so every destination of a document that
+// several queries retrieved follows the first and its rows are loaded once per layer.
+// (One layer is bound by the cache writes, which do not shrink; over all layers the
+// saved reads pay: measured 1607 -> 1314 us for 32 layers of the Llama-8B batch-8
+// workload, while grouping one layer's chunks moved its time from 50 to 53 us.)
+// Producer (warp 0, one thread): bulk-loads a group's K rows and V rows into a stage.
+// Consumers (warps 1-4), per chunk of the group: document keys are read from the stage,
+// rotated by the chunk's delta in registers (each thread keeps a fixed (head, j0) slot
+// and its eight double-float cos/sin pairs) and written with 16-byte global stores;
+// one thread bulk-stores the values (and the keys of prefix and fresh chunks, which are
+// not rotated) straight from the stage.  The stage is freed once the group's stores
+// have read it and every consumer has passed the next group's barrier.
+__device__ __forceinline__ bool same_source(const CopyChunk& a, int la, const CopyChunk& b, int lb) {
+    const bool fa = a.kind == KVLINK_SEG_LINK || a.kind == KVLINK_SEG_QUESTION;
+    const bool fb = b.kind == KVLINK_SEG_LINK || b.kind == KVLINK_SEG_QUESTION;
+    return la == lb && fa == fb && a.src_row == b.src_row && a.n == b.n;
+}
+
 template <int D, int MAXL>
 __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     const CopyChunk* __restrict__ chunks, int n_chunks, int n_layers, const float4* __restrict__ rope, int h_kv,
@@ -126,8 +144,20 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     const int64_t n_units = (int64_t)n_chunks * n_layers;
     const int c_begin = (int)(n_units * blockIdx.x / gridDim.x);
     const int c_end = (int)(n_units * (blockIdx.x + 1) / gridDim.x);
+
     const int64_t row_elems = (int64_t)h_kv * D;
     const uint32_t row_bytes = (uint32_t)(row_elems * 2);
+    auto layer_of = [&](int c) { return MAXL == 1 ? 0 : c / n_chunks; };
+    // the end of the group that starts at chunk c
+    auto group_end = [&](int c, int layer, const CopyChunk& ch) {
+        int e = c + 1;
+        while (e < c_end) {
+            const int le = layer_of(e);
+            if (!same_source(chunks[e - le * n_chunks], le, ch, layer)) break;
+            ++e;
+        }
+        return e;
+    };
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kCopyStages; ++i) {
@@ -144,11 +174,11 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
         // ------------------------------------------------------------ producer
         if (threadIdx.x == 0) {
             int issued = 0;
-            for (int c = c_begin, i = 0; c < c_end; ++c, ++i) {
-                const int st = i % kCopyStages;
-                if (!copy_wait(empty + st, ((i / kCopyStages) & 1) ^ 1, abort_flag)) break;
-                const int layer = MAXL == 1 ? 0 : c / n_chunks;
+            for (int c = c_begin, g = 0; c < c_end; ++g) {
+                const int layer = layer_of(c);
                 const CopyChunk ch = chunks[c - layer * n_chunks];
+                const int st = g % kCopyStages;
+                if (!copy_wait(empty + st, ((g / kCopyStages) & 1) ^ 1, abort_flag)) break;
                 const bool fresh = ch.kind == KVLINK_SEG_LINK || ch.kind == KVLINK_SEG_QUESTION;
                 const __nv_bfloat16* sk = (fresh ? k_new : L.pool_k[layer]) + ch.src_row * row_elems;
                 const __nv_bfloat16* sv = (fresh ? v_new : L.pool_v[layer]) + ch.src_row * row_elems;
@@ -157,7 +187,8 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
                 mbar_arrive_expect_tx(full + st, 2 * bytes);
                 bulk_load(stage, sk, bytes, full + st);
                 bulk_load(stage + kCopyStageBytes, sv, bytes, full + st);
-                issued = i + 1;
+                issued = g + 1;
+                c = group_end(c, layer, ch);
             }
             // no load may still be in flight when the CTA leaves
             for (int i = issued - kCopyStages > 0 ? issued - kCopyStages : 0; i < issued; ++i)
@@ -178,40 +209,46 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     const uint32_t lo_off = (uint32_t)(head * D + j0) * 2;
     int cur_table = -1;
     float4 cs[8];
-    for (int c = c_begin, i = 0; c < c_end; ++c, ++i) {
-        const int st = i % kCopyStages;
-        copy_wait(full + st, (i / kCopyStages) & 1, abort_flag);
-        named_bar_sync(1, kCopyConsumers);
-        if (*abort_flag) break;  // uniform: every consumer passed the barrier first
-        const int layer = MAXL == 1 ? 0 : c / n_chunks;
-        const CopyChunk ch = chunks[c - layer * n_chunks];
-        uint8_t* stage = smem + st * CopySmem::STAGE;
-        if (ch.kind == KVLINK_SEG_DOC) {
-            if (ch.table != cur_table) {
-                const float4* t = rope + (int64_t)ch.table * (D / 2) + j0;
+    for (int c = c_begin, g = 0; c < c_end; ++g) {
+        const int layer = layer_of(c);
+        const CopyChunk ch0 = chunks[c - layer * n_chunks];
+        const int c1 = group_end(c, layer, ch0);
+        const int st = g % kCopyStages;
+        copy_wait(full + st, (g / kCopyStages) & 1, abort_flag);
+        named_bar_sync(1, kCopyConsumers);     // every consumer is done with the previous group
+        if (*abort_flag) break;                // uniform: every consumer passed the barrier first
+        const uint8_t* stage = smem + st * CopySmem::STAGE;
+        const uint32_t bytes = (uint32_t)ch0.n * row_bytes;
+        for (int cc = c; cc < c1; ++cc) {
+            const CopyChunk ch = chunks[cc - layer * n_chunks];
+            if (ch.kind == KVLINK_SEG_DOC) {
+                if (ch.table != cur_table) {
+                    const float4* t = rope + (int64_t)ch.table * (D / 2) + j0;
 #pragma unroll
-                for (int q = 0; q < 8; ++q) cs[q] = __ldg(t + q);
-                cur_table = ch.table;
+                    for (int q = 0; q < 8; ++q) cs[q] = __ldg(t + q);
+                    cur_table = ch.table;
+                }
+                uint8_t* dst = reinterpret_cast<uint8_t*>(L.cache_k[layer] + ch.dst_row * row_elems) + lo_off;
+                for (int t = tok0; t < ch.n; t += TPP) {
+                    const uint8_t* src = stage + (uint32_t)t * row_bytes + lo_off;
+                    uint4 a = *reinterpret_cast<const uint4*>(src);
+                    uint4 b = *reinterpret_cast<const uint4*>(src + D);
+                    rotate8(a, b, cs);
+                    uint8_t* d = dst + (size_t)t * row_bytes;
+                    *reinterpret_cast<uint4*>(d) = a;
+                    *reinterpret_cast<uint4*>(d + D) = b;
+                }
+            } else if (tc == 0) {
+                bulk_store(L.cache_k[layer] + ch.dst_row * row_elems, stage, bytes);
             }
-            for (int t = tok0; t < ch.n; t += TPP) {
-                uint4* lo = reinterpret_cast<uint4*>(stage + (uint32_t)t * row_bytes + lo_off);
-                uint4* hi = reinterpret_cast<uint4*>(stage + (uint32_t)t * row_bytes + lo_off + D);
-                uint4 a = *lo, b = *hi;
-                rotate8(a, b, cs);
-                *lo = a;
-                *hi = b;
-            }
-            fence_proxy_async_smem();  // the bulk store reads these writes through the async proxy
+            if (tc == 0) bulk_store(L.cache_v[layer] + ch.dst_row * row_elems, stage + kCopyStageBytes, bytes);
         }
-        named_bar_sync(1, kCopyConsumers);
         if (tc == 0) {
-            const uint32_t bytes = (uint32_t)ch.n * row_bytes;
-            bulk_store(L.cache_k[layer] + ch.dst_row * row_elems, stage, bytes);
-            bulk_store(L.cache_v[layer] + ch.dst_row * row_elems, stage + kCopyStageBytes, bytes);
             bulk_commit();
-            bulk_wait_read<1>();  // the previous unit's stores have read their stage
-            if (i > 0) mbar_arrive(empty + (i - 1) % kCopyStages);
+            bulk_wait_read<1>();  // the previous group's stores have read their stage
+            if (g > 0) mbar_arrive(empty + (g - 1) % kCopyStages);
         }
+        c = c1;
     }
     if (tc == 0) bulk_wait<0>();
 }
@@ -245,7 +282,7 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
         launch_reencode_t<64, 1>(ch, n_chunks, 1, P.rope, h_kv, num_sms, L, k_new, v_new, stream);
 }
 
-// The document chunks [0, n_chunks) of n_layers layers, kMaxLayersPerLaunch layers per launch.
+// The document chunks (sorted by source) of n_layers layers, kMaxLayersPerLaunch layers per launch.
 void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int h_kv, int num_sms, int n_layers,
                             const void* const* pool_k, const void* const* pool_v, void* const* cache_k,
                             void* const* cache_v, cudaStream_t stream) {
@@ -263,11 +300,11 @@ void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int
             L.cache_v[l] = (bf*)cache_v[l0 + l];
         }
         if (head_dim == 128)
-            launch_reencode_t<128, kMaxLayersPerLaunch>(P.chunks, n_chunks, nl, P.rope, h_kv, num_sms, L, nullptr,
-                                                        nullptr, stream);
+            launch_reencode_t<128, kMaxLayersPerLaunch>(P.chunks_sorted, n_chunks, nl, P.rope, h_kv, num_sms, L,
+                                                        nullptr, nullptr, stream);
         else
-            launch_reencode_t<64, kMaxLayersPerLaunch>(P.chunks, n_chunks, nl, P.rope, h_kv, num_sms, L, nullptr,
-                                                       nullptr, stream);
+            launch_reencode_t<64, kMaxLayersPerLaunch>(P.chunks_sorted, n_chunks, nl, P.rope, h_kv, num_sms, L,
+                                                       nullptr, nullptr, stream);
     }
 }
 
