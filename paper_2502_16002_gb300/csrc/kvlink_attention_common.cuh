@@ -239,37 +239,50 @@ __device__ __forceinline__ void softmax_role(const AttnItem& it, const DevicePla
         tmem_ld32(s_col + 96, *reinterpret_cast<uint32_t(*)[32]>(s + 96));
         tmem_ld_wait();
 
-        // raw row max (scale > 0 commutes with max); masked keys become -inf.  Eight
-        // independent running maxima keep the dependency chain short.  A tile lies in one
-        // run of rows (cached rows, or the fresh rows at the end), where the visible keys
-        // are those below one limit; only a tile holding the end of the cached rows and the
-        // start of the fresh rows needs both comparisons.
+        // raw row max (scale > 0 commutes with max).  A tile lies in one run of rows (cached
+        // rows, or the fresh rows at the end), where a row sees the keys below one limit, so
+        // for each row the tile is fully visible, fully masked, or holds the row's limit.
+        // Only the last case needs a per-column select (a compare and select per column
+        // cost ~800 cycles a tile on the softmax warps), and a warp takes that path only
+        // when one of its rows has its limit in the tile; a fully masked row instead drops
+        // its max and gets p = 0 from an infinite exponent offset.  Only a tile holding the
+        // end of the cached rows and the start of the fresh rows compares twice per column.
         const int key0 = item_tile(it, it.kv_tile0 + j) * kAttnBN;
         float mx8[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
+        constexpr uint32_t kNegInf = 0xff800000u;
+        bool dead = false;  // the row sees no key of this tile
+        bool plain = true;
         if (key0 + kAttnBN > it.min_vis) {  // some row of the tile may not see every key
             if (key0 + kAttnBN <= F || key0 >= F) {
-                const int lim = key0 >= F ? F + (int)vis_b : vis_a;
+                const int nv = (key0 >= F ? F + (int)vis_b : vis_a) - key0;  // columns [0, nv) visible
+                dead = nv <= 0;
+                if (__any_sync(0xffffffffu, nv > 0 && nv < kAttnBN)) {
+                    plain = false;
 #pragma unroll
-                for (int c = 0; c < 128; ++c) {
-                    if (key0 + c >= lim) s[c] = __float_as_uint(-INFINITY);
-                    mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
+                    for (int c = 0; c < 128; ++c) {
+                        s[c] = c < nv ? s[c] : kNegInf;
+                        mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
+                    }
                 }
             } else {
+                plain = false;
 #pragma unroll
                 for (int c = 0; c < 128; ++c) {
                     const int kr = key0 + c;
-                    if (!(kr < vis_a || (uint32_t)(kr - F) < vis_b)) s[c] = __float_as_uint(-INFINITY);
+                    if (!(kr < vis_a || (uint32_t)(kr - F) < vis_b)) s[c] = kNegInf;
                     mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
                 }
             }
-        } else {
+        }
+        if (plain) {
 #pragma unroll
             for (int c = 0; c < 128; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(s[c]));
         }
-        const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                               fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+        const float mx = dead ? -INFINITY
+                              : fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                      fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
         const float m_new = fmaxf(m, mx * scale_log2);
         const bool resc = m_new > m + kRescaleThreshold;
         float alpha = 1.f;
@@ -295,7 +308,8 @@ __device__ __forceinline__ void softmax_role(const AttnItem& it, const DevicePla
         }
         // p = exp2(s * scale - m) on column pairs (packed f32x2 arithmetic); pairs with
         // (c % 8) >= KVLINK_EXP_POLY_FROM go to the FMA pipe (exp2_poly2), the rest to MUFU
-        const float mu = (m == -INFINITY) ? 0.f : m;
+        // a fully masked row: s * scale - inf = -inf, so every p is 0
+        const float mu = dead ? INFINITY : ((m == -INFINITY) ? 0.f : m);
         const uint64_t sc2 = f2_pack(scale_log2, scale_log2);
         const uint64_t nmu2 = f2_pack(-mu, -mu);
         uint64_t acc[4];
