@@ -48,7 +48,7 @@ UNIT = "us/query"
 # summaries under profiles/, keyed by (kernel, workload); None until captured for
 # the current kernel version.
 NCU_TRAFFIC = {
-    ("attention", 3): 263778816,   # profiles/attention_tc_llama8b_b8_zipf.md
+    ("attention", 3): 259171328,   # profiles/attention_tc_llama8b_b8_zipf.md
     ("reencode", 3): 228434176,    # profiles/reencode_llama8b_b8_zipf.md
 }
 
