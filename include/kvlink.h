@@ -162,6 +162,14 @@ typedef struct {
  * result is deterministic.  On success *out owns host memory until
  * kvlink_plan_destroy.  Errors: EINVAL, EBOUNDS, EUNSUPPORTED. */
 int kvlink_plan_create(const kvlink_batch_desc_t* desc, kvlink_plan_t** out);
+/* Rebuild an existing plan for another batch, as kvlink_plan_create would, reusing the
+ * plan's host storage: a serving loop that keeps one plan per stream avoids allocating
+ * (and first touching) its per-position tables for every batch.  The plan must be
+ * uploaded again before use; device work already enqueued with the old tables is not
+ * affected (kvlink_plan_upload orders its copy after it on the upload's stream).  On error
+ * the plan holds no batch: rebuild it or destroy it.  Errors: as kvlink_plan_create. */
+int kvlink_plan_rebuild(kvlink_plan_t* plan, const kvlink_batch_desc_t* desc);
+/* Waits for the plan's last upload copy, then frees its host memory. */
 void kvlink_plan_destroy(kvlink_plan_t* plan);
 int kvlink_plan_get_info(const kvlink_plan_t* plan, kvlink_plan_info_t* info);
 
@@ -183,8 +191,10 @@ int kvlink_plan_get_sources(const kvlink_plan_t* plan, kvlink_source_t* src, int
  * delta_i * theta^(-2j/D) for every cached document i and j < D/2, with the angle
  * formed and reduced in float64 and stored as float32 (Sec. 2.2; done once per
  * batch, shared by all layers).  The plan records d_buf; later calls read it.
- * d_buf must stay valid, and the plan alive, until the last call using them has
- * completed on the device.  Errors: EINVAL, ECAPACITY, ECUDA. */
+ * Asynchronous: the tables go through a pinned staging buffer owned by the plan, and the
+ * call returns once the copy is enqueued (a later upload of the same plan first waits for
+ * it).  d_buf must stay valid, and the plan alive, until the last call using them has
+ * completed on the device.  Errors: EINVAL (not built), ECAPACITY, ECUDA. */
 int kvlink_plan_upload(kvlink_plan_t* plan, double theta, void* d_buf, size_t bytes,
                        kvlink_stream_t stream);
 

@@ -94,6 +94,39 @@ const char* kvlink_strerror(int code) {
 
 const char* kvlink_last_cuda_error(void) { return g_last_cuda_error.c_str(); }
 
+namespace kvlink {
+PinnedStaging::~PinnedStaging() {
+    // errors are ignored: at process exit the runtime may already be gone
+    if (done) {
+        cudaEventSynchronize(done);
+        cudaEventDestroy(done);
+    }
+    if (ptr) cudaFreeHost(ptr);
+}
+
+// Room for `bytes` in the staging buffer, once the last copy out of it has completed.
+static int staging_reserve(PinnedStaging& st, size_t bytes) {
+    if (st.done) {
+        cudaError_t e = cudaEventSynchronize(st.done);
+        if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload: previous copy");
+    } else {
+        cudaError_t e = cudaEventCreateWithFlags(&st.done, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload: event");
+    }
+    if (st.bytes >= bytes) return KVLINK_OK;
+    if (st.ptr) cudaFreeHost(st.ptr);
+    st.ptr = nullptr;
+    st.bytes = 0;
+    void* h = nullptr;
+    cudaError_t e = cudaHostAlloc(&h, bytes, cudaHostAllocDefault);
+    if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload: pinned staging");
+    std::memset(h, 0, bytes);
+    st.ptr = (char*)h;
+    st.bytes = bytes;
+    return KVLINK_OK;
+}
+}  // namespace kvlink
+
 int kvlink_plan_create(const kvlink_batch_desc_t* desc, kvlink_plan_t** out) {
     if (!desc || !out) return KVLINK_EINVAL;
     *out = nullptr;
@@ -110,8 +143,36 @@ int kvlink_plan_create(const kvlink_batch_desc_t* desc, kvlink_plan_t** out) {
         delete p;
         return rc;
     }
+    p->built = true;
     *out = p;
     return KVLINK_OK;
+}
+
+int kvlink_plan_rebuild(kvlink_plan_t* p, const kvlink_batch_desc_t* desc) {
+    if (!p || !desc) return KVLINK_EINVAL;
+    // a fresh plan that takes over the old one's table storage (cleared, capacity kept, so
+    // the tables are rebuilt in memory that is already mapped) and its staging buffer
+    kvlink_plan q;
+    q.staging = std::move(p->staging);
+#define KVLINK_RECYCLE(m) \
+    q.m.swap(p->m);       \
+    q.m.clear();
+    KVLINK_RECYCLE(pool_start) KVLINK_RECYCLE(pool_len) KVLINK_RECYCLE(pool_block_table) KVLINK_RECYCLE(seg)
+    KVLINK_RECYCLE(chunks) KVLINK_RECYCLE(chunks_sorted) KVLINK_RECYCLE(cu_ctx) KVLINK_RECYCLE(cu_fresh)
+    KVLINK_RECYCLE(fresh_pos) KVLINK_RECYCLE(fresh_query) KVLINK_RECYCLE(src) KVLINK_RECYCLE(src_row)
+    KVLINK_RECYCLE(fresh_vis) KVLINK_RECYCLE(fresh_row0) KVLINK_RECYCLE(cu_grp) KVLINK_RECYCLE(grp_src)
+    KVLINK_RECYCLE(items) KVLINK_RECYCLE(merges)
+#undef KVLINK_RECYCLE
+    std::string why;
+    int rc;
+    try {
+        rc = build_plan(desc, resolve_num_sms(desc->num_sms), &q, &why);
+    } catch (...) {
+        rc = KVLINK_ECAPACITY;
+    }
+    q.built = rc == KVLINK_OK;
+    *p = std::move(q);
+    return rc;
 }
 
 void kvlink_plan_destroy(kvlink_plan_t* plan) { delete plan; }
@@ -172,9 +233,12 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     if (!(theta > 1.0)) return KVLINK_EINVAL;
     if (((uintptr_t)d_buf & 255u) != 0) return KVLINK_EINVAL;
     if (bytes < p->device_bytes) return KVLINK_ECAPACITY;
-    std::vector<char> host(p->device_bytes, 0);
+    if (!p->built) return KVLINK_EINVAL;
+    int rc = staging_reserve(p->staging, p->device_bytes);
+    if (rc != KVLINK_OK) return rc;
+    char* host = p->staging.ptr;
     auto put = [&](size_t off, const void* src, size_t n) {
-        if (n) std::memcpy(host.data() + off, src, n);
+        if (n) std::memcpy(host + off, src, n);
     };
     put(p->off_seg, p->seg.data(), p->seg.size() * sizeof(kvlink_segment_t));
     put(p->off_chunks, p->chunks.data(), p->chunks.size() * sizeof(CopyChunk));
@@ -194,11 +258,11 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     put(p->off_fresh_vis, p->fresh_vis.data(), p->fresh_vis.size() * sizeof(int32_t));
     put(p->off_fresh_row0, p->fresh_row0.data(), p->fresh_row0.size() * sizeof(int32_t));
     cudaStream_t s = (cudaStream_t)stream;
-    cudaError_t e = cudaMemcpyAsync(d_buf, host.data(), p->device_bytes, cudaMemcpyHostToDevice, s);
+    cudaError_t e = cudaMemcpyAsync(d_buf, host, p->device_bytes, cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload copy");
-    // pageable source: wait so that `host` may be released on return
-    e = cudaStreamSynchronize(s);
-    if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload sync");
+    // asynchronous: the next upload (or the plan's destruction) waits for this copy
+    e = cudaEventRecord(p->staging.done, s);
+    if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload event");
     char* b = (char*)d_buf;
     DevicePlan& d = p->dev;
     d.seg = (const kvlink_segment_t*)(b + p->off_seg);
@@ -220,7 +284,7 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     d.fresh_vis = (const int32_t*)(b + p->off_fresh_vis);
     d.fresh_row0 = (const int32_t*)(b + p->off_fresh_row0);
     launch_rope_table(d.seg, (int)p->seg.size(), (float4*)(b + p->off_rope), p->head_dim, theta, s);
-    int rc = check_launch("rope_table_kernel");
+    rc = check_launch("rope_table_kernel");
     if (rc != KVLINK_OK) return rc;
     p->theta = theta;
     p->d_buf = d_buf;

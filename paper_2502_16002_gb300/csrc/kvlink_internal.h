@@ -6,6 +6,7 @@
 #include <vector_types.h>
 
 #include <string>
+#include <utility>
 #include <vector>
 
 #include "kvlink.h"
@@ -107,6 +108,30 @@ constexpr int32_t kGrpRowMask = kGrpFresh - 1;
 
 }  // namespace kvlink
 
+namespace kvlink {
+// Pinned host buffer of the plan upload, reused by later uploads.  `done` is recorded on
+// the upload's stream after its copy; the buffer is rewritten only once it has completed.
+struct PinnedStaging {
+    char* ptr = nullptr;
+    size_t bytes = 0;
+    cudaEvent_t done = nullptr;
+    PinnedStaging() = default;
+    PinnedStaging(const PinnedStaging&) = delete;
+    PinnedStaging& operator=(const PinnedStaging&) = delete;
+    PinnedStaging(PinnedStaging&& o) noexcept { swap(o); }
+    PinnedStaging& operator=(PinnedStaging&& o) noexcept {
+        swap(o);
+        return *this;
+    }
+    ~PinnedStaging();
+    void swap(PinnedStaging& o) noexcept {
+        std::swap(ptr, o.ptr);
+        std::swap(bytes, o.bytes);
+        std::swap(done, o.done);
+    }
+};
+}  // namespace kvlink
+
 struct kvlink_plan {
     // scalars of the description
     int32_t batch = 0, n_link = 0, h_q = 0, h_kv = 0, head_dim = 0;
@@ -145,6 +170,9 @@ struct kvlink_plan {
            off_fresh_vis = 0, off_fresh_row0 = 0,
            device_bytes = 0;
     size_t workspace_bytes = 0;
+
+    bool built = false;                 // holds a batch (a failed rebuild clears it)
+    kvlink::PinnedStaging staging;
 
     // set by kvlink_plan_upload
     bool uploaded = false;

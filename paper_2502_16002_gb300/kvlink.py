@@ -103,6 +103,7 @@ def _load():
         "kvlink_linked_prefill_fused": (C.c_int, [P, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_linked_prefill_layers": (C.c_int, [P, C.c_int32, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_reencode_concat_layers": (C.c_int, [P, C.c_int32, V, V, V, V, V]),
+        "kvlink_plan_rebuild": (C.c_int, [P, C.POINTER(kvlink_batch_desc_t)]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
         "kvlink_selftest_wait_timeout": (C.c_int, [C.c_uint32, V]),
@@ -124,7 +125,7 @@ DECLARED = [
     "kvlink_device_status", "kvlink_clear_device_status", "kvlink_strerror",
     "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc", "kvlink_rope_fresh",
     "kvlink_plan_get_sources", "kvlink_linked_prefill_fused", "kvlink_linked_prefill_layers",
-    "kvlink_reencode_concat_layers",
+    "kvlink_reencode_concat_layers", "kvlink_plan_rebuild",
     "kvlink_selftest_wait_timeout",
 ]
 
@@ -173,9 +174,9 @@ class Plan:
         self.close()
 
 
-def kvlink_plan_create(*, n_link, h_q, h_kv, head_dim, pool_len, pool_start, pool_rows,
-                       prefix_doc, n_docs, doc_ids, q_len, pool_block_size=0,
-                       pool_block_table=None, num_sms=0, layout=KVLINK_LAYOUT_INTERLEAVED) -> Plan:
+def _batch_desc(n_link, h_q, h_kv, head_dim, pool_len, pool_start, pool_rows, prefix_doc, n_docs, doc_ids,
+                q_len, pool_block_size, pool_block_table, num_sms, layout):
+    """A kvlink_batch_desc_t and the arrays it points into (kept alive by the caller)."""
     arrs = dict(pool_len=_i32(pool_len), pool_start=_i64(pool_start), prefix_doc=_i32(prefix_doc),
                 n_docs=_i32(n_docs), doc_ids=_i32(doc_ids), q_len=_i32(q_len))
     bt = _i32(pool_block_table) if pool_block_table is not None else None
@@ -195,9 +196,25 @@ def kvlink_plan_create(*, n_link, h_q, h_kv, head_dim, pool_len, pool_start, poo
     d.q_len = _ptr(arrs["q_len"], C.c_int32)
     d.num_sms = int(num_sms)
     d.layout = int(layout)
+    return d, (arrs, bt)
+
+
+def kvlink_plan_create(*, n_link, h_q, h_kv, head_dim, pool_len, pool_start, pool_rows,
+                       prefix_doc, n_docs, doc_ids, q_len, pool_block_size=0,
+                       pool_block_table=None, num_sms=0, layout=KVLINK_LAYOUT_INTERLEAVED) -> Plan:
+    d, keep = _batch_desc(n_link, h_q, h_kv, head_dim, pool_len, pool_start, pool_rows, prefix_doc, n_docs,
+                          doc_ids, q_len, pool_block_size, pool_block_table, num_sms, layout)
     h = C.c_void_p()
     _check(lib.kvlink_plan_create(C.byref(d), C.byref(h)), "kvlink_plan_create")
     return Plan(h)
+
+
+def kvlink_plan_rebuild(plan: Plan, *, n_link, h_q, h_kv, head_dim, pool_len, pool_start, pool_rows,
+                        prefix_doc, n_docs, doc_ids, q_len, pool_block_size=0,
+                        pool_block_table=None, num_sms=0, layout=KVLINK_LAYOUT_INTERLEAVED) -> None:
+    d, keep = _batch_desc(n_link, h_q, h_kv, head_dim, pool_len, pool_start, pool_rows, prefix_doc, n_docs,
+                          doc_ids, q_len, pool_block_size, pool_block_table, num_sms, layout)
+    _check(lib.kvlink_plan_rebuild(plan.handle, C.byref(d)), "kvlink_plan_rebuild")
 
 
 def kvlink_plan_get_info(plan: Plan) -> kvlink_plan_info_t:

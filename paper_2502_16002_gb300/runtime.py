@@ -59,6 +59,26 @@ class LinkedPrefill:
                    pool_block_table=batch.pool_block_table, num_sms=num_sms, layout=layout,
                    device=device, stream=stream)
 
+    def rebuild_from_batch(self, batch, num_sms=0, stream=None, layout=K.KVLINK_LAYOUT_INTERLEAVED):
+        """Reuse this object for another batch: the plan is rebuilt in place (its host storage
+        reused) and uploaded into the same plan buffer and workspace when they are large
+        enough.  The upload is ordered after the work already enqueued on `stream`."""
+        cfg = batch.cfg
+        K.kvlink_plan_rebuild(self.plan, n_link=cfg.n_link, h_q=cfg.h_q, h_kv=cfg.h_kv, head_dim=cfg.head_dim,
+                              pool_len=batch.pool_len, pool_start=batch.pool_start, pool_rows=batch.pool_rows,
+                              prefix_doc=batch.prefix_doc, n_docs=batch.n_docs, doc_ids=batch.doc_ids,
+                              q_len=batch.q_len, pool_block_size=cfg.pool_block_size,
+                              pool_block_table=batch.pool_block_table, num_sms=num_sms, layout=layout)
+        self.info = K.kvlink_plan_get_info(self.plan)
+        self.theta = float(cfg.theta)
+        if int(self.info.device_bytes) > self.plan_buf.numel():
+            self.plan_buf = torch.empty(int(self.info.device_bytes), dtype=torch.uint8, device=self.device)
+        if int(self.info.workspace_bytes) > self.workspace.numel():
+            self.workspace = torch.empty(int(self.info.workspace_bytes), dtype=torch.uint8, device=self.device)
+        K.kvlink_plan_upload(self.plan, self.theta, self.plan_buf.data_ptr(), self.plan_buf.numel(),
+                             _stream_handle(stream))
+        return self
+
     def sources(self) -> np.ndarray:
         """Per-position sources (kvlink_source_t records) of the plan."""
         return K.kvlink_plan_get_sources(self.plan)
@@ -124,7 +144,7 @@ class LinkedPrefill:
         K.kvlink_reencode_concat_layers(self.plan, *ptrs, _stream_handle(stream))
 
     def linked_prefill_layers_from_host(self, pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new,
-                                        cache_k, cache_v, out, h_out, streams=None):
+                                        cache_k, cache_v, out, h_out, streams=None, wait=True):
         """Every layer of the linked prefill with the fresh rows in host memory.
 
         Per layer l: h_q[l], h_k_new[l], h_v_new[l] (pinned host tensors) are copied to
@@ -134,20 +154,33 @@ class LinkedPrefill:
         kernels of the layers around it.  Returns after the last output has arrived.
 
         streams: optional (input, compute, output) torch.cuda.Stream triple.
+        wait=False returns once everything is enqueued, so that the host can prepare the
+        next batch (e.g. rebuild_from_batch on the compute stream) while this one runs.
+        Calls on the same object then chain through per-layer events: a layer's inputs are
+        overwritten only after the previous call's kernels of that layer have read them, and
+        its output only after the previous call's copy of it to the host.
         """
         if streams is None:
             streams = (torch.cuda.Stream(self.device), torch.cuda.current_stream(self.device),
                        torch.cuda.Stream(self.device))
         s_in, s_c, s_out = streams
         n = len(pool_k)
+        prev = getattr(self, "_host_chain", None)
+        if prev is not None and len(prev[0]) != n:
+            prev = None
+        done_c, done_o = [], []
         for l in range(n):
             ev_in = torch.cuda.Event()
             with torch.cuda.stream(s_in):
+                if prev is not None:
+                    s_in.wait_event(prev[0][l])      # the previous call's layer l read q, k_new, v_new
                 q[l].copy_(h_q[l], non_blocking=True)
                 k_new[l].copy_(h_k_new[l], non_blocking=True)
                 v_new[l].copy_(h_v_new[l], non_blocking=True)
                 ev_in.record(s_in)
             s_c.wait_event(ev_in)
+            if prev is not None:
+                s_c.wait_event(prev[1][l])           # the previous call's out[l] reached the host
             self.linked_prefill(pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l],
                                 out[l], stream=s_c)
             ev_out = torch.cuda.Event()
@@ -155,4 +188,10 @@ class LinkedPrefill:
             s_out.wait_event(ev_out)
             with torch.cuda.stream(s_out):
                 h_out[l].copy_(out[l], non_blocking=True)
-        s_out.synchronize()
+                ev_d2h = torch.cuda.Event()
+                ev_d2h.record(s_out)
+            done_c.append(ev_out)
+            done_o.append(ev_d2h)
+        self._host_chain = (done_c, done_o)
+        if wait:
+            s_out.synchronize()

@@ -233,3 +233,45 @@ def test_attention_exp2_polynomial_accuracy():
     want = np.exp2(x[normal].astype(np.float64))
     assert np.max(np.abs(got[normal] / want - 1)) < 1e-4
     assert np.all(got[~normal] < 2.0 ** -124)   # at or near the clamp: negligible, never negative
+
+
+def _plan_kwargs(batch, **over):
+    cfg = batch.cfg
+    kw = dict(n_link=cfg.n_link, h_q=cfg.h_q, h_kv=cfg.h_kv, head_dim=cfg.head_dim,
+              pool_len=batch.pool_len, pool_start=batch.pool_start, pool_rows=batch.pool_rows,
+              prefix_doc=batch.prefix_doc, n_docs=batch.n_docs, doc_ids=batch.doc_ids,
+              q_len=batch.q_len, pool_block_size=cfg.pool_block_size,
+              pool_block_table=batch.pool_block_table, num_sms=152)
+    kw.update(over)
+    return kw
+
+
+def _tables(K, plan):
+    info = K.kvlink_plan_get_info(plan)
+    fields = {f: getattr(info, f) for f, _ in type(info)._fields_}
+    return (fields, K.kvlink_plan_get_segments(plan).tobytes(), [a.tobytes() for a in K.kvlink_plan_get_offsets(plan)],
+            K.kvlink_plan_get_fresh_positions(plan).tobytes(), K.kvlink_plan_get_sources(plan).tobytes())
+
+
+def test_rebuilt_plan_equals_a_created_one(K):
+    """kvlink_plan_rebuild reuses a plan's storage for another batch (other shapes, a paged
+    pool, the other layout) and must give exactly the tables kvlink_plan_create gives."""
+    plan = _plan(K, W.draw_batch(W.get_config(3)))
+    for cfg_index, layout in ((2, 0), (5, 0), (3, 1), (1, 0), (3, 0)):
+        batch = W.draw_batch(W.get_config(cfg_index))
+        K.kvlink_plan_rebuild(plan, **_plan_kwargs(batch, layout=layout))
+        assert _tables(K, plan) == _tables(K, _plan(K, batch, layout=layout)), (cfg_index, layout)
+
+
+def test_failed_rebuild_leaves_no_batch(K):
+    batch = W.draw_batch(W.get_config(1))
+    plan = _plan(K, batch)
+    bad = np.array(batch.doc_ids, copy=True)
+    bad[0] = len(batch.pool_len) + 5                  # a document id outside the pool
+    with pytest.raises(K.KvlinkError):
+        K.kvlink_plan_rebuild(plan, **_plan_kwargs(batch, doc_ids=bad))
+    with pytest.raises(K.KvlinkError) as e:           # nothing to upload
+        K.kvlink_plan_upload(plan, 1e4, 1 << 20, 1 << 20, 0)
+    assert e.value.code == K.KVLINK_EINVAL
+    K.kvlink_plan_rebuild(plan, **_plan_kwargs(batch))  # usable again
+    assert _tables(K, plan) == _tables(K, _plan(K, batch))

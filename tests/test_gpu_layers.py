@@ -85,3 +85,55 @@ def test_reencode_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers):
         assert torch.equal(caches[layer][0].view(torch.int16), ck.view(torch.int16)), layer
         assert torch.equal(caches[layer][1].view(torch.int16), cv.view(torch.int16)), layer
     assert K.kvlink_device_status() == 0
+
+
+def test_pipelined_host_path_chains_calls(RT):
+    """Two batches through linked_prefill_layers_from_host(wait=False) on one object and one
+    set of device buffers, the plan rebuilt for the second while the first runs: each call's
+    host outputs must equal the per-layer kvlink_linked_prefill of its own inputs, bit for bit
+    (the second call overwrites q, k_new, v_new and out only after the first is done with them)."""
+    dev = torch.device("cuda:0")
+    n_layers = 3
+    ba, bb = W.draw_batch(W.get_config(2)), W.draw_batch(W.get_config(2), seed=7)
+    lp = RT.LinkedPrefill.from_batch(ba, device=dev)
+    T = max(int(lp.info.n_fresh), int(RT.LinkedPrefill.from_batch(bb, device=dev).info.n_fresh))
+    cfg = ba.cfg
+
+    def host_inputs(batch):
+        xs = [W.fresh_qkv(batch, l) for l in range(n_layers)]
+        pad = lambda a: np.pad(a, ((0, T - a.shape[0]),) + ((0, 0),) * (a.ndim - 1))
+        return [torch.stack([RT.bf16_from_bits(pad(x[i]), None) for x in xs]).pin_memory() for i in range(3)]
+
+    pools = {id(b): [W.pool_kv(b, l) for l in range(n_layers)] for b in (ba, bb)}
+    pk = {k: [RT.bf16_from_bits(p[0], dev) for p in v] for k, v in pools.items()}
+    pv = {k: [RT.bf16_from_bits(p[1], dev) for p in v] for k, v in pools.items()}
+    hin = {id(b): host_inputs(b) for b in (ba, bb)}
+    q = torch.empty((n_layers, T, cfg.h_q, cfg.head_dim), dtype=torch.bfloat16, device=dev)
+    kn = torch.empty((n_layers, T, cfg.h_kv, cfg.head_dim), dtype=torch.bfloat16, device=dev)
+    vn = torch.empty_like(kn)
+    ctx = max(int(lp.info.ctx_rows), int(RT.LinkedPrefill.from_batch(bb, device=dev).info.ctx_rows))
+    ck = torch.empty((n_layers, ctx, cfg.h_kv, cfg.head_dim), dtype=torch.bfloat16, device=dev)
+    cv = torch.empty_like(ck)
+    out = torch.empty_like(q)
+    h_out = {id(b): torch.empty(out.shape, dtype=out.dtype, pin_memory=True) for b in (ba, bb)}
+    streams = (torch.cuda.Stream(dev), torch.cuda.current_stream(dev), torch.cuda.Stream(dev))
+    for b in (ba, bb):
+        if b is bb:
+            lp.rebuild_from_batch(bb, stream=streams[1])
+        h_q, h_kn, h_vn = hin[id(b)]
+        lp.linked_prefill_layers_from_host(pk[id(b)], pv[id(b)], h_q, h_kn, h_vn, q, kn, vn, ck, cv, out,
+                                           h_out[id(b)], streams=streams, wait=False)
+    torch.cuda.synchronize(dev)
+    from paper_2502_16002_gb300 import kvlink as K
+    assert K.kvlink_device_status() == 0
+    for b in (ba, bb):
+        ref_lp = RT.LinkedPrefill.from_batch(b, device=dev)
+        n = int(ref_lp.info.n_fresh)
+        h_q, h_kn, h_vn = hin[id(b)]
+        for l in range(n_layers):
+            c_k, c_v = ref_lp.empty_cache()
+            ref = torch.empty(ref_lp.fresh_shape(cfg.h_q), dtype=torch.bfloat16, device=dev)
+            ref_lp.linked_prefill(pk[id(b)][l], pv[id(b)][l], h_q[l, :n].to(dev), h_kn[l, :n].to(dev),
+                                  h_vn[l, :n].to(dev), c_k, c_v, ref)
+            torch.cuda.synchronize(dev)
+            assert torch.equal(h_out[id(b)][l, :n].view(torch.int16), ref.cpu().view(torch.int16)), (l,)
