@@ -2,9 +2,9 @@
 """Linked-prefill benchmark (KVLink, arXiv 2502.16002) on GB300.
 
 One step = the whole linked prefill of one batch, over every layer, through
-kvlink_linked_prefill_layers: per layer, re-encode + concatenate the retrieved
-documents' cached K/V and place the fresh link/question K/V (one launch), then run
-the suffix attention.
+kvlink_linked_prefill_layers_overlapped: the retrieved documents' cached K/V of every
+layer re-encoded + concatenated on a second stream, and per layer, once its caches are
+in place, the fresh link/question K/V placed and the suffix attention run.
 
 Default workload: Llama-3.1-8B shape (32 layers, 32 query / 8 KV heads, head dim
 128), batch 8, each query 20 of 200 pooled 256-token documents drawn by Zipf(1.1),
@@ -13,11 +13,13 @@ tokens per query).  Inputs are synthetic N(0,1) bf16, resident in HBM; every lay
 has its own pool, cache and fresh tensors, so each step streams well over L2.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config 3] [--impl ours|reference]
-                  [--path two-kernel|one-kernel|one-kernel-k-only] [--layout interleaved|links_at_end]
+                  [--path two-kernel|two-kernel-serial|one-kernel|one-kernel-k-only] [--layout interleaved|links_at_end]
 
---path selects the library entry point: kvlink_linked_prefill_layers (the default,
-above), or kvlink_linked_prefill_fused per layer (one kernel per layer; -k-only leaves
-the values in the pool).
+--path selects the library entry point: kvlink_linked_prefill_layers_overlapped (the
+default, above), two-kernel-serial (kvlink_linked_prefill_layers: per layer one launch
+that re-encodes and places the fresh rows, then the attention, on one stream), or
+kvlink_linked_prefill_fused per layer (one kernel per layer; -k-only leaves the values
+in the pool).
 --layout selects the physical order of the linked cache.
 
 Prints one JSON line (rank 0).  --impl reference times the fp64 CPU oracle on the
@@ -231,7 +233,7 @@ def run_ours(args, rank, world, local_rank):
     ws, wsb = lp.workspace.data_ptr(), lp.workspace.numel()
     plan = lp.plan
 
-    one_kernel = args.path != "two-kernel"
+    one_kernel = args.path.startswith("one-kernel")
 
     def layer_call(l):
         if one_kernel:
@@ -245,14 +247,18 @@ def run_ours(args, rank, world, local_rank):
                                     out[l].data_ptr(), ws, wsb, sh)
 
     ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, q, kn, vn, ck, cv, out)]
+    re_stream = torch.cuda.Stream(dev)
+    re_sh = int(re_stream.cuda_stream)
     layer_ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, ck, cv)]
 
     def step():
         if one_kernel:
             for l in range(L):
                 layer_call(l)
-        else:
+        elif args.path == "two-kernel-serial":
             K.kvlink_linked_prefill_layers(plan, *ptrs, ws, wsb, sh)
+        else:
+            K.kvlink_linked_prefill_layers_overlapped(plan, *ptrs, ws, wsb, sh, re_sh)
 
     def barrier():
         if world > 1:
@@ -388,7 +394,7 @@ def run_ours(args, rank, world, local_rank):
                 "traffic": NCU_TRAFFIC.get(("reencode", cfg.index)) if default_path else None,
                 "peak_kind": f"HBM copy, {peaks['source']}"}
     n_merge = 1 if info.n_attn_splits > 0 else 0
-    launches_per_step = L * ((1 if one_kernel else 2) + n_merge)
+    launches_per_step = L * ((1 if one_kernel else 2 if args.path == "two-kernel-serial" else 3) + n_merge)
     attn_entry = {"us_per_launch": round(t_at * 1e6, 2), "TFLOP_per_s": round(at_tfs, 2),
                   "frac_bf16_sustained": round(at_frac, 4),
                   "frac_bf16_burst": round(at_tfs / peaks["bf16_tflops"], 4),
@@ -499,7 +505,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--path", choices=["two-kernel", "one-kernel", "one-kernel-k-only"], default="two-kernel")
+    ap.add_argument("--path", choices=["two-kernel", "two-kernel-serial", "one-kernel", "one-kernel-k-only"],
+                    default="two-kernel")
     ap.add_argument("--layout", choices=["interleaved", "links_at_end"], default="interleaved")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":

@@ -303,6 +303,23 @@ int kvlink_linked_prefill_layers(const kvlink_plan_t* plan, int32_t n_layers, co
                                  void* const* d_cache_v, void* const* d_out, void* d_workspace,
                                  size_t workspace_bytes, kvlink_stream_t stream);
 
+/* The same results as kvlink_linked_prefill_layers, bit for bit, with the re-encode on a
+ * second stream.  reencode_stream first waits for the work already enqueued on `stream`,
+ * then re-encodes every layer's document caches (kvlink_reencode_concat) back to back;
+ * layer l's fresh-row placement and suffix attention run on `stream` once layer l's
+ * caches are in place.  The document caches do not depend on the forward pass, so the
+ * re-encode of later layers fills the SMs that the attention of earlier layers leaves
+ * idle (the ends of its grid, the gaps between launches).  When the call returns,
+ * `stream` is ordered after all of its work.  The plan keeps the events it uses: calls
+ * with one plan must not run concurrently.  Errors: as kvlink_linked_prefill_layers;
+ * EINVAL also when the two streams are the same. */
+int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
+                                            const void* const* d_pool_v, const void* const* d_q,
+                                            const void* const* d_k_new, const void* const* d_v_new,
+                                            void* const* d_cache_k, void* const* d_cache_v, void* const* d_out,
+                                            void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream,
+                                            kvlink_stream_t reencode_stream);
+
 /* Allocation-free variant of kvlink_suffix_attention.  The paper has no counterpart:
  * this entry point serves callers that may not allocate device memory at all, such as
  * a serving loop whose memory budget is fixed at start-up (cudaMalloc can synchronise

@@ -104,6 +104,20 @@ PinnedStaging::~PinnedStaging() {
     if (ptr) cudaFreeHost(ptr);
 }
 
+EventPool::~EventPool() {
+    for (cudaEvent_t e : ev) cudaEventDestroy(e);
+}
+
+static int events_reserve(EventPool& pool, size_t n) {
+    while (pool.ev.size() < n) {
+        cudaEvent_t e = nullptr;
+        cudaError_t err = cudaEventCreateWithFlags(&e, cudaEventDisableTiming);
+        if (err != cudaSuccess) return cuda_fail(err, "event");
+        pool.ev.push_back(e);
+    }
+    return KVLINK_OK;
+}
+
 // Room for `bytes` in the staging buffer, once the last copy out of it has completed.
 static int staging_reserve(PinnedStaging& st, size_t bytes) {
     if (st.done) {
@@ -439,6 +453,55 @@ int kvlink_linked_prefill_layers(const kvlink_plan_t* p, int32_t n_layers, const
     for (int l = 0; l < n_layers; ++l) {
         rc = kvlink_linked_prefill(p, pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l],
                                    out[l], ws, ws_bytes, stream);
+        if (rc) return rc;
+    }
+    return KVLINK_OK;
+}
+
+int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* p, int32_t n_layers, const void* const* pool_k,
+                                            const void* const* pool_v, const void* const* q,
+                                            const void* const* k_new, const void* const* v_new,
+                                            void* const* cache_k, void* const* cache_v, void* const* out, void* ws,
+                                            size_t ws_bytes, kvlink_stream_t stream,
+                                            kvlink_stream_t reencode_stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (n_layers <= 0 || !pool_k || !pool_v || !q || !k_new || !v_new || !cache_k || !cache_v || !out)
+        return KVLINK_EINVAL;
+    if (stream == reencode_stream) return KVLINK_EINVAL;
+    // every argument is checked before the first launch
+    if (!all_aligned(n_layers, pool_k) || !all_aligned(n_layers, pool_v) ||
+        !all_aligned(n_layers, (const void* const*)cache_k) || !all_aligned(n_layers, (const void* const*)cache_v) ||
+        !all_aligned(n_layers, q) || !all_aligned(n_layers, k_new) || !all_aligned(n_layers, v_new) ||
+        !all_aligned(n_layers, (const void* const*)out))
+        return KVLINK_EINVAL;
+    if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
+    if (ws && !aligned16(ws)) return KVLINK_EINVAL;
+    rc = events_reserve(p->events, (size_t)n_layers + 1);
+    if (rc) return rc;
+    cudaStream_t s = (cudaStream_t)stream, r = (cudaStream_t)reencode_stream;
+    cudaEvent_t* ev = p->events.ev.data();
+    // the re-encode stream starts after the work already on `stream` (the plan upload, the
+    // pool), then re-encodes every layer's document caches back to back
+    cudaError_t e = cudaEventRecord(ev[n_layers], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(r, ev[n_layers], 0);
+    if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_overlapped: stream order");
+    for (int l = 0; l < n_layers; ++l) {
+        launch_reencode(p->dev, 0, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, pool_k[l], pool_v[l],
+                        nullptr, nullptr, cache_k[l], cache_v[l], r);
+        rc = check_launch("reencode_kernel (overlapped)");
+        if (rc) return rc;
+        e = cudaEventRecord(ev[l], r);
+        if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_overlapped: event");
+    }
+    // per layer on `stream`: once its caches are in place, the fresh rows and the attention;
+    // the last wait also orders every re-encode before later work on `stream`
+    for (int l = 0; l < n_layers; ++l) {
+        e = cudaStreamWaitEvent(s, ev[l], 0);
+        if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_overlapped: wait");
+        rc = place_fresh(p, k_new[l], v_new[l], cache_k[l], cache_v[l], s);
+        if (rc) return rc;
+        rc = attention_common(p, q[l], cache_k[l], cache_v[l], out[l], ws, ws_bytes, s);
         if (rc) return rc;
     }
     return KVLINK_OK;

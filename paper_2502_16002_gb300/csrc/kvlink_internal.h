@@ -130,6 +130,19 @@ struct PinnedStaging {
         std::swap(done, o.done);
     }
 };
+// Events reused by the calls of one plan (created on first use, destroyed with the plan).
+struct EventPool {
+    std::vector<cudaEvent_t> ev;
+    EventPool() = default;
+    EventPool(const EventPool&) = delete;
+    EventPool& operator=(const EventPool&) = delete;
+    EventPool(EventPool&& o) noexcept { ev.swap(o.ev); }
+    EventPool& operator=(EventPool&& o) noexcept {
+        ev.swap(o.ev);
+        return *this;
+    }
+    ~EventPool();
+};
 }  // namespace kvlink
 
 struct kvlink_plan {
@@ -173,6 +186,7 @@ struct kvlink_plan {
 
     bool built = false;                 // holds a batch (a failed rebuild clears it)
     kvlink::PinnedStaging staging;
+    kvlink::EventPool events;           // per-layer events of the overlapped all-layers call
 
     // set by kvlink_plan_upload
     bool uploaded = false;

@@ -104,6 +104,8 @@ def _load():
         "kvlink_linked_prefill_layers": (C.c_int, [P, C.c_int32, V, V, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_reencode_concat_layers": (C.c_int, [P, C.c_int32, V, V, V, V, V]),
         "kvlink_plan_rebuild": (C.c_int, [P, C.POINTER(kvlink_batch_desc_t)]),
+        "kvlink_linked_prefill_layers_overlapped": (C.c_int, [P, C.c_int32, V, V, V, V, V, V, V, V, V, C.c_size_t,
+                                                              V, V]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
         "kvlink_selftest_wait_timeout": (C.c_int, [C.c_uint32, V]),
@@ -125,7 +127,7 @@ DECLARED = [
     "kvlink_device_status", "kvlink_clear_device_status", "kvlink_strerror",
     "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc", "kvlink_rope_fresh",
     "kvlink_plan_get_sources", "kvlink_linked_prefill_fused", "kvlink_linked_prefill_layers",
-    "kvlink_reencode_concat_layers", "kvlink_plan_rebuild",
+    "kvlink_reencode_concat_layers", "kvlink_plan_rebuild", "kvlink_linked_prefill_layers_overlapped",
     "kvlink_selftest_wait_timeout",
 ]
 
@@ -316,6 +318,18 @@ def kvlink_linked_prefill_layers(plan: Plan, pool_k, pool_v, q, k_new, v_new, ca
         raise ValueError("every per-layer pointer list needs one entry per layer")
     _check(lib.kvlink_linked_prefill_layers(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs], workspace,
                                             workspace_bytes, stream), "kvlink_linked_prefill_layers")
+
+
+def kvlink_linked_prefill_layers_overlapped(plan: Plan, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out,
+                                            workspace, workspace_bytes: int, stream: int, reencode_stream: int) -> None:
+    """As kvlink_linked_prefill_layers, with the re-encode on reencode_stream."""
+    n = len(pool_k)
+    arrs = [_ptr_array(x) for x in (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out)]
+    if any(len(a) != n for a in arrs):
+        raise ValueError("every per-layer pointer list needs one entry per layer")
+    _check(lib.kvlink_linked_prefill_layers_overlapped(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs],
+                                                       workspace, workspace_bytes, stream, reencode_stream),
+           "kvlink_linked_prefill_layers_overlapped")
 
 
 def kvlink_reencode_concat_layers(plan: Plan, pool_k, pool_v, cache_k, cache_v, stream: int = 0) -> None:

@@ -138,6 +138,20 @@ class LinkedPrefill:
         K.kvlink_linked_prefill_layers(self.plan, *ptrs, self.workspace.data_ptr(), self.workspace.numel(),
                                        _stream_handle(stream))
 
+    def linked_prefill_layers_overlapped(self, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out,
+                                         stream=None, reencode_stream=None):
+        """All layers in one ABI call, the re-encode on a second stream (created if not given)."""
+        if reencode_stream is None:
+            reencode_stream = self._reencode_stream()
+        ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out)]
+        K.kvlink_linked_prefill_layers_overlapped(self.plan, *ptrs, self.workspace.data_ptr(), self.workspace.numel(),
+                                                  _stream_handle(stream), _stream_handle(reencode_stream))
+
+    def _reencode_stream(self):
+        if getattr(self, "_re_stream", None) is None:
+            self._re_stream = torch.cuda.Stream(self.device)
+        return self._re_stream
+
     def reencode_concat_layers(self, pool_k, pool_v, cache_k, cache_v, stream=None):
         """The document caches of all layers in one launch (sequences of per-layer tensors)."""
         ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, cache_k, cache_v)]
@@ -147,11 +161,13 @@ class LinkedPrefill:
                                         cache_k, cache_v, out, h_out, streams=None, wait=True):
         """Every layer of the linked prefill with the fresh rows in host memory.
 
-        Per layer l: h_q[l], h_k_new[l], h_v_new[l] (pinned host tensors) are copied to
-        q[l], k_new[l], v_new[l] on an input stream, kvlink_linked_prefill runs on the
-        compute stream once they have landed, and out[l] is copied to h_out[l] (pinned) on
-        an output stream once it is written.  The copies of one layer thus overlap the
-        kernels of the layers around it.  Returns after the last output has arrived.
+        The document caches of every layer are re-encoded on a fourth stream, as in
+        kvlink_linked_prefill_layers_overlapped.  Per layer l: h_q[l], h_k_new[l], h_v_new[l]
+        (pinned host tensors) are copied to q[l], k_new[l], v_new[l] on an input stream; the
+        fresh-row placement and the suffix attention run on the compute stream once they have
+        landed and layer l's caches are in place; out[l] is copied to h_out[l] (pinned) on an
+        output stream once it is written.  The copies of one layer thus overlap the kernels of
+        the layers around it.  Returns after the last output has arrived.
 
         streams: optional (input, compute, output) torch.cuda.Stream triple.
         wait=False returns once everything is enqueued, so that the host can prepare the
@@ -164,10 +180,26 @@ class LinkedPrefill:
             streams = (torch.cuda.Stream(self.device), torch.cuda.current_stream(self.device),
                        torch.cuda.Stream(self.device))
         s_in, s_c, s_out = streams
+        s_re = self._reencode_stream()
         n = len(pool_k)
         prev = getattr(self, "_host_chain", None)
         if prev is not None and len(prev[0]) != n:
             prev = None
+        # the document caches of every layer on the re-encode stream (after the work already on
+        # the compute stream, e.g. the plan upload); a layer's cache is rewritten only after the
+        # previous call's attention of that layer has read it
+        ev0 = torch.cuda.Event()
+        ev0.record(s_c)
+        s_re.wait_event(ev0)
+        ev_re = []
+        for l in range(n):
+            if prev is not None:
+                s_re.wait_event(prev[0][l])
+            K.kvlink_reencode_concat(self.plan, pool_k[l].data_ptr(), pool_v[l].data_ptr(), cache_k[l].data_ptr(),
+                                     cache_v[l].data_ptr(), _stream_handle(s_re))
+            e = torch.cuda.Event()
+            e.record(s_re)
+            ev_re.append(e)
         done_c, done_o = [], []
         for l in range(n):
             ev_in = torch.cuda.Event()
@@ -179,10 +211,10 @@ class LinkedPrefill:
                 v_new[l].copy_(h_v_new[l], non_blocking=True)
                 ev_in.record(s_in)
             s_c.wait_event(ev_in)
+            s_c.wait_event(ev_re[l])
             if prev is not None:
                 s_c.wait_event(prev[1][l])           # the previous call's out[l] reached the host
-            self.linked_prefill(pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l],
-                                out[l], stream=s_c)
+            self.suffix_attention(q[l], k_new[l], v_new[l], cache_k[l], cache_v[l], out[l], stream=s_c)
             ev_out = torch.cuda.Event()
             ev_out.record(s_c)
             s_out.wait_event(ev_out)

@@ -1,4 +1,5 @@
-"""GPU check of the all-layers calls.  kvlink_linked_prefill_layers must give, for every
+"""GPU check of the all-layers calls.  kvlink_linked_prefill_layers and
+kvlink_linked_prefill_layers_overlapped (re-encode on a second stream) must give, for every
 layer, exactly (bit for bit) what the per-layer kvlink_linked_prefill gives, and
 kvlink_reencode_concat_layers exactly what kvlink_reencode_concat gives per layer,
 including across the kernel's per-launch layer limit; one query of the last layer is
@@ -31,8 +32,9 @@ def _sentinel_cache(lp):
     return ck, cv
 
 
+@pytest.mark.parametrize("overlapped", [False, True])
 @pytest.mark.parametrize("cfg_index,n_layers,layout", [(2, 3, 0), (5, 2, 0), (3, 2, 1)])
-def test_all_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers, layout):
+def test_all_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers, layout, overlapped):
     from paper_2502_16002_gb300 import kvlink as K
     dev = torch.device("cuda:0")
     batch = W.draw_batch(W.get_config(cfg_index))
@@ -46,7 +48,10 @@ def test_all_layers_call_equals_per_layer_calls(RT, cfg_index, n_layers, layout)
     lp = RT.LinkedPrefill.from_batch(batch, device=dev, layout=layout)
     caches = [_sentinel_cache(lp) for _ in range(n_layers)]
     outs = [torch.full_like(x, float("nan")) for x in q]
-    lp.linked_prefill_layers(pk, pv, q, kn, vn, [c[0] for c in caches], [c[1] for c in caches], outs)
+    if overlapped:      # the re-encode on a second stream
+        lp.linked_prefill_layers_overlapped(pk, pv, q, kn, vn, [c[0] for c in caches], [c[1] for c in caches], outs)
+    else:
+        lp.linked_prefill_layers(pk, pv, q, kn, vn, [c[0] for c in caches], [c[1] for c in caches], outs)
     for layer in range(n_layers):
         ck, cv = _sentinel_cache(lp)
         ref = torch.full_like(q[layer], float("nan"))
