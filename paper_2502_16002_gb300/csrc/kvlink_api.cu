@@ -18,6 +18,8 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
 void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int h_kv, int num_sms, int n_layers,
                             const void* const* pool_k, const void* const* pool_v, void* const* cache_k,
                             void* const* cache_v, cudaStream_t stream);
+void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int row_bytes, const void* k_new,
+                        const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
 int read_copy_status(int32_t* status);
 void launch_rope_fresh(const int32_t* d_fresh_pos, int n_fresh, int head_dim, double theta, void* q, int h_q,
                        void* k, int h_kv, cudaStream_t stream);
@@ -174,7 +176,8 @@ int kvlink_plan_rebuild(kvlink_plan_t* p, const kvlink_batch_desc_t* desc) {
     KVLINK_RECYCLE(pool_start) KVLINK_RECYCLE(pool_len) KVLINK_RECYCLE(pool_block_table) KVLINK_RECYCLE(seg)
     KVLINK_RECYCLE(chunks) KVLINK_RECYCLE(chunks_sorted) KVLINK_RECYCLE(cu_ctx) KVLINK_RECYCLE(cu_fresh)
     KVLINK_RECYCLE(fresh_pos) KVLINK_RECYCLE(fresh_query) KVLINK_RECYCLE(src) KVLINK_RECYCLE(src_row)
-    KVLINK_RECYCLE(fresh_vis) KVLINK_RECYCLE(fresh_row0) KVLINK_RECYCLE(cu_grp) KVLINK_RECYCLE(grp_src)
+    KVLINK_RECYCLE(fresh_vis) KVLINK_RECYCLE(fresh_row0) KVLINK_RECYCLE(fresh_dst) KVLINK_RECYCLE(cu_grp)
+    KVLINK_RECYCLE(grp_src)
     KVLINK_RECYCLE(items) KVLINK_RECYCLE(merges)
 #undef KVLINK_RECYCLE
     std::string why;
@@ -271,6 +274,7 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     put(p->off_src_row, p->src_row.data(), p->src_row.size() * sizeof(kvlink_source_t));
     put(p->off_fresh_vis, p->fresh_vis.data(), p->fresh_vis.size() * sizeof(int32_t));
     put(p->off_fresh_row0, p->fresh_row0.data(), p->fresh_row0.size() * sizeof(int32_t));
+    put(p->off_fresh_dst, p->fresh_dst.data(), p->fresh_dst.size() * sizeof(int32_t));
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = cudaMemcpyAsync(d_buf, host, p->device_bytes, cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload copy");
@@ -297,6 +301,7 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     d.src_row = (const kvlink_source_t*)(b + p->off_src_row);
     d.fresh_vis = (const int32_t*)(b + p->off_fresh_vis);
     d.fresh_row0 = (const int32_t*)(b + p->off_fresh_row0);
+    d.fresh_dst = (const int32_t*)(b + p->off_fresh_dst);
     launch_rope_table(d.seg, (int)p->seg.size(), (float4*)(b + p->off_rope), p->head_dim, theta, s);
     rc = check_launch("rope_table_kernel");
     if (rc != KVLINK_OK) return rc;
@@ -340,10 +345,9 @@ int kvlink_reencode_concat_layers(const kvlink_plan_t* p, int32_t n_layers, cons
 
 static int place_fresh(const kvlink_plan_t* p, const void* k_new, const void* v_new, void* cache_k,
                        void* cache_v, cudaStream_t s) {
-    const int n_all = (int)p->chunks.size();
-    launch_reencode(p->dev, p->n_chunks_cached, n_all - p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms,
-                    nullptr, nullptr, k_new, v_new, cache_k, cache_v, s);
-    return check_launch("fresh placement");
+    launch_place_fresh(p->dev.fresh_dst, p->cu_fresh.back(), p->h_kv * p->head_dim * 2, k_new, v_new, cache_k,
+                       cache_v, s);
+    return check_launch("place_fresh_kernel");
 }
 
 static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k, void* cache_v,

@@ -97,6 +97,7 @@ struct DevicePlan {
     // index among the query's fresh rows (interleaved: fresh_row0 = kNoFreshRegion).
     const int32_t* fresh_vis;    // [n_fresh]
     const int32_t* fresh_row0;   // [B], query-relative
+    const int32_t* fresh_dst;    // [n_fresh] batch cache row of every fresh row
     // Groups of 8 cache rows (8m .. 8m+7 of a query), at cu_grp[b] + m: the first source
     // row when the group's 8 rows are consecutive in one tensor (one 8-row TMA copy), else
     // -1 (rows copied one by one; also the query's last, partial group).
@@ -167,7 +168,7 @@ struct kvlink_plan {
     std::vector<int32_t> fresh_pos;
     std::vector<int32_t> fresh_query;
     std::vector<kvlink_source_t> src, src_row;
-    std::vector<int32_t> fresh_vis, fresh_row0;
+    std::vector<int32_t> fresh_vis, fresh_row0, fresh_dst;
     std::vector<int32_t> cu_grp, grp_src;
     std::vector<kvlink::AttnItem> items;
     std::vector<kvlink::MergeGroup> merges;
@@ -180,7 +181,7 @@ struct kvlink_plan {
     size_t off_seg = 0, off_chunks = 0, off_rope = 0, off_pool_start = 0, off_pool_bt = 0,
            off_cu_ctx = 0, off_cu_fresh = 0, off_fresh_pos = 0, off_fresh_query = 0,
            off_items = 0, off_merges = 0, off_src = 0, off_cu_grp = 0, off_grp_src = 0, off_src_row = 0,
-           off_fresh_vis = 0, off_fresh_row0 = 0,
+           off_fresh_vis = 0, off_fresh_row0 = 0, off_fresh_dst = 0,
            device_bytes = 0;
     size_t workspace_bytes = 0;
 

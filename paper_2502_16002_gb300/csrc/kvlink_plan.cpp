@@ -202,6 +202,12 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         }
     }
 
+    // ---- the cache row of every fresh row (the fresh-row placement)
+    p->fresh_dst.assign(p->fresh_pos.size(), 0);
+    for (const kvlink_segment_t& sg : p->seg)
+        if (sg.kind == KVLINK_SEG_LINK || sg.kind == KVLINK_SEG_QUESTION)
+            for (int t = 0; t < sg.len; ++t) p->fresh_dst[(size_t)sg.src + t] = (int32_t)(sg.dst + t);
+
     // ---- groups of 8 cache rows whose sources are consecutive in one tensor: each is one
     // 8-row TMA copy in the one-kernel path
     p->cu_grp.assign(B + 1, 0);
@@ -371,6 +377,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     p->off_src_row = take(p->src_row.size() * sizeof(kvlink_source_t));
     p->off_fresh_vis = take(p->fresh_vis.size() * sizeof(int32_t));
     p->off_fresh_row0 = take(p->fresh_row0.size() * sizeof(int32_t));
+    p->off_fresh_dst = take(p->fresh_dst.size() * sizeof(int32_t));
     p->device_bytes = off;
     p->uploaded = false;
     return KVLINK_OK;

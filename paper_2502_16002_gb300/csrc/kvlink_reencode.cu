@@ -309,6 +309,54 @@ void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int
 }
 
 // --------------------------------------------------------------------------
+// A4: the fresh link/question rows to their cache rows (bit copies).  A few MB per layer
+// on the path of the attention that follows, so the copy is built for latency: one warp
+// per row and 16-byte accesses, all of a lane's loads issued before its stores.
+// --------------------------------------------------------------------------
+constexpr int kPlaceWarps = 8;
+
+__global__ void __launch_bounds__(32 * kPlaceWarps) place_fresh_kernel(const int32_t* __restrict__ fresh_dst,
+                                                                       int n_fresh, int row_vec,
+                                                                       const uint4* __restrict__ k_new,
+                                                                       const uint4* __restrict__ v_new,
+                                                                       uint4* __restrict__ cache_k,
+                                                                       uint4* __restrict__ cache_v) {
+    // after a recorded failure, later launches skip their work
+    if (*reinterpret_cast<volatile int32_t*>(&g_copy_status) != 0) return;
+    const int row = blockIdx.x * kPlaceWarps + threadIdx.x / 32, lane = threadIdx.x % 32;
+    if (row >= n_fresh) return;
+    const int64_t src = (int64_t)row * row_vec, dst = (int64_t)fresh_dst[row] * row_vec;
+    for (int i0 = lane; i0 < row_vec; i0 += 4 * 32) {
+        uint4 k[4], v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int i = i0 + u * 32;
+            if (i < row_vec) {
+                k[u] = __ldg(k_new + src + i);
+                v[u] = __ldg(v_new + src + i);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int i = i0 + u * 32;
+            if (i < row_vec) {
+                cache_k[dst + i] = k[u];
+                cache_v[dst + i] = v[u];
+            }
+        }
+    }
+}
+
+void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int row_bytes, const void* k_new, const void* v_new,
+                        void* cache_k, void* cache_v, cudaStream_t stream) {
+    if (n_fresh <= 0) return;
+    const int blocks = (n_fresh + kPlaceWarps - 1) / kPlaceWarps;
+    place_fresh_kernel<<<blocks, 32 * kPlaceWarps, 0, stream>>>(d_fresh_dst, n_fresh, row_bytes / 16,
+                                                                (const uint4*)k_new, (const uint4*)v_new,
+                                                                (uint4*)cache_k, (uint4*)cache_v);
+}
+
+// --------------------------------------------------------------------------
 // RoPE of the fresh rows at their global positions (Sec. 2.2: a token at position i
 // carries R_i).  One thread per (fresh row, j < D/2): the angle pos * theta^(-2j/D) is
 // formed in float64, cos/sin are split into float pairs, and pair (j, j + D/2) of every
