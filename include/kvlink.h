@@ -320,6 +320,34 @@ int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* plan, int32_t n_layer
                                             void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream,
                                             kvlink_stream_t reencode_stream);
 
+/* The linked prefill of n_layers layers end to end from host memory, as a serving step
+ * runs it: the same results as kvlink_linked_prefill_layers_overlapped, bit for bit, with
+ * every layer's fresh rows brought in from, and its output taken back to, host memory.
+ *   h_q[l], h_k_new[l], h_v_new[l]: host rows of layer l, [n_fresh][h_q or h_kv][D] bf16,
+ *     copied to d_q[l], d_k_new[l], d_v_new[l] on copy_in_stream (pinned memory makes the
+ *     copies asynchronous);
+ *   the document caches of every layer are re-encoded on reencode_stream, which first
+ *     waits for the work already on `stream` (the plan upload);
+ *   layer l's fresh-row placement and suffix attention run on `stream` once its inputs
+ *     and caches are in place;
+ *   d_out[l] is copied to h_out[l] ([n_fresh][h_q][D]) on copy_out_stream.
+ * Returns once everything is enqueued: the outputs are on the host when copy_out_stream
+ * has completed the call's work.  Successive calls with one plan (also across
+ * kvlink_plan_rebuild) chain through events the plan keeps: a layer's device inputs and
+ * caches are rewritten only after the previous call's kernels of that layer have read
+ * them, and its device output only after the previous call's copy of it to the host, so
+ * a caller may prepare and enqueue the next batch while one runs.  The four streams must
+ * be distinct.  Errors: as kvlink_linked_prefill_layers; EINVAL also for a NULL host
+ * pointer or repeated streams. */
+int kvlink_linked_prefill_layers_host(kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
+                                      const void* const* d_pool_v, const void* const* h_q,
+                                      const void* const* h_k_new, const void* const* h_v_new, void* const* d_q,
+                                      void* const* d_k_new, void* const* d_v_new, void* const* d_cache_k,
+                                      void* const* d_cache_v, void* const* d_out, void* const* h_out,
+                                      void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream,
+                                      kvlink_stream_t reencode_stream, kvlink_stream_t copy_in_stream,
+                                      kvlink_stream_t copy_out_stream);
+
 /* Allocation-free variant of kvlink_suffix_attention.  The paper has no counterpart:
  * this entry point serves callers that may not allocate device memory at all, such as
  * a serving loop whose memory budget is fixed at start-up (cudaMalloc can synchronise

@@ -170,6 +170,9 @@ int kvlink_plan_rebuild(kvlink_plan_t* p, const kvlink_batch_desc_t* desc) {
     // the tables are rebuilt in memory that is already mapped) and its staging buffer
     kvlink_plan q;
     q.staging = std::move(p->staging);
+    // the events of earlier calls still order this plan's next calls after them
+    q.events = std::move(p->events);
+    q.host_chain_layers = p->host_chain_layers;
 #define KVLINK_RECYCLE(m) \
     q.m.swap(p->m);       \
     q.m.clear();
@@ -508,6 +511,84 @@ int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* p, int32_t n_layers, 
         rc = attention_common(p, q[l], cache_k[l], cache_v[l], out[l], ws, ws_bytes, s);
         if (rc) return rc;
     }
+    return KVLINK_OK;
+}
+
+int kvlink_linked_prefill_layers_host(kvlink_plan_t* p, int32_t n_layers, const void* const* pool_k,
+                                      const void* const* pool_v, const void* const* h_q, const void* const* h_k_new,
+                                      const void* const* h_v_new, void* const* q, void* const* k_new,
+                                      void* const* v_new, void* const* cache_k, void* const* cache_v,
+                                      void* const* out, void* const* h_out, void* ws, size_t ws_bytes,
+                                      kvlink_stream_t stream, kvlink_stream_t reencode_stream,
+                                      kvlink_stream_t copy_in_stream, kvlink_stream_t copy_out_stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (n_layers <= 0 || !pool_k || !pool_v || !h_q || !h_k_new || !h_v_new || !q || !k_new || !v_new ||
+        !cache_k || !cache_v || !out || !h_out)
+        return KVLINK_EINVAL;
+    if (stream == reencode_stream || stream == copy_in_stream || stream == copy_out_stream ||
+        reencode_stream == copy_in_stream || reencode_stream == copy_out_stream || copy_in_stream == copy_out_stream)
+        return KVLINK_EINVAL;
+    auto cv = [](void* const* a) { return (const void* const*)a; };
+    if (!all_aligned(n_layers, pool_k) || !all_aligned(n_layers, pool_v) || !all_aligned(n_layers, cv(q)) ||
+        !all_aligned(n_layers, cv(k_new)) || !all_aligned(n_layers, cv(v_new)) || !all_aligned(n_layers, cv(cache_k)) ||
+        !all_aligned(n_layers, cv(cache_v)) || !all_aligned(n_layers, cv(out)))
+        return KVLINK_EINVAL;
+    for (int l = 0; l < n_layers; ++l)
+        if (!h_q[l] || !h_k_new[l] || !h_v_new[l] || !h_out[l]) return KVLINK_EINVAL;
+    if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
+    if (ws && !aligned16(ws)) return KVLINK_EINVAL;
+    // events: [0, L) caches in place, [L, 2L) inputs in place, [2L, 3L) layer computed,
+    // [3L, 4L) output on the host, 4L the call's start.  The previous call's records of the
+    // last two kinds order this call's rewrites of the same buffers after their readers.
+    const bool chained = p->host_chain_layers == n_layers;
+    rc = events_reserve(p->events, 4 * (size_t)n_layers + 1);
+    if (rc) return rc;
+    cudaEvent_t* ev = p->events.ev.data();
+    cudaEvent_t *ev_re = ev, *ev_in = ev + n_layers, *ev_c = ev + 2 * n_layers, *ev_o = ev + 3 * n_layers;
+    cudaStream_t s = (cudaStream_t)stream, r = (cudaStream_t)reencode_stream, ci = (cudaStream_t)copy_in_stream,
+                 co = (cudaStream_t)copy_out_stream;
+    const size_t n_fresh = (size_t)p->cu_fresh.back();
+    const size_t q_bytes = n_fresh * p->h_q * p->head_dim * 2, kv_bytes = n_fresh * p->h_kv * p->head_dim * 2;
+    cudaError_t e = cudaEventRecord(ev[4 * n_layers], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(r, ev[4 * n_layers], 0);
+    if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host: stream order");
+    // the document caches of every layer, on the re-encode stream
+    for (int l = 0; l < n_layers; ++l) {
+        if (chained && (e = cudaStreamWaitEvent(r, ev_c[l], 0)) != cudaSuccess)
+            return cuda_fail(e, "linked_prefill_layers_host: wait");
+        launch_reencode(p->dev, 0, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, pool_k[l], pool_v[l],
+                        nullptr, nullptr, cache_k[l], cache_v[l], r);
+        rc = check_launch("reencode_kernel (host path)");
+        if (rc) return rc;
+        if ((e = cudaEventRecord(ev_re[l], r)) != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host");
+    }
+    for (int l = 0; l < n_layers; ++l) {
+        // fresh rows in from the host
+        if (chained && (e = cudaStreamWaitEvent(ci, ev_c[l], 0)) != cudaSuccess)
+            return cuda_fail(e, "linked_prefill_layers_host: wait");
+        e = cudaMemcpyAsync(q[l], h_q[l], q_bytes, cudaMemcpyHostToDevice, ci);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(k_new[l], h_k_new[l], kv_bytes, cudaMemcpyHostToDevice, ci);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(v_new[l], h_v_new[l], kv_bytes, cudaMemcpyHostToDevice, ci);
+        if (e == cudaSuccess) e = cudaEventRecord(ev_in[l], ci);
+        // the layer, once its inputs and caches are in place (and the previous call's output
+        // of this layer has left)
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev_in[l], 0);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev_re[l], 0);
+        if (e == cudaSuccess && chained) e = cudaStreamWaitEvent(s, ev_o[l], 0);
+        if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host: inputs");
+        rc = place_fresh(p, k_new[l], v_new[l], cache_k[l], cache_v[l], s);
+        if (rc) return rc;
+        rc = attention_common(p, q[l], cache_k[l], cache_v[l], out[l], ws, ws_bytes, s);
+        if (rc) return rc;
+        // the output back to the host
+        e = cudaEventRecord(ev_c[l], s);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(co, ev_c[l], 0);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(h_out[l], out[l], q_bytes, cudaMemcpyDeviceToHost, co);
+        if (e == cudaSuccess) e = cudaEventRecord(ev_o[l], co);
+        if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host: output");
+    }
+    p->host_chain_layers = n_layers;
     return KVLINK_OK;
 }
 

@@ -187,7 +187,8 @@ struct kvlink_plan {
 
     bool built = false;                 // holds a batch (a failed rebuild clears it)
     kvlink::PinnedStaging staging;
-    kvlink::EventPool events;           // per-layer events of the overlapped all-layers call
+    kvlink::EventPool events;           // per-layer events of the overlapped all-layers calls
+    int32_t host_chain_layers = 0;      // layers of the last host-path call (its events chain the next)
 
     // set by kvlink_plan_upload
     bool uploaded = false;

@@ -106,6 +106,7 @@ def _load():
         "kvlink_plan_rebuild": (C.c_int, [P, C.POINTER(kvlink_batch_desc_t)]),
         "kvlink_linked_prefill_layers_overlapped": (C.c_int, [P, C.c_int32, V, V, V, V, V, V, V, V, V, C.c_size_t,
                                                               V, V]),
+        "kvlink_linked_prefill_layers_host": (C.c_int, [P, C.c_int32] + [V] * 13 + [C.c_size_t, V, V, V, V]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
         "kvlink_selftest_wait_timeout": (C.c_int, [C.c_uint32, V]),
@@ -128,6 +129,7 @@ DECLARED = [
     "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc", "kvlink_rope_fresh",
     "kvlink_plan_get_sources", "kvlink_linked_prefill_fused", "kvlink_linked_prefill_layers",
     "kvlink_reencode_concat_layers", "kvlink_plan_rebuild", "kvlink_linked_prefill_layers_overlapped",
+    "kvlink_linked_prefill_layers_host",
     "kvlink_selftest_wait_timeout",
 ]
 
@@ -330,6 +332,20 @@ def kvlink_linked_prefill_layers_overlapped(plan: Plan, pool_k, pool_v, q, k_new
     _check(lib.kvlink_linked_prefill_layers_overlapped(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs],
                                                        workspace, workspace_bytes, stream, reencode_stream),
            "kvlink_linked_prefill_layers_overlapped")
+
+
+def kvlink_linked_prefill_layers_host(plan: Plan, pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new, cache_k,
+                                      cache_v, out, h_out, workspace, workspace_bytes: int, stream: int,
+                                      reencode_stream: int, copy_in_stream: int, copy_out_stream: int) -> None:
+    """Per-layer pointer sequences (h_*: host, the rest device); see include/kvlink.h."""
+    n = len(pool_k)
+    seqs = (pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new, cache_k, cache_v, out, h_out)
+    arrs = [_ptr_array(x) for x in seqs]
+    if any(len(a) != n for a in arrs):
+        raise ValueError("every per-layer pointer list needs one entry per layer")
+    _check(lib.kvlink_linked_prefill_layers_host(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs], workspace,
+                                                 workspace_bytes, stream, reencode_stream, copy_in_stream,
+                                                 copy_out_stream), "kvlink_linked_prefill_layers_host")
 
 
 def kvlink_reencode_concat_layers(plan: Plan, pool_k, pool_v, cache_k, cache_v, stream: int = 0) -> None:

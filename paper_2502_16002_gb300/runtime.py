@@ -159,71 +159,30 @@ class LinkedPrefill:
 
     def linked_prefill_layers_from_host(self, pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new,
                                         cache_k, cache_v, out, h_out, streams=None, wait=True):
-        """Every layer of the linked prefill with the fresh rows in host memory.
+        """Every layer of the linked prefill with the fresh rows and outputs in host memory, in
+        one kvlink_linked_prefill_layers_host call.
 
-        The document caches of every layer are re-encoded on a fourth stream, as in
-        kvlink_linked_prefill_layers_overlapped.  Per layer l: h_q[l], h_k_new[l], h_v_new[l]
-        (pinned host tensors) are copied to q[l], k_new[l], v_new[l] on an input stream; the
-        fresh-row placement and the suffix attention run on the compute stream once they have
-        landed and layer l's caches are in place; out[l] is copied to h_out[l] (pinned) on an
-        output stream once it is written.  The copies of one layer thus overlap the kernels of
-        the layers around it.  Returns after the last output has arrived.
+        h_q, h_k_new, h_v_new, h_out: pinned host tensors [L, n_fresh, heads, D]; the rest
+        device tensors, one per layer (or [L, ...]).  Per layer the fresh rows are copied in on
+        an input stream, the document caches re-encoded on a fourth stream, the placement and
+        attention run on the compute stream, and the output is copied back on an output
+        stream.  streams: optional (input, compute, output) torch.cuda.Stream triple.
 
-        streams: optional (input, compute, output) torch.cuda.Stream triple.
-        wait=False returns once everything is enqueued, so that the host can prepare the
-        next batch (e.g. rebuild_from_batch on the compute stream) while this one runs.
-        Calls on the same object then chain through per-layer events: a layer's inputs are
-        overwritten only after the previous call's kernels of that layer have read them, and
-        its output only after the previous call's copy of it to the host.
+        wait=False returns once everything is enqueued, so that the host can prepare the next
+        batch (rebuild_from_batch on the compute stream) while this one runs; successive calls
+        on this object chain through events the plan keeps.
         """
         if streams is None:
             streams = (torch.cuda.Stream(self.device), torch.cuda.current_stream(self.device),
                        torch.cuda.Stream(self.device))
         s_in, s_c, s_out = streams
-        s_re = self._reencode_stream()
-        n = len(pool_k)
-        prev = getattr(self, "_host_chain", None)
-        if prev is not None and len(prev[0]) != n:
-            prev = None
-        # the document caches of every layer on the re-encode stream (after the work already on
-        # the compute stream, e.g. the plan upload); a layer's cache is rewritten only after the
-        # previous call's attention of that layer has read it
-        ev0 = torch.cuda.Event()
-        ev0.record(s_c)
-        s_re.wait_event(ev0)
-        ev_re = []
-        for l in range(n):
-            if prev is not None:
-                s_re.wait_event(prev[0][l])
-            K.kvlink_reencode_concat(self.plan, pool_k[l].data_ptr(), pool_v[l].data_ptr(), cache_k[l].data_ptr(),
-                                     cache_v[l].data_ptr(), _stream_handle(s_re))
-            e = torch.cuda.Event()
-            e.record(s_re)
-            ev_re.append(e)
-        done_c, done_o = [], []
-        for l in range(n):
-            ev_in = torch.cuda.Event()
-            with torch.cuda.stream(s_in):
-                if prev is not None:
-                    s_in.wait_event(prev[0][l])      # the previous call's layer l read q, k_new, v_new
-                q[l].copy_(h_q[l], non_blocking=True)
-                k_new[l].copy_(h_k_new[l], non_blocking=True)
-                v_new[l].copy_(h_v_new[l], non_blocking=True)
-                ev_in.record(s_in)
-            s_c.wait_event(ev_in)
-            s_c.wait_event(ev_re[l])
-            if prev is not None:
-                s_c.wait_event(prev[1][l])           # the previous call's out[l] reached the host
-            self.suffix_attention(q[l], k_new[l], v_new[l], cache_k[l], cache_v[l], out[l], stream=s_c)
-            ev_out = torch.cuda.Event()
-            ev_out.record(s_c)
-            s_out.wait_event(ev_out)
-            with torch.cuda.stream(s_out):
-                h_out[l].copy_(out[l], non_blocking=True)
-                ev_d2h = torch.cuda.Event()
-                ev_d2h.record(s_out)
-            done_c.append(ev_out)
-            done_o.append(ev_d2h)
-        self._host_chain = (done_c, done_o)
+        for seq in (h_q, h_k_new, h_v_new, h_out):
+            if not all(t.is_pinned() for t in seq):
+                raise ValueError("host tensors must be pinned")
+        ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new,
+                                                      cache_k, cache_v, out, h_out)]
+        K.kvlink_linked_prefill_layers_host(self.plan, *ptrs, self.workspace.data_ptr(), self.workspace.numel(),
+                                            _stream_handle(s_c), _stream_handle(self._reencode_stream()),
+                                            _stream_handle(s_in), _stream_handle(s_out))
         if wait:
             s_out.synchronize()
