@@ -366,11 +366,11 @@ def run_ours(args, rank, world, local_rank):
         e2e = {"value": round(whole_job_us_per_query(e2e_ms, cfg.batch, world), 3), "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(h_out.numel() * 2),
                "steps": e2e_steps,
-               "note": "per step: host plan rebuild + table upload; per layer, fresh q/k/v H2D from pinned "
-                       "memory, linked prefill, output D2H to pinned memory, on three streams so that "
-                       "copies overlap the neighbouring layers' kernels; steps pipelined (the host "
-                       "prepares the next batch while one runs), wall clock from the first step's "
-                       "start to the last output on the host; document pool resident in HBM"}
+               "note": "per step: host plan rebuild + table upload, then kvlink_linked_prefill_layers_host: "
+                       "per layer fresh q/k/v H2D from pinned memory, document re-encode on its own "
+                       "stream, placement + attention, output D2H to pinned memory (four streams); steps "
+                       "pipelined (the host prepares the next batch while one runs), wall clock from the "
+                       "first step's start to the last output on the host; document pool resident in HBM"}
 
     peaks = _peaks()
     cnt = algorithmic_counts(batch, info)
