@@ -400,3 +400,63 @@ def test_paged_pool_reads_the_same_documents():
         rows = O.pool_doc_rows(paged, d, starts, lens, table, bs)
         for t in range(lens[d]):
             assert np.array_equal(rows[t], paged[table[starts[d] + t // bs], t % bs])
+
+
+def test_no_link_tokens_is_block_reuse_with_causal_question():
+    """K = 0 link tokens (the PromptCache / block-attention style reuse the paper compares
+    with): the question attends causally over [prefix, documents in retrieval order,
+    question], every cached key rotated straight to its global position."""
+    rng = np.random.default_rng(11)
+    H, Hq, D, theta = 2, 4, 16, 10000.0
+    P, lens, Q = 3, [5, 2, 4], 3                      # pool entries 0..2: documents, 3: prefix
+    raw = [rng.standard_normal((n, H, D)) for n in lens + [P]]
+    stored = [O.f64_to_bf16_bits(O.rope_rotate(x, np.arange(len(x))[:, None], theta)) for x in raw]
+    pk = np.concatenate(stored)
+    pv = W.f32_to_bf16_bits(rng.standard_normal((sum(lens) + P, H, D)).astype(np.float32))
+    st = np.cumsum([0] + lens)[:4].astype(np.int64)
+    ln = np.asarray(lens + [P], np.int32)
+    order = [2, 0, 1]                                  # retrieval order
+    kn = W.f32_to_bf16_bits(rng.standard_normal((Q, H, D)).astype(np.float32))
+    vn = W.f32_to_bf16_bits(rng.standard_normal((Q, H, D)).astype(np.float32))
+    qn = rng.standard_normal((Q, Hq, D))
+    c = O.reencode_concat(pk, pv, st, ln, 3, order, 0, kn, vn, Q, theta)
+    ours = O.suffix_attention(qn, c.k_exact, O.bf16_bits_to_f64(c.v_bits), c.layout.fresh_pos)
+
+    # the full sequence written out by hand: each entry un-rotated from its local positions
+    # and rotated at its global ones
+    ks, vs, pos = [], [], 0
+    for e in [3] + order:
+        n = int(ln[e])
+        local = np.arange(n)[:, None]
+        raw_k = O.rope_rotate(O.bf16_bits_to_f64(stored[e]), -local, theta)
+        ks.append(O.rope_rotate(raw_k, pos + local, theta))
+        vs.append(O.bf16_bits_to_f64(pv[st[e]:st[e] + n]))
+        pos += n
+    assert pos == P + sum(lens)
+    seq_k = np.concatenate(ks + [O.bf16_bits_to_f64(kn)])
+    seq_v = np.concatenate(vs + [O.bf16_bits_to_f64(vn)])
+    C = pos + Q
+    causal = [[j <= r for j in range(C)] for r in range(C)]
+    seq_q = np.zeros((C, Hq, D)); seq_q[pos:] = qn
+    full = _bruteforce_full_attention(seq_q.tolist(), seq_k.tolist(), seq_v.tolist(), causal, Hq, H)
+    np.testing.assert_allclose(ours, full[pos:], rtol=0, atol=1e-9)
+
+
+def test_byte_model_of_the_8b_shape():
+    """The paper's cache size for Llama-3-8B, about 131 MB per 1000 tokens, is K and V x 32
+    layers x 8 KV heads x 128 dims x 2 bytes = 131072 B per token.  The 8B-shaped workloads
+    and the bench's algorithmic byte count (cache bytes written per cached token and layer)
+    must follow the same formula."""
+    import bench
+    for idx in (3, 4, 5):
+        cfg = W.get_config(idx)
+        assert 2 * cfg.layers * cfg.h_kv * cfg.head_dim * 2 == 131072, idx
+    assert abs(131072 * 1000 / 1e6 - 131) < 0.1
+
+    class Info:                                        # the plan fields the count reads
+        cached_tokens, n_fresh, ctx_rows, attn_pairs = 1000, 0, 1000, 0
+
+    batch = W.draw_batch(W.get_config(3))
+    cnt = bench.algorithmic_counts(batch, Info())
+    written_per_layer = cnt["reencode_bytes"] - 2 * batch.cfg.h_kv * batch.cfg.head_dim * 2 * cnt["unique_pool_tokens"]
+    assert written_per_layer * batch.cfg.layers == 131072 * 1000
