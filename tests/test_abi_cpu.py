@@ -275,3 +275,25 @@ def test_failed_rebuild_leaves_no_batch(K):
     assert e.value.code == K.KVLINK_EINVAL
     K.kvlink_plan_rebuild(plan, **_plan_kwargs(batch))  # usable again
     assert _tables(K, plan) == _tables(K, _plan(K, batch))
+
+
+def test_null_tables_in_the_description_are_rejected(K):
+    """A NULL host table in kvlink_batch_desc_t (or a NULL description / output) is EINVAL."""
+    import ctypes as C
+    batch = W.draw_batch(W.get_config(1))
+    d, keep = K._batch_desc(batch.cfg.n_link, batch.cfg.h_q, batch.cfg.h_kv, batch.cfg.head_dim, batch.pool_len,
+                            batch.pool_start, batch.pool_rows, batch.prefix_doc, batch.n_docs, batch.doc_ids,
+                            batch.q_len, 0, None, 152, 0)
+    h = C.c_void_p()
+    assert K.lib.kvlink_plan_create(C.byref(d), C.byref(h)) == 0
+    K.lib.kvlink_plan_destroy(h)
+    for field in ("pool_len", "pool_start", "prefix_doc", "n_docs", "q_len", "doc_ids"):
+        saved = getattr(d, field)
+        setattr(d, field, None)
+        h = C.c_void_p()
+        assert K.lib.kvlink_plan_create(C.byref(d), C.byref(h)) == K.KVLINK_EINVAL, field
+        assert not h.value
+        setattr(d, field, saved)
+    assert K.lib.kvlink_plan_create(None, C.byref(h)) == K.KVLINK_EINVAL
+    assert K.lib.kvlink_plan_create(C.byref(d), None) == K.KVLINK_EINVAL
+    assert K.lib.kvlink_plan_rebuild(None, C.byref(d)) == K.KVLINK_EINVAL
