@@ -377,6 +377,11 @@ int kvlink_suffix_attention_noalloc(const kvlink_plan_t* plan, const void* d_q, 
  * current device.  Errors: ECUDA. */
 #define KVLINK_STATUS_WAIT_TIMEOUT 0x41
 #define KVLINK_STATUS_COPY_TIMEOUT 0x21
+/* Only in the build with KVLINK_DEBUG_CHECKS (libkvlink_debug.so): a work item or merge
+ * group of the suffix attention (0x42), or a re-encode unit or fresh-row destination (0x22),
+ * lies outside the plan's tables; the CTA that found it did nothing else. */
+#define KVLINK_STATUS_BAD_INDEX_ATTN 0x42
+#define KVLINK_STATUS_BAD_INDEX_COPY 0x22
 int kvlink_device_status(int32_t* status);
 int kvlink_clear_device_status(void);
 

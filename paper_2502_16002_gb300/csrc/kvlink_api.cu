@@ -18,8 +18,8 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
 void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int h_kv, int num_sms, int n_layers,
                             const void* const* pool_k, const void* const* pool_v, void* const* cache_k,
                             void* const* cache_v, cudaStream_t stream);
-void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int row_bytes, const void* k_new,
-                        const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
+void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int64_t ctx_rows, int row_bytes,
+                        const void* k_new, const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
 int read_copy_status(int32_t* status);
 void launch_rope_fresh(const int32_t* d_fresh_pos, int n_fresh, int head_dim, double theta, void* q, int h_q,
                        void* k, int h_kv, cudaStream_t stream);
@@ -305,6 +305,13 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     d.fresh_vis = (const int32_t*)(b + p->off_fresh_vis);
     d.fresh_row0 = (const int32_t*)(b + p->off_fresh_row0);
     d.fresh_dst = (const int32_t*)(b + p->off_fresh_dst);
+    d.batch = p->batch;
+    d.h_kv = p->h_kv;
+    d.n_fresh = p->cu_fresh.back();
+    d.n_slots = p->n_slots;
+    d.n_rope_rows = p->n_rope_rows;
+    d.ctx_rows = p->cu_ctx.back();
+    d.pool_rows = p->pool_rows;
     launch_rope_table(d.seg, (int)p->seg.size(), (float4*)(b + p->off_rope), p->head_dim, theta, s);
     rc = check_launch("rope_table_kernel");
     if (rc != KVLINK_OK) return rc;
@@ -348,8 +355,8 @@ int kvlink_reencode_concat_layers(const kvlink_plan_t* p, int32_t n_layers, cons
 
 static int place_fresh(const kvlink_plan_t* p, const void* k_new, const void* v_new, void* cache_k,
                        void* cache_v, cudaStream_t s) {
-    launch_place_fresh(p->dev.fresh_dst, p->cu_fresh.back(), p->h_kv * p->head_dim * 2, k_new, v_new, cache_k,
-                       cache_v, s);
+    launch_place_fresh(p->dev.fresh_dst, p->cu_fresh.back(), p->cu_ctx.back(), p->h_kv * p->head_dim * 2, k_new,
+                       v_new, cache_k, cache_v, s);
     return check_launch("place_fresh_kernel");
 }
 

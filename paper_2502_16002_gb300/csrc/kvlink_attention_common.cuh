@@ -22,6 +22,19 @@ namespace kvlink {
 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 constexpr int32_t kAttnStatusWaitTimeout = 0x41;
+constexpr int32_t kAttnStatusBadIndex = 0x42;    // KVLINK_DEBUG_CHECKS: a table entry out of bounds
+
+// Whether a work item lies inside the plan's tables (checked by the KVLINK_DEBUG_CHECKS build
+// before any access through the item).  Key-tile rows past a query's cache are read as zeros
+// by TMA, so only the plan's own indices need checking.
+__device__ __forceinline__ bool item_in_bounds(const AttnItem& it, const DevicePlan& P) {
+    if (it.query < 0 || it.query >= P.batch || it.kv_head < 0 || it.kv_head >= P.h_kv) return false;
+    const int n_fresh_q = P.cu_fresh[it.query + 1] - P.cu_fresh[it.query];
+    if (it.tok0 < 0 || it.tok0 >= it.tok1 || it.tok1 > n_fresh_q) return false;
+    if (it.kv_tile0 < 0 || it.kv_tile1 < it.kv_tile0 || it.a_tiles < 0 || it.b_tile0 < 0) return false;
+    if (it.slot < -1 || it.slot >= P.n_slots) return false;
+    return true;
+}
 constexpr float kRescaleThreshold = 8.0f;         // log2 units: rescale O when the max grows by > 2^8
 #ifndef KVLINK_EXP_POLY_FROM
 #define KVLINK_EXP_POLY_FROM 8                     // column pairs c with (c % 8) >= this use exp2_poly2

@@ -86,6 +86,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         // after a recorded failure, later launches skip their work instead of waiting out their bounds
         *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_attn_status) != 0 ? 1 : 0;
+#ifdef KVLINK_DEBUG_CHECKS
+        if (!*abort_flag && !item_in_bounds(it, P)) {
+            atomicCAS(&g_attn_status, 0, kAttnStatusBadIndex);
+            *abort_flag = 1;
+        }
+#endif
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
@@ -102,7 +108,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
     const bool skip = *abort_flag != 0;  // written before the barrier: uniform across the CTA
-    const int ctx0 = (int)P.cu_ctx[it.query];
+    const int ctx0 = skip ? 0 : (int)P.cu_ctx[it.query];
 
     if (skip) {
         // nothing issued: fall through to the teardown
@@ -152,6 +158,14 @@ template <int D>
 __global__ void __launch_bounds__(256) attn_merge_kernel(DevicePlan P, const float* __restrict__ ws,
                                                          __nv_bfloat16* __restrict__ out, int h_q, int G) {
     const MergeGroup mg = P.merges[blockIdx.x];
+#ifdef KVLINK_DEBUG_CHECKS
+    if (mg.query < 0 || mg.query >= P.batch || mg.kv_head < 0 || mg.kv_head >= P.h_kv || mg.tok0 < 0 ||
+        mg.tok1 < mg.tok0 || mg.tok1 > P.cu_fresh[mg.query + 1] - P.cu_fresh[mg.query] || mg.slot0 < 0 ||
+        mg.n_split < 1 || mg.slot0 + mg.n_split > P.n_slots) {
+        if (threadIdx.x == 0) atomicCAS(&g_attn_status, 0, kAttnStatusBadIndex);
+        return;
+    }
+#endif
     const int n_rows = (mg.tok1 - mg.tok0) * G;
     const int f0 = P.cu_fresh[mg.query];
     const int64_t slot_floats = (int64_t)kAttnBM * (D + 2);

@@ -65,6 +65,14 @@ __host__ __device__ inline int32_t item_tile(const AttnItem& it, int32_t v) {
 // fresh_row0 of a query without a fresh region at the end (interleaved layout)
 constexpr int32_t kNoFreshRegion = 0x3fffffff;
 
+// Bounds of the re-encode and placement kernels' tables (device-side checks).
+struct CopyBounds {
+    int64_t ctx_rows;    // rows of the linked cache
+    int64_t pool_rows;   // rows of the pool tensor
+    int32_t n_fresh;     // fresh rows
+    int32_t n_rope_rows; // rows of the RoPE delta table
+};
+
 // Rows of one (query, KV head, M-tile) whose KV range was split over several items.
 struct MergeGroup {
     int32_t query;
@@ -98,6 +106,9 @@ struct DevicePlan {
     const int32_t* fresh_vis;    // [n_fresh]
     const int32_t* fresh_row0;   // [B], query-relative
     const int32_t* fresh_dst;    // [n_fresh] batch cache row of every fresh row
+    // sizes the tables index into (checked on the device by the KVLINK_DEBUG_CHECKS build)
+    int32_t batch, h_kv, n_fresh, n_slots, n_rope_rows;
+    int64_t ctx_rows, pool_rows;
     // Groups of 8 cache rows (8m .. 8m+7 of a query), at cu_grp[b] + m: the first source
     // row when the group's 8 rows are consecutive in one tensor (one 8-row TMA copy), else
     // -1 (rows copied one by one; also the query's last, partial group).

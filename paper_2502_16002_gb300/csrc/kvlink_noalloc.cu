@@ -26,8 +26,8 @@ namespace kvlink {
 void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv, int num_sms,
                      const void* pool_k, const void* pool_v, const void* k_new, const void* v_new, void* cache_k,
                      void* cache_v, cudaStream_t stream);
-void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int row_bytes, const void* k_new,
-                        const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
+void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int64_t ctx_rows, int row_bytes,
+                        const void* k_new, const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
 int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t ctx_rows,
                         int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err);
@@ -74,8 +74,8 @@ extern "C" int kvlink_suffix_attention_noalloc(const kvlink_plan_t* p, const voi
     if (rc != KVLINK_OK) return rc;
     cudaStream_t s = (cudaStream_t)stream;
     if (k_new) {
-        kvlink::launch_place_fresh(p->dev.fresh_dst, p->cu_fresh.back(), p->h_kv * p->head_dim * 2, k_new, v_new,
-                                   cache_k, cache_v, s);
+        kvlink::launch_place_fresh(p->dev.fresh_dst, p->cu_fresh.back(), p->cu_ctx.back(), p->h_kv * p->head_dim * 2,
+                                   k_new, v_new, cache_k, cache_v, s);
         if (cudaGetLastError() != cudaSuccess) return KVLINK_ECUDA;
     }
     cudaError_t err = cudaSuccess;

@@ -61,6 +61,7 @@ constexpr int kCopyThreads = 32 + kCopyConsumers;    // + 1 producer warp
 constexpr int kCopyStages = 3;
 constexpr uint64_t kCopyWaitLimitNs = 2000000000ull;
 constexpr int32_t kCopyStatusWaitTimeout = 0x21;
+constexpr int32_t kCopyStatusBadIndex = 0x22;   // KVLINK_DEBUG_CHECKS: a table entry out of bounds
 
 static __device__ int32_t g_copy_status;
 
@@ -132,7 +133,8 @@ __device__ __forceinline__ bool same_source(const CopyChunk& a, int la, const Co
 template <int D, int MAXL>
 __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     const CopyChunk* __restrict__ chunks, int n_chunks, int n_layers, const float4* __restrict__ rope, int h_kv,
-    const LayerPtrs<MAXL> L, const __nv_bfloat16* __restrict__ k_new, const __nv_bfloat16* __restrict__ v_new) {
+    const LayerPtrs<MAXL> L, const __nv_bfloat16* __restrict__ k_new, const __nv_bfloat16* __restrict__ v_new,
+    const CopyBounds bounds) {
     using namespace sm100;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
@@ -165,6 +167,24 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
             mbar_init(empty + i, 1);
         }
         *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_copy_status) != 0 ? 1 : 0;
+#ifdef KVLINK_DEBUG_CHECKS
+        // every unit of this CTA inside its tensors, before any copy uses one
+        const int max_rows = kCopyStageBytes / (int)row_bytes;
+        for (int c = c_begin; c < c_end && !*abort_flag; ++c) {
+            const int layer = MAXL == 1 ? 0 : c / n_chunks;
+            const CopyChunk ch = chunks[c - layer * n_chunks];
+            const bool fresh = ch.kind == KVLINK_SEG_LINK || ch.kind == KVLINK_SEG_QUESTION;
+            const bool ok = ch.n >= 1 && ch.n <= max_rows && ch.dst_row >= 0 && ch.dst_row + ch.n <= bounds.ctx_rows &&
+                            ch.src_row >= 0 &&
+                            ch.src_row + ch.n <= (fresh ? (int64_t)bounds.n_fresh : bounds.pool_rows) &&
+                            (fresh ? (k_new != nullptr && v_new != nullptr) : (L.pool_k[layer] != nullptr)) &&
+                            (ch.kind != KVLINK_SEG_DOC || (ch.table >= 0 && ch.table < bounds.n_rope_rows));
+            if (!ok) {
+                atomicCAS(&g_copy_status, 0, kCopyStatusBadIndex);
+                *abort_flag = 1;
+            }
+        }
+#endif
         fence_mbar_init();
     }
     __syncthreads();
@@ -256,7 +276,7 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
 template <int D, int MAXL>
 static void launch_reencode_t(const CopyChunk* ch, int n_chunks, int n_layers, const float4* rope, int h_kv,
                               int num_sms, const LayerPtrs<MAXL>& L, const void* k_new, const void* v_new,
-                              cudaStream_t stream) {
+                              const CopyBounds& bounds, cudaStream_t stream) {
     static bool attr = false;
     if (!attr) {
         cudaFuncSetAttribute(reencode_kernel<D, MAXL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -266,7 +286,7 @@ static void launch_reencode_t(const CopyChunk* ch, int n_chunks, int n_layers, c
     const int64_t n_units = (int64_t)n_chunks * n_layers;
     const int grid = n_units < num_sms ? (int)n_units : num_sms;
     reencode_kernel<D, MAXL><<<grid, kCopyThreads, CopySmem::BYTES, stream>>>(
-        ch, n_chunks, n_layers, rope, h_kv, L, (const __nv_bfloat16*)k_new, (const __nv_bfloat16*)v_new);
+        ch, n_chunks, n_layers, rope, h_kv, L, (const __nv_bfloat16*)k_new, (const __nv_bfloat16*)v_new, bounds);
 }
 
 void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv, int num_sms,
@@ -276,10 +296,11 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
     using bf = __nv_bfloat16;
     LayerPtrs<1> L{{(const bf*)pool_k}, {(const bf*)pool_v}, {(bf*)cache_k}, {(bf*)cache_v}};
     const CopyChunk* ch = P.chunks + chunk_base;
+    const CopyBounds bounds{P.ctx_rows, P.pool_rows, P.n_fresh, P.n_rope_rows};
     if (head_dim == 128)
-        launch_reencode_t<128, 1>(ch, n_chunks, 1, P.rope, h_kv, num_sms, L, k_new, v_new, stream);
+        launch_reencode_t<128, 1>(ch, n_chunks, 1, P.rope, h_kv, num_sms, L, k_new, v_new, bounds, stream);
     else
-        launch_reencode_t<64, 1>(ch, n_chunks, 1, P.rope, h_kv, num_sms, L, k_new, v_new, stream);
+        launch_reencode_t<64, 1>(ch, n_chunks, 1, P.rope, h_kv, num_sms, L, k_new, v_new, bounds, stream);
 }
 
 // The document chunks (sorted by source) of n_layers layers, kMaxLayersPerLaunch layers per launch.
@@ -299,12 +320,13 @@ void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int
             L.cache_k[l] = (bf*)cache_k[l0 + l];
             L.cache_v[l] = (bf*)cache_v[l0 + l];
         }
+        const CopyBounds bounds{P.ctx_rows, P.pool_rows, P.n_fresh, P.n_rope_rows};
         if (head_dim == 128)
             launch_reencode_t<128, kMaxLayersPerLaunch>(P.chunks_sorted, n_chunks, nl, P.rope, h_kv, num_sms, L,
-                                                        nullptr, nullptr, stream);
+                                                        nullptr, nullptr, bounds, stream);
         else
             launch_reencode_t<64, kMaxLayersPerLaunch>(P.chunks_sorted, n_chunks, nl, P.rope, h_kv, num_sms, L,
-                                                       nullptr, nullptr, stream);
+                                                       nullptr, nullptr, bounds, stream);
     }
 }
 
@@ -316,7 +338,7 @@ void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int
 constexpr int kPlaceWarps = 8;
 
 __global__ void __launch_bounds__(32 * kPlaceWarps) place_fresh_kernel(const int32_t* __restrict__ fresh_dst,
-                                                                       int n_fresh, int row_vec,
+                                                                       int n_fresh, int64_t ctx_rows, int row_vec,
                                                                        const uint4* __restrict__ k_new,
                                                                        const uint4* __restrict__ v_new,
                                                                        uint4* __restrict__ cache_k,
@@ -325,6 +347,12 @@ __global__ void __launch_bounds__(32 * kPlaceWarps) place_fresh_kernel(const int
     if (*reinterpret_cast<volatile int32_t*>(&g_copy_status) != 0) return;
     const int row = blockIdx.x * kPlaceWarps + threadIdx.x / 32, lane = threadIdx.x % 32;
     if (row >= n_fresh) return;
+#ifdef KVLINK_DEBUG_CHECKS
+    if (fresh_dst[row] < 0 || fresh_dst[row] >= ctx_rows) {
+        if (lane == 0) atomicCAS(&g_copy_status, 0, kCopyStatusBadIndex);
+        return;
+    }
+#endif
     const int64_t src = (int64_t)row * row_vec, dst = (int64_t)fresh_dst[row] * row_vec;
     for (int i0 = lane; i0 < row_vec; i0 += 4 * 32) {
         uint4 k[4], v[4];
@@ -347,11 +375,11 @@ __global__ void __launch_bounds__(32 * kPlaceWarps) place_fresh_kernel(const int
     }
 }
 
-void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int row_bytes, const void* k_new, const void* v_new,
-                        void* cache_k, void* cache_v, cudaStream_t stream) {
+void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int64_t ctx_rows, int row_bytes, const void* k_new,
+                        const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream) {
     if (n_fresh <= 0) return;
     const int blocks = (n_fresh + kPlaceWarps - 1) / kPlaceWarps;
-    place_fresh_kernel<<<blocks, 32 * kPlaceWarps, 0, stream>>>(d_fresh_dst, n_fresh, row_bytes / 16,
+    place_fresh_kernel<<<blocks, 32 * kPlaceWarps, 0, stream>>>(d_fresh_dst, n_fresh, ctx_rows, row_bytes / 16,
                                                                 (const uint4*)k_new, (const uint4*)v_new,
                                                                 (uint4*)cache_k, (uint4*)cache_v);
 }

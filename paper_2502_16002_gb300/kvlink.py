@@ -29,6 +29,7 @@ KVLINK_SEG_PREFIX, KVLINK_SEG_DOC, KVLINK_SEG_LINK, KVLINK_SEG_QUESTION = 0, 1, 
 KVLINK_LAYOUT_INTERLEAVED, KVLINK_LAYOUT_LINKS_AT_END = 0, 1
 KVLINK_SRC_POOL, KVLINK_SRC_FRESH = 0, 1
 KVLINK_STATUS_WAIT_TIMEOUT, KVLINK_STATUS_COPY_TIMEOUT = 0x41, 0x21
+KVLINK_STATUS_BAD_INDEX_ATTN, KVLINK_STATUS_BAD_INDEX_COPY = 0x42, 0x22
 
 
 class kvlink_batch_desc_t(C.Structure):

@@ -39,6 +39,16 @@ def test_library_exports_every_declared_function(K):
     assert set(names) == set(K.DECLARED)
 
 
+def test_debug_build_exports_the_same_functions(K):
+    """libkvlink_debug.so (device-side index checks) is the same C ABI."""
+    path = os.path.join(os.path.dirname(K._LIB_PATH), "libkvlink_debug.so")
+    if not os.path.exists(path):
+        pytest.skip("the debug library has not been built")
+    lib = ctypes.CDLL(path)
+    for n in _declared_functions():
+        assert hasattr(lib, n), n
+
+
 def _plan(K, batch, **over):
     cfg = batch.cfg
     kw = dict(n_link=cfg.n_link, h_q=cfg.h_q, h_kv=cfg.h_kv, head_dim=cfg.head_dim,
