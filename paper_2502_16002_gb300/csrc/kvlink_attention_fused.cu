@@ -436,13 +436,12 @@ template <int D, int G>
 static cudaError_t launch_fused_dg(const FusedMaps& M, const DevicePlan& P, const FusedArgs& A, int n_items,
                                    cudaStream_t stream) {
     using C = FusedCfg<D>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(attn_fused_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)C::SMEM_BYTES);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<uint64_t> attr_set{0};
+    cudaError_t ea = once_per_device(attr_set, [] {
+        return cudaFuncSetAttribute(attn_fused_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)C::SMEM_BYTES);
+    });
+    if (ea != cudaSuccess) return ea;
     if (n_items > 0) attn_fused_kernel<D, G><<<n_items, kFusedThreads, C::SMEM_BYTES, stream>>>(M, P, A);
     return cudaGetLastError();
 }

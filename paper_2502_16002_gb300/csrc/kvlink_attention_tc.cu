@@ -220,13 +220,12 @@ static cudaError_t launch_tc_dg(const CUtensorMap& mq, const CUtensorMap& mk, co
                                 const DevicePlan& P, int n_items, int n_merges, void* out, float* ws, int h_q,
                                 float scale_log2, cudaStream_t stream) {
     using C = TcCfg<D>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)C::SMEM_BYTES);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<uint64_t> attr_set{0};
+    cudaError_t ea = once_per_device(attr_set, [] {
+        return cudaFuncSetAttribute(attn_tc_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)C::SMEM_BYTES);
+    });
+    if (ea != cudaSuccess) return ea;
     if (n_items > 0)
         attn_tc_kernel<D, G><<<n_items, kTcThreads, C::SMEM_BYTES, stream>>>(
             mq, mk, mv, P, (__nv_bfloat16*)out, ws, h_q, scale_log2);

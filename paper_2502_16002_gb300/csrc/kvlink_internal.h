@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 #include <vector_types.h>
 
+#include <atomic>
 #include <string>
 #include <utility>
 #include <vector>
@@ -64,6 +65,21 @@ __host__ __device__ inline int32_t item_tile(const AttnItem& it, int32_t v) {
 
 // fresh_row0 of a query without a fresh region at the end (interleaved layout)
 constexpr int32_t kNoFreshRegion = 0x3fffffff;
+
+// Runs `fn` (a kernel attribute setter) once per device: such attributes belong to the
+// device's context, so a process that launches on several devices needs the call on each.
+// Thread-safe; concurrent first calls may both run `fn`, which is idempotent.
+template <typename Fn>
+inline cudaError_t once_per_device(std::atomic<uint64_t>& done, Fn&& fn) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = dev >= 0 && dev < 64 ? (uint64_t)1 << dev : 0;
+    if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+    e = fn();
+    if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+    return e;
+}
 
 // Bounds of the re-encode and placement kernels' tables (device-side checks).
 struct CopyBounds {

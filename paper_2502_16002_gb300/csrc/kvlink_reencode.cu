@@ -277,12 +277,12 @@ template <int D, int MAXL>
 static void launch_reencode_t(const CopyChunk* ch, int n_chunks, int n_layers, const float4* rope, int h_kv,
                               int num_sms, const LayerPtrs<MAXL>& L, const void* k_new, const void* v_new,
                               const CopyBounds& bounds, cudaStream_t stream) {
-    static bool attr = false;
-    if (!attr) {
-        cudaFuncSetAttribute(reencode_kernel<D, MAXL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)CopySmem::BYTES);
-        attr = true;
-    }
+    // a failure here surfaces as the launch error, which the caller checks
+    static std::atomic<uint64_t> attr{0};
+    once_per_device(attr, [] {
+        return cudaFuncSetAttribute(reencode_kernel<D, MAXL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)CopySmem::BYTES);
+    });
     const int64_t n_units = (int64_t)n_chunks * n_layers;
     const int grid = n_units < num_sms ? (int)n_units : num_sms;
     reencode_kernel<D, MAXL><<<grid, kCopyThreads, CopySmem::BYTES, stream>>>(
