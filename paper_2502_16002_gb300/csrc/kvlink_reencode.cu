@@ -61,7 +61,9 @@ constexpr int kCopyThreads = 32 + kCopyConsumers;    // + 1 producer warp
 constexpr int kCopyStages = 3;
 constexpr uint64_t kCopyWaitLimitNs = 2000000000ull;
 constexpr int32_t kCopyStatusWaitTimeout = 0x21;
-constexpr int32_t kCopyStatusBadIndex = 0x22;   // KVLINK_DEBUG_CHECKS: a table entry out of bounds
+#ifdef KVLINK_DEBUG_CHECKS
+constexpr int32_t kCopyStatusBadIndex = 0x22;   // a table entry out of bounds
+#endif
 
 static __device__ int32_t g_copy_status;
 
