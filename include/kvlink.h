@@ -8,17 +8,28 @@
  * attending over the linked cache under KVLink's mask (Sec. 2.3, Fig. 2).  This
  * library is the per-layer attention-side work of that step:
  *
- *   kvlink_plan_create / kvlink_plan_upload     segment table and RoPE delta table
+ *   kvlink_plan_create / _rebuild / _upload     segment table and RoPE delta table
  *   kvlink_reencode_concat                      re-encode + gather/concat cached K/V
  *   kvlink_suffix_attention                     fresh rows attend over the linked cache
  *   kvlink_linked_prefill                       both, chained, for one layer
+ *   kvlink_linked_prefill_layers[_overlapped]   every layer in one call (the re-encode of
+ *                                               all layers on a second stream)
+ *   kvlink_linked_prefill_layers_host           the same from and to host memory
+ *   kvlink_linked_prefill_fused                 one kernel per layer (keys rotated on load)
+ *   kvlink_reencode_concat_layers, kvlink_rope_fresh, kvlink_suffix_attention_simt,
+ *   kvlink_suffix_attention_noalloc, kvlink_device_status, kvlink_selftest_wait_timeout
+ *
+ * libkvlink_debug.so is the same ABI built with device-side checks of every index table
+ * entry the kernels use (KVLINK_STATUS_BAD_INDEX_*).
  *
  * Conventions shared by every call
  *   - Tensors are bf16, "NHD" per layer: [rows][heads][head_dim], rows contiguous.
  *   - Pointers named d_* or documented as "device" are device memory; "host"
  *     pointers are read during the call only.  The caller owns every buffer; the
- *     library allocates no device memory.  kvlink_plan_create allocates the plan's
- *     host tables (freed by kvlink_plan_destroy).
+ *     library allocates no device memory.  A plan owns host memory only: its tables
+ *     (kvlink_plan_create), a pinned staging buffer (kvlink_plan_upload) and the CUDA
+ *     events of the all-layers calls, all freed by kvlink_plan_destroy.  Calls that use
+ *     one plan must not run concurrently from several host threads.
  *   - Device work is enqueued on `stream` (a cudaStream_t; NULL = legacy default)
  *     and is asynchronous.  Arguments are validated on the host before anything is
  *     launched; a call that returns an error has launched nothing.
@@ -213,7 +224,8 @@ int kvlink_reencode_concat(const kvlink_plan_t* plan, const void* d_pool_k, cons
 
 /* Suffix attention of one layer (Sec. 2.3, "inference"):
  *   if d_k_new/d_v_new are non-NULL, fresh rows are first written to their slots:
- *     cache_k[cu_ctx[b] + fresh_pos[r]] = k_new[r] (same for v);
+ *     cache_k[slot(r)] = k_new[r] (same for v), slot(r) = cu_ctx[b] + fresh_pos[r] in
+ *     the interleaved layout, the query's fresh region in the links-at-end layout;
  *   then for every fresh row r of query b (global position p_r), query head h,
  *   KV head g = h / G:
  *     out[r][h] = sum_j softmax_j(q[r][h] . cache_k[j][g] / sqrt(D)) cache_v[j][g]
