@@ -348,9 +348,12 @@ int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* plan, int32_t n_layer
  * kvlink_plan_rebuild) chain through events the plan keeps: a layer's device inputs and
  * caches are rewritten only after the previous call's kernels of that layer have read
  * them, and its device output only after the previous call's copy of it to the host, so
- * a caller may prepare and enqueue the next batch while one runs.  The four streams must
- * be distinct.  Errors: as kvlink_linked_prefill_layers; EINVAL also for a NULL host
- * pointer or repeated streams. */
+ * a caller may prepare and enqueue the next batch while one runs.  The chain links calls
+ * of this function only: other work that touches the same buffers in between (another
+ * entry point, the caller's kernels) must be ordered by the caller, e.g. by making
+ * copy_in_stream wait for it.  The four streams must be distinct.  Errors: as
+ * kvlink_linked_prefill_layers; EINVAL also for a NULL host pointer or repeated
+ * streams. */
 int kvlink_linked_prefill_layers_host(kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
                                       const void* const* d_pool_v, const void* const* h_q,
                                       const void* const* h_k_new, const void* const* h_v_new, void* const* d_q,
