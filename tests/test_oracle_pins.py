@@ -388,18 +388,65 @@ def test_one_document_no_links_is_standard_causal_attention():
     np.testing.assert_allclose(ours, full[P + L:], rtol=0, atol=1e-9)
 
 
-def test_paged_pool_reads_the_same_documents():
-    rng = np.random.default_rng(10)
-    H, D, bs = 2, 8, 4
-    lens = np.asarray([5, 9, 4], np.int32)
-    nblk = (lens + bs - 1) // bs
-    starts = np.concatenate([[0], np.cumsum(nblk)[:-1]]).astype(np.int64)
-    table = rng.permutation(int(nblk.sum())).astype(np.int32)
-    paged = rng.integers(0, 2**15, size=(int(nblk.sum()), bs, H, D)).astype(np.uint16)
-    for d in range(3):
-        rows = O.pool_doc_rows(paged, d, starts, lens, table, bs)
-        for t in range(lens[d]):
-            assert np.array_equal(rows[t], paged[table[starts[d] + t // bs], t % bs])
+def _page_out(contig, starts, lens, bs, rng):
+    """Store a contiguous pool as pages, the way a paged cache manager would: each
+    document's rows are padded to whole blocks (the padding filled with values that occur
+    nowhere in the documents), cut into [blocks, bs] with a reshape, and the blocks are
+    written to physical pages drawn as a random permutation.  Returns (pages, block table,
+    first logical block of each document)."""
+    H, D = contig.shape[1:]
+    nblk = [(int(L) + bs - 1) // bs for L in lens]
+    first = np.concatenate([[0], np.cumsum(nblk)[:-1]]).astype(np.int64)
+    n_pages = int(sum(nblk)) + 3                   # spare pages nothing maps to
+    table = rng.permutation(n_pages)[: int(sum(nblk))].astype(np.int32)
+    pages = np.full((n_pages, bs, H, D), 0xFFFF, dtype=np.uint16)     # NaN patterns
+    for d, L in enumerate(lens):
+        padded = np.full((nblk[d] * bs, H, D), 0xFFFE, dtype=np.uint16)
+        padded[:L] = contig[starts[d]: starts[d] + L]
+        for i, blk in enumerate(padded.reshape(nblk[d], bs, H, D)):
+            pages[table[first[d] + i]] = blk
+    return pages, table, first
+
+
+@pytest.mark.parametrize("bs", [16, 8])
+def test_paged_pool_reads_the_same_documents(bs):
+    """The paged read of every document equals its contiguous slice, for lengths around
+    the block size (1, bs-1, bs, bs+1) and a long one, through a block table drawn
+    independently of the reader: the pages are written by a reshape of each padded
+    document, not by the row arithmetic the oracle reads them with."""
+    rng = np.random.default_rng(10 + bs)
+    H, D = 2, 8
+    lens = np.asarray([1, bs - 1, bs, bs + 1, 100, 37], np.int32)
+    starts = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int64)
+    contig = rng.integers(0, 2**15, size=(int(lens.sum()), H, D)).astype(np.uint16)
+    pages, table, first = _page_out(contig, starts, lens, bs, rng)
+    for d in range(len(lens)):
+        want = O.pool_doc_rows(contig, d, starts, lens)
+        assert np.array_equal(want, contig[starts[d]: starts[d] + lens[d]])
+        got = O.pool_doc_rows(pages, d, first, lens, table, bs)
+        assert got.shape == want.shape
+        assert np.array_equal(got, want), f"document {d} (length {lens[d]})"
+
+
+def test_paged_pool_gives_the_contiguous_linked_cache():
+    """The whole re-encode + concat from a paged pool equals the one from the same
+    documents stored contiguously, bit for bit (keys and values)."""
+    rng = np.random.default_rng(12)
+    H, D, bs, K, theta = 2, 16, 16, 2, 10000.0
+    lens = np.asarray([17, 1, 16, 40, 15], np.int32)
+    starts = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int64)
+    ck = rng.integers(0, 2**15, size=(int(lens.sum()), H, D)).astype(np.uint16) & 0xBFFF   # finite
+    cv = rng.integers(0, 2**15, size=(int(lens.sum()), H, D)).astype(np.uint16) & 0xBFFF
+    pk, table, first = _page_out(ck, starts, lens, bs, np.random.default_rng(1))
+    pv, table_v, _ = _page_out(cv, starts, lens, bs, np.random.default_rng(1))
+    assert np.array_equal(table, table_v)
+    docs, prefix, Q = [3, 0, 1], 4, 3
+    T = len(docs) * K + Q
+    kn = rng.integers(0, 2**15, size=(T, H, D)).astype(np.uint16) & 0xBFFF
+    vn = rng.integers(0, 2**15, size=(T, H, D)).astype(np.uint16) & 0xBFFF
+    a = O.reencode_concat(ck, cv, starts, lens, prefix, docs, K, kn, vn, Q, theta)
+    b = O.reencode_concat(pk, pv, first, lens, prefix, docs, K, kn, vn, Q, theta, block_table=table, block_size=bs)
+    assert np.array_equal(a.k_bits, b.k_bits) and np.array_equal(a.v_bits, b.v_bits)
 
 
 def test_no_link_tokens_is_block_reuse_with_causal_question():
