@@ -345,10 +345,13 @@ int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* plan, int32_t n_layer
  *   d_out[l] is copied to h_out[l] ([n_fresh][h_q][D]) on copy_out_stream.
  * Returns once everything is enqueued: the outputs are on the host when copy_out_stream
  * has completed the call's work.  Successive calls with one plan (also across
- * kvlink_plan_rebuild) chain through events the plan keeps: a layer's device inputs and
- * caches are rewritten only after the previous call's kernels of that layer have read
- * them, and its device output only after the previous call's copy of it to the host, so
- * a caller may prepare and enqueue the next batch while one runs.  The chain links calls
+ * kvlink_plan_rebuild) chain through events the plan keeps for this function alone: a
+ * layer's device inputs and caches are rewritten only after the previous call's kernels of
+ * that layer have read them, and its device output only after the previous call's copy of
+ * it to the host, so a caller may prepare and enqueue the next batch while one runs.  A
+ * call with another layer count than the previous one is ordered after the whole previous
+ * call instead (its copies in and its re-encode start after the previous call's last
+ * output copy).  The chain links calls
  * of this function only: other work that touches the same buffers in between (another
  * entry point, the caller's kernels) must be ordered by the caller, e.g. by making
  * copy_in_stream wait for it.  The four streams must be distinct.  Errors: as
@@ -375,7 +378,10 @@ int kvlink_linked_prefill_layers_host(kvlink_plan_t* plan, int32_t n_layers, con
  *     rejected with KVLINK_ECAPACITY before anything is launched.
  *   - The first call on a device looks up the array's device address (once per
  *     device, with that device current); make that first call before any stream
- *     capture.
+ *     capture.  The address is kept for the life of the process: resetting the device
+ *     (cudaDeviceReset) after that first call is not supported.
+ *   - CUDA failures are recorded for kvlink_last_cuda_error() like those of every
+ *     other entry point.
  *   - All calls share the array and it keeps the last call's contents; nothing in it
  *     needs to start at zero.  Calls whose work overlaps on the GPU race on it.
  * Errors: EINVAL, ECAPACITY, EUNSUPPORTED, ECUDA. */

@@ -2,6 +2,7 @@
 // host, plan upload, and the launches of the linked-prefill kernels.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstring>
 #include <new>
 #include <string>
@@ -56,6 +57,16 @@ int check_launch(const char* where) {
     const cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? KVLINK_OK : cuda_fail(e, where);
 }
+
+}  // namespace
+
+namespace kvlink {
+// The recorder above, for entry points defined in other translation units.
+int record_cuda_error(cudaError_t e, const char* where) { return cuda_fail(e, where); }
+int record_launch_error(const char* where) { return check_launch(where); }
+}  // namespace kvlink
+
+namespace {
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
@@ -172,6 +183,7 @@ int kvlink_plan_rebuild(kvlink_plan_t* p, const kvlink_batch_desc_t* desc) {
     q.staging = std::move(p->staging);
     // the events of earlier calls still order this plan's next calls after them
     q.events = std::move(p->events);
+    q.host_events = std::move(p->host_events);
     q.host_chain_layers = p->host_chain_layers;
 #define KVLINK_RECYCLE(m) \
     q.m.swap(p->m);       \
@@ -545,20 +557,29 @@ int kvlink_linked_prefill_layers_host(kvlink_plan_t* p, int32_t n_layers, const 
         if (!h_q[l] || !h_k_new[l] || !h_v_new[l] || !h_out[l]) return KVLINK_EINVAL;
     if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
     if (ws && !aligned16(ws)) return KVLINK_EINVAL;
-    // events: [0, L) caches in place, [L, 2L) inputs in place, [2L, 3L) layer computed,
-    // [3L, 4L) output on the host, 4L the call's start.  The previous call's records of the
-    // last two kinds order this call's rewrites of the same buffers after their readers.
-    const bool chained = p->host_chain_layers == n_layers;
-    rc = events_reserve(p->events, 4 * (size_t)n_layers + 1);
+    // events (the plan's host-path pool, used by no other entry point): [0, L) caches in
+    // place, [L, 2L) inputs in place, [2L, 3L) layer computed, [3L, 4L) output on the host,
+    // 4L the call's start.  When the previous call had as many layers, its records of the
+    // last two kinds order this call's rewrites of the same buffers after their readers,
+    // layer by layer.  Otherwise this call is ordered after the whole previous call: `stream`
+    // waits for its last output copy (which followed every layer it computed), and the copy
+    // and re-encode streams wait for this call's start on `stream`.
+    const int32_t prev_layers = p->host_chain_layers;
+    const bool chained = prev_layers == n_layers;
+    rc = events_reserve(p->host_events, 4 * (size_t)std::max(n_layers, prev_layers) + 1);
     if (rc) return rc;
-    cudaEvent_t* ev = p->events.ev.data();
+    cudaEvent_t* ev = p->host_events.ev.data();
     cudaEvent_t *ev_re = ev, *ev_in = ev + n_layers, *ev_c = ev + 2 * n_layers, *ev_o = ev + 3 * n_layers;
     cudaStream_t s = (cudaStream_t)stream, r = (cudaStream_t)reencode_stream, ci = (cudaStream_t)copy_in_stream,
                  co = (cudaStream_t)copy_out_stream;
     const size_t n_fresh = (size_t)p->cu_fresh.back();
     const size_t q_bytes = n_fresh * p->h_q * p->head_dim * 2, kv_bytes = n_fresh * p->h_kv * p->head_dim * 2;
-    cudaError_t e = cudaEventRecord(ev[4 * n_layers], s);
+    cudaError_t e = cudaSuccess;
+    // the previous call's last output copy: waited for before any event is recorded again
+    if (!chained && prev_layers > 0) e = cudaStreamWaitEvent(s, ev[4 * prev_layers - 1], 0);
+    if (e == cudaSuccess) e = cudaEventRecord(ev[4 * n_layers], s);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(r, ev[4 * n_layers], 0);
+    if (e == cudaSuccess && !chained) e = cudaStreamWaitEvent(ci, ev[4 * n_layers], 0);
     if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host: stream order");
     // the document caches of every layer, on the re-encode stream
     for (int l = 0; l < n_layers; ++l) {

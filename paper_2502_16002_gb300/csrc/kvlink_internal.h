@@ -215,6 +215,7 @@ struct kvlink_plan {
     bool built = false;                 // holds a batch (a failed rebuild clears it)
     kvlink::PinnedStaging staging;
     kvlink::EventPool events;           // per-layer events of the overlapped all-layers calls
+    kvlink::EventPool host_events;      // events of the host-path calls (kept apart from the above)
     int32_t host_chain_layers = 0;      // layers of the last host-path call (its events chain the next)
 
     // set by kvlink_plan_upload
@@ -225,6 +226,11 @@ struct kvlink_plan {
 };
 
 namespace kvlink {
+// Record a failed CUDA call for kvlink_last_cuda_error() and return KVLINK_ECUDA
+// (kvlink_api.cu); record_launch_error checks cudaGetLastError() the same way and returns
+// KVLINK_OK when there is nothing to record.
+int record_cuda_error(cudaError_t e, const char* where);
+int record_launch_error(const char* where);
 // Host plan builder (kvlink_plan.cpp).  num_sms must be resolved (> 0).
 int build_plan(const kvlink_batch_desc_t* desc, int32_t num_sms, kvlink_plan* plan,
                std::string* why);

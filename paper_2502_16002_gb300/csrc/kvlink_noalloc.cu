@@ -15,7 +15,9 @@
 // capture.  All calls share the array and it keeps the last call's contents: nothing
 // in it needs to start at zero, because every partial slot the merge reads is written
 // by the same call first.  Two calls whose work overlaps on the GPU (different streams,
-// or different host threads on one device) race on the array.
+// or different host threads on one device) race on the array.  The looked-up address
+// stays cached for the life of the process, so resetting a device (cudaDeviceReset) after
+// the first call on it is not supported: the next call would launch with a stale address.
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -44,12 +46,16 @@ void* g_scratch_addr[kMaxDevices] = {};
 // Device address of the scratch array on the current device (looked up once per device).
 int scratch_on_current_device(void** addr) {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return KVLINK_ECUDA;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return kvlink::record_cuda_error(e, "kvlink_suffix_attention_noalloc: device");
     if (dev < 0 || dev >= kMaxDevices) return KVLINK_EUNSUPPORTED;
     std::lock_guard<std::mutex> lock(g_scratch_mu);
     if (!g_scratch_addr[dev]) {
         void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return KVLINK_ECUDA;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) return kvlink::record_cuda_error(e, "kvlink_suffix_attention_noalloc: scratch address");
+        if (!p)
+            return kvlink::record_cuda_error(cudaErrorInvalidSymbol, "kvlink_suffix_attention_noalloc: scratch address");
         g_scratch_addr[dev] = p;
     }
     *addr = g_scratch_addr[dev];
@@ -76,10 +82,13 @@ extern "C" int kvlink_suffix_attention_noalloc(const kvlink_plan_t* p, const voi
     if (k_new) {
         kvlink::launch_place_fresh(p->dev.fresh_dst, p->cu_fresh.back(), p->cu_ctx.back(), p->h_kv * p->head_dim * 2,
                                    k_new, v_new, cache_k, cache_v, s);
-        if (cudaGetLastError() != cudaSuccess) return KVLINK_ECUDA;
+        rc = kvlink::record_launch_error("place_fresh_kernel (noalloc)");
+        if (rc != KVLINK_OK) return rc;
     }
     cudaError_t err = cudaSuccess;
-    return kvlink::launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
-                                       p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, ws,
-                                       s, &err);
+    rc = kvlink::launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
+                                     p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, ws, s,
+                                     &err);
+    if (rc == KVLINK_ECUDA) return kvlink::record_cuda_error(err, "suffix attention launch (noalloc)");
+    return rc;
 }

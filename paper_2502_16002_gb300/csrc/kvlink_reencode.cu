@@ -236,9 +236,12 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
         const CopyChunk ch0 = chunks[c - layer * n_chunks];
         const int c1 = group_end(c, layer, ch0);
         const int st = g % kCopyStages;
-        copy_wait(full + st, (g / kCopyStages) & 1, abort_flag);
-        named_bar_sync(1, kCopyConsumers);     // every consumer is done with the previous group
-        if (*abort_flag) break;                // uniform: every consumer passed the barrier first
+        const bool loaded = copy_wait(full + st, (g / kCopyStages) & 1, abort_flag);
+        // Every consumer is done with the previous group, and all of them take one decision:
+        // the producer may raise the abort flag at any moment (its own wait ran out), so each
+        // consumer's read of the flag could differ; the barrier ORs them, so either all 128
+        // leave the loop or none does, and no consumer is left waiting at the next barrier.
+        if (named_bar_any(1, kCopyConsumers, !loaded || *abort_flag != 0)) break;
         const uint8_t* stage = smem + st * CopySmem::STAGE;
         const uint32_t bytes = (uint32_t)ch0.n * row_bytes;
         for (int cc = c; cc < c1; ++cc) {

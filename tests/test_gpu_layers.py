@@ -142,3 +142,50 @@ def test_pipelined_host_path_chains_calls(RT):
                                   h_vn[l, :n].to(dev), c_k, c_v, ref)
             torch.cuda.synchronize(dev)
             assert torch.equal(h_out[id(b)][l, :n].view(torch.int16), ref.cpu().view(torch.int16)), (l,)
+
+
+def test_host_path_calls_with_different_layer_counts(RT):
+    """Host-path calls of 4, then 2, then 4 layers, enqueued back to back (wait=False) on one
+    plan and one set of device buffers, each with its own inputs: a call whose layer count
+    differs from the previous one must still rewrite the shared device inputs, caches and
+    outputs only after the previous call is done with them.  Every call's host outputs must
+    equal per-layer kvlink_linked_prefill of its own inputs, bit for bit; the last layer of
+    the last call is also checked against the fp64 oracle."""
+    from paper_2502_16002_gb300 import kvlink as K
+    dev = torch.device("cuda:0")
+    batch = W.draw_batch(W.get_config(2))
+    cfg = batch.cfg
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    calls = [list(range(0, 4)), list(range(4, 6)), list(range(6, 10))]   # source layer of every slot
+    raw = {l: W.pool_kv(batch, l) + W.fresh_qkv(batch, l) for c in calls for l in c}
+    T = int(lp.info.n_fresh)
+    q = torch.empty((4, T, cfg.h_q, cfg.head_dim), dtype=torch.bfloat16, device=dev)
+    kn = torch.empty((4, T, cfg.h_kv, cfg.head_dim), dtype=torch.bfloat16, device=dev)
+    vn = torch.empty_like(kn)
+    ck = torch.empty((4,) + lp.cache_shape(), dtype=torch.bfloat16, device=dev)
+    cv = torch.empty_like(ck)
+    out = torch.empty_like(q)
+    streams = (torch.cuda.Stream(dev), torch.cuda.current_stream(dev), torch.cuda.Stream(dev))
+    results = []
+    for c in calls:
+        n = len(c)
+        pk = [RT.bf16_from_bits(raw[l][0], dev) for l in c]
+        pv = [RT.bf16_from_bits(raw[l][1], dev) for l in c]
+        h_q, h_kn, h_vn = (torch.stack([RT.bf16_from_bits(raw[l][i], None) for l in c]).pin_memory()
+                           for i in (2, 3, 4))
+        h_out = torch.empty((n, T, cfg.h_q, cfg.head_dim), dtype=torch.bfloat16, pin_memory=True)
+        lp.linked_prefill_layers_from_host(pk, pv, h_q, h_kn, h_vn, q[:n], kn[:n], vn[:n], ck[:n], cv[:n],
+                                           out[:n], h_out, streams=streams, wait=False)
+        results.append((c, pk, pv, h_q, h_kn, h_vn, h_out))
+    torch.cuda.synchronize(dev)
+    assert K.kvlink_device_status() == 0
+    for c, pk, pv, h_q, h_kn, h_vn, h_out in results:
+        for i, l in enumerate(c):
+            c_k, c_v = lp.empty_cache()
+            ref = torch.empty(lp.fresh_shape(cfg.h_q), dtype=torch.bfloat16, device=dev)
+            lp.linked_prefill(pk[i], pv[i], h_q[i].to(dev), h_kn[i].to(dev), h_vn[i].to(dev), c_k, c_v, ref)
+            torch.cuda.synchronize(dev)
+            assert torch.equal(h_out[i].view(torch.int16), ref.cpu().view(torch.int16)), (c, l)
+    c, *_, h_out = results[-1]
+    gk, gv = RT.bits_from_bf16(ck[len(c) - 1]), RT.bits_from_bf16(cv[len(c) - 1])
+    check_query(batch, 0, lp, gk, gv, h_out[len(c) - 1].float().numpy().astype(np.float64), raw[c[-1]])
