@@ -29,6 +29,7 @@ from __future__ import annotations
 
 import argparse
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -46,13 +47,33 @@ import workloads as W  # noqa: E402
 METRIC = "linked-prefill us/query (all layers, 8B-shape)"
 UNIT = "us/query"
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch from the committed ncu
-# summaries under profiles/, keyed by (kernel, workload); None until captured for
-# the current kernel version.
-NCU_TRAFFIC = {
-    ("attention", 3): 259171328,   # profiles/attention_tc_llama8b_b8_zipf.md
-    ("reencode", 3): 214893056,    # profiles/reencode_llama8b_b8_zipf.md (cached rows)
+# dram__bytes_read.sum + dram__bytes_write.sum per launch, from one ncu capture of the
+# kernel on the workload, keyed by (kernel, workload).  Each figure carries the hash of the
+# sources that built the captured kernel (and planned its launch): when they change, the
+# figure no longer describes the kernel being timed and the line reports traffic null.
+KERNEL_SOURCES = {
+    "attention": ["kvlink_attention_tc.cu", "kvlink_attention_common.cuh", "kvlink_sm100.cuh",
+                  "kvlink_internal.h", "kvlink_plan.cpp"],
+    "reencode": ["kvlink_reencode.cu", "kvlink_rope.cuh", "kvlink_sm100.cuh", "kvlink_internal.h",
+                 "kvlink_plan.cpp"],
 }
+NCU_TRAFFIC = {}    # (kernel, workload index) -> (bytes per launch, source hash)
+
+
+def source_hash(kernel: str) -> str:
+    """sha256 (first 16 hex digits) over the sources of one kernel."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES[kernel]:
+        with open(os.path.join(ROOT, "paper_2502_16002_gb300", "csrc", f), "rb") as fh:
+            h.update(f.encode() + b"\0" + fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(kernel: str, workload: int):
+    """Measured DRAM bytes per launch when the capture matches the current sources, else None."""
+    rec = NCU_TRAFFIC.get((kernel, workload))
+    return rec[0] if rec and rec[1] == source_hash(kernel) else None
 
 
 def _peaks():
@@ -75,7 +96,7 @@ def _cores():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 200 ms in a background reader.
+    """nvidia-smi clocks and throttle reasons sampled every interval_ms in a background reader.
 
     Each line is stamped when it arrives; summary() keeps the samples that fall inside
     the window marked with start() / stop()."""
@@ -84,8 +105,9 @@ class ClockSampler:
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, interval_ms: int = 50):
         self.gpu = gpu_index
+        self.interval_ms = int(interval_ms)
         self.proc = None
         self.lines = []
         self.t0 = self.t1 = None
@@ -95,7 +117,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", str(self.interval_ms)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except (FileNotFoundError, OSError):
             self.proc = None
             return self
@@ -136,7 +158,8 @@ class ClockSampler:
             if len(f) < 8:
                 continue
             n_all += 1
-            if self.t0 is not None and not (self.t0 - 0.2 <= t <= self.t1 + 0.2):
+            pad = self.interval_ms / 1000.0
+            if self.t0 is not None and not (self.t0 - pad <= t <= self.t1 + pad):
                 continue
             try:
                 sm.append(float(f[0]))
@@ -201,238 +224,303 @@ def rank_batch_seed(rank: int) -> int:
 
 # ------------------------------------------------------------------ our arm
 
-def run_ours(args, rank, world, local_rank):
-    import torch
+class Workload:
+    """One workload resident on the device: its plan, every layer's pool, fresh rows, linked
+    cache and output, and the library calls of one step."""
 
-    from paper_2502_16002_gb300 import kvlink as K
-    from paper_2502_16002_gb300.runtime import LinkedPrefill
+    def __init__(self, args, cfg_index, rank, dev):
+        import torch
 
-    dev = torch.device("cuda", local_rank)
-    torch.cuda.set_device(dev)
-    cfg = W.get_config(args.config)
-    batch = W.draw_batch(cfg, seed=rank_batch_seed(rank))   # every rank serves its own batch
-    L = args.layers or cfg.layers
-    layout = {"interleaved": K.KVLINK_LAYOUT_INTERLEAVED, "links_at_end": K.KVLINK_LAYOUT_LINKS_AT_END}[args.layout]
-    lp = LinkedPrefill.from_batch(batch, device=dev, layout=layout)
-    info = lp.info
-    ctx, T = int(info.ctx_rows), int(info.n_fresh)
-    H, Hq, D = cfg.h_kv, cfg.h_q, cfg.head_dim
-    pool_shape = ((batch.pool_rows // cfg.pool_block_size, cfg.pool_block_size, H, D)
-                  if cfg.pool_block_size else (batch.pool_rows, H, D))
-    base = 1_000_000 * (rank + 1)
-    pool_k = [W.normal_bf16_torch(pool_shape, base + 10 * l + 1, dev) for l in range(L)]
-    pool_v = [W.normal_bf16_torch(pool_shape, base + 10 * l + 2, dev) for l in range(L)]
-    q = W.normal_bf16_torch((L, T, Hq, D), base + 3, dev)
-    kn = W.normal_bf16_torch((L, T, H, D), base + 4, dev)
-    vn = W.normal_bf16_torch((L, T, H, D), base + 5, dev)
-    ck = torch.empty((L, ctx, H, D), dtype=torch.bfloat16, device=dev)
-    cv = torch.empty_like(ck)
-    out = torch.empty((L, T, Hq, D), dtype=torch.bfloat16, device=dev)
-    stream = torch.cuda.current_stream(dev)
-    sh = int(stream.cuda_stream)
-    ws, wsb = lp.workspace.data_ptr(), lp.workspace.numel()
-    plan = lp.plan
+        from paper_2502_16002_gb300 import kvlink as K
+        from paper_2502_16002_gb300.runtime import LinkedPrefill
 
-    one_kernel = args.path.startswith("one-kernel")
+        self.K = K
+        self.dev = dev
+        self.cfg = cfg = W.get_config(cfg_index)
+        self.batch = W.draw_batch(cfg, seed=rank_batch_seed(rank))   # every rank serves its own batch
+        self.L = L = args.layers or cfg.layers
+        self.path, self.layout = args.path, args.layout
+        layout = {"interleaved": K.KVLINK_LAYOUT_INTERLEAVED, "links_at_end": K.KVLINK_LAYOUT_LINKS_AT_END}
+        self.lp = LinkedPrefill.from_batch(self.batch, device=dev, layout=layout[args.layout])
+        self.info = info = self.lp.info
+        ctx, T = int(info.ctx_rows), int(info.n_fresh)
+        H, Hq, D = cfg.h_kv, cfg.h_q, cfg.head_dim
+        pool_shape = ((self.batch.pool_rows // cfg.pool_block_size, cfg.pool_block_size, H, D)
+                      if cfg.pool_block_size else (self.batch.pool_rows, H, D))
+        base = 1_000_000 * (rank + 1) + 100_000 * cfg_index
+        self.pool_k = [W.normal_bf16_torch(pool_shape, base + 10 * l + 1, dev) for l in range(L)]
+        self.pool_v = [W.normal_bf16_torch(pool_shape, base + 10 * l + 2, dev) for l in range(L)]
+        self.q = W.normal_bf16_torch((L, T, Hq, D), base + 3, dev)
+        self.kn = W.normal_bf16_torch((L, T, H, D), base + 4, dev)
+        self.vn = W.normal_bf16_torch((L, T, H, D), base + 5, dev)
+        self.ck = torch.empty((L, ctx, H, D), dtype=torch.bfloat16, device=dev)
+        self.cv = torch.empty_like(self.ck)
+        self.out = torch.empty((L, T, Hq, D), dtype=torch.bfloat16, device=dev)
+        self.stream = torch.cuda.current_stream(dev)
+        self.sh = int(self.stream.cuda_stream)
+        self.ws, self.wsb = self.lp.workspace.data_ptr(), self.lp.workspace.numel()
+        self.plan = self.lp.plan
+        self.one_kernel = args.path.startswith("one-kernel")
+        self.ptrs = [[t.data_ptr() for t in seq]
+                     for seq in (self.pool_k, self.pool_v, self.q, self.kn, self.vn, self.ck, self.cv, self.out)]
+        self.re_stream = torch.cuda.Stream(dev)
+        self.re_sh = int(self.re_stream.cuda_stream)
+        self.layer_ptrs = [[t.data_ptr() for t in seq] for seq in (self.pool_k, self.pool_v, self.ck, self.cv)]
 
-    def layer_call(l):
-        if one_kernel:
-            K.kvlink_linked_prefill_fused(plan, pool_k[l].data_ptr(), pool_v[l].data_ptr(), q[l].data_ptr(),
-                                          kn[l].data_ptr(), vn[l].data_ptr(), ck[l].data_ptr(),
-                                          None if args.path == "one-kernel-k-only" else cv[l].data_ptr(),
-                                          out[l].data_ptr(), ws, wsb, sh)
+    def layer_call(self, l):
+        K = self.K
+        if self.one_kernel:
+            K.kvlink_linked_prefill_fused(self.plan, self.pool_k[l].data_ptr(), self.pool_v[l].data_ptr(),
+                                          self.q[l].data_ptr(), self.kn[l].data_ptr(), self.vn[l].data_ptr(),
+                                          self.ck[l].data_ptr(),
+                                          None if self.path == "one-kernel-k-only" else self.cv[l].data_ptr(),
+                                          self.out[l].data_ptr(), self.ws, self.wsb, self.sh)
         else:
-            K.kvlink_linked_prefill(plan, pool_k[l].data_ptr(), pool_v[l].data_ptr(), q[l].data_ptr(),
-                                    kn[l].data_ptr(), vn[l].data_ptr(), ck[l].data_ptr(), cv[l].data_ptr(),
-                                    out[l].data_ptr(), ws, wsb, sh)
+            K.kvlink_linked_prefill(self.plan, self.pool_k[l].data_ptr(), self.pool_v[l].data_ptr(),
+                                    self.q[l].data_ptr(), self.kn[l].data_ptr(), self.vn[l].data_ptr(),
+                                    self.ck[l].data_ptr(), self.cv[l].data_ptr(), self.out[l].data_ptr(),
+                                    self.ws, self.wsb, self.sh)
 
-    ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, q, kn, vn, ck, cv, out)]
-    re_stream = torch.cuda.Stream(dev)
-    re_sh = int(re_stream.cuda_stream)
-    layer_ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, ck, cv)]
-
-    def step():
-        if one_kernel:
-            for l in range(L):
-                layer_call(l)
-        elif args.path == "two-kernel-serial":
-            K.kvlink_linked_prefill_layers(plan, *ptrs, ws, wsb, sh)
+    def step(self):
+        K = self.K
+        if self.one_kernel:
+            for l in range(self.L):
+                self.layer_call(l)
+        elif self.path == "two-kernel-serial":
+            K.kvlink_linked_prefill_layers(self.plan, *self.ptrs, self.ws, self.wsb, self.sh)
         else:
-            K.kvlink_linked_prefill_layers_overlapped(plan, *ptrs, ws, wsb, sh, re_sh)
+            K.kvlink_linked_prefill_layers_overlapped(self.plan, *self.ptrs, self.ws, self.wsb, self.sh, self.re_sh)
 
-    def barrier():
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
+    def launches_per_step(self):
+        n_merge = 1 if self.info.n_attn_splits > 0 else 0
+        per_layer = 1 if self.one_kernel else 2 if self.path == "two-kernel-serial" else 3
+        return self.L * (per_layer + n_merge)
 
-    for _ in range(args.warmup):
-        step()
-    torch.cuda.synchronize(dev)
-    assert K.kvlink_device_status() == 0
+    def timed_steps(self, n, world, clock_ms, local_rank):
+        """ms per step over n steps, CUDA events on the launching stream, barrier and synchronize
+        on both sides, max over ranks; with the clocks sampled during the timed region."""
+        import torch
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with ClockSampler(local_rank, clock_ms) as clk:
+            barrier(world)
+            torch.cuda.synchronize(self.dev)
+            clk.start()
+            e0.record(self.stream)
+            for _ in range(n):
+                self.step()
+            e1.record(self.stream)
+            torch.cuda.synchronize(self.dev)
+            clk.stop()
+            barrier(world)
+        assert self.K.kvlink_device_status() == 0
+        return max_over_ranks(e0.elapsed_time(e1), world, self.dev) / n, clk.summary()
 
-    # ---- timed region: the production path
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(local_rank) as clk:
-        barrier()
-        torch.cuda.synchronize(dev)
-        clk.start()
-        e0.record(stream)
-        for _ in range(args.steps):
-            step()
-        e1.record(stream)
-        torch.cuda.synchronize(dev)
-        clk.stop()
-        barrier()
-    ms_total = max_over_ranks(e0.elapsed_time(e1), world, dev)
-    ms_per_step = ms_total / args.steps
-    us_per_query = ms_per_step * 1e3 / cfg.batch      # per rank; ranks run in parallel
-    value = whole_job_us_per_query(ms_per_step, cfg.batch, world)
-    assert K.kvlink_device_status() == 0
+    def kernel_pass(self, k_steps):
+        """The step's kernels timed one launch at a time with events around each call: per layer
+        the re-encode of its document caches, then the attention kernel alone (the fresh rows
+        already in the cache); and every layer's re-encode in one launch, for comparison.
+        Returns seconds per launch (re-encode, attention, all-layer re-encode)."""
+        import torch
+        K, dev, stream, sh, L = self.K, self.dev, self.stream, self.sh, self.L
 
-    # ---- per-kernel pass: same work through the separate calls, events around each
-    k_steps = min(args.steps, 20)
+        def timed(fn, n):
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+            torch.cuda.synchronize(dev)
+            for j, (a, b_) in enumerate(evs):
+                a.record(stream)
+                fn(j)
+                b_.record(stream)
+            torch.cuda.synchronize(dev)
+            return float(np.mean([a.elapsed_time(b_) for a, b_ in evs])) * 1e-3
 
-    def timed(fn, n):
-        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
-        torch.cuda.synchronize(dev)
-        for j, (a, b_) in enumerate(evs):
-            a.record(stream)
-            fn(j)
-            b_.record(stream)
-        torch.cuda.synchronize(dev)
-        return float(np.mean([a.elapsed_time(b_) for a, b_ in evs])) * 1e-3      # s per call
-
-    t_re = t_re_all = float("nan")
-    if one_kernel:      # the whole layer is one kernel: timed as the "attention" launch
-        t_at = timed(lambda j: layer_call(j % L), k_steps * L)
-    else:
-        # per layer, as the step runs them: the re-encode of the layer's document caches,
-        # then the attention kernel alone (the fresh rows are already in the cache)
+        if self.one_kernel:      # the whole layer is one kernel: timed as the "attention" launch
+            return float("nan"), timed(lambda j: self.layer_call(j % L), k_steps * L), float("nan")
         ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(L * k_steps)]
         torch.cuda.synchronize(dev)
         for j, (a, b_, c) in enumerate(ev):
             l = j % L
             a.record(stream)
-            K.kvlink_reencode_concat(plan, pool_k[l].data_ptr(), pool_v[l].data_ptr(), ck[l].data_ptr(),
-                                     cv[l].data_ptr(), sh)
+            K.kvlink_reencode_concat(self.plan, self.pool_k[l].data_ptr(), self.pool_v[l].data_ptr(),
+                                     self.ck[l].data_ptr(), self.cv[l].data_ptr(), sh)
             b_.record(stream)
-            K.kvlink_suffix_attention(plan, q[l].data_ptr(), None, None, ck[l].data_ptr(), cv[l].data_ptr(),
-                                      out[l].data_ptr(), ws, wsb, sh)
+            K.kvlink_suffix_attention(self.plan, self.q[l].data_ptr(), None, None, self.ck[l].data_ptr(),
+                                      self.cv[l].data_ptr(), self.out[l].data_ptr(), self.ws, self.wsb, sh)
             c.record(stream)
         torch.cuda.synchronize(dev)
-        t_re = float(np.mean([a.elapsed_time(b_) for a, b_, _ in ev])) * 1e-3   # s per launch
+        t_re = float(np.mean([a.elapsed_time(b_) for a, b_, _ in ev])) * 1e-3
         t_at = float(np.mean([b_.elapsed_time(c) for _, b_, c in ev])) * 1e-3
-        # every layer's document caches in one launch, for comparison (not on the step's path)
-        t_re_all = timed(lambda j: K.kvlink_reencode_concat_layers(plan, *layer_ptrs, sh), k_steps)
-    assert K.kvlink_device_status() == 0
+        t_re_all = timed(lambda j: K.kvlink_reencode_concat_layers(self.plan, *self.layer_ptrs, sh), k_steps)
+        assert K.kvlink_device_status() == 0
+        return t_re, t_at, t_re_all
 
-    # ---- end to end through the public API with host buffers
-    e2e = None
-    if not args.no_e2e and not one_kernel and args.layout == "interleaved":
-        h_q = torch.empty(q.shape, dtype=q.dtype, pin_memory=True)
-        h_kn = torch.empty(kn.shape, dtype=kn.dtype, pin_memory=True)
-        h_vn = torch.empty(vn.shape, dtype=vn.dtype, pin_memory=True)
-        h_out = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
-        h_q.copy_(q)
-        h_kn.copy_(kn)
-        h_vn.copy_(vn)
-        e2e_steps = max(1, min(args.steps, 10))
+    def roofline(self, t_re, t_at, t_re_all, peaks):
+        """Per-kernel figures and the roofline entry of the dominant kernel.  Both kernels are
+        timed alone, launch by launch, so the attention's fraction is of the burst bf16 peak
+        (the sustained fraction is reported beside it)."""
+        cnt = algorithmic_counts(self.batch, self.info)
+        at_tfs = cnt["attn_flops"] / t_at / 1e12
+        at_frac = at_tfs / peaks["bf16_tflops"]
+        default_path = not self.one_kernel and self.layout == "interleaved"
+        attn_entry = {"us_per_launch": round(t_at * 1e6, 2), "TFLOP_per_s": round(at_tfs, 2),
+                      "frac_bf16_burst": round(at_frac, 4),
+                      "frac_bf16_sustained": round(at_tfs / peaks["bf16_tflops_sustained"], 4),
+                      "algorithmic_flops": cnt["attn_flops"],
+                      "hbm_bound_us": round(cnt["attn_bytes"] / peaks["hbm_gbs"] / 1e3, 2),
+                      "traffic": ncu_traffic("attention", self.cfg.index) if default_path else None}
+        if self.one_kernel:
+            kernels = {"linked_prefill_fused": attn_entry}
+            re_gbs = float("nan")
+        else:
+            re_gbs = cnt["reencode_bytes"] / t_re / 1e9
+            re_all_gbs = self.L * cnt["reencode_bytes"] / t_re_all / 1e9
+            kernels = {"reencode_concat": {"us_per_launch": round(t_re * 1e6, 2), "GB_per_s": round(re_gbs, 1),
+                                           "frac_hbm": round(re_gbs / peaks["hbm_gbs"], 4),
+                                           "frac_8TBs": round(re_gbs / 8000.0, 4),
+                                           "algorithmic_bytes": cnt["reencode_bytes"],
+                                           "bytes_per_query_doc_count": cnt["reencode_bytes_naive"],
+                                           "traffic": ncu_traffic("reencode", self.cfg.index) if default_path
+                                           else None},
+                       "reencode_concat_all_layers": {"us_per_launch": round(t_re_all * 1e6, 2), "layers": self.L,
+                                                      "GB_per_s": round(re_all_gbs, 1),
+                                                      "frac_hbm": round(re_all_gbs / peaks["hbm_gbs"], 4),
+                                                      "note": "every layer in one launch; not on the step's path"},
+                       "suffix_attention": attn_entry}
+        if self.one_kernel or t_at >= t_re:
+            name = ("kvlink linked_prefill_fused (one kernel)" if self.one_kernel else
+                    "kvlink suffix attention" + ("" if self.layout == "interleaved" else " (rows gathered)"))
+            roof = {"kernel": name, "bound": "tensor", "achieved": round(at_tfs, 2), "peak": peaks["bf16_tflops"],
+                    "unit": "TFLOP/s", "frac": round(at_frac, 4), "traffic": attn_entry["traffic"],
+                    "peak_kind": f"bf16 dense burst ({peaks['source']}): the kernel is timed alone, launch by launch",
+                    "algorithmic_unit": "4 * h_q * head_dim flops per unmasked (fresh row, key) pair",
+                    "algorithmic_per_launch": cnt["attn_flops"]}
+        else:
+            roof = {"kernel": "kvlink reencode_concat", "bound": "hbm", "achieved": round(re_gbs, 1),
+                    "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(re_gbs / peaks["hbm_gbs"], 4),
+                    "traffic": kernels["reencode_concat"]["traffic"], "peak_kind": f"HBM copy ({peaks['source']})",
+                    "algorithmic_unit": "unique pool K+V rows read + linked-cache K+V rows written",
+                    "algorithmic_per_launch": cnt["reencode_bytes"]}
+        return roof, kernels
 
-        streams = (torch.cuda.Stream(dev), stream, torch.cuda.Stream(dev))
+    def config(self, world):
+        cfg, info = self.cfg, self.info
+        return {"workload": cfg.name, "index": cfg.index, "batch_per_gpu": cfg.batch, "layers": self.L,
+                "h_q": cfg.h_q,
+                "h_kv": cfg.h_kv, "head_dim": cfg.head_dim, "docs_per_query": cfg.docs_per_query,
+                "n_link": cfg.n_link, "ctx_tokens_per_query": int(info.ctx_rows) // cfg.batch,
+                "fresh_rows": int(info.n_fresh), "pool": "paged, 16-token blocks" if cfg.pool_block_size else
+                "contiguous", "parallelism": f"replicas x{world} (independent batches)", "path": self.path,
+                "layout": self.layout,
+                "l2": "inputs larger than L2: each layer has its own pool "
+                      f"({self.pool_k[0].numel() * 4 / 1e6:.0f} MB K+V) and cache "
+                      f"({self.ck[0].numel() * 4 / 1e6:.0f} MB K+V)"}
 
-        p_e2e = LinkedPrefill.from_batch(batch, device=dev, stream=stream)
 
-        def e2e_step():
-            # a new batch: the plan rebuilt on the host and uploaded (ordered after the previous
-            # batch's kernels), then every layer with its fresh rows copied in from pinned host
-            # memory and its output copied back to pinned host memory, pipelined per layer; the
-            # host prepares the next batch while this one runs
-            p_e2e.rebuild_from_batch(batch, stream=stream)
-            p_e2e.linked_prefill_layers_from_host(pool_k, pool_v, h_q, h_kn, h_vn, q, kn, vn, ck, cv, out, h_out,
-                                                  streams=streams, wait=False)
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
 
+
+def run_e2e(wl, args, world):
+    """The same metric through the public API with host buffers (kvlink_linked_prefill_layers_host)."""
+    import torch
+
+    from paper_2502_16002_gb300.runtime import LinkedPrefill
+    dev, stream, batch, cfg = wl.dev, wl.stream, wl.batch, wl.cfg
+    h_q = torch.empty(wl.q.shape, dtype=wl.q.dtype, pin_memory=True)
+    h_kn = torch.empty(wl.kn.shape, dtype=wl.kn.dtype, pin_memory=True)
+    h_vn = torch.empty(wl.vn.shape, dtype=wl.vn.dtype, pin_memory=True)
+    h_out = torch.empty(wl.out.shape, dtype=wl.out.dtype, pin_memory=True)
+    h_q.copy_(wl.q)
+    h_kn.copy_(wl.kn)
+    h_vn.copy_(wl.vn)
+    e2e_steps = max(1, min(args.steps, 10))
+    streams = (torch.cuda.Stream(dev), stream, torch.cuda.Stream(dev))
+    p_e2e = LinkedPrefill.from_batch(batch, device=dev, stream=stream)
+
+    def e2e_step():
+        # a new batch: the plan rebuilt on the host and uploaded (ordered after the previous
+        # batch's kernels), then every layer with its fresh rows copied in from pinned host
+        # memory and its output copied back to pinned host memory, pipelined per layer; the
+        # host prepares the next batch while this one runs
+        p_e2e.rebuild_from_batch(batch, stream=stream)
+        p_e2e.linked_prefill_layers_from_host(wl.pool_k, wl.pool_v, h_q, h_kn, h_vn, wl.q, wl.kn, wl.vn, wl.ck,
+                                              wl.cv, wl.out, h_out, streams=streams, wait=False)
+
+    e2e_step()
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
         e2e_step()
-        torch.cuda.synchronize(dev)
-        barrier()
-        torch.cuda.synchronize(dev)
-        t0 = time.perf_counter()
-        for _ in range(e2e_steps):
-            e2e_step()
-        torch.cuda.synchronize(dev)          # every step's output is on the host
-        t1 = time.perf_counter()
-        barrier()
-        e2e_ms = max_over_ranks((t1 - t0) * 1e3, world, dev) / e2e_steps
-        h2d = (h_q.numel() + h_kn.numel() + h_vn.numel()) * 2 + int(info.device_bytes)
-        e2e = {"value": round(whole_job_us_per_query(e2e_ms, cfg.batch, world), 3), "unit": UNIT,
-               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(h_out.numel() * 2),
-               "steps": e2e_steps,
-               "note": "per step: host plan rebuild + table upload, then kvlink_linked_prefill_layers_host: "
-                       "per layer fresh q/k/v H2D from pinned memory, document re-encode on its own "
-                       "stream, placement + attention, output D2H to pinned memory (four streams); steps "
-                       "pipelined (the host prepares the next batch while one runs), wall clock from the "
-                       "first step's start to the last output on the host; document pool resident in HBM"}
+    torch.cuda.synchronize(dev)          # every step's output is on the host
+    t1 = time.perf_counter()
+    barrier(world)
+    e2e_ms = max_over_ranks((t1 - t0) * 1e3, world, dev) / e2e_steps
+    h2d = (h_q.numel() + h_kn.numel() + h_vn.numel()) * 2 + int(wl.info.device_bytes)
+    return {"value": round(whole_job_us_per_query(e2e_ms, cfg.batch, world), 3), "unit": UNIT,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(h_out.numel() * 2),
+            "steps": e2e_steps,
+            "note": "per step: host plan rebuild + table upload, then kvlink_linked_prefill_layers_host: "
+                    "per layer fresh q/k/v H2D from pinned memory, document re-encode on its own "
+                    "stream, placement + attention, output D2H to pinned memory (four streams); steps "
+                    "pipelined (the host prepares the next batch while one runs), wall clock from the "
+                    "first step's start to the last output on the host; document pool resident in HBM"}
 
-    peaks = _peaks()
-    cnt = algorithmic_counts(batch, info)
-    re_gbs = cnt["reencode_bytes"] / t_re / 1e9
-    re_all_gbs = L * cnt["reencode_bytes"] / t_re_all / 1e9
-    at_tfs = cnt["attn_flops"] / t_at / 1e12
-    re_frac = re_gbs / peaks["hbm_gbs"]
-    at_frac = at_tfs / peaks["bf16_tflops_sustained"]
-    dominant = "attention" if one_kernel or t_at >= t_re else "reencode"
-    default_path = not one_kernel and args.layout == "interleaved"
-    if dominant == "attention":
-        name = ("kvlink linked_prefill_fused (one kernel)" if one_kernel else
-                "kvlink suffix attention" + ("" if args.layout == "interleaved" else " (rows gathered)"))
-        roof = {"kernel": name, "bound": "tensor", "achieved": round(at_tfs, 2),
-                "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s", "frac": round(at_frac, 4),
-                "traffic": NCU_TRAFFIC.get(("attention", cfg.index)) if default_path else None,
-                "peak_kind": f"bf16 sustained, {peaks['source']}"}
-    else:
-        roof = {"kernel": "kvlink reencode_concat", "bound": "hbm", "achieved": round(re_gbs, 1),
-                "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(re_frac, 4),
-                "traffic": NCU_TRAFFIC.get(("reencode", cfg.index)) if default_path else None,
-                "peak_kind": f"HBM copy, {peaks['source']}"}
-    n_merge = 1 if info.n_attn_splits > 0 else 0
-    launches_per_step = L * ((1 if one_kernel else 2 if args.path == "two-kernel-serial" else 3) + n_merge)
-    attn_entry = {"us_per_launch": round(t_at * 1e6, 2), "TFLOP_per_s": round(at_tfs, 2),
-                  "frac_bf16_sustained": round(at_frac, 4),
-                  "frac_bf16_burst": round(at_tfs / peaks["bf16_tflops"], 4),
-                  "algorithmic_flops": cnt["attn_flops"],
-                  "hbm_bound_us": round(cnt["attn_bytes"] / peaks["hbm_gbs"] / 1e3, 2)}
-    if one_kernel:
-        kernels = {"linked_prefill_fused": attn_entry}
-    else:
-        kernels = {"reencode_concat": {"us_per_launch": round(t_re * 1e6, 2), "GB_per_s": round(re_gbs, 1),
-                                       "frac_hbm": round(re_frac, 4),
-                                       "frac_8TBs": round(re_gbs / 8000.0, 4),
-                                       "algorithmic_bytes": cnt["reencode_bytes"],
-                                       "bytes_per_query_doc_count": cnt["reencode_bytes_naive"]},
-                   "reencode_concat_all_layers": {"us_per_launch": round(t_re_all * 1e6, 2), "layers": L,
-                                                  "GB_per_s": round(re_all_gbs, 1),
-                                                  "frac_hbm": round(re_all_gbs / peaks["hbm_gbs"], 4),
-                                                  "note": "every layer in one launch; not on the step's path"},
-                   "suffix_attention": attn_entry}
+
+def run_ours(args, rank, world, local_rank, cfg_index, main=True):
+    """One workload: the timed K steps (the line's value), the per-kernel pass and roofline,
+    and for the main workload also a sustained run of at least a second with its clocks and
+    the end-to-end leg."""
+    import torch
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    wl = Workload(args, cfg_index, rank, dev)
+    for _ in range(args.warmup):
+        wl.step()
+    torch.cuda.synchronize(dev)
+    assert wl.K.kvlink_device_status() == 0
+
+    # ---- timed region: the production path, exactly K steps
+    ms_per_step, clocks = wl.timed_steps(args.steps, world, args.clock_ms, local_rank)
+    value = whole_job_us_per_query(ms_per_step, wl.cfg.batch, world)
+
+    # ---- the same step for at least a second, so that the clock record has many samples
+    sustained = None
+    if main and not args.no_sustained:
+        n = int(min(5000, max(args.steps, math.ceil(1.2e3 / max(ms_per_step, 1e-3)))))
+        ms_s, clk_s = wl.timed_steps(n, world, args.clock_ms, local_rank)
+        sustained = {"steps": n, "ms_per_step": round(ms_s, 4),
+                     "value": round(whole_job_us_per_query(ms_s, wl.cfg.batch, world), 3), "unit": UNIT,
+                     "timed_s": round(n * ms_s / 1e3, 3), "clocks": clk_s}
+
+    t_re, t_at, t_re_all = wl.kernel_pass(min(args.steps, 20) if main else min(args.steps, 5))
+    roof, kernels = wl.roofline(t_re, t_at, t_re_all, _peaks())
+
+    e2e = None
+    if main and not args.no_e2e and not wl.one_kernel and args.layout == "interleaved":
+        e2e = run_e2e(wl, args, world)
+
     res = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
         "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic N(0,1) bf16, seeded; document pool resident in HBM",
-        "config": {"workload": cfg.name, "batch_per_gpu": cfg.batch, "layers": L, "h_q": Hq, "h_kv": H,
-                   "head_dim": D, "docs_per_query": cfg.docs_per_query, "n_link": cfg.n_link,
-                   "ctx_tokens_per_query": ctx // cfg.batch, "fresh_rows": T,
-                   "parallelism": f"replicas x{world} (independent batches)",
-                   "path": args.path, "layout": args.layout,
-                   "l2": "inputs larger than L2: each layer has its own pool "
-                         f"({pool_k[0].numel() * 4 / 1e6:.0f} MB K+V) and cache "
-                         f"({ck[0].numel() * 4 / 1e6:.0f} MB K+V)"},
+        "config": wl.config(world),
         "roofline": roof,
         "kernels": kernels,
-        "per_rank_us_per_query": round(us_per_query, 3),
-        "gpu_launches": int(args.steps * launches_per_step),
-        "clocks": clk.summary(),
-        "e2e": e2e,
+        "per_rank_us_per_query": round(ms_per_step * 1e3 / wl.cfg.batch, 3),
+        "gpu_launches": int(args.steps * wl.launches_per_step()),
+        "clocks": clocks,
     }
+    if main:
+        res["sustained"] = sustained
+        res["e2e"] = e2e
+    del wl
+    torch.cuda.synchronize(dev)
+    torch.cuda.empty_cache()
     return res
 
 
@@ -508,7 +596,15 @@ def main():
     ap.add_argument("--path", choices=["two-kernel", "two-kernel-serial", "one-kernel", "one-kernel-k-only"],
                     default="two-kernel")
     ap.add_argument("--layout", choices=["interleaved", "links_at_end"], default="interleaved")
+    ap.add_argument("--extra-configs", type=int, nargs="*", default=None,
+                    help="further workloads timed after the main one and reported under 'workloads' "
+                         "(default: 4 and 5 when the main workload is 3)")
+    ap.add_argument("--clock-ms", type=int, default=50, help="nvidia-smi sampling interval")
+    ap.add_argument("--no-sustained", action="store_true",
+                    help="skip the run of at least a second that gives the clock record many samples")
     args = ap.parse_args()
+    if args.extra_configs is None:
+        args.extra_configs = [4, 5] if args.config == 3 and not args.layers else []
     if args.warmup < 3 and args.impl == "ours":
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
 
@@ -526,12 +622,23 @@ def main():
         import torch.distributed as dist
         torch.cuda.set_device(local_rank)
         dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
-    res = run_ours(args, rank, world, local_rank)
+    res = run_ours(args, rank, world, local_rank, args.config)
+    extra = {}
+    for c in args.extra_configs:
+        r = run_ours(args, rank, world, local_rank, c, main=False)
+        extra[r["config"]["workload"]] = {k: r[k] for k in ("value", "unit", "ms_per_step", "steps", "config",
+                                                             "roofline", "kernels", "clocks", "gpu_launches")}
+    if extra:
+        res["workloads"] = extra
     if rank == 0:
         if not args.no_cpu_baseline and world == 1:
-            v, spent, desc = oracle_sample(W.get_config(args.config))
-            res["cpu_baseline"] = {"value": round(v, 1), "unit": UNIT, "cores": _cores(), "kind": "oracle",
-                                   "sample": desc, "seconds": round(spent, 1)}
+            def baseline(cfg_index, seconds):
+                v, spent, desc = oracle_sample(W.get_config(cfg_index), max_seconds=seconds)
+                return {"value": round(v, 1), "unit": UNIT, "cores": _cores(), "kind": "oracle",
+                        "sample": desc, "seconds": round(spent, 1)}
+            res["cpu_baseline"] = baseline(args.config, 20.0)
+            for name, r in extra.items():
+                r["cpu_baseline"] = baseline(r["config"]["index"], 8.0)
         print(json.dumps(res), flush=True)
     if world > 1:
         import torch.distributed as dist

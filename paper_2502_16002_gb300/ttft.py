@@ -114,9 +114,13 @@ def _time(fn, warmup=10, iters=40):
     return e0.elapsed_time(e1) / iters
 
 
-def measure(doc_len, n_docs, n_link, q_len, host_caches, device, layer):
-    """ms per layer of (standard, linked) for n_docs documents of doc_len tokens."""
+def layer_arms(doc_len, n_docs, n_link, q_len, host_caches, device, layer):
+    """The two arms of the comparison on one layer, as callables (standard, linked), and a
+    dict in which each run leaves what the library read and wrote: under "standard" the
+    zero-document plan, q/k/v after RoPE and the attention output; under "linked" the plan,
+    the document pool, q/k/v after RoPE, the linked cache and the attention output."""
     n_ctx = n_docs * doc_len + q_len
+    seen = {}
     # ---- standard prefill: every token through the layer, causal attention over all of them
     std = _plan([], 0, n_ctx, device)
     x_std = torch.randn(n_ctx, HIDDEN, device=device, dtype=torch.bfloat16)
@@ -127,6 +131,7 @@ def measure(doc_len, n_docs, n_link, q_len, host_caches, device, layer):
         q, k, v = _qkv(layer, x_std)
         std.rope_fresh(q, k)
         std.suffix_attention(q, k, v, ck_s, cv_s, out_s)
+        seen["standard"] = dict(plan=std, q=q, k=k, v=v, out=out_s)
         return _finish(layer, x_std, out_s)
 
     # ---- linked prefill: fresh link/question rows only, documents from the cache pool
@@ -149,8 +154,16 @@ def measure(doc_len, n_docs, n_link, q_len, host_caches, device, layer):
         q, k, v = _qkv(layer, x_new)
         lp.rope_fresh(q, k)
         lp.linked_prefill(pool_k, pool_v, q, k, v, ck, cv, out)
+        seen["linked"] = dict(plan=lp, pool_k=pool_k, pool_v=pool_v, q=q, k=k, v=v, cache_k=ck, cache_v=cv,
+                              out=out, doc_len=doc_len, n_docs=n_docs, n_link=n_link, q_len=q_len)
         return _finish(layer, x_new, out)
 
+    return standard, linked, seen, n_ctx, T
+
+
+def measure(doc_len, n_docs, n_link, q_len, host_caches, device, layer):
+    """ms per layer of (standard, linked) for n_docs documents of doc_len tokens."""
+    standard, linked, _, n_ctx, T = layer_arms(doc_len, n_docs, n_link, q_len, host_caches, device, layer)
     t_std = _time(_graphed(standard))
     t_lnk = _time(_graphed(linked))
     assert K.kvlink_device_status() == 0

@@ -97,7 +97,8 @@ def custom_batch(index, *, h_q, h_kv, D, n_link, prefix, doc_lens_per_query, q_l
     cfg = W.WorkloadConfig(index=index, name=f"edge{index}", batch=len(q_lens), layers=1, h_q=h_q,
                            h_kv=h_kv, head_dim=D, theta=theta, prefix_len=prefix, n_link=n_link,
                            docs_per_query=0, pool_docs=len(lens), pool_block_size=pool_block_size)
-    pool_len = np.asarray(lens + ([prefix] if prefix else []), np.int32)
+    # a pool needs one entry: with no documents and no prefix it holds one that no query uses
+    pool_len = np.asarray(lens + ([prefix] if prefix else []) or [1], np.int32)
     ids, off = [], 0
     for q in doc_lens_per_query:
         ids.extend(range(off, off + len(q)))
@@ -137,6 +138,12 @@ EDGE = {
                                      doc_lens_per_query=[[6000, 300]], q_lens=[40]),
     "paged_pool_ragged": dict(h_q=16, h_kv=4, D=128, n_link=5, prefix=0, pool_block_size=16,
                               doc_lens_per_query=[[15, 16, 17, 100], [33]], q_lens=[12, 5]),
+    # the standard full prefill that the TTFT comparison times: no documents, no prefix, the
+    # whole context as one causal run of fresh rows
+    "no_documents_causal_context": dict(h_q=32, h_kv=8, D=128, n_link=5, prefix=0,
+                                        doc_lens_per_query=[[]], q_lens=[1523]),
+    "prefix_only_no_documents": dict(h_q=32, h_kv=8, D=128, n_link=5, prefix=300,
+                                     doc_lens_per_query=[[], [7]], q_lens=[200, 3]),
 }
 
 

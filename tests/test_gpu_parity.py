@@ -69,9 +69,10 @@ def test_reencode_leaves_fresh_slots_untouched(RT):
 
 # ----------------------------------------------------------------- full-size workloads, sampled
 
-def test_llama8b_batch8_zipf_sampled(RT):
+@pytest.mark.parametrize("layer", [0, 31])
+def test_llama8b_batch8_zipf_sampled(RT, layer):
     batch = W.draw_batch(W.get_config(3))
-    lp, gk, gv, gout, inp = run_layer(RT, batch, 31)
+    lp, gk, gv, gout, inp = run_layer(RT, batch, layer)
     for b in range(batch.cfg.batch):
         check_query(batch, b, lp, gk, gv, gout, inp, attention=b in (0, 7))
 
@@ -80,7 +81,8 @@ def test_llama8b_long_context_sampled(RT):
     batch = W.draw_batch(W.get_config(4))
     lp, gk, gv, gout, inp = run_layer(RT, batch, 0)
     T = int(batch.n_fresh[0])
-    rows = [0, 1, 4, 5, 9, 31, 32, 127, 128, 255, 256, 400, 499, 500, 501, 563, T - 2, T - 1]
+    rows = ([0, 1, 4, 5, 9, 31, 32, 127, 128, 255, 256, 400, 499, 500, 501, 563] + list(range(540, 561)) +
+            list(range(600, T)))
     check_query(batch, 0, lp, gk, gv, gout, inp, rows=rows)
 
 
@@ -152,3 +154,34 @@ def test_ttft_comparison_harness_runs(RT):
     t_std, t_lnk, n_ctx, T = ttft.measure(64, 3, 5, 16, True, dev, layer)
     assert n_ctx == 3 * 64 + 16 and T == 3 * 5 + 16
     assert t_std > 0 and t_lnk > 0
+
+
+def test_ttft_arms_match_the_oracle(RT):
+    """One layer of each TTFT arm, run once outside any graph: the standard arm's attention
+    (a zero-document plan, the whole context as causal fresh rows) and the linked arm's
+    linked cache and attention, each against the fp64 oracle on the tensors the arm gave the
+    library (q, k, v after the projection and RoPE, the document pool)."""
+    from paper_2502_16002_gb300 import kvlink as K, ttft
+    dev = torch.device("cuda:0")
+    layer = ttft.Layer(dev)
+    standard, linked, seen, n_ctx, T = ttft.layer_arms(100, 4, 5, 24, True, dev, layer)
+    standard()
+    linked()
+    torch.cuda.synchronize(dev)
+    assert K.kvlink_device_status() == 0
+    bits = RT.bits_from_bf16
+    s = seen["standard"]
+    f64 = lambda t: O.bf16_bits_to_f64(bits(t))
+    ref = O.suffix_attention(f64(s["q"]), f64(s["k"]), f64(s["v"]), np.arange(n_ctx))
+    err = np.abs(s["out"].float().cpu().numpy() - ref)
+    assert err.max() <= 1e-2 and err.mean() <= 1e-3, (err.max(), err.mean())
+    ln = seen["linked"]
+    cache = O.reencode_concat(bits(ln["pool_k"]), bits(ln["pool_v"]), np.arange(4) * 100, np.full(4, 100), -1,
+                              [0, 1, 2, 3], 5, bits(ln["k"]), bits(ln["v"]), 24, ttft.THETA)
+    gk, gv = bits(ln["cache_k"]), bits(ln["cache_v"])
+    assert np.array_equal(gv, cache.v_bits)
+    assert ulp_distance(gk, cache.k_bits).max() <= 1
+    ref = O.suffix_attention(f64(ln["q"]), O.bf16_bits_to_f64(cache.k_bits), O.bf16_bits_to_f64(cache.v_bits),
+                             cache.layout.fresh_pos)
+    err = np.abs(ln["out"].float().cpu().numpy() - ref)
+    assert err.max() <= 1e-2 and err.mean() <= 1e-3, (err.max(), err.mean())
