@@ -296,10 +296,11 @@ class Workload:
         per_layer = 1 if self.one_kernel else 2 if self.path == "two-kernel-serial" else 3
         return self.L * (per_layer + n_merge)
 
-    def timed_steps(self, n, world, clock_ms, local_rank):
+    def timed_steps(self, n, world, clock_ms, local_rank, step=None):
         """ms per step over n steps, CUDA events on the launching stream, barrier and synchronize
         on both sides, max over ranks; with the clocks sampled during the timed region."""
         import torch
+        step = step or self.step
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with ClockSampler(local_rank, clock_ms) as clk:
             barrier(world)
@@ -307,7 +308,7 @@ class Workload:
             clk.start()
             e0.record(self.stream)
             for _ in range(n):
-                self.step()
+                step()
             e1.record(self.stream)
             torch.cuda.synchronize(self.dev)
             clk.stop()
@@ -400,6 +401,48 @@ class Workload:
                     "algorithmic_unit": "unique pool K+V rows read + linked-cache K+V rows written",
                     "algorithmic_per_launch": cnt["reencode_bytes"]}
         return roof, kernels
+
+    def host_pool_leg(self, args, world, local_rank):
+        """The same step with every layer's document cache pool in page-locked host memory
+        (kvlink_linked_prefill_layers_host_pool: each layer's documents read over the host link
+        by the re-encode, on the load stream, while earlier layers' attention runs), and one
+        layer's host-pool re-encode timed alone."""
+        import torch
+        K = self.K
+        h_k = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in self.pool_k]
+        h_v = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in self.pool_v]
+        for h, d in zip(h_k + h_v, self.pool_k + self.pool_v):
+            h.copy_(d)
+        ptrs = [[t.data_ptr() for t in seq] for seq in (h_k, h_v, self.q, self.kn, self.vn, self.ck, self.cv, self.out)]
+
+        def step():
+            K.kvlink_linked_prefill_layers_host_pool(self.plan, *ptrs, self.ws, self.wsb, self.sh, self.re_sh)
+
+        for _ in range(args.warmup):
+            step()
+        torch.cuda.synchronize(self.dev)
+        ms, clocks = self.timed_steps(args.steps, world, args.clock_ms, local_rank, step)
+        n = min(args.steps, 5) * self.L
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        for j, (a, b_) in enumerate(evs):
+            l = j % self.L
+            a.record(self.stream)
+            K.kvlink_reencode_concat_host_pool(self.plan, h_k[l].data_ptr(), h_v[l].data_ptr(), self.ck[l].data_ptr(),
+                                               self.cv[l].data_ptr(), self.sh)
+            b_.record(self.stream)
+        torch.cuda.synchronize(self.dev)
+        assert K.kvlink_device_status() == 0
+        t = float(np.mean([a.elapsed_time(b_) for a, b_ in evs])) * 1e-3
+        cnt = algorithmic_counts(self.batch, self.info)
+        read = cnt["reencode_bytes"] - 2 * self.cfg.h_kv * self.cfg.head_dim * 2 * int(self.info.cached_tokens)
+        return {"value": round(whole_job_us_per_query(ms, self.cfg.batch, world), 3), "unit": UNIT,
+                "ms_per_step": round(ms, 4), "steps": args.steps, "clocks": clocks,
+                "reencode_host_pool_us_per_launch": round(t * 1e6, 2),
+                "host_read_GB_per_s": round(read / t / 1e9, 1),
+                "device_write_GB_per_s": round((cnt["reencode_bytes"] - read) / t / 1e9, 1),
+                "host_bytes_read_per_layer": int(read),
+                "note": "every layer's document pool in pinned host memory, read over NVLink-C2C by the "
+                        "re-encode (kvlink_linked_prefill_layers_host_pool); fresh rows resident in HBM"}
 
     def config(self, world):
         cfg, info = self.cfg, self.info
@@ -499,9 +542,11 @@ def run_ours(args, rank, world, local_rank, cfg_index, main=True):
     t_re, t_at, t_re_all = wl.kernel_pass(min(args.steps, 20) if main else min(args.steps, 5))
     roof, kernels = wl.roofline(t_re, t_at, t_re_all, _peaks())
 
-    e2e = None
+    e2e = host_pool = None
     if main and not args.no_e2e and not wl.one_kernel and args.layout == "interleaved":
         e2e = run_e2e(wl, args, world)
+    if main and not args.no_host_pool and not wl.one_kernel and args.layout == "interleaved":
+        host_pool = wl.host_pool_leg(args, world, local_rank)
 
     res = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
@@ -518,6 +563,7 @@ def run_ours(args, rank, world, local_rank, cfg_index, main=True):
     if main:
         res["sustained"] = sustained
         res["e2e"] = e2e
+        res["host_pool"] = host_pool
     del wl
     torch.cuda.synchronize(dev)
     torch.cuda.empty_cache()
@@ -600,6 +646,8 @@ def main():
                     help="further workloads timed after the main one and reported under 'workloads' "
                          "(default: 4 and 5 when the main workload is 3)")
     ap.add_argument("--clock-ms", type=int, default=50, help="nvidia-smi sampling interval")
+    ap.add_argument("--no-host-pool", action="store_true",
+                    help="skip the leg with the document pool in pinned host memory")
     ap.add_argument("--no-sustained", action="store_true",
                     help="skip the run of at least a second that gives the clock record many samples")
     args = ap.parse_args()

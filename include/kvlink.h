@@ -15,6 +15,8 @@
  *   kvlink_linked_prefill_layers[_overlapped]   every layer in one call (the re-encode of
  *                                               all layers on a second stream)
  *   kvlink_linked_prefill_layers_host           the same from and to host memory
+ *   kvlink_reencode_concat_host_pool,           the document cache pool in host memory
+ *   kvlink_linked_prefill_layers_host_pool      (Sec. 3.3), read over the host link
  *   kvlink_linked_prefill_fused                 one kernel per layer (keys rotated on load)
  *   kvlink_reencode_concat_layers, kvlink_rope_fresh, kvlink_suffix_attention_simt,
  *   kvlink_suffix_attention_noalloc, kvlink_device_status, kvlink_selftest_wait_timeout
@@ -365,6 +367,37 @@ int kvlink_linked_prefill_layers_host(kvlink_plan_t* plan, int32_t n_layers, con
                                       void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream,
                                       kvlink_stream_t reencode_stream, kvlink_stream_t copy_in_stream,
                                       kvlink_stream_t copy_out_stream);
+
+/* Re-encode + concat of one layer (as kvlink_reencode_concat, the same bits) with that
+ * layer's document cache pool in host memory (Sec. 3.3: the precomputed caches are kept in
+ * CPU memory and loaded for every request).  h_pool_k / h_pool_v: page-locked host memory
+ * (cudaHostAlloc, or cudaHostRegister'ed) holding the pool in the plan's layout; the kernel
+ * reads the rows it needs through the device's mapping of that memory (NVLink-C2C on a
+ * Grace system), rotates the document keys and writes the linked cache in device memory, so
+ * the rows cross the host link once and are never staged.  The host memory must stay valid
+ * and unchanged until the work has completed on the device.  Errors: EINVAL (also for
+ * pageable or device memory), ECUDA. */
+int kvlink_reencode_concat_host_pool(const kvlink_plan_t* plan, const void* h_pool_k, const void* h_pool_v,
+                                     void* d_cache_k, void* d_cache_v, kvlink_stream_t stream);
+
+/* The linked prefill of n_layers layers with every layer's document cache pool in host
+ * memory: the same results as kvlink_linked_prefill_layers_overlapped, bit for bit, with
+ * kvlink_reencode_concat_host_pool in place of the device-pool re-encode.  load_stream
+ * first waits for the work already on `stream`, then loads and re-encodes every layer's
+ * document caches from host memory back to back; layer l's fresh-row placement and suffix
+ * attention run on `stream` once layer l's caches are in place, so the loading of later
+ * layers overlaps the attention of earlier ones.  h_pool_k / h_pool_v: HOST arrays of
+ * n_layers page-locked host pointers; the other arrays as for
+ * kvlink_linked_prefill_layers_overlapped.  When the call returns, `stream` is ordered after
+ * all of its work.  The plan keeps the events it uses: calls with one plan must not run
+ * concurrently.  Errors: as kvlink_linked_prefill_layers_overlapped; EINVAL also for a pool
+ * pointer that is not page-locked host memory, or when the two streams are the same. */
+int kvlink_linked_prefill_layers_host_pool(kvlink_plan_t* plan, int32_t n_layers, const void* const* h_pool_k,
+                                           const void* const* h_pool_v, const void* const* d_q,
+                                           const void* const* d_k_new, const void* const* d_v_new,
+                                           void* const* d_cache_k, void* const* d_cache_v, void* const* d_out,
+                                           void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream,
+                                           kvlink_stream_t load_stream);
 
 /* Allocation-free variant of kvlink_suffix_attention.  The paper has no counterpart:
  * this entry point serves callers that may not allocate device memory at all, such as

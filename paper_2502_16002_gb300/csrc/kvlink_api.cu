@@ -19,6 +19,8 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
 void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int h_kv, int num_sms, int n_layers,
                             const void* const* pool_k, const void* const* pool_v, void* const* cache_k,
                             void* const* cache_v, cudaStream_t stream);
+void launch_reencode_host(const DevicePlan& P, int n_chunks, int head_dim, int h_kv, int num_sms,
+                          const void* pool_k, const void* pool_v, void* cache_k, void* cache_v, cudaStream_t stream);
 void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int64_t ctx_rows, int row_bytes,
                         const void* k_new, const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
 int read_copy_status(int32_t* status);
@@ -617,6 +619,80 @@ int kvlink_linked_prefill_layers_host(kvlink_plan_t* p, int32_t n_layers, const 
         if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host: output");
     }
     p->host_chain_layers = n_layers;
+    return KVLINK_OK;
+}
+
+// The device's address of page-locked host memory (cudaHostAlloc, cudaHostRegister): the
+// kernels read the pool through it.  Pageable memory and device memory are rejected.
+static int host_pool_view(const void* h, const void** d) {
+    if (!h) return KVLINK_EINVAL;
+    cudaPointerAttributes a;
+    const cudaError_t e = cudaPointerGetAttributes(&a, h);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return KVLINK_EINVAL;
+    }
+    if (a.type != cudaMemoryTypeHost || !a.devicePointer || !aligned16(a.devicePointer)) return KVLINK_EINVAL;
+    *d = a.devicePointer;
+    return KVLINK_OK;
+}
+
+int kvlink_reencode_concat_host_pool(const kvlink_plan_t* p, const void* h_pool_k, const void* h_pool_v,
+                                     void* cache_k, void* cache_v, kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (!cache_k || !cache_v || !aligned16(cache_k) || !aligned16(cache_v)) return KVLINK_EINVAL;
+    const void *dk = nullptr, *dv = nullptr;
+    if ((rc = host_pool_view(h_pool_k, &dk)) || (rc = host_pool_view(h_pool_v, &dv))) return rc;
+    launch_reencode_host(p->dev, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, dk, dv, cache_k, cache_v,
+                         (cudaStream_t)stream);
+    return check_launch("reencode_host_kernel");
+}
+
+int kvlink_linked_prefill_layers_host_pool(kvlink_plan_t* p, int32_t n_layers, const void* const* h_pool_k,
+                                           const void* const* h_pool_v, const void* const* q,
+                                           const void* const* k_new, const void* const* v_new, void* const* cache_k,
+                                           void* const* cache_v, void* const* out, void* ws, size_t ws_bytes,
+                                           kvlink_stream_t stream, kvlink_stream_t load_stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (n_layers <= 0 || !h_pool_k || !h_pool_v || !q || !k_new || !v_new || !cache_k || !cache_v || !out)
+        return KVLINK_EINVAL;
+    if (stream == load_stream) return KVLINK_EINVAL;
+    if (!all_aligned(n_layers, (const void* const*)cache_k) || !all_aligned(n_layers, (const void* const*)cache_v) ||
+        !all_aligned(n_layers, q) || !all_aligned(n_layers, k_new) || !all_aligned(n_layers, v_new) ||
+        !all_aligned(n_layers, (const void* const*)out))
+        return KVLINK_EINVAL;
+    if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
+    if (ws && !aligned16(ws)) return KVLINK_EINVAL;
+    // every host pool pointer is resolved (and checked) before the first launch
+    std::vector<const void*> dk((size_t)n_layers), dv((size_t)n_layers);
+    for (int l = 0; l < n_layers; ++l)
+        if ((rc = host_pool_view(h_pool_k[l], &dk[l])) || (rc = host_pool_view(h_pool_v[l], &dv[l]))) return rc;
+    rc = events_reserve(p->events, (size_t)n_layers + 1);
+    if (rc) return rc;
+    cudaStream_t s = (cudaStream_t)stream, r = (cudaStream_t)load_stream;
+    cudaEvent_t* ev = p->events.ev.data();
+    cudaError_t e = cudaEventRecord(ev[n_layers], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(r, ev[n_layers], 0);
+    if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host_pool: stream order");
+    // every layer's document caches loaded from host memory and re-encoded, back to back
+    for (int l = 0; l < n_layers; ++l) {
+        launch_reencode_host(p->dev, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, dk[l], dv[l], cache_k[l],
+                             cache_v[l], r);
+        rc = check_launch("reencode_host_kernel (layers)");
+        if (rc) return rc;
+        e = cudaEventRecord(ev[l], r);
+        if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host_pool: event");
+    }
+    for (int l = 0; l < n_layers; ++l) {
+        e = cudaStreamWaitEvent(s, ev[l], 0);
+        if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host_pool: wait");
+        rc = place_fresh(p, k_new[l], v_new[l], cache_k[l], cache_v[l], s);
+        if (rc) return rc;
+        rc = attention_common(p, q[l], cache_k[l], cache_v[l], out[l], ws, ws_bytes, s);
+        if (rc) return rc;
+    }
     return KVLINK_OK;
 }
 

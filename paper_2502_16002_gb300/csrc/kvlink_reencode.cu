@@ -336,6 +336,107 @@ void launch_reencode_layers(const DevicePlan& P, int n_chunks, int head_dim, int
 }
 
 // --------------------------------------------------------------------------
+// A3 with the document caches in host memory (Sec. 3.3: the caches start in CPU memory and
+// are loaded for every request).  On GB300 the SMs reach page-locked Grace memory over
+// NVLink-C2C, so the rows are loaded straight from the host pool by the re-encode itself
+// and written once, rotated, to the linked cache in HBM: no staging copy.  Plain 16-byte
+// loads (the bulk-copy path of reencode_kernel is kept to device memory).  One warp per
+// work unit at a time; a lane owns (head, j0) pairs of the row (elements j0..j0+7 and
+// j0+D/2..j0+D/2+7 of one head) and issues the loads of two token rows before any store, so
+// each lane keeps eight 16-byte host loads in flight.  The rotation is the one of
+// reencode_kernel (rotate8), so the cache bits are identical.
+// --------------------------------------------------------------------------
+constexpr int kHostWarps = 8;
+constexpr int kHostPairsPerLane = 2;        // rows of up to 64 pairs (the 8B shape) in one pass
+
+template <int D>
+__global__ void __launch_bounds__(32 * kHostWarps) reencode_host_kernel(
+    const CopyChunk* __restrict__ chunks, int n_chunks, const float4* __restrict__ rope, int h_kv,
+    const uint4* __restrict__ pool_k, const uint4* __restrict__ pool_v, uint4* __restrict__ cache_k,
+    uint4* __restrict__ cache_v, const CopyBounds bounds) {
+    if (*reinterpret_cast<volatile int32_t*>(&g_copy_status) != 0) return;   // a recorded failure
+    constexpr int PAIRS_PER_HEAD = D / 16;
+    constexpr int PAIRS_PER_PASS = 32 * kHostPairsPerLane;
+    const int U = h_kv * PAIRS_PER_HEAD;              // (lo, hi) pairs of 16-byte words per row
+    const int row_vec = h_kv * D / 8;                 // 16-byte words per row
+    const int lane = threadIdx.x % 32;
+    const int warp = blockIdx.x * kHostWarps + threadIdx.x / 32;
+    const int n_warps = gridDim.x * kHostWarps;
+    for (int c = warp; c < n_chunks; c += n_warps) {
+        const CopyChunk ch = chunks[c];
+#ifdef KVLINK_DEBUG_CHECKS
+        if (ch.n < 1 || ch.dst_row < 0 || ch.dst_row + ch.n > bounds.ctx_rows || ch.src_row < 0 ||
+            ch.src_row + ch.n > bounds.pool_rows ||
+            (ch.kind == KVLINK_SEG_DOC && (ch.table < 0 || ch.table >= bounds.n_rope_rows))) {
+            if (lane == 0) atomicCAS(&g_copy_status, 0, kCopyStatusBadIndex);
+            continue;
+        }
+#endif
+        const bool rot = ch.kind == KVLINK_SEG_DOC;
+        for (int p0 = 0; p0 < U; p0 += PAIRS_PER_PASS) {     // one pass for rows of <= 64 pairs
+            int lo_idx[kHostPairsPerLane];
+            bool has[kHostPairsPerLane];
+            float4 cs[kHostPairsPerLane][8];
+#pragma unroll
+            for (int i = 0; i < kHostPairsPerLane; ++i) {
+                const int p = p0 + lane + 32 * i;
+                has[i] = p < U;
+                lo_idx[i] = (p / PAIRS_PER_HEAD) * (D / 8) + p % PAIRS_PER_HEAD;
+                if (rot && has[i]) {
+                    const float4* t = rope + (int64_t)ch.table * (D / 2) + (p % PAIRS_PER_HEAD) * 8;
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) cs[i][q] = __ldg(t + q);
+                }
+            }
+            for (int t0 = 0; t0 < ch.n; t0 += 2) {
+                uint4 k[2][kHostPairsPerLane][2], v[2][kHostPairsPerLane][2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int64_t src = (ch.src_row + t0 + u) * row_vec;
+#pragma unroll
+                    for (int i = 0; i < kHostPairsPerLane; ++i)
+                        if (has[i] && t0 + u < ch.n) {
+                            k[u][i][0] = pool_k[src + lo_idx[i]];
+                            k[u][i][1] = pool_k[src + lo_idx[i] + D / 16];
+                            v[u][i][0] = pool_v[src + lo_idx[i]];
+                            v[u][i][1] = pool_v[src + lo_idx[i] + D / 16];
+                        }
+                }
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int64_t dst = (ch.dst_row + t0 + u) * row_vec;
+#pragma unroll
+                    for (int i = 0; i < kHostPairsPerLane; ++i)
+                        if (has[i] && t0 + u < ch.n) {
+                            if (rot) rotate8(k[u][i][0], k[u][i][1], cs[i]);
+                            cache_k[dst + lo_idx[i]] = k[u][i][0];
+                            cache_k[dst + lo_idx[i] + D / 16] = k[u][i][1];
+                            cache_v[dst + lo_idx[i]] = v[u][i][0];
+                            cache_v[dst + lo_idx[i] + D / 16] = v[u][i][1];
+                        }
+                }
+            }
+        }
+    }
+}
+
+// The cached chunks of one layer from a device-accessible host pool.
+void launch_reencode_host(const DevicePlan& P, int n_chunks, int head_dim, int h_kv, int num_sms,
+                          const void* pool_k, const void* pool_v, void* cache_k, void* cache_v, cudaStream_t stream) {
+    if (n_chunks <= 0) return;
+    const CopyBounds bounds{P.ctx_rows, P.pool_rows, P.n_fresh, P.n_rope_rows};
+    const int grid = std::max(1, std::min((n_chunks + kHostWarps - 1) / kHostWarps, 4 * num_sms));
+    if (head_dim == 128)
+        reencode_host_kernel<128><<<grid, 32 * kHostWarps, 0, stream>>>(
+            P.chunks, n_chunks, P.rope, h_kv, (const uint4*)pool_k, (const uint4*)pool_v, (uint4*)cache_k,
+            (uint4*)cache_v, bounds);
+    else
+        reencode_host_kernel<64><<<grid, 32 * kHostWarps, 0, stream>>>(
+            P.chunks, n_chunks, P.rope, h_kv, (const uint4*)pool_k, (const uint4*)pool_v, (uint4*)cache_k,
+            (uint4*)cache_v, bounds);
+}
+
+// --------------------------------------------------------------------------
 // A4: the fresh link/question rows to their cache rows (bit copies).  A few MB per layer
 // on the path of the attention that follows, so the copy is built for latency: one warp
 // per row and 16-byte accesses, all of a lane's loads issued before its stores.

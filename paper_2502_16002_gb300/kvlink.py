@@ -108,6 +108,8 @@ def _load():
         "kvlink_linked_prefill_layers_overlapped": (C.c_int, [P, C.c_int32, V, V, V, V, V, V, V, V, V, C.c_size_t,
                                                               V, V]),
         "kvlink_linked_prefill_layers_host": (C.c_int, [P, C.c_int32] + [V] * 13 + [C.c_size_t, V, V, V, V]),
+        "kvlink_reencode_concat_host_pool": (C.c_int, [P, V, V, V, V, V]),
+        "kvlink_linked_prefill_layers_host_pool": (C.c_int, [P, C.c_int32] + [V] * 9 + [C.c_size_t, V, V]),
         "kvlink_device_status": (C.c_int, [C.POINTER(C.c_int32)]),
         "kvlink_clear_device_status": (C.c_int, []),
         "kvlink_selftest_wait_timeout": (C.c_int, [C.c_uint32, V]),
@@ -130,7 +132,7 @@ DECLARED = [
     "kvlink_last_cuda_error", "kvlink_version", "kvlink_suffix_attention_noalloc", "kvlink_rope_fresh",
     "kvlink_plan_get_sources", "kvlink_linked_prefill_fused", "kvlink_linked_prefill_layers",
     "kvlink_reencode_concat_layers", "kvlink_plan_rebuild", "kvlink_linked_prefill_layers_overlapped",
-    "kvlink_linked_prefill_layers_host",
+    "kvlink_linked_prefill_layers_host", "kvlink_reencode_concat_host_pool", "kvlink_linked_prefill_layers_host_pool",
     "kvlink_selftest_wait_timeout",
 ]
 
@@ -347,6 +349,25 @@ def kvlink_linked_prefill_layers_host(plan: Plan, pool_k, pool_v, h_q, h_k_new, 
     _check(lib.kvlink_linked_prefill_layers_host(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs], workspace,
                                                  workspace_bytes, stream, reencode_stream, copy_in_stream,
                                                  copy_out_stream), "kvlink_linked_prefill_layers_host")
+
+
+def kvlink_reencode_concat_host_pool(plan: Plan, h_pool_k: int, h_pool_v: int, cache_k: int, cache_v: int,
+                                     stream: int = 0) -> None:
+    """h_pool_k / h_pool_v: page-locked host memory; cache_k / cache_v: device memory."""
+    _check(lib.kvlink_reencode_concat_host_pool(plan.handle, h_pool_k, h_pool_v, cache_k, cache_v, stream),
+           "kvlink_reencode_concat_host_pool")
+
+
+def kvlink_linked_prefill_layers_host_pool(plan: Plan, h_pool_k, h_pool_v, q, k_new, v_new, cache_k, cache_v, out,
+                                           workspace, workspace_bytes: int, stream: int, load_stream: int) -> None:
+    """Per-layer pointer sequences: h_pool_*: page-locked host memory, the rest device memory."""
+    n = len(h_pool_k)
+    arrs = [_ptr_array(x) for x in (h_pool_k, h_pool_v, q, k_new, v_new, cache_k, cache_v, out)]
+    if any(len(a) != n for a in arrs):
+        raise ValueError("every per-layer pointer list needs one entry per layer")
+    _check(lib.kvlink_linked_prefill_layers_host_pool(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs],
+                                                      workspace, workspace_bytes, stream, load_stream),
+           "kvlink_linked_prefill_layers_host_pool")
 
 
 def kvlink_reencode_concat_layers(plan: Plan, pool_k, pool_v, cache_k, cache_v, stream: int = 0) -> None:

@@ -152,6 +152,24 @@ class LinkedPrefill:
             self._re_stream = torch.cuda.Stream(self.device)
         return self._re_stream
 
+    def reencode_concat_host_pool(self, h_pool_k, h_pool_v, cache_k, cache_v, stream=None):
+        """One layer's re-encode + concat with its pool in pinned host memory."""
+        for t in (h_pool_k, h_pool_v):
+            if not t.is_pinned():
+                raise ValueError("the host pool must be pinned")
+        K.kvlink_reencode_concat_host_pool(self.plan, h_pool_k.data_ptr(), h_pool_v.data_ptr(), cache_k.data_ptr(),
+                                           cache_v.data_ptr(), _stream_handle(stream))
+
+    def linked_prefill_layers_host_pool(self, h_pool_k, h_pool_v, q, k_new, v_new, cache_k, cache_v, out,
+                                        stream=None, load_stream=None):
+        """All layers in one ABI call with every layer's pool in pinned host memory (sequences of
+        per-layer tensors); the loading and re-encode run on load_stream (created if not given)."""
+        if load_stream is None:
+            load_stream = self._reencode_stream()
+        ptrs = [[t.data_ptr() for t in seq] for seq in (h_pool_k, h_pool_v, q, k_new, v_new, cache_k, cache_v, out)]
+        K.kvlink_linked_prefill_layers_host_pool(self.plan, *ptrs, self.workspace.data_ptr(), self.workspace.numel(),
+                                                 _stream_handle(stream), _stream_handle(load_stream))
+
     def reencode_concat_layers(self, pool_k, pool_v, cache_k, cache_v, stream=None):
         """The document caches of all layers in one launch (sequences of per-layer tensors)."""
         ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, cache_k, cache_v)]

@@ -38,13 +38,14 @@ HIDDEN, H_Q, H_KV, HEAD_DIM, FFN, LAYERS, THETA = 4096, 32, 8, 128, 14336, 32, 5
 
 
 class Layer:
-    """Random bf16 weights of one Llama-3.1-8B-shaped layer."""
+    """Random bf16 weights of one Llama-3.1-8B-shaped layer, N(0, 1/fan_in): after the RMSNorm
+    the projected q, k and v have unit variance, the value distribution of the workloads."""
 
     def __init__(self, device, seed=0):
         g = torch.Generator(device=device)
         g.manual_seed(seed)
         def w(o, i):
-            return (torch.randn(o, i, generator=g, device=device, dtype=torch.float32) * 0.02).to(torch.bfloat16)
+            return (torch.randn(o, i, generator=g, device=device, dtype=torch.float32) / i ** 0.5).to(torch.bfloat16)
         self.wqkv = w((H_Q + 2 * H_KV) * HEAD_DIM, HIDDEN)
         self.wo = w(HIDDEN, H_Q * HEAD_DIM)
         self.wgu = w(2 * FFN, HIDDEN)

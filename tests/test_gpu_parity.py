@@ -160,7 +160,10 @@ def test_ttft_arms_match_the_oracle(RT):
     """One layer of each TTFT arm, run once outside any graph: the standard arm's attention
     (a zero-document plan, the whole context as causal fresh rows) and the linked arm's
     linked cache and attention, each against the fp64 oracle on the tensors the arm gave the
-    library (q, k, v after the projection and RoPE, the document pool)."""
+    library (q, k, v after the projection and RoPE, the document pool).  The harness's
+    weights give q, k and v unit variance, as in the workloads, so the attention bar is the
+    same (an output of magnitude 4 or more would already carry a bf16 rounding error near
+    the 1e-2 bar)."""
     from paper_2502_16002_gb300 import kvlink as K, ttft
     dev = torch.device("cuda:0")
     layer = ttft.Layer(dev)
