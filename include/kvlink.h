@@ -167,6 +167,8 @@ typedef struct {
     size_t device_bytes;      /* size of the device buffer kvlink_plan_upload needs   */
     size_t workspace_bytes;   /* scratch of kvlink_suffix_attention / linked_prefill  */
     int64_t attn_pairs;       /* unmasked (fresh row, key) pairs, per KV head group   */
+    int32_t n_attn_ctas;      /* CTAs of the persistent suffix attention (one per SM at
+                                 most), each running its own list of work items       */
 } kvlink_plan_info_t;
 
 /* Build the host tables of a batch: the layout of every query (Sec. 2.3), the

@@ -30,7 +30,7 @@ int clear_copy_status();
 void launch_attention_simt(const DevicePlan& P, int n_fresh, int head_dim, int h_q, int h_kv,
                            const void* q, const void* cache_k, const void* cache_v, void* out,
                            cudaStream_t stream);
-int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t ctx_rows,
+int launch_attention_tc(const DevicePlan& P, int n_items, int n_ctas, int n_merges, int n_fresh, int64_t ctx_rows,
                         int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err);
 int read_attention_status(int32_t* status);
@@ -195,7 +195,7 @@ int kvlink_plan_rebuild(kvlink_plan_t* p, const kvlink_batch_desc_t* desc) {
     KVLINK_RECYCLE(fresh_pos) KVLINK_RECYCLE(fresh_query) KVLINK_RECYCLE(src) KVLINK_RECYCLE(src_row)
     KVLINK_RECYCLE(fresh_vis) KVLINK_RECYCLE(fresh_row0) KVLINK_RECYCLE(fresh_dst) KVLINK_RECYCLE(cu_grp)
     KVLINK_RECYCLE(grp_src)
-    KVLINK_RECYCLE(items) KVLINK_RECYCLE(merges)
+    KVLINK_RECYCLE(items) KVLINK_RECYCLE(merges) KVLINK_RECYCLE(sched) KVLINK_RECYCLE(cu_sched)
 #undef KVLINK_RECYCLE
     std::string why;
     int rc;
@@ -231,6 +231,7 @@ int kvlink_plan_get_info(const kvlink_plan_t* p, kvlink_plan_info_t* info) {
     info->device_bytes = p->device_bytes;
     info->workspace_bytes = p->workspace_bytes;
     info->attn_pairs = p->attn_pairs;
+    info->n_attn_ctas = p->cu_sched.empty() ? 0 : (int32_t)p->cu_sched.size() - 1;
     return KVLINK_OK;
 }
 
@@ -292,6 +293,8 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     put(p->off_fresh_vis, p->fresh_vis.data(), p->fresh_vis.size() * sizeof(int32_t));
     put(p->off_fresh_row0, p->fresh_row0.data(), p->fresh_row0.size() * sizeof(int32_t));
     put(p->off_fresh_dst, p->fresh_dst.data(), p->fresh_dst.size() * sizeof(int32_t));
+    put(p->off_sched, p->sched.data(), p->sched.size() * sizeof(int32_t));
+    put(p->off_cu_sched, p->cu_sched.data(), p->cu_sched.size() * sizeof(int32_t));
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = cudaMemcpyAsync(d_buf, host, p->device_bytes, cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload copy");
@@ -319,11 +322,14 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     d.fresh_vis = (const int32_t*)(b + p->off_fresh_vis);
     d.fresh_row0 = (const int32_t*)(b + p->off_fresh_row0);
     d.fresh_dst = (const int32_t*)(b + p->off_fresh_dst);
+    d.sched = (const int32_t*)(b + p->off_sched);
+    d.cu_sched = (const int32_t*)(b + p->off_cu_sched);
     d.batch = p->batch;
     d.h_kv = p->h_kv;
     d.n_fresh = p->cu_fresh.back();
     d.n_slots = p->n_slots;
     d.n_rope_rows = p->n_rope_rows;
+    d.n_items = (int32_t)p->items.size();
     d.ctx_rows = p->cu_ctx.back();
     d.pool_rows = p->pool_rows;
     launch_rope_table(d.seg, (int)p->seg.size(), (float4*)(b + p->off_rope), p->head_dim, theta, s);
@@ -382,7 +388,8 @@ static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k
     if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
     if (ws && !aligned16(ws)) return KVLINK_EINVAL;
     cudaError_t err = cudaSuccess;
-    const int rc = launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
+    const int rc = launch_attention_tc(p->dev, (int)p->items.size(), (int)p->cu_sched.size() - 1,
+                                       (int)p->merges.size(), p->cu_fresh.back(),
                                        p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out,
                                        ws, s, &err);
     if (rc == KVLINK_ECUDA) return cuda_fail(err, "suffix attention launch");

@@ -218,15 +218,18 @@ __device__ __forceinline__ void mma_pv_role(uint8_t* smem, uint32_t off_v, uint3
     drain_bar(bar_drain, 0, status);
 }
 
-// Softmax + epilogue role, run by warps 0-3 (threadIdx.x = tile row).  TMEM holds NB
-// S/P buffers of kAttnBN columns from column tmem_s and the O accumulator at tmem_o.
+// Softmax over the key tiles of one item, run by warps 0-3 (threadIdx.x = tile row).  TMEM
+// holds NB S/P buffers of kAttnBN columns from column tmem_s and the O accumulator at tmem_o.
+// g0 is the running count of key tiles before this item's first one: a kernel that runs
+// several items one after another keeps its S buffers and barrier phases going across them
+// (tile j of the item uses buffer (g0 + j) % NB).  O is touched only to rescale it, after the
+// item's previous PV has finished.  Leaves the row's running max m (log2 units) and sum l.
 template <int D, int G, int NB>
-__device__ __forceinline__ void softmax_role(const AttnItem& it, const DevicePlan& P, uint32_t tmem_s,
-                                             uint32_t tmem_o, int n_tiles, uint64_t* bar_s_full,
+__device__ __forceinline__ bool softmax_item(const AttnItem& it, const DevicePlan& P, uint32_t tmem_s,
+                                             uint32_t tmem_o, int n_tiles, int g0, uint64_t* bar_s_full,
                                              uint64_t* bar_p_full, uint64_t* bar_o_done,
-                                             volatile int32_t* abort_flag, int32_t* status,
-                                             __nv_bfloat16* __restrict__ out, float* __restrict__ ws, int h_q,
-                                             float scale_log2) {
+                                             volatile int32_t* abort_flag, int32_t* status, float scale_log2,
+                                             float& m_out, float& l_out) {
     using namespace sm100;
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int r = threadIdx.x;  // tile row == TMEM lane
@@ -239,10 +242,10 @@ __device__ __forceinline__ void softmax_role(const AttnItem& it, const DevicePla
     const uint32_t vis_b = valid ? (uint32_t)(tok + 1) : 0u;
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
     float m = -INFINITY, l = 0.f;
-    bool ok = true;
     for (int j = 0; j < n_tiles; ++j) {
-        const int b = j % NB;
-        if (!(ok = warp_wait(bar_s_full + b, (j / NB) & 1, abort_flag, status))) break;
+        const int g = g0 + j;
+        const int b = g % NB;
+        if (!warp_wait(bar_s_full + b, (g / NB) & 1, abort_flag, status)) return false;
         tc_fence_after();
         uint32_t s[128];
         const uint32_t s_col = lane_base + tmem_s + b * kAttnBN;
@@ -306,7 +309,7 @@ __device__ __forceinline__ void softmax_role(const AttnItem& it, const DevicePla
         }
         if (j > 0 && __any_sync(0xffffffffu, resc)) {
             // O is touched only while no PV is in flight: PV_{j-1} done, PV_j not yet issued
-            if (!(ok = warp_wait(bar_o_done + (j - 1) % NB, ((j - 1) / NB) & 1, abort_flag, status))) break;
+            if (!warp_wait(bar_o_done + (g - 1) % NB, ((g - 1) / NB) & 1, abort_flag, status)) return false;
             tc_fence_after();
 #pragma unroll
             for (int c4 = 0; c4 < D / 32; ++c4) {
@@ -356,44 +359,69 @@ __device__ __forceinline__ void softmax_role(const AttnItem& it, const DevicePla
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_p_full + b);
     }
-    if (ok && n_tiles > 0)
-        ok = warp_wait(bar_o_done + (n_tiles - 1) % NB, ((n_tiles - 1) / NB) & 1, abort_flag, status);
-    if (!ok) return;
-    tc_fence_after();
+    m_out = m;
+    l_out = l;
+    return true;
+}
+
+// Row r of an item's result from the values o[] of its O row: the output row normalised by
+// l (bf16), or, for an item whose KV range was split, the unnormalised partial (O, m, l).
+template <int D, int G>
+__device__ __forceinline__ void store_result(const AttnItem& it, const DevicePlan& P, int r, const uint32_t* o,
+                                             int c0, int nc, float m, float l, __nv_bfloat16* __restrict__ out,
+                                             float* __restrict__ ws, int h_q) {
+    const int tok = it.tok0 + r / G;
     if (it.slot < 0) {
+        if (tok >= it.tok1) return;
         const float inv = 1.f / l;
-        __nv_bfloat16* orow = out + ((int64_t)frow * h_q + it.kv_head * G + (r % G)) * D;
-#pragma unroll
-        for (int c4 = 0; c4 < D / 32; ++c4) {
-            uint32_t o[32];
-            tmem_ld32(lane_base + tmem_o + c4 * 32, o);
-            tmem_ld_wait();
-            if (valid) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint4 w;
-                    w.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * inv, __uint_as_float(o[8 * q + 1]) * inv);
-                    w.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv);
-                    w.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv);
-                    w.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv);
-                    *reinterpret_cast<uint4*>(orow + c4 * 32 + 8 * q) = w;
-                }
-            }
+        const int frow = P.cu_fresh[it.query] + tok;
+        __nv_bfloat16* orow = out + ((int64_t)frow * h_q + it.kv_head * G + (r % G)) * D + c0;
+        for (int q = 0; q < nc / 8; ++q) {
+            uint4 w;
+            w.x = pack2_bf16(__uint_as_float(o[8 * q + 0]) * inv, __uint_as_float(o[8 * q + 1]) * inv);
+            w.y = pack2_bf16(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv);
+            w.z = pack2_bf16(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv);
+            w.w = pack2_bf16(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv);
+            *reinterpret_cast<uint4*>(orow + 8 * q) = w;
         }
     } else {
         float* wo = ws + (int64_t)it.slot * kAttnBM * (D + 2);
-#pragma unroll
-        for (int c4 = 0; c4 < D / 32; ++c4) {
-            uint32_t o[32];
-            tmem_ld32(lane_base + tmem_o + c4 * 32, o);
-            tmem_ld_wait();
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-                *reinterpret_cast<uint4*>(wo + r * D + c4 * 32 + 4 * q) =
-                    make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+        for (int q = 0; q < nc / 4; ++q)
+            *reinterpret_cast<uint4*>(wo + r * D + c0 + 4 * q) = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2],
+                                                                           o[4 * q + 3]);
+        if (c0 == 0) {
+            wo[kAttnBM * D + r] = m;
+            wo[kAttnBM * D + kAttnBM + r] = l;
         }
-        wo[kAttnBM * D + r] = m;
-        wo[kAttnBM * D + kAttnBM + r] = l;
+    }
+}
+
+// Softmax + epilogue role of the one-item-per-CTA kernels, run by warps 0-3: the item's
+// tiles, then (once its last PV has finished) its result from O in TMEM.
+template <int D, int G, int NB>
+__device__ __forceinline__ void softmax_role(const AttnItem& it, const DevicePlan& P, uint32_t tmem_s,
+                                             uint32_t tmem_o, int n_tiles, uint64_t* bar_s_full,
+                                             uint64_t* bar_p_full, uint64_t* bar_o_done,
+                                             volatile int32_t* abort_flag, int32_t* status,
+                                             __nv_bfloat16* __restrict__ out, float* __restrict__ ws, int h_q,
+                                             float scale_log2) {
+    using namespace sm100;
+    float m, l;
+    if (!softmax_item<D, G, NB>(it, P, tmem_s, tmem_o, n_tiles, 0, bar_s_full, bar_p_full, bar_o_done, abort_flag,
+                                status, scale_log2, m, l))
+        return;
+    if (n_tiles > 0 &&
+        !warp_wait(bar_o_done + (n_tiles - 1) % NB, ((n_tiles - 1) / NB) & 1, abort_flag, status))
+        return;
+    tc_fence_after();
+    const int r = threadIdx.x;
+    const uint32_t lane_base = (uint32_t)((threadIdx.x / 32) * 32) << 16;
+#pragma unroll
+    for (int c4 = 0; c4 < D / 32; ++c4) {
+        uint32_t o[32];
+        tmem_ld32(lane_base + tmem_o + c4 * 32, o);
+        tmem_ld_wait();
+        store_result<D, G>(it, P, r, o, c4 * 32, 32, m, l, out, ws, h_q);
     }
 }
 

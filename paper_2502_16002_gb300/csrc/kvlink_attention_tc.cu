@@ -153,6 +153,293 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
 }
 
+// ------------------------------------------------------------------------------------------
+// Persistent form: one CTA per SM runs its list of items (the plan's per-CTA schedule) back to
+// back.  Every role walks the same list on its own and keeps its ring slots, TMEM buffers and
+// barrier phases going across items, so an item's start (Q, the first key tiles) and finish
+// (reading O out of TMEM, normalising, storing) overlap the neighbouring items' tile loops
+// instead of idling the tensor cores, and no CTA is launched per item.
+//   warps 0-3   softmax (softmax_item); at the end of an item its m and l go to shared memory
+//   warp 4      TMA: K tiles into the NK-stage ring; Q of each item once the previous item's
+//               S MMAs have read theirs (the next Q is brought into L2 ahead of time)
+//   warp 5      TMEM allocation; the thread issuing S = Q K^T
+//   warp 6      TMA: V tiles into the NV-stage ring
+//   warp 7      the thread issuing O += P V; an item's first PV waits until the epilogue has
+//               read the previous item's O
+//   warps 8-11  epilogue: once an item's last PV has finished, O is read out of TMEM (the
+//               accumulator is then free for the next item) and normalised and stored from
+//               registers
+// Registers: launched at 168 per thread (384 x 168 <= 64K); the TMA/MMA warpgroup drops to
+// 56 and the softmax warpgroup rises to 240 (240 + 56 + 168 per SM sub-partition).
+constexpr int kPtThreads = 384;
+constexpr int kPtEpiWarp0 = 8;
+constexpr uint32_t kPtSoftmaxRegs = 240, kPtIdleRegs = 56;
+static_assert(kPtThreads * 168 <= 65536, "launch register budget");
+static_assert(128 * (kPtSoftmaxRegs + kPtIdleRegs + 168) <= kPtThreads * 168, "register split");
+
+template <int D>
+struct PtCfg {
+    using T = TcCfg<D>;
+    static constexpr int NK = T::NK, NV = T::NV, NB = T::NB, ATOMS = T::ATOMS;
+    static constexpr uint32_t ATOM_BYTES = T::ATOM_BYTES, Q_BYTES = T::Q_BYTES, KV_BYTES = T::KV_BYTES;
+    static constexpr uint32_t OFF_Q = T::OFF_Q, OFF_K = T::OFF_K, OFF_V = T::OFF_V;
+    static constexpr uint32_t OFF_STATS = OFF_V + NV * KV_BYTES;        // m[128], l[128] of one item
+    static constexpr uint32_t OFF_BAR = OFF_STATS + 2 * kAttnBM * 4;
+    // q_full, q_empty, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB], p_full[NB],
+    // o_done[NB], o_full, o_free, st_full, st_empty, drain x2
+    static constexpr int N_BARS = 2 + 2 * NK + 2 * NV + 3 * NB + 6;
+    static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
+    static constexpr uint32_t TMEM_S = T::TMEM_S, TMEM_O = T::TMEM_O;
+    static_assert(SMEM_BYTES <= 232448, "shared memory budget");
+};
+
+template <int D, int G>
+__global__ void __launch_bounds__(kPtThreads, 1)
+    attn_tc_persistent_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                              const __grid_constant__ CUtensorMap tm_v, DevicePlan P,
+                              __nv_bfloat16* __restrict__ out, float* __restrict__ ws, int h_q, float scale_log2) {
+    using C = PtCfg<D>;
+    constexpr int NK = C::NK, NV = C::NV, NB = C::NB;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
+
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+    uint64_t* bar_q_full = bars;
+    uint64_t* bar_q_empty = bar_q_full + 1;
+    uint64_t* bar_k_full = bar_q_empty + 1;
+    uint64_t* bar_k_empty = bar_k_full + NK;
+    uint64_t* bar_v_full = bar_k_empty + NK;
+    uint64_t* bar_v_empty = bar_v_full + NV;
+    uint64_t* bar_s_full = bar_v_empty + NV;
+    uint64_t* bar_p_full = bar_s_full + NB;
+    uint64_t* bar_o_done = bar_p_full + NB;
+    uint64_t* bar_o_full = bar_o_done + NB;
+    uint64_t* bar_o_free = bar_o_full + 1;
+    uint64_t* bar_st_full = bar_o_free + 1;
+    uint64_t* bar_st_empty = bar_st_full + 1;
+    uint64_t* bar_drain = bar_st_empty + 1;
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + C::N_BARS);
+    volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(tmem_holder + 1);
+    float* st_m = reinterpret_cast<float*>(smem + C::OFF_STATS);
+    float* st_l = st_m + kAttnBM;
+
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int first = P.cu_sched[blockIdx.x], n_mine = P.cu_sched[blockIdx.x + 1] - first;
+    int32_t* status = &g_attn_status;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < C::N_BARS; ++i) {
+            uint64_t* b = bars + i;
+            // arrivals per phase: one per softmax / epilogue warp, else one (thread or commit)
+            const bool four = (b >= bar_p_full && b < bar_p_full + NB) || b == bar_o_free || b == bar_st_full ||
+                              b == bar_st_empty;
+            mbar_init(b, four ? 4 : 1);
+        }
+        // after a recorded failure, later launches skip their work instead of waiting out their bounds
+        *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_attn_status) != 0 ? 1 : 0;
+#ifdef KVLINK_DEBUG_CHECKS
+        for (int k = 0; k < n_mine && !*abort_flag; ++k) {
+            const int idx = P.sched[first + k];
+            if (idx < 0 || idx >= P.n_items || !item_in_bounds(P.items[idx], P) ||
+                P.items[idx].kv_tile1 <= P.items[idx].kv_tile0) {
+                atomicCAS(&g_attn_status, 0, kAttnStatusBadIndex);
+                *abort_flag = 1;
+            }
+        }
+#endif
+        fence_mbar_init();
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(tmem_holder, kTmemCols);
+        tmem_relinquish();
+    }
+    if (warp == kTmaKWarp && lane == 0) {
+        prefetch_tensormap(&tm_q);
+        prefetch_tensormap(&tm_k);
+        prefetch_tensormap(&tm_v);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+    const bool skip = *abort_flag != 0;  // written before the barrier: uniform across the CTA
+
+    if (skip) {
+        // nothing issued: fall through to the teardown
+    } else if (warp >= kSoftmaxWarps && warp < kPtEpiWarp0) {
+        setmaxnreg_dec<kPtIdleRegs>();
+        if (warp == kTmaKWarp && lane == 0) {
+            // ------------------------------------------------ Q of every item, and the K ring
+            int g = 0, q_issued = 0;
+            bool ok = true;
+            auto load_k = [&](const AttnItem& it, int ctx0, int j) -> bool {
+                const int st = g % NK;
+                if (!wait_bar(bar_k_empty + st, ((g / NK) & 1) ^ 1, abort_flag, status)) return false;
+                const int row = ctx0 + item_tile(it, it.kv_tile0 + j) * kAttnBN;
+                mbar_arrive_expect_tx(bar_k_full + st, C::KV_BYTES);
+#pragma unroll
+                for (int a = 0; a < C::ATOMS; ++a)
+                    tma_load_3d(smem + C::OFF_K + st * C::KV_BYTES + a * C::ATOM_BYTES, &tm_k, a * 64, it.kv_head,
+                                row, bar_k_full + st);
+                ++g;
+                return true;
+            };
+            for (int k = 0; ok && k < n_mine; ++k) {
+                const AttnItem it = P.items[P.sched[first + k]];
+                const int n = it.kv_tile1 - it.kv_tile0, ctx0 = (int)P.cu_ctx[it.query];
+                // the key tiles that fit in the ring go ahead of Q: their slots free up before the
+                // previous item's last S MMA has finished reading the Q buffer
+                const int ahead = k == 0 ? 0 : (n < NK ? n : NK);
+                for (int j = 0; ok && j < ahead; ++j) ok = load_k(it, ctx0, j);
+                if (!ok) break;
+                if (k > 0 && !(ok = wait_bar(bar_q_empty, (k - 1) & 1, abort_flag, status))) break;
+                mbar_arrive_expect_tx(bar_q_full, C::Q_BYTES);
+#pragma unroll
+                for (int a = 0; a < C::ATOMS; ++a)
+                    tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &tm_q, a * 64, it.kv_head * G,
+                                P.cu_fresh[it.query] + it.tok0, bar_q_full);
+                ++q_issued;
+                if (k + 1 < n_mine) {       // the next item's Q into L2 while this one runs
+                    const AttnItem nx = P.items[P.sched[first + k + 1]];
+#pragma unroll
+                    for (int a = 0; a < C::ATOMS; ++a)
+                        tma_prefetch_l2_3d(&tm_q, a * 64, nx.kv_head * G, P.cu_fresh[nx.query] + nx.tok0);
+                }
+                for (int j = ahead; ok && j < n; ++j) ok = load_k(it, ctx0, j);
+            }
+            // no copy may still be in flight when the CTA leaves
+            for (int gg = g - NK > 0 ? g - NK : 0; gg < g; ++gg) drain_bar(bar_k_full + gg % NK, (gg / NK) & 1, status);
+            if (q_issued > 0) drain_bar(bar_q_full, (q_issued - 1) & 1, status);
+        } else if (warp == kTmaVWarp && lane == 0) {
+            // ------------------------------------------------ the V ring
+            int g = 0;
+            bool ok = true;
+            for (int k = 0; ok && k < n_mine; ++k) {
+                const AttnItem it = P.items[P.sched[first + k]];
+                const int n = it.kv_tile1 - it.kv_tile0, ctx0 = (int)P.cu_ctx[it.query];
+                for (int j = 0; j < n; ++j, ++g) {
+                    const int st = g % NV;
+                    if (!(ok = wait_bar(bar_v_empty + st, ((g / NV) & 1) ^ 1, abort_flag, status))) break;
+                    const int row = ctx0 + item_tile(it, it.kv_tile0 + j) * kAttnBN;
+                    mbar_arrive_expect_tx(bar_v_full + st, C::KV_BYTES);
+#pragma unroll
+                    for (int a = 0; a < C::ATOMS; ++a)
+                        tma_load_3d(smem + C::OFF_V + st * C::KV_BYTES + a * C::ATOM_BYTES, &tm_v, a * 64, it.kv_head,
+                                    row, bar_v_full + st);
+                }
+            }
+            for (int gg = g - NV > 0 ? g - NV : 0; gg < g; ++gg) drain_bar(bar_v_full + gg % NV, (gg / NV) & 1, status);
+        } else if (warp == kMmaWarp && lane == 0) {
+            // ------------------------------------------------ S = Q K^T
+            constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
+            const uint32_t sQ = smem_u32(smem + C::OFF_Q);
+            int g = 0;
+            bool ok = true;
+            for (int k = 0; ok && k < n_mine; ++k) {
+                const AttnItem it = P.items[P.sched[first + k]];
+                const int n = it.kv_tile1 - it.kv_tile0;
+                if (!(ok = wait_bar(bar_q_full, k & 1, abort_flag, status))) break;
+                for (int j = 0; j < n; ++j, ++g) {
+                    const int sk = g % NK, b = g % NB;
+                    if (!(ok = wait_bar(bar_k_full + sk, (g / NK) & 1, abort_flag, status))) break;
+                    // buffer b last held P of tile g - NB: its PV must have finished reading it
+                    if (g >= NB && !(ok = wait_bar(bar_o_done + b, ((g - NB) / NB) & 1, abort_flag, status))) break;
+                    tc_fence_after();
+                    const uint32_t sK = smem_u32(smem + C::OFF_K + sk * C::KV_BYTES);
+#pragma unroll
+                    for (int kk = 0; kk < D / 16; ++kk) {
+                        const uint32_t koff = (kk >> 2) * C::ATOM_BYTES + (kk & 3) * 32;
+                        mma_bf16_ss(tmem + C::TMEM_S + b * kAttnBN, sdesc_sw128(sQ + koff, 16, 1024),
+                                    sdesc_sw128(sK + koff, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(bar_s_full + b);
+                    mma_commit(bar_k_empty + sk);
+                }
+                if (ok) mma_commit(bar_q_empty);   // arrives once this item's S MMAs have read Q
+            }
+            mma_commit(bar_drain);
+            drain_bar(bar_drain, 0, status);
+        } else if (warp == kPvWarp && lane == 0) {
+            // ------------------------------------------------ O += P V
+            constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
+            int g = 0;
+            bool ok = true;
+            for (int k = 0; ok && k < n_mine; ++k) {
+                const AttnItem it = P.items[P.sched[first + k]];
+                const int n = it.kv_tile1 - it.kv_tile0;
+                for (int i = 0; i < n; ++i, ++g) {
+                    const int b = g % NB, sv = g % NV;
+                    if (!(ok = wait_bar(bar_p_full + b, (g / NB) & 1, abort_flag, status))) break;
+                    if (!(ok = wait_bar(bar_v_full + sv, (g / NV) & 1, abort_flag, status))) break;
+                    // the item's first PV overwrites O: the epilogue must have read the previous item's
+                    if (i == 0 && k > 0 && !(ok = wait_bar(bar_o_free, (k - 1) & 1, abort_flag, status))) break;
+                    tc_fence_after();
+                    const uint32_t sV = smem_u32(smem + C::OFF_V + sv * C::KV_BYTES);
+                    const uint32_t pcol = tmem + C::TMEM_S + b * kAttnBN;
+#pragma unroll
+                    for (int kk = 0; kk < kAttnBN / 16; ++kk)
+                        mma_bf16_ts(tmem + C::TMEM_O, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, C::ATOM_BYTES, 1024),
+                                    idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
+                    mma_commit(bar_o_done + b);
+                    mma_commit(bar_v_empty + sv);
+                }
+                if (ok) mma_commit(bar_o_full);    // arrives once the item's last PV has finished
+            }
+            mma_commit(bar_drain + 1);
+            drain_bar(bar_drain + 1, 0, status);
+        }
+    } else if (warp < kSoftmaxWarps) {
+        // ---------------------------------------------------- softmax (warps 0-3)
+        setmaxnreg_inc<kPtSoftmaxRegs>();
+        int g = 0;
+        for (int k = 0; k < n_mine; ++k) {
+            const AttnItem it = P.items[P.sched[first + k]];
+            const int n = it.kv_tile1 - it.kv_tile0;
+            float m, l;
+            if (!softmax_item<D, G, NB>(it, P, tmem + C::TMEM_S, tmem + C::TMEM_O, n, g, bar_s_full, bar_p_full,
+                                        bar_o_done, abort_flag, status, scale_log2, m, l))
+                break;
+            g += n;
+            // the row's m and l to the epilogue, once it has taken the previous item's
+            if (!warp_wait(bar_st_empty, (k & 1) ^ 1, abort_flag, status)) break;
+            st_m[threadIdx.x] = m;
+            st_l[threadIdx.x] = l;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_st_full);
+        }
+    } else {
+        // ---------------------------------------------------- epilogue (warps 8-11)
+        const int r = threadIdx.x - kPtEpiWarp0 * 32;                   // tile row == TMEM lane
+        const uint32_t lane_base = (uint32_t)((warp % 4) * 32) << 16;
+        for (int k = 0; k < n_mine; ++k) {
+            const AttnItem it = P.items[P.sched[first + k]];
+            if (!warp_wait(bar_o_full, k & 1, abort_flag, status)) break;
+            if (!warp_wait(bar_st_full, k & 1, abort_flag, status)) break;
+            const float m = st_m[r], l = st_l[r];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_st_empty);
+            tc_fence_after();
+            uint32_t o[D];
+#pragma unroll
+            for (int c4 = 0; c4 < D / 32; ++c4)
+                tmem_ld32(lane_base + tmem + C::TMEM_O + c4 * 32, *reinterpret_cast<uint32_t(*)[32]>(o + 32 * c4));
+            tmem_ld_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_o_free);     // O may now take the next item's PVs
+            store_result<D, G>(it, P, r, o, 0, D, m, l, out, ws, h_q);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
 // Combine the partial results of split KV ranges: O = sum_s O_s 2^(m_s - M) / sum_s l_s 2^(m_s - M).
 template <int D>
 __global__ void __launch_bounds__(256) attn_merge_kernel(DevicePlan P, const float* __restrict__ ws,
@@ -217,17 +504,23 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uin
 
 template <int D, int G>
 static cudaError_t launch_tc_dg(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv,
-                                const DevicePlan& P, int n_items, int n_merges, void* out, float* ws, int h_q,
-                                float scale_log2, cudaStream_t stream) {
-    using C = TcCfg<D>;
+                                const DevicePlan& P, int n_items, int n_ctas, int n_merges, void* out, float* ws,
+                                int h_q, float scale_log2, cudaStream_t stream) {
     static std::atomic<uint64_t> attr_set{0};
     cudaError_t ea = once_per_device(attr_set, [] {
-        return cudaFuncSetAttribute(attn_tc_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)C::SMEM_BYTES);
+        cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)TcCfg<D>::SMEM_BYTES);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(attn_tc_persistent_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)PtCfg<D>::SMEM_BYTES);
+        return e;
     });
     if (ea != cudaSuccess) return ea;
-    if (n_items > 0)
-        attn_tc_kernel<D, G><<<n_items, kTcThreads, C::SMEM_BYTES, stream>>>(
+    if (n_items > 0 && n_ctas > 0)
+        attn_tc_persistent_kernel<D, G><<<n_ctas, kPtThreads, PtCfg<D>::SMEM_BYTES, stream>>>(
+            mq, mk, mv, P, (__nv_bfloat16*)out, ws, h_q, scale_log2);
+    else if (n_items > 0)
+        attn_tc_kernel<D, G><<<n_items, kTcThreads, TcCfg<D>::SMEM_BYTES, stream>>>(
             mq, mk, mv, P, (__nv_bfloat16*)out, ws, h_q, scale_log2);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -247,7 +540,8 @@ cudaError_t launch_attn_merge(const DevicePlan& P, int n_merges, const float* ws
 }
 
 // Returns 0, or KVLINK_ECUDA / KVLINK_EUNSUPPORTED.
-int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t ctx_rows,
+// n_ctas > 0: the persistent kernel over the plan's per-CTA schedule; 0: one CTA per item.
+int launch_attention_tc(const DevicePlan& P, int n_items, int n_ctas, int n_merges, int n_fresh, int64_t ctx_rows,
                         int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err) {
     const int G = h_q / h_kv;
@@ -261,8 +555,8 @@ int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fr
     float* w = (float*)ws;
     cudaError_t e = cudaErrorInvalidValue;
 #define KVLINK_TC_CASE(DD, GG)                                                                         \
-    if (head_dim == DD && G == GG) e = launch_tc_dg<DD, GG>(mq, mk, mv, P, n_items, n_merges, out, w, h_q, sl2, \
-                                                            stream);
+    if (head_dim == DD && G == GG) e = launch_tc_dg<DD, GG>(mq, mk, mv, P, n_items, n_ctas, n_merges, out, w, h_q, \
+                                                            sl2, stream);
     KVLINK_TC_CASE(128, 1) KVLINK_TC_CASE(128, 2) KVLINK_TC_CASE(128, 4) KVLINK_TC_CASE(128, 8)
     KVLINK_TC_CASE(128, 16) KVLINK_TC_CASE(64, 1) KVLINK_TC_CASE(64, 2) KVLINK_TC_CASE(64, 4)
     KVLINK_TC_CASE(64, 8) KVLINK_TC_CASE(64, 16)

@@ -123,13 +123,16 @@ struct DevicePlan {
     const int32_t* fresh_row0;   // [B], query-relative
     const int32_t* fresh_dst;    // [n_fresh] batch cache row of every fresh row
     // sizes the tables index into (checked on the device by the KVLINK_DEBUG_CHECKS build)
-    int32_t batch, h_kv, n_fresh, n_slots, n_rope_rows;
+    int32_t batch, h_kv, n_fresh, n_slots, n_rope_rows, n_items;
     int64_t ctx_rows, pool_rows;
     // Groups of 8 cache rows (8m .. 8m+7 of a query), at cu_grp[b] + m: the first source
     // row when the group's 8 rows are consecutive in one tensor (one 8-row TMA copy), else
     // -1 (rows copied one by one; also the query's last, partial group).
     const int32_t* cu_grp;       // [B+1]
     const int32_t* grp_src;      // pool row, or kGrpFresh | fresh row
+    // Persistent attention: CTA c runs items sched[cu_sched[c] .. cu_sched[c+1]) in order.
+    const int32_t* sched;        // [n_items] item indices
+    const int32_t* cu_sched;     // [n_ctas + 1]
 };
 constexpr int32_t kGrpFresh = 1 << 30;
 constexpr int32_t kGrpRowMask = kGrpFresh - 1;
@@ -199,6 +202,7 @@ struct kvlink_plan {
     std::vector<int32_t> cu_grp, grp_src;
     std::vector<kvlink::AttnItem> items;
     std::vector<kvlink::MergeGroup> merges;
+    std::vector<int32_t> sched, cu_sched;   // the persistent attention's item list per CTA
     int32_t n_slots = 0;
     int64_t cached_tokens = 0;
     int64_t attn_pairs = 0;
@@ -208,7 +212,7 @@ struct kvlink_plan {
     size_t off_seg = 0, off_chunks = 0, off_rope = 0, off_pool_start = 0, off_pool_bt = 0,
            off_cu_ctx = 0, off_cu_fresh = 0, off_fresh_pos = 0, off_fresh_query = 0,
            off_items = 0, off_merges = 0, off_src = 0, off_cu_grp = 0, off_grp_src = 0, off_src_row = 0,
-           off_fresh_vis = 0, off_fresh_row0 = 0, off_fresh_dst = 0,
+           off_fresh_vis = 0, off_fresh_row0 = 0, off_fresh_dst = 0, off_sched = 0, off_cu_sched = 0,
            device_bytes = 0;
     size_t workspace_bytes = 0;
 

@@ -30,7 +30,7 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
                      void* cache_v, cudaStream_t stream);
 void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int64_t ctx_rows, int row_bytes,
                         const void* k_new, const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
-int launch_attention_tc(const DevicePlan& P, int n_items, int n_merges, int n_fresh, int64_t ctx_rows,
+int launch_attention_tc(const DevicePlan& P, int n_items, int n_ctas, int n_merges, int n_fresh, int64_t ctx_rows,
                         int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err);
 }  // namespace kvlink
@@ -86,7 +86,8 @@ extern "C" int kvlink_suffix_attention_noalloc(const kvlink_plan_t* p, const voi
         if (rc != KVLINK_OK) return rc;
     }
     cudaError_t err = cudaSuccess;
-    rc = kvlink::launch_attention_tc(p->dev, (int)p->items.size(), (int)p->merges.size(), p->cu_fresh.back(),
+    rc = kvlink::launch_attention_tc(p->dev, (int)p->items.size(), (int)p->cu_sched.size() - 1,
+                                     (int)p->merges.size(), p->cu_fresh.back(),
                                      p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, ws, s,
                                      &err);
     if (rc == KVLINK_ECUDA) return kvlink::record_cuda_error(err, "suffix attention launch (noalloc)");

@@ -5,6 +5,7 @@
 #include <cstdint>
 #include <cstring>
 #include <numeric>
+#include <queue>
 #include <string>
 
 #include "kvlink_internal.h"
@@ -299,46 +300,42 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
             }
         }
     }
-    // Split long KV ranges (into partials merged afterwards) only when there are fewer
-    // items than SMs: with at least one item per SM the merges and the extra prologues
-    // cost more than the balance they buy (measured on the 8B-shape workloads).
-    int32_t max_tiles = INT32_MAX;
-    if ((int64_t)tiles.size() < (int64_t)num_sms)
-        max_tiles = (int32_t)std::max<int64_t>(8, (work + num_sms - 1) / num_sms);
-    p->items.clear();
-    p->merges.clear();
-    p->n_slots = 0;
-    for (const Tile& t : tiles) {
-        const int32_t n_split = (t.n_tiles + max_tiles - 1) / max_tiles;
-        if (n_split <= 1) {
-            p->items.push_back({t.b, t.g, t.t0, t.t1, 0, t.n_tiles, -1, t.min_vis, t.owner, t.a_tiles, t.b_tile0});
-            continue;
+    // Split KV ranges into pieces of at most max_tiles key tiles (partials merged afterwards).
+    auto make_items = [&](int32_t max_tiles, std::vector<AttnItem>& items, std::vector<MergeGroup>& merges,
+                          int32_t& n_slots) {
+        items.clear();
+        merges.clear();
+        n_slots = 0;
+        for (const Tile& t : tiles) {
+            const int32_t n_split = (t.n_tiles + max_tiles - 1) / max_tiles;
+            if (n_split <= 1) {
+                items.push_back({t.b, t.g, t.t0, t.t1, 0, t.n_tiles, -1, t.min_vis, t.owner, t.a_tiles, t.b_tile0});
+                continue;
+            }
+            merges.push_back({t.b, t.g, t.t0, t.t1, n_slots, n_split, 0, 0});
+            for (int s = 0; s < n_split; ++s) {
+                const int32_t a = (int32_t)((int64_t)t.n_tiles * s / n_split);
+                const int32_t e = (int32_t)((int64_t)t.n_tiles * (s + 1) / n_split);
+                items.push_back({t.b, t.g, t.t0, t.t1, a, e, n_slots + s, t.min_vis, t.owner, t.a_tiles, t.b_tile0});
+            }
+            n_slots += n_split;
         }
-        p->merges.push_back({t.b, t.g, t.t0, t.t1, p->n_slots, n_split, 0, 0});
-        for (int s = 0; s < n_split; ++s) {
-            const int32_t a = (int32_t)((int64_t)t.n_tiles * s / n_split);
-            const int32_t e = (int32_t)((int64_t)t.n_tiles * (s + 1) / n_split);
-            p->items.push_back({t.b, t.g, t.t0, t.t1, a, e, p->n_slots + s, t.min_vis, t.owner, t.a_tiles, t.b_tile0});
-        }
-        p->n_slots += n_split;
-    }
-    // Launch order.  The items of one (query, KV head) stay adjacent, so that CTAs running
-    // at the same time read the same K/V tiles (served from L2 after the first); groups go
-    // longest first, and so do the items inside a group.  Items of at most 55% of the
-    // longest item's key tiles are held back to the end, longest first: run inside their
-    // groups they leave the long items of the last groups to start late and run alone at
-    // the end of the grid, while at the end they fill the gaps of the last wave (their K/V
-    // tiles, a prefix of their group's, are read once more).
-    {
+        // Launch order.  The items of one (query, KV head) stay adjacent, so that CTAs running
+        // at the same time read the same K/V tiles (served from L2 after the first); groups go
+        // longest first, and so do the items inside a group.  Items of at most 55% of the
+        // longest item's key tiles are held back to the end, longest first: run inside their
+        // groups they leave the long items of the last groups to start late and run alone at
+        // the end of the grid, while at the end they fill the gaps of the last wave (their K/V
+        // tiles, a prefix of their group's, are read once more).
         std::vector<int64_t> group_cost((size_t)B * d->h_kv, 0);
         int64_t longest = 0;
-        for (const AttnItem& it : p->items) {
+        for (const AttnItem& it : items) {
             const int64_t c = it.kv_tile1 - it.kv_tile0;
             int64_t& g = group_cost[(size_t)it.query * d->h_kv + it.kv_head];
             g = std::max(g, c);
             longest = std::max(longest, c);
         }
-        std::stable_sort(p->items.begin(), p->items.end(), [&](const AttnItem& x, const AttnItem& y) {
+        std::stable_sort(items.begin(), items.end(), [&](const AttnItem& x, const AttnItem& y) {
             const int64_t cx = x.kv_tile1 - x.kv_tile0, cy = y.kv_tile1 - y.kv_tile0;
             const bool late_x = cx * 100 <= longest * 55, late_y = cy * 100 <= longest * 55;
             if (late_x != late_y) return late_y;
@@ -353,8 +350,89 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
             if (x.kv_head != y.kv_head) return x.kv_head < y.kv_head;
             return cx > cy;
         });
+    };
+
+    // The persistent attention's schedule: one CTA per SM (fewer with fewer items), each item
+    // handed to the CTA that would be free first (list scheduling on the estimated cost in
+    // half tiles: two per key tile, one for the item's own start and finish, two more for a
+    // piece of a split range, whose partial is stored and merged).  Two hand-out orders are
+    // estimated: the launch order (the items of one (query, KV head) run together and share
+    // their K/V tiles in L2) and longest first over all items; the launch order is kept
+    // unless longest first finishes more than 3% earlier (a few long groups filling the
+    // grid: one long query's last KV head would otherwise start only after a first item
+    // elsewhere).
+    using Slot = std::pair<int64_t, int32_t>;
+    auto cost = [](const AttnItem& it) { return 2 * (int64_t)(it.kv_tile1 - it.kv_tile0) + 1 + (it.slot >= 0 ? 2 : 0); };
+    auto schedule = [&](const std::vector<AttnItem>& items, const std::vector<int32_t>& order, int32_t n_ctas,
+                        std::vector<std::vector<int32_t>>* lists) {
+        std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> free_at;
+        for (int32_t c = 0; c < n_ctas; ++c) free_at.push({0, c});
+        if (lists) lists->assign((size_t)n_ctas, {});
+        int64_t makespan = 0;
+        for (int32_t i : order) {
+            const Slot sl = free_at.top();
+            free_at.pop();
+            if (lists) (*lists)[(size_t)sl.second].push_back(i);
+            makespan = std::max(makespan, sl.first + cost(items[(size_t)i]));
+            free_at.push({sl.first + cost(items[(size_t)i]), sl.second});
+        }
+        return makespan;
+    };
+    // returns the estimated makespan and the better order
+    auto best_order = [&](const std::vector<AttnItem>& items, int32_t n_ctas, std::vector<int32_t>& order) {
+        std::vector<int32_t> launch(items.size()), longest_first;
+        std::iota(launch.begin(), launch.end(), 0);
+        longest_first = launch;
+        std::stable_sort(longest_first.begin(), longest_first.end(),
+                         [&](int32_t a, int32_t b) { return cost(items[(size_t)a]) > cost(items[(size_t)b]); });
+        const int64_t m_launch = schedule(items, launch, n_ctas, nullptr);
+        const int64_t m_longest = schedule(items, longest_first, n_ctas, nullptr);
+        const bool use_longest = m_longest * 103 < m_launch * 100;
+        order = use_longest ? longest_first : launch;
+        return use_longest ? m_longest : m_launch;
+    };
+
+    // Split granularity: pieces of at most W / (k * SMs) key tiles (W the batch's key tiles),
+    // for the k in 1..4 whose estimated time is shortest (a larger k only when it is more
+    // than 2% shorter): with many short items nothing is split; one long query, or a batch
+    // whose longest items would hold the grid up, is split just enough to balance.  The
+    // estimate adds the merge pass, which runs after the attention and reads every partial
+    // (O, m, l: about 130 KB for head_dim 128, written once and read once): at HBM speed
+    // one half tile of attention time moves about 19 partials, plus about 5 half tiles for
+    // the launch.
+    int64_t best_span = INT64_MAX;
+    std::vector<int32_t> best_ord;
+    for (int k = 1; k <= 4; ++k) {
+        const int32_t max_tiles = (int32_t)std::max<int64_t>(8, (work + (int64_t)num_sms * k - 1) / ((int64_t)num_sms * k));
+        std::vector<AttnItem> items;
+        std::vector<MergeGroup> merges;
+        int32_t n_slots = 0;
+        make_items(max_tiles, items, merges, n_slots);
+        const int32_t n_ctas = std::min<int32_t>(num_sms, (int32_t)items.size());
+        std::vector<int32_t> order;
+        const int64_t span = best_order(items, n_ctas, order) + (n_slots > 0 ? 5 + n_slots / 19 : 0);
+        if (k == 1 || span * 100 < best_span * 98) {
+            best_span = span;
+            p->items.swap(items);
+            p->merges.swap(merges);
+            p->n_slots = n_slots;
+            best_ord.swap(order);
+        }
+        if (max_tiles == 8) break;   // finer pieces are not made
     }
     p->workspace_bytes = (size_t)p->n_slots * (size_t)kAttnBM * ((size_t)d->head_dim + 2) * sizeof(float);
+    {
+        const int32_t n_ctas = std::min<int32_t>(num_sms, (int32_t)p->items.size());
+        std::vector<std::vector<int32_t>> lists;
+        schedule(p->items, best_ord, n_ctas, &lists);
+        p->sched.clear();
+        p->cu_sched.assign((size_t)n_ctas + 1, 0);
+        for (int32_t c = 0; c < n_ctas; ++c) {
+            p->cu_sched[(size_t)c] = (int32_t)p->sched.size();
+            p->sched.insert(p->sched.end(), lists[(size_t)c].begin(), lists[(size_t)c].end());
+        }
+        p->cu_sched[(size_t)n_ctas] = (int32_t)p->sched.size();
+    }
 
     // ---- device buffer layout (256-byte aligned tables)
     size_t off = 0;
@@ -378,6 +456,8 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     p->off_fresh_vis = take(p->fresh_vis.size() * sizeof(int32_t));
     p->off_fresh_row0 = take(p->fresh_row0.size() * sizeof(int32_t));
     p->off_fresh_dst = take(p->fresh_dst.size() * sizeof(int32_t));
+    p->off_sched = take(p->sched.size() * sizeof(int32_t));
+    p->off_cu_sched = take(p->cu_sched.size() * sizeof(int32_t));
     p->device_bytes = off;
     p->uploaded = false;
     return KVLINK_OK;

@@ -73,7 +73,7 @@ class kvlink_plan_info_t(C.Structure):
         ("n_copy_chunks", C.c_int32), ("n_attn_items", C.c_int32), ("n_attn_splits", C.c_int32),
         ("num_sms", C.c_int32),
         ("device_bytes", C.c_size_t), ("workspace_bytes", C.c_size_t),
-        ("attn_pairs", C.c_int64),
+        ("attn_pairs", C.c_int64), ("n_attn_ctas", C.c_int32),
     ]
 
 

@@ -32,6 +32,7 @@ import numpy as np
 import torch
 
 from . import kvlink as K
+from .clocks import ClockSampler
 from .runtime import LinkedPrefill
 
 HIDDEN, H_Q, H_KV, HEAD_DIM, FFN, LAYERS, THETA = 4096, 32, 8, 128, 14336, 32, 500000.0
@@ -102,16 +103,32 @@ def _graphed(fn):
     return g.replay
 
 
-def _time(fn, warmup=10, iters=40):
+CLOCKS = {}     # arm -> clock record of its last timed region (filled by _time)
+
+
+def _time(fn, warmup=10, iters=40, arm=None, min_seconds=1.0):
+    """ms per call from CUDA events around `iters` calls (raised so that the timed region lasts
+    at least min_seconds), with the GPU clocks sampled during the timed region."""
     for _ in range(warmup):
         fn()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     e0.record()
-    for _ in range(iters):
-        fn()
+    fn()
     e1.record()
     torch.cuda.synchronize()
+    iters = max(iters, int(min_seconds * 1e3 / max(e0.elapsed_time(e1), 1e-3)) + 1)
+    with ClockSampler(torch.cuda.current_device(), 50) as clk:
+        torch.cuda.synchronize()
+        clk.start()
+        e0.record()
+        for _ in range(iters):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        clk.stop()
+    if arm is not None:
+        CLOCKS[arm] = dict(clk.summary(), iters=iters)
     return e0.elapsed_time(e1) / iters
 
 
@@ -165,8 +182,8 @@ def layer_arms(doc_len, n_docs, n_link, q_len, host_caches, device, layer):
 def measure(doc_len, n_docs, n_link, q_len, host_caches, device, layer):
     """ms per layer of (standard, linked) for n_docs documents of doc_len tokens."""
     standard, linked, _, n_ctx, T = layer_arms(doc_len, n_docs, n_link, q_len, host_caches, device, layer)
-    t_std = _time(_graphed(standard))
-    t_lnk = _time(_graphed(linked))
+    t_std = _time(_graphed(standard), arm="standard")
+    t_lnk = _time(_graphed(linked), arm="linked")
     assert K.kvlink_device_status() == 0
     return t_std, t_lnk, n_ctx, T
 
@@ -227,8 +244,8 @@ def measure_pipelined(doc_len, n_docs, n_link, q_len, device, layer, layers=LAYE
         compute.wait_stream(copy_stream)
         return x
 
-    t_std = _time(_graphed(standard), warmup=3, iters=10)
-    t_lnk = _time(_graphed(linked), warmup=3, iters=10)
+    t_std = _time(_graphed(standard), warmup=3, iters=10, arm="standard")
+    t_lnk = _time(_graphed(linked), warmup=3, iters=10, arm="linked")
     assert K.kvlink_device_status() == 0
     return t_std, t_lnk, n_ctx, T
 
@@ -254,8 +271,8 @@ def main():
                     "context_tokens": n_ctx, "fresh_tokens": T, "ttft_standard_ms": round(t_std, 3),
                     "ttft_linked_ms": round(t_lnk, 3), "reduction_pct": round(100 * (1 - t_lnk / t_std), 1),
                     "caches": "pinned host memory, per-layer copies overlapped with the previous layer",
-                    "layers": LAYERS, "shape": "Llama-3.1-8B, random bf16 weights, whole model in one graph"}),
-                    flush=True)
+                    "layers": LAYERS, "shape": "Llama-3.1-8B, random bf16 weights, whole model in one graph",
+                    "clocks": dict(CLOCKS)}), flush=True)
         return
     for n_link in args.links:
         for L in args.lengths:
@@ -266,7 +283,8 @@ def main():
                 "ttft_standard_ms": round(t_std * LAYERS, 3), "ttft_linked_ms": round(t_lnk * LAYERS, 3),
                 "reduction_pct": round(100 * (1 - t_lnk / t_std), 1),
                 "caches": "pinned host memory, copied per layer" if args.host_caches else "resident in HBM",
-                "layers": LAYERS, "shape": "Llama-3.1-8B, random bf16 weights"}), flush=True)
+                "layers": LAYERS, "shape": "Llama-3.1-8B, random bf16 weights", "clocks": dict(CLOCKS)}),
+                flush=True)
 
 
 if __name__ == "__main__":
