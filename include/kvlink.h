@@ -206,6 +206,8 @@ int kvlink_plan_get_sources(const kvlink_plan_t* plan, kvlink_source_t* src, int
  * delta_i * theta^(-2j/D) for every cached document i and j < D/2, with the angle
  * formed and reduced in float64 and stored as float32 (Sec. 2.2; done once per
  * batch, shared by all layers).  The plan records d_buf; later calls read it.
+ * The buffer also holds the arrival counters of the attention's in-kernel merges, which the
+ * upload zeroes and the attention kernels update (the buffer is not read-only on the device).
  * Asynchronous: the tables go through a pinned staging buffer owned by the plan, and the
  * call returns once the copy is enqueued (a later upload of the same plan first waits for
  * it).  d_buf must stay valid, and the plan alive, until the last call using them has
@@ -239,6 +241,11 @@ int kvlink_reencode_concat(const kvlink_plan_t* plan, const void* d_pool_k, cons
  * d_q: [n_fresh][h_q][D]; d_k_new/d_v_new: [n_fresh][h_kv][D]; d_out: [n_fresh][h_q][D];
  * all bf16.  Scores and softmax in fp32, products of bf16 on the tensor cores.
  * d_workspace: >= workspace_bytes of scratch (may be NULL when that is 0).
+ * The attention runs as one persistent kernel, one CTA per SM over its share of the work;
+ * a KV range cut between CTAs is merged inside the kernel through arrival counters kept in
+ * the plan's device buffer (zeroed by kvlink_plan_upload), so attention calls with one plan
+ * must not overlap on the device, and after a wait that ran out (kvlink_device_status) the
+ * plan must be uploaded again before its next use.
  * Errors: EINVAL, ECAPACITY, EUNSUPPORTED, ECUDA. */
 int kvlink_suffix_attention(const kvlink_plan_t* plan, const void* d_q, const void* d_k_new,
                             const void* d_v_new, void* d_cache_k, void* d_cache_v, void* d_out,

@@ -196,6 +196,7 @@ int kvlink_plan_rebuild(kvlink_plan_t* p, const kvlink_batch_desc_t* desc) {
     KVLINK_RECYCLE(fresh_vis) KVLINK_RECYCLE(fresh_row0) KVLINK_RECYCLE(fresh_dst) KVLINK_RECYCLE(cu_grp)
     KVLINK_RECYCLE(grp_src)
     KVLINK_RECYCLE(items) KVLINK_RECYCLE(merges) KVLINK_RECYCLE(sched) KVLINK_RECYCLE(cu_sched)
+    KVLINK_RECYCLE(slot_group)
 #undef KVLINK_RECYCLE
     std::string why;
     int rc;
@@ -295,6 +296,8 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     put(p->off_fresh_dst, p->fresh_dst.data(), p->fresh_dst.size() * sizeof(int32_t));
     put(p->off_sched, p->sched.data(), p->sched.size() * sizeof(int32_t));
     put(p->off_cu_sched, p->cu_sched.data(), p->cu_sched.size() * sizeof(int32_t));
+    put(p->off_slot_group, p->slot_group.data(), p->slot_group.size() * sizeof(int32_t));
+    std::memset(host + p->off_merge_count, 0, p->merges.size() * sizeof(unsigned long long));
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = cudaMemcpyAsync(d_buf, host, p->device_bytes, cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return cuda_fail(e, "kvlink_plan_upload copy");
@@ -324,6 +327,9 @@ int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes
     d.fresh_dst = (const int32_t*)(b + p->off_fresh_dst);
     d.sched = (const int32_t*)(b + p->off_sched);
     d.cu_sched = (const int32_t*)(b + p->off_cu_sched);
+    d.slot_group = (const int32_t*)(b + p->off_slot_group);
+    d.merge_count = (unsigned long long*)(b + p->off_merge_count);
+    d.n_merges = (int32_t)p->merges.size();
     d.batch = p->batch;
     d.h_kv = p->h_kv;
     d.n_fresh = p->cu_fresh.back();

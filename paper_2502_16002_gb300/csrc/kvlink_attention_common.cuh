@@ -385,13 +385,95 @@ __device__ __forceinline__ void store_result(const AttnItem& it, const DevicePla
             *reinterpret_cast<uint4*>(orow + 8 * q) = w;
         }
     } else {
+        // column-major [D][kAttnBM]: the 32 rows of a warp write 128 contiguous bytes per column
         float* wo = ws + (int64_t)it.slot * kAttnBM * (D + 2);
-        for (int q = 0; q < nc / 4; ++q)
-            *reinterpret_cast<uint4*>(wo + r * D + c0 + 4 * q) = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2],
-                                                                           o[4 * q + 3]);
+        for (int e = 0; e < nc; ++e) wo[(c0 + e) * kAttnBM + r] = __uint_as_float(o[e]);
         if (c0 == 0) {
             wo[kAttnBM * D + r] = m;
             wo[kAttnBM * D + kAttnBM + r] = l;
+        }
+    }
+}
+
+// Merge of the partial results (O, m, l) of one split KV range, row r (Sec. 2.3 attention
+// computed over disjoint key ranges and combined): with M = max_s m_s and f_s = 2^(m_s - M),
+// out = sum_s O_s f_s * (1 / sum_s l_s f_s), summed in slot order.  O_s is column-major:
+// element (r, d) of a slot at d * kAttnBM + r.  The separate merge kernel and
+// the persistent attention's in-kernel merge both use these, so they give the same bits.
+// Partials are read through L2 (ld.global.cg): another CTA may have written them.
+template <int D>
+__device__ __forceinline__ float merge_max(const float* ws, int slot0, int n, int r) {
+    const int64_t slot_floats = (int64_t)kAttnBM * (D + 2);
+    float M = -INFINITY;
+#pragma unroll 4
+    for (int s = 0; s < n; ++s) M = fmaxf(M, __ldcg(ws + (slot0 + s) * slot_floats + kAttnBM * D + r));
+    return M;
+}
+template <int D>
+__device__ __forceinline__ float merge_factor(const float* ws, int slot, int r, float M) {
+    const float ms = __ldcg(ws + (int64_t)slot * kAttnBM * (D + 2) + kAttnBM * D + r);
+    return (ms == -INFINITY) ? 0.f : sm100::ex2_approx(ms - M);
+}
+template <int D>
+__device__ __forceinline__ float merge_sum(const float* ws, int slot0, int n, int r, float M) {
+    float L = 0.f;
+#pragma unroll 4
+    for (int s = 0; s < n; ++s)
+        L = __fmaf_rn(__ldcg(ws + (int64_t)(slot0 + s) * kAttnBM * (D + 2) + kAttnBM * D + kAttnBM + r),
+                      merge_factor<D>(ws, slot0 + s, r, M), L);
+    return L;
+}
+template <int D>
+__device__ __forceinline__ float merge_value(const float* ws, int slot0, int n, int r, int d, float M, float L) {
+    float O = 0.f;
+    for (int s = 0; s < n; ++s)
+        O = __fmaf_rn(__ldcg(ws + (int64_t)(slot0 + s) * kAttnBM * (D + 2) + d * kAttnBM + r),
+                      merge_factor<D>(ws, slot0 + s, r, M), O);
+    return __fmul_rn(O, __frcp_rn(L));
+}
+
+// Row r of a merge group's output, written as bf16 to orow, with the arithmetic of
+// merge_value (the same factors, the same fused multiply-adds in slot order, the same
+// reciprocal).  Built for latency: the partials are column-major, so the 32 rows of a warp
+// read 128 contiguous bytes per column, and each 32-column chunk issues the loads of two
+// slots (their m and 32 values each) before any arithmetic.
+template <int D>
+__device__ __noinline__ void merge_row_store(const float* ws, int slot0, int n, int r,
+                                             __nv_bfloat16* __restrict__ orow) {
+    const float M = merge_max<D>(ws, slot0, n, r);
+    const float inv = __frcp_rn(merge_sum<D>(ws, slot0, n, r, M));
+    const int64_t slot_floats = (int64_t)kAttnBM * (D + 2);
+    for (int c0 = 0; c0 < D; c0 += 32) {
+        float acc[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) acc[e] = 0.f;
+        for (int s0 = 0; s0 < n; s0 += 2) {
+            const bool two = s0 + 1 < n;
+            const float* w0 = ws + (slot0 + s0) * slot_floats;
+            const float* w1 = two ? w0 + slot_floats : w0;
+            const float m0 = __ldcg(w0 + kAttnBM * D + r), m1 = __ldcg(w1 + kAttnBM * D + r);
+            float v0[32], v1[32];
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+                v0[e] = __ldcg(w0 + (c0 + e) * kAttnBM + r);
+                v1[e] = __ldcg(w1 + (c0 + e) * kAttnBM + r);
+            }
+            const float f0 = (m0 == -INFINITY) ? 0.f : sm100::ex2_approx(m0 - M);
+            const float f1 = (m1 == -INFINITY) ? 0.f : sm100::ex2_approx(m1 - M);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+                acc[e] = __fmaf_rn(v0[e], f0, acc[e]);
+                if (two) acc[e] = __fmaf_rn(v1[e], f1, acc[e]);
+            }
+        }
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+            uint4 w;
+            w.x = pack2_bf16(__fmul_rn(acc[8 * h + 0], inv), __fmul_rn(acc[8 * h + 1], inv));
+            w.y = pack2_bf16(__fmul_rn(acc[8 * h + 2], inv), __fmul_rn(acc[8 * h + 3], inv));
+            w.z = pack2_bf16(__fmul_rn(acc[8 * h + 4], inv), __fmul_rn(acc[8 * h + 5], inv));
+            w.w = pack2_bf16(__fmul_rn(acc[8 * h + 6], inv), __fmul_rn(acc[8 * h + 7], inv));
+            *reinterpret_cast<uint4*>(orow + c0 + 8 * h) = w;
         }
     }
 }

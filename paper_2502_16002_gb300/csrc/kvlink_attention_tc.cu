@@ -160,15 +160,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // (reading O out of TMEM, normalising, storing) overlap the neighbouring items' tile loops
 // instead of idling the tensor cores, and no CTA is launched per item.
 //   warps 0-3   softmax (softmax_item); at the end of an item its m and l go to shared memory
-//   warp 4      TMA: K tiles into the NK-stage ring; Q of each item once the previous item's
-//               S MMAs have read theirs (the next Q is brought into L2 ahead of time)
+//   warp 4      TMA: Q of each item into one of two Q buffers (so it lands while the previous
+//               item runs), and the K tiles into the NK-stage ring
 //   warp 5      TMEM allocation; the thread issuing S = Q K^T
 //   warp 6      TMA: V tiles into the NV-stage ring
 //   warp 7      the thread issuing O += P V; an item's first PV waits until the epilogue has
 //               read the previous item's O
 //   warps 8-11  epilogue: once an item's last PV has finished, O is read out of TMEM (the
 //               accumulator is then free for the next item) and normalised and stored from
-//               registers
+//               registers.  A piece of a split KV range stores its partial (O, m, l); the
+//               piece that completes its group (a per-group arrival counter in the plan
+//               buffer) merges the group's partials into the output, so no merge launch follows
 // Registers: launched at 168 per thread (384 x 168 <= 64K); the TMA/MMA warpgroup drops to
 // 56 and the softmax warpgroup rises to 240 (240 + 56 + 168 per SM sub-partition).
 constexpr int kPtThreads = 384;
@@ -177,21 +179,68 @@ constexpr uint32_t kPtSoftmaxRegs = 240, kPtIdleRegs = 56;
 static_assert(kPtThreads * 168 <= 65536, "launch register budget");
 static_assert(128 * (kPtSoftmaxRegs + kPtIdleRegs + 168) <= kPtThreads * 168, "register split");
 
+// Shared memory: two Q buffers (the next item's Q lands while the current item runs), the K
+// ring and the V ring (one stage fewer than the one-item kernel's for head_dim 128: a V tile
+// is needed a softmax later than its K tile), m and l of one item, a flag, the barriers.
 template <int D>
 struct PtCfg {
-    using T = TcCfg<D>;
-    static constexpr int NK = T::NK, NV = T::NV, NB = T::NB, ATOMS = T::ATOMS;
-    static constexpr uint32_t ATOM_BYTES = T::ATOM_BYTES, Q_BYTES = T::Q_BYTES, KV_BYTES = T::KV_BYTES;
-    static constexpr uint32_t OFF_Q = T::OFF_Q, OFF_K = T::OFF_K, OFF_V = T::OFF_V;
+    static constexpr int ATOMS = D / 64;
+    static constexpr int NK = (D == 128) ? 3 : 5;
+    static constexpr int NV = (D == 128) ? 2 : 4;
+    static constexpr int NB = 3;
+    static constexpr uint32_t ATOM_BYTES = 128 * 128;
+    static constexpr uint32_t Q_BYTES = ATOMS * ATOM_BYTES, KV_BYTES = ATOMS * ATOM_BYTES;
+    static constexpr uint32_t OFF_Q = 0;                                // two buffers
+    static constexpr uint32_t OFF_K = OFF_Q + 2 * Q_BYTES;
+    static constexpr uint32_t OFF_V = OFF_K + NK * KV_BYTES;
     static constexpr uint32_t OFF_STATS = OFF_V + NV * KV_BYTES;        // m[128], l[128] of one item
-    static constexpr uint32_t OFF_BAR = OFF_STATS + 2 * kAttnBM * 4;
-    // q_full, q_empty, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB], p_full[NB],
-    // o_done[NB], o_full, o_free, st_full, st_empty, drain x2
-    static constexpr int N_BARS = 2 + 2 * NK + 2 * NV + 3 * NB + 6;
+    static constexpr uint32_t OFF_FLAG = OFF_STATS + 2 * kAttnBM * 4;   // the epilogue's merge decision
+    static constexpr uint32_t OFF_BAR = OFF_FLAG + 16;
+    // q_full[2], q_empty[2], k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB],
+    // p_full[NB], o_done[NB], o_full, o_free, st_full, st_empty, drain x2
+    static constexpr int N_BARS = 4 + 2 * NK + 2 * NV + 3 * NB + 6;
     static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
-    static constexpr uint32_t TMEM_S = T::TMEM_S, TMEM_O = T::TMEM_O;
+    static constexpr uint32_t TMEM_S = 0, TMEM_O = NB * kAttnBN;
+    static_assert(TMEM_O + D <= kTmemCols, "TMEM budget");
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
 };
+
+// The epilogue warps' part of an item (thread r = TMEM lane r): O read out of TMEM (then the
+// accumulator is free for the next item's PVs), normalised and stored; for a piece of a split
+// range its partial is stored, and the piece that completes its merge group combines all the
+// group's partials into the output.  The four warps take every decision together (named
+// barrier 1 over their 128 threads).
+template <int D, int G>
+__device__ __forceinline__ void epilogue_item(const AttnItem& it, const DevicePlan& P, int r, uint32_t o_taddr,
+                                              float m, float l, uint64_t* bar_o_free, volatile int32_t* flag,
+                                              __nv_bfloat16* __restrict__ out, float* __restrict__ ws, int h_q) {
+    uint32_t o[D];
+#pragma unroll
+    for (int c4 = 0; c4 < D / 32; ++c4) tmem_ld32(o_taddr + c4 * 32, *reinterpret_cast<uint32_t(*)[32]>(o + 32 * c4));
+    tmem_ld_wait();
+    tc_fence_before();
+    __syncwarp();
+    if (threadIdx.x % 32 == 0) mbar_arrive(bar_o_free);     // O may now take the next item's PVs
+    store_result<D, G>(it, P, r, o, 0, D, m, l, out, ws, h_q);
+    if (it.slot < 0) return;
+    // a piece of a split range: the last of its group to arrive merges
+    const int grp = P.slot_group[it.slot];
+    const MergeGroup mg = P.merges[grp];
+    // The four warps' partial stores are ordered before thread 0's arrival by the barrier, and
+    // the arrival (release, cumulative) publishes them to every CTA; the arrival that completes
+    // the group also acquires the other pieces' partials, which the barrier then orders before
+    // this CTA's reads of them.
+    named_bar_sync(1, 128);
+    if (r == 0) *flag = ((atom_add_acq_rel_gpu(P.merge_count + grp, 1ull) + 1) % (unsigned long long)mg.n_split) == 0;
+    named_bar_sync(1, 128);
+    const bool last = *flag != 0;
+    named_bar_sync(1, 128);                 // every thread has read the flag before it is reused
+    if (!last) return;
+    const int tok = mg.tok0 + r / G;
+    if (tok >= mg.tok1) return;
+    merge_row_store<D>(ws, mg.slot0, mg.n_split, r,
+                       out + ((int64_t)(P.cu_fresh[mg.query] + tok) * h_q + mg.kv_head * G + (r % G)) * D);
+}
 
 template <int D, int G>
 __global__ void __launch_bounds__(kPtThreads, 1)
@@ -205,9 +254,9 @@ __global__ void __launch_bounds__(kPtThreads, 1)
     uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
 
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
-    uint64_t* bar_q_full = bars;
-    uint64_t* bar_q_empty = bar_q_full + 1;
-    uint64_t* bar_k_full = bar_q_empty + 1;
+    uint64_t* bar_q_full = bars;                 // [2]
+    uint64_t* bar_q_empty = bar_q_full + 2;      // [2]
+    uint64_t* bar_k_full = bar_q_empty + 2;
     uint64_t* bar_k_empty = bar_k_full + NK;
     uint64_t* bar_v_full = bar_k_empty + NK;
     uint64_t* bar_v_empty = bar_v_full + NV;
@@ -223,6 +272,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(tmem_holder + 1);
     float* st_m = reinterpret_cast<float*>(smem + C::OFF_STATS);
     float* st_l = st_m + kAttnBM;
+    volatile int32_t* merge_flag = reinterpret_cast<volatile int32_t*>(smem + C::OFF_FLAG);
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int first = P.cu_sched[blockIdx.x], n_mine = P.cu_sched[blockIdx.x + 1] - first;
@@ -241,8 +291,14 @@ __global__ void __launch_bounds__(kPtThreads, 1)
 #ifdef KVLINK_DEBUG_CHECKS
         for (int k = 0; k < n_mine && !*abort_flag; ++k) {
             const int idx = P.sched[first + k];
-            if (idx < 0 || idx >= P.n_items || !item_in_bounds(P.items[idx], P) ||
-                P.items[idx].kv_tile1 <= P.items[idx].kv_tile0) {
+            bool ok = idx >= 0 && idx < P.n_items && item_in_bounds(P.items[idx], P) &&
+                      P.items[idx].kv_tile1 > P.items[idx].kv_tile0;
+            if (ok && P.items[idx].slot >= 0) {
+                const int grp = P.slot_group[P.items[idx].slot];
+                ok = grp >= 0 && grp < P.n_merges && P.merges[grp].n_split >= 1 &&
+                     P.merges[grp].slot0 >= 0 && P.merges[grp].slot0 + P.merges[grp].n_split <= P.n_slots;
+            }
+            if (!ok) {
                 atomicCAS(&g_attn_status, 0, kAttnStatusBadIndex);
                 *abort_flag = 1;
             }
@@ -273,44 +329,33 @@ __global__ void __launch_bounds__(kPtThreads, 1)
             // ------------------------------------------------ Q of every item, and the K ring
             int g = 0, q_issued = 0;
             bool ok = true;
-            auto load_k = [&](const AttnItem& it, int ctx0, int j) -> bool {
-                const int st = g % NK;
-                if (!wait_bar(bar_k_empty + st, ((g / NK) & 1) ^ 1, abort_flag, status)) return false;
-                const int row = ctx0 + item_tile(it, it.kv_tile0 + j) * kAttnBN;
-                mbar_arrive_expect_tx(bar_k_full + st, C::KV_BYTES);
-#pragma unroll
-                for (int a = 0; a < C::ATOMS; ++a)
-                    tma_load_3d(smem + C::OFF_K + st * C::KV_BYTES + a * C::ATOM_BYTES, &tm_k, a * 64, it.kv_head,
-                                row, bar_k_full + st);
-                ++g;
-                return true;
-            };
             for (int k = 0; ok && k < n_mine; ++k) {
                 const AttnItem it = P.items[P.sched[first + k]];
                 const int n = it.kv_tile1 - it.kv_tile0, ctx0 = (int)P.cu_ctx[it.query];
-                // the key tiles that fit in the ring go ahead of Q: their slots free up before the
-                // previous item's last S MMA has finished reading the Q buffer
-                const int ahead = k == 0 ? 0 : (n < NK ? n : NK);
-                for (int j = 0; ok && j < ahead; ++j) ok = load_k(it, ctx0, j);
-                if (!ok) break;
-                if (k > 0 && !(ok = wait_bar(bar_q_empty, (k - 1) & 1, abort_flag, status))) break;
-                mbar_arrive_expect_tx(bar_q_full, C::Q_BYTES);
+                // Q buffer k % 2, once the S MMAs of item k - 2 have read it
+                const int qb = k & 1;
+                if (!(ok = wait_bar(bar_q_empty + qb, ((k >> 1) & 1) ^ 1, abort_flag, status))) break;
+                mbar_arrive_expect_tx(bar_q_full + qb, C::Q_BYTES);
 #pragma unroll
                 for (int a = 0; a < C::ATOMS; ++a)
-                    tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &tm_q, a * 64, it.kv_head * G,
-                                P.cu_fresh[it.query] + it.tok0, bar_q_full);
+                    tma_load_3d(smem + C::OFF_Q + qb * C::Q_BYTES + a * C::ATOM_BYTES, &tm_q, a * 64,
+                                it.kv_head * G, P.cu_fresh[it.query] + it.tok0, bar_q_full + qb);
                 ++q_issued;
-                if (k + 1 < n_mine) {       // the next item's Q into L2 while this one runs
-                    const AttnItem nx = P.items[P.sched[first + k + 1]];
+                for (int j = 0; j < n; ++j, ++g) {
+                    const int st = g % NK;
+                    if (!(ok = wait_bar(bar_k_empty + st, ((g / NK) & 1) ^ 1, abort_flag, status))) break;
+                    const int row = ctx0 + item_tile(it, it.kv_tile0 + j) * kAttnBN;
+                    mbar_arrive_expect_tx(bar_k_full + st, C::KV_BYTES);
 #pragma unroll
                     for (int a = 0; a < C::ATOMS; ++a)
-                        tma_prefetch_l2_3d(&tm_q, a * 64, nx.kv_head * G, P.cu_fresh[nx.query] + nx.tok0);
+                        tma_load_3d(smem + C::OFF_K + st * C::KV_BYTES + a * C::ATOM_BYTES, &tm_k, a * 64, it.kv_head,
+                                    row, bar_k_full + st);
                 }
-                for (int j = ahead; ok && j < n; ++j) ok = load_k(it, ctx0, j);
             }
             // no copy may still be in flight when the CTA leaves
             for (int gg = g - NK > 0 ? g - NK : 0; gg < g; ++gg) drain_bar(bar_k_full + gg % NK, (gg / NK) & 1, status);
-            if (q_issued > 0) drain_bar(bar_q_full, (q_issued - 1) & 1, status);
+            for (int k = q_issued - 2 > 0 ? q_issued - 2 : 0; k < q_issued; ++k)
+                drain_bar(bar_q_full + (k & 1), (k >> 1) & 1, status);
         } else if (warp == kTmaVWarp && lane == 0) {
             // ------------------------------------------------ the V ring
             int g = 0;
@@ -333,13 +378,14 @@ __global__ void __launch_bounds__(kPtThreads, 1)
         } else if (warp == kMmaWarp && lane == 0) {
             // ------------------------------------------------ S = Q K^T
             constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
-            const uint32_t sQ = smem_u32(smem + C::OFF_Q);
             int g = 0;
             bool ok = true;
             for (int k = 0; ok && k < n_mine; ++k) {
                 const AttnItem it = P.items[P.sched[first + k]];
                 const int n = it.kv_tile1 - it.kv_tile0;
-                if (!(ok = wait_bar(bar_q_full, k & 1, abort_flag, status))) break;
+                const int qb = k & 1;
+                if (!(ok = wait_bar(bar_q_full + qb, (k >> 1) & 1, abort_flag, status))) break;
+                const uint32_t sQ = smem_u32(smem + C::OFF_Q + qb * C::Q_BYTES);
                 for (int j = 0; j < n; ++j, ++g) {
                     const int sk = g % NK, b = g % NB;
                     if (!(ok = wait_bar(bar_k_full + sk, (g / NK) & 1, abort_flag, status))) break;
@@ -356,7 +402,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
                     mma_commit(bar_s_full + b);
                     mma_commit(bar_k_empty + sk);
                 }
-                if (ok) mma_commit(bar_q_empty);   // arrives once this item's S MMAs have read Q
+                if (ok) mma_commit(bar_q_empty + qb);   // arrives once this item's S MMAs have read Q
             }
             mma_commit(bar_drain);
             drain_bar(bar_drain, 0, status);
@@ -414,21 +460,15 @@ __global__ void __launch_bounds__(kPtThreads, 1)
         const uint32_t lane_base = (uint32_t)((warp % 4) * 32) << 16;
         for (int k = 0; k < n_mine; ++k) {
             const AttnItem it = P.items[P.sched[first + k]];
-            if (!warp_wait(bar_o_full, k & 1, abort_flag, status)) break;
-            if (!warp_wait(bar_st_full, k & 1, abort_flag, status)) break;
+            bool ok = warp_wait(bar_o_full, k & 1, abort_flag, status);
+            ok = ok && warp_wait(bar_st_full, k & 1, abort_flag, status);
+            // the four epilogue warps leave together (they meet at named barriers below)
+            if (named_bar_any(1, 128, !ok)) break;
             const float m = st_m[r], l = st_l[r];
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_st_empty);
             tc_fence_after();
-            uint32_t o[D];
-#pragma unroll
-            for (int c4 = 0; c4 < D / 32; ++c4)
-                tmem_ld32(lane_base + tmem + C::TMEM_O + c4 * 32, *reinterpret_cast<uint32_t(*)[32]>(o + 32 * c4));
-            tmem_ld_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar_o_free);     // O may now take the next item's PVs
-            store_result<D, G>(it, P, r, o, 0, D, m, l, out, ws, h_q);
+            epilogue_item<D, G>(it, P, r, lane_base + tmem + C::TMEM_O, m, l, bar_o_free, merge_flag, out, ws, h_q);
         }
     }
 
@@ -455,21 +495,13 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(DevicePlan P, const flo
 #endif
     const int n_rows = (mg.tok1 - mg.tok0) * G;
     const int f0 = P.cu_fresh[mg.query];
-    const int64_t slot_floats = (int64_t)kAttnBM * (D + 2);
     for (int idx = threadIdx.x; idx < n_rows * D; idx += blockDim.x) {
-        const int r = idx / D, d = idx % D;
-        float M = -INFINITY;
-        for (int s = 0; s < mg.n_split; ++s) M = fmaxf(M, ws[(mg.slot0 + s) * slot_floats + kAttnBM * D + r]);
-        float L = 0.f, O = 0.f;
-        for (int s = 0; s < mg.n_split; ++s) {
-            const float* w = ws + (mg.slot0 + s) * slot_floats;
-            const float ms = w[kAttnBM * D + r];
-            const float f = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
-            L += w[kAttnBM * D + kAttnBM + r] * f;
-            O += w[r * D + d] * f;
-        }
+        const int r = idx % n_rows, d = idx / n_rows;   // neighbouring threads: neighbouring rows
+        const float M = merge_max<D>(ws, mg.slot0, mg.n_split, r);
+        const float L = merge_sum<D>(ws, mg.slot0, mg.n_split, r, M);
         const int frow = f0 + mg.tok0 + r / G;
-        out[((int64_t)frow * h_q + mg.kv_head * G + (r % G)) * D + d] = __float2bfloat16_rn(O / L);
+        out[((int64_t)frow * h_q + mg.kv_head * G + (r % G)) * D + d] =
+            __float2bfloat16_rn(merge_value<D>(ws, mg.slot0, mg.n_split, r, d, M, L));
     }
 }
 
@@ -516,10 +548,12 @@ static cudaError_t launch_tc_dg(const CUtensorMap& mq, const CUtensorMap& mk, co
         return e;
     });
     if (ea != cudaSuccess) return ea;
-    if (n_items > 0 && n_ctas > 0)
+    if (n_items > 0 && n_ctas > 0) {       // split ranges are merged inside the kernel
         attn_tc_persistent_kernel<D, G><<<n_ctas, kPtThreads, PtCfg<D>::SMEM_BYTES, stream>>>(
             mq, mk, mv, P, (__nv_bfloat16*)out, ws, h_q, scale_log2);
-    else if (n_items > 0)
+        return cudaGetLastError();
+    }
+    if (n_items > 0)
         attn_tc_kernel<D, G><<<n_items, kTcThreads, TcCfg<D>::SMEM_BYTES, stream>>>(
             mq, mk, mv, P, (__nv_bfloat16*)out, ws, h_q, scale_log2);
     cudaError_t e = cudaGetLastError();

@@ -133,6 +133,13 @@ struct DevicePlan {
     // Persistent attention: CTA c runs items sched[cu_sched[c] .. cu_sched[c+1]) in order.
     const int32_t* sched;        // [n_items] item indices
     const int32_t* cu_sched;     // [n_ctas + 1]
+    // Split KV ranges merged inside the persistent attention: the merge group of every
+    // partial slot, and one arrival counter per group.  A counter only ever grows (each
+    // launch adds its group's n_split), so the piece that brings it to a multiple of n_split
+    // is the last of its launch and merges; kvlink_plan_upload zeroes the counters.
+    const int32_t* slot_group;   // [n_slots]
+    unsigned long long* merge_count;   // [n_merges], in the plan buffer (written by the kernel)
+    int32_t n_merges;
 };
 constexpr int32_t kGrpFresh = 1 << 30;
 constexpr int32_t kGrpRowMask = kGrpFresh - 1;
@@ -203,6 +210,7 @@ struct kvlink_plan {
     std::vector<kvlink::AttnItem> items;
     std::vector<kvlink::MergeGroup> merges;
     std::vector<int32_t> sched, cu_sched;   // the persistent attention's item list per CTA
+    std::vector<int32_t> slot_group;        // merge group of every partial slot
     int32_t n_slots = 0;
     int64_t cached_tokens = 0;
     int64_t attn_pairs = 0;
@@ -213,6 +221,7 @@ struct kvlink_plan {
            off_cu_ctx = 0, off_cu_fresh = 0, off_fresh_pos = 0, off_fresh_query = 0,
            off_items = 0, off_merges = 0, off_src = 0, off_cu_grp = 0, off_grp_src = 0, off_src_row = 0,
            off_fresh_vis = 0, off_fresh_row0 = 0, off_fresh_dst = 0, off_sched = 0, off_cu_sched = 0,
+           off_slot_group = 0, off_merge_count = 0,
            device_bytes = 0;
     size_t workspace_bytes = 0;
 

@@ -300,139 +300,204 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
             }
         }
     }
-    // Split KV ranges into pieces of at most max_tiles key tiles (partials merged afterwards).
-    auto make_items = [&](int32_t max_tiles, std::vector<AttnItem>& items, std::vector<MergeGroup>& merges,
-                          int32_t& n_slots) {
-        items.clear();
-        merges.clear();
-        n_slots = 0;
-        for (const Tile& t : tiles) {
-            const int32_t n_split = (t.n_tiles + max_tiles - 1) / max_tiles;
-            if (n_split <= 1) {
-                items.push_back({t.b, t.g, t.t0, t.t1, 0, t.n_tiles, -1, t.min_vis, t.owner, t.a_tiles, t.b_tile0});
-                continue;
-            }
-            merges.push_back({t.b, t.g, t.t0, t.t1, n_slots, n_split, 0, 0});
-            for (int s = 0; s < n_split; ++s) {
-                const int32_t a = (int32_t)((int64_t)t.n_tiles * s / n_split);
-                const int32_t e = (int32_t)((int64_t)t.n_tiles * (s + 1) / n_split);
-                items.push_back({t.b, t.g, t.t0, t.t1, a, e, n_slots + s, t.min_vis, t.owner, t.a_tiles, t.b_tile0});
-            }
-            n_slots += n_split;
+    // ---- work items and the persistent attention's schedule.
+    // Costs are in half tiles: two per key tile, one for an item's own start and finish.  Two
+    // schedules are built and the one with the shorter estimated time is kept:
+    //  A  whole M-tiles in launch order, each to the CTA with the least work so far (list
+    //     scheduling; also tried longest first over all M-tiles).  The launch order keeps the
+    //     M-tiles of one (query, KV head) together, groups with the longest M-tile first, so
+    //     that CTAs working at the same time share their K/V tiles in L2; M-tiles of at most
+    //     55% of the longest are held back to the end, longest first, where they fill the
+    //     gaps of the last wave (when the longest M-tile is more than a quarter of a CTA's
+    //     share; otherwise the groups simply go by their key tiles).  Balance is limited by the
+    //     M-tile size: a CTA holding two long M-tiles ends late.
+    //  B  the same list scheduling (M-tiles of a group together, groups with the most key
+    //     tiles first) with every CTA capped at an equal share of the whole: an M-tile that
+    //     would carry a CTA past its share is cut, the CTA keeps the key tiles that fit and the
+    //     rest goes on to the next CTA with the least work.  The pieces of a cut M-tile write
+    //     partial results (O, m, l), merged inside the persistent kernel by the piece that
+    //     completes the group (or by attn_merge_kernel after the one-item-per-CTA kernels).
+    //     The estimate charges every CTA holding a piece kMergeCost for the partial store and
+    //     the merge (epilogue work that also takes issue slots from the softmax), so B is also
+    //     tried with shares 5% and 10% above the mean, where fewer M-tiles are cut.  One long
+    //     query (M-tiles of a few hundred key tiles) needs B.
+    // Small batches use fewer CTAs (at least kMinShare half tiles each) and never cut a piece
+    // under kMinPiece key tiles.
+    struct Sched {
+        std::vector<AttnItem> items;
+        std::vector<MergeGroup> merges;
+        std::vector<std::vector<int32_t>> lists;
+        int32_t n_slots = 0;
+        int64_t span = 0;
+    };
+    constexpr int64_t kMinShare = 2 * 8 + 1;
+    constexpr int32_t kMinPiece = 4;
+    constexpr int64_t kMergeCost = 14;
+    int64_t total = 0;
+    for (const Tile& t : tiles) total += 2 * (int64_t)t.n_tiles + 1;
+    const int32_t n_ctas = (int32_t)std::max<int64_t>(1, std::min<int64_t>(num_sms, total / kMinShare));
+    using Slot = std::pair<int64_t, int32_t>;      // (work so far, CTA)
+    auto item_of = [](const Tile& t, int32_t a, int32_t e) {
+        return AttnItem{t.b, t.g, t.t0, t.t1, a, e, -1, t.min_vis, t.owner, t.a_tiles, t.b_tile0};
+    };
+    auto group_key = [&](const std::vector<int64_t>& gc, const Tile& t) { return gc[(size_t)t.b * d->h_kv + t.g]; };
+
+    // A: whole M-tiles, list scheduled in the given order
+    auto schedule_whole = [&](const std::vector<Tile>& order) {
+        Sched s;
+        s.lists.assign((size_t)n_ctas, {});
+        std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> least;
+        for (int32_t c = 0; c < n_ctas; ++c) least.push({0, c});
+        for (const Tile& t : order) {
+            const Slot sl = least.top();
+            least.pop();
+            s.lists[(size_t)sl.second].push_back((int32_t)s.items.size());
+            s.items.push_back(item_of(t, 0, t.n_tiles));
+            const int64_t load = sl.first + 2 * (int64_t)t.n_tiles + 1;
+            s.span = std::max(s.span, load);
+            least.push({load, sl.second});
         }
-        // Launch order.  The items of one (query, KV head) stay adjacent, so that CTAs running
-        // at the same time read the same K/V tiles (served from L2 after the first); groups go
-        // longest first, and so do the items inside a group.  Items of at most 55% of the
-        // longest item's key tiles are held back to the end, longest first: run inside their
-        // groups they leave the long items of the last groups to start late and run alone at
-        // the end of the grid, while at the end they fill the gaps of the last wave (their K/V
-        // tiles, a prefix of their group's, are read once more).
-        std::vector<int64_t> group_cost((size_t)B * d->h_kv, 0);
-        int64_t longest = 0;
-        for (const AttnItem& it : items) {
-            const int64_t c = it.kv_tile1 - it.kv_tile0;
-            int64_t& g = group_cost[(size_t)it.query * d->h_kv + it.kv_head];
-            g = std::max(g, c);
-            longest = std::max(longest, c);
+        return s;
+    };
+    // B: capped shares, M-tiles cut at the cap
+    auto schedule_capped = [&](const std::vector<Tile>& order, int slack_pct) {
+        Sched s;
+        s.lists.assign((size_t)n_ctas, {});
+        std::vector<int32_t> pieces_on((size_t)n_ctas, 0);
+        // the equal share, plus room for the starts of two more pieces and slack_pct percent:
+        // with slack, an M-tile is cut only where a CTA would otherwise end well past the mean
+        int64_t share = (total + n_ctas - 1) / n_ctas * (100 + slack_pct) / 100 + 2;
+        std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> least;
+        for (int32_t c = 0; c < n_ctas; ++c) least.push({0, c});
+        for (const Tile& t : order) {
+            const size_t first_piece = s.items.size();
+            std::vector<int32_t> ctas;
+            int32_t done = 0;
+            while (done < t.n_tiles) {
+                // every CTA full (a cut adds a start the shares did not count): all shares grow
+                while (least.top().first + 3 > share) share += 2;
+                const Slot sl = least.top();
+                least.pop();
+                const int32_t rest = t.n_tiles - done;
+                int32_t m = (int32_t)std::min<int64_t>(rest, (share - sl.first - 1) / 2);
+                // no piece under kMinPiece key tiles: the CTA rather runs a little past its share
+                if (m < rest) {
+                    if (m < kMinPiece) m = std::min(rest, kMinPiece);
+                    else if (rest - m < kMinPiece) m = rest;
+                }
+                s.lists[(size_t)sl.second].push_back((int32_t)s.items.size());
+                s.items.push_back(item_of(t, done, done + m));
+                ctas.push_back(sl.second);
+                least.push({sl.first + 2 * (int64_t)m + 1, sl.second});
+                done += m;
+            }
+            const int32_t n_split = (int32_t)(s.items.size() - first_piece);
+            if (n_split > 1) {
+                s.merges.push_back({t.b, t.g, t.t0, t.t1, s.n_slots, n_split, 0, 0});
+                for (int32_t i = 0; i < n_split; ++i) s.items[first_piece + (size_t)i].slot = s.n_slots + i;
+                s.n_slots += n_split;
+                for (int32_t c : ctas) ++pieces_on[(size_t)c];
+            }
         }
-        std::stable_sort(items.begin(), items.end(), [&](const AttnItem& x, const AttnItem& y) {
-            const int64_t cx = x.kv_tile1 - x.kv_tile0, cy = y.kv_tile1 - y.kv_tile0;
-            const bool late_x = cx * 100 <= longest * 55, late_y = cy * 100 <= longest * 55;
+        while (!least.empty()) {
+            const Slot sl = least.top();
+            least.pop();
+            s.span = std::max(s.span, sl.first + kMergeCost * pieces_on[(size_t)sl.second]);
+        }
+        return s;
+    };
+
+    std::vector<int64_t> longest_in_group((size_t)B * d->h_kv, 0), tiles_in_group((size_t)B * d->h_kv, 0);
+    int64_t longest = 0;
+    for (const Tile& t : tiles) {
+        int64_t& lg = longest_in_group[(size_t)t.b * d->h_kv + t.g];
+        lg = std::max<int64_t>(lg, t.n_tiles);
+        tiles_in_group[(size_t)t.b * d->h_kv + t.g] += t.n_tiles;
+        longest = std::max<int64_t>(longest, t.n_tiles);
+    }
+    auto by_group = [&](const std::vector<int64_t>& gc, bool defer_short) {
+        std::vector<Tile> v = tiles;
+        std::stable_sort(v.begin(), v.end(), [&](const Tile& x, const Tile& y) {
+            const int64_t cx = x.n_tiles, cy = y.n_tiles;
+            const bool late_x = defer_short && cx * 100 <= longest * 55, late_y = defer_short && cy * 100 <= longest * 55;
             if (late_x != late_y) return late_y;
             if (!late_x) {
-                const int64_t gx = group_cost[(size_t)x.query * d->h_kv + x.kv_head];
-                const int64_t gy = group_cost[(size_t)y.query * d->h_kv + y.kv_head];
+                const int64_t gx = group_key(gc, x), gy = group_key(gc, y);
                 if (gx != gy) return gx > gy;
             } else if (cx != cy) {
                 return cx > cy;
             }
-            if (x.query != y.query) return x.query < y.query;
-            if (x.kv_head != y.kv_head) return x.kv_head < y.kv_head;
+            if (x.b != y.b) return x.b < y.b;
+            if (x.g != y.g) return x.g < y.g;
             return cx > cy;
         });
+        return v;
     };
-
-    // The persistent attention's schedule: one CTA per SM (fewer with fewer items), each item
-    // handed to the CTA that would be free first (list scheduling on the estimated cost in
-    // half tiles: two per key tile, one for the item's own start and finish, two more for a
-    // piece of a split range, whose partial is stored and merged).  Two hand-out orders are
-    // estimated: the launch order (the items of one (query, KV head) run together and share
-    // their K/V tiles in L2) and longest first over all items; the launch order is kept
-    // unless longest first finishes more than 3% earlier (a few long groups filling the
-    // grid: one long query's last KV head would otherwise start only after a first item
-    // elsewhere).
-    using Slot = std::pair<int64_t, int32_t>;
-    auto cost = [](const AttnItem& it) { return 2 * (int64_t)(it.kv_tile1 - it.kv_tile0) + 1 + (it.slot >= 0 ? 2 : 0); };
-    auto schedule = [&](const std::vector<AttnItem>& items, const std::vector<int32_t>& order, int32_t n_ctas,
-                        std::vector<std::vector<int32_t>>* lists) {
-        std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> free_at;
-        for (int32_t c = 0; c < n_ctas; ++c) free_at.push({0, c});
-        if (lists) lists->assign((size_t)n_ctas, {});
-        int64_t makespan = 0;
-        for (int32_t i : order) {
-            const Slot sl = free_at.top();
-            free_at.pop();
-            if (lists) (*lists)[(size_t)sl.second].push_back(i);
-            makespan = std::max(makespan, sl.first + cost(items[(size_t)i]));
-            free_at.push({sl.first + cost(items[(size_t)i]), sl.second});
-        }
-        return makespan;
-    };
-    // returns the estimated makespan and the better order
-    auto best_order = [&](const std::vector<AttnItem>& items, int32_t n_ctas, std::vector<int32_t>& order) {
-        std::vector<int32_t> launch(items.size()), longest_first;
-        std::iota(launch.begin(), launch.end(), 0);
-        longest_first = launch;
-        std::stable_sort(longest_first.begin(), longest_first.end(),
-                         [&](int32_t a, int32_t b) { return cost(items[(size_t)a]) > cost(items[(size_t)b]); });
-        const int64_t m_launch = schedule(items, launch, n_ctas, nullptr);
-        const int64_t m_longest = schedule(items, longest_first, n_ctas, nullptr);
-        const bool use_longest = m_longest * 103 < m_launch * 100;
-        order = use_longest ? longest_first : launch;
-        return use_longest ? m_longest : m_launch;
-    };
-
-    // Split granularity: pieces of at most W / (k * SMs) key tiles (W the batch's key tiles),
-    // for the k in 1..4 whose estimated time is shortest (a larger k only when it is more
-    // than 2% shorter): with many short items nothing is split; one long query, or a batch
-    // whose longest items would hold the grid up, is split just enough to balance.  The
-    // estimate adds the merge pass, which runs after the attention and reads every partial
-    // (O, m, l: about 130 KB for head_dim 128, written once and read once): at HBM speed
-    // one half tile of attention time moves about 19 partials, plus about 5 half tiles for
-    // the launch.
-    int64_t best_span = INT64_MAX;
-    std::vector<int32_t> best_ord;
-    for (int k = 1; k <= 4; ++k) {
-        const int32_t max_tiles = (int32_t)std::max<int64_t>(8, (work + (int64_t)num_sms * k - 1) / ((int64_t)num_sms * k));
-        std::vector<AttnItem> items;
-        std::vector<MergeGroup> merges;
-        int32_t n_slots = 0;
-        make_items(max_tiles, items, merges, n_slots);
-        const int32_t n_ctas = std::min<int32_t>(num_sms, (int32_t)items.size());
-        std::vector<int32_t> order;
-        const int64_t span = best_order(items, n_ctas, order) + (n_slots > 0 ? 5 + n_slots / 19 : 0);
-        if (k == 1 || span * 100 < best_span * 98) {
-            best_span = span;
-            p->items.swap(items);
-            p->merges.swap(merges);
-            p->n_slots = n_slots;
-            best_ord.swap(order);
-        }
-        if (max_tiles == 8) break;   // finer pieces are not made
-    }
-    p->workspace_bytes = (size_t)p->n_slots * (size_t)kAttnBM * ((size_t)d->head_dim + 2) * sizeof(float);
+    std::vector<Tile> longest_first = tiles;
+    std::stable_sort(longest_first.begin(), longest_first.end(),
+                     [](const Tile& x, const Tile& y) { return x.n_tiles > y.n_tiles; });
+    // holding short M-tiles back pays when the longest M-tile is a large part of a CTA's share
+    // (its tail decides when the grid ends); otherwise the plain group order keeps the
+    // groups' K/V tiles together longer
+    const bool defer_short = 2 * longest * 4 > (total + n_ctas - 1) / n_ctas;
+    Sched a_launch = schedule_whole(defer_short ? by_group(longest_in_group, true) : by_group(tiles_in_group, false));
+    Sched a_longest = schedule_whole(longest_first);
+    Sched best = std::move(a_longest.span * 103 < a_launch.span * 100 ? a_longest : a_launch);
+    // A repaired: while the most loaded CTA ends more than two piece costs after the least
+    // loaded one, its last whole M-tile is cut in two and the second piece moves to the end of
+    // the least loaded CTA (a two-piece merge); only the CTAs that hold the grid up are cut.
     {
-        const int32_t n_ctas = std::min<int32_t>(num_sms, (int32_t)p->items.size());
-        std::vector<std::vector<int32_t>> lists;
-        schedule(p->items, best_ord, n_ctas, &lists);
-        p->sched.clear();
-        p->cu_sched.assign((size_t)n_ctas + 1, 0);
-        for (int32_t c = 0; c < n_ctas; ++c) {
-            p->cu_sched[(size_t)c] = (int32_t)p->sched.size();
-            p->sched.insert(p->sched.end(), lists[(size_t)c].begin(), lists[(size_t)c].end());
+        Sched r = best;
+        std::vector<int64_t> load((size_t)n_ctas, 0);
+        for (int32_t c = 0; c < n_ctas; ++c)
+            for (int32_t i : r.lists[(size_t)c]) load[(size_t)c] += 2 * (int64_t)(r.items[(size_t)i].kv_tile1 - r.items[(size_t)i].kv_tile0) + 1;
+        for (int32_t step = 0; step < n_ctas; ++step) {
+            const int32_t hi = (int32_t)(std::max_element(load.begin(), load.end()) - load.begin());
+            const int32_t lo = (int32_t)(std::min_element(load.begin(), load.end()) - load.begin());
+            const int64_t gap = load[(size_t)hi] - load[(size_t)lo];
+            if (gap <= 4 * kMergeCost || r.lists[(size_t)hi].empty()) break;
+            const int32_t idx = r.lists[(size_t)hi].back();
+            AttnItem& it = r.items[(size_t)idx];
+            if (it.slot >= 0) break;
+            const int32_t n = it.kv_tile1 - it.kv_tile0;
+            // move x tiles so that both ends meet: 2x = (gap - 1) / 2 (each side pays kMergeCost)
+            int32_t x = (int32_t)std::min<int64_t>(n - kMinPiece, (gap - 1) / 4);
+            if (x < kMinPiece) break;
+            AttnItem moved = it;
+            moved.kv_tile0 = it.kv_tile1 - x;
+            it.kv_tile1 = moved.kv_tile0;
+            it.slot = r.n_slots;
+            moved.slot = r.n_slots + 1;
+            r.merges.push_back({it.query, it.kv_head, it.tok0, it.tok1, r.n_slots, 2, 0, 0});
+            r.n_slots += 2;
+            r.lists[(size_t)lo].push_back((int32_t)r.items.size());
+            r.items.push_back(moved);
+            load[(size_t)hi] += -2 * (int64_t)x + kMergeCost;
+            load[(size_t)lo] += 2 * (int64_t)x + 1 + kMergeCost;
         }
-        p->cu_sched[(size_t)n_ctas] = (int32_t)p->sched.size();
+        r.span = *std::max_element(load.begin(), load.end());
+        if (r.span * 100 < best.span * 97) best = std::move(r);
     }
+    for (int slack : {0, 5, 10}) {
+        Sched capped = schedule_capped(by_group(tiles_in_group, false), slack);
+        if (capped.span * 100 < best.span * 97) best = std::move(capped);
+    }
+
+    p->items.swap(best.items);
+    p->merges.swap(best.merges);
+    p->n_slots = best.n_slots;
+    p->sched.clear();
+    p->cu_sched.assign((size_t)n_ctas + 1, 0);
+    for (int32_t c = 0; c < n_ctas; ++c) {
+        p->cu_sched[(size_t)c] = (int32_t)p->sched.size();
+        p->sched.insert(p->sched.end(), best.lists[(size_t)c].begin(), best.lists[(size_t)c].end());
+    }
+    p->cu_sched[(size_t)n_ctas] = (int32_t)p->sched.size();
+    (void)work;
+    p->workspace_bytes = (size_t)p->n_slots * (size_t)kAttnBM * ((size_t)d->head_dim + 2) * sizeof(float);
+    p->slot_group.assign((size_t)p->n_slots, -1);
+    for (size_t g = 0; g < p->merges.size(); ++g)
+        for (int32_t s = 0; s < p->merges[g].n_split; ++s) p->slot_group[(size_t)(p->merges[g].slot0 + s)] = (int32_t)g;
 
     // ---- device buffer layout (256-byte aligned tables)
     size_t off = 0;
@@ -458,6 +523,8 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     p->off_fresh_dst = take(p->fresh_dst.size() * sizeof(int32_t));
     p->off_sched = take(p->sched.size() * sizeof(int32_t));
     p->off_cu_sched = take(p->cu_sched.size() * sizeof(int32_t));
+    p->off_slot_group = take(p->slot_group.size() * sizeof(int32_t));
+    p->off_merge_count = take(p->merges.size() * sizeof(unsigned long long));
     p->device_bytes = off;
     p->uploaded = false;
     return KVLINK_OK;

@@ -360,9 +360,12 @@ __global__ void __launch_bounds__(32 * kHostWarps) reencode_host_kernel(
     const int U = h_kv * PAIRS_PER_HEAD;              // (lo, hi) pairs of 16-byte words per row
     const int row_vec = h_kv * D / 8;                 // 16-byte words per row
     const int lane = threadIdx.x % 32;
-    const int warp = blockIdx.x * kHostWarps + threadIdx.x / 32;
-    const int n_warps = gridDim.x * kHostWarps;
-    for (int c = warp; c < n_chunks; c += n_warps) {
+    // CTA b walks the contiguous range [n*b/grid, n*(b+1)/grid) of the units sorted by source
+    // row, its warps on neighbouring units: the host rows in flight at any time lie in a few
+    // short runs per CTA instead of all over the pool
+    const int c_begin = (int)((int64_t)n_chunks * blockIdx.x / gridDim.x);
+    const int c_end = (int)((int64_t)n_chunks * (blockIdx.x + 1) / gridDim.x);
+    for (int c = c_begin + (int)threadIdx.x / 32; c < c_end; c += kHostWarps) {
         const CopyChunk ch = chunks[c];
 #ifdef KVLINK_DEBUG_CHECKS
         if (ch.n < 1 || ch.dst_row < 0 || ch.dst_row + ch.n > bounds.ctx_rows || ch.src_row < 0 ||
@@ -425,14 +428,15 @@ void launch_reencode_host(const DevicePlan& P, int n_chunks, int head_dim, int h
                           const void* pool_k, const void* pool_v, void* cache_k, void* cache_v, cudaStream_t stream) {
     if (n_chunks <= 0) return;
     const CopyBounds bounds{P.ctx_rows, P.pool_rows, P.n_fresh, P.n_rope_rows};
-    const int grid = std::max(1, std::min((n_chunks + kHostWarps - 1) / kHostWarps, 4 * num_sms));
+    const int grid = std::max(1, std::min((n_chunks + kHostWarps - 1) / kHostWarps, 2 * num_sms));
+    // the cached units sorted by source row (the same set as the plan's cached units)
     if (head_dim == 128)
         reencode_host_kernel<128><<<grid, 32 * kHostWarps, 0, stream>>>(
-            P.chunks, n_chunks, P.rope, h_kv, (const uint4*)pool_k, (const uint4*)pool_v, (uint4*)cache_k,
+            P.chunks_sorted, n_chunks, P.rope, h_kv, (const uint4*)pool_k, (const uint4*)pool_v, (uint4*)cache_k,
             (uint4*)cache_v, bounds);
     else
         reencode_host_kernel<64><<<grid, 32 * kHostWarps, 0, stream>>>(
-            P.chunks, n_chunks, P.rope, h_kv, (const uint4*)pool_k, (const uint4*)pool_v, (uint4*)cache_k,
+            P.chunks_sorted, n_chunks, P.rope, h_kv, (const uint4*)pool_k, (const uint4*)pool_v, (uint4*)cache_k,
             (uint4*)cache_v, bounds);
 }
 

@@ -61,6 +61,22 @@ def test_one_kernel_equals_two_kernel_path_bitwise(RT, cfg_index, layer, layout)
         check_query(batch, b, lp, gk, gv, gout, inp, layout=lo)
 
 
+@pytest.mark.parametrize("layout", sorted(LAYOUTS))
+def test_split_ranges_merge_to_the_same_bits(RT, layout):
+    """A plan whose KV ranges are cut between CTAs: the one-kernel path merges the partials in
+    a separate merge kernel, the persistent suffix attention inside the kernel, with the same
+    arithmetic, so the outputs must be the same bits."""
+    name = "long_single_doc_split_kv"
+    batch = custom_batch(50 + sorted(EDGE).index(name), **EDGE[name])
+    lo = LAYOUTS[layout]
+    lp, gk, gv, gout, inp = run_layer(RT, batch, 0, "onekernel", layout=lo)
+    assert lp.info.n_attn_splits > 0
+    _, rk, rv, rout, _ = run_layer(RT, batch, 0, "fused", layout=lo)
+    assert np.array_equal(gk, rk) and np.array_equal(gv, rv)
+    assert _same_bits(gout, rout), "in-kernel merge differs from the merge kernel"
+    check_query(batch, 0, lp, gk, gv, gout, inp, layout=lo)
+
+
 @pytest.mark.parametrize("name", sorted(EDGE))
 @pytest.mark.parametrize("layout", sorted(LAYOUTS))
 def test_one_kernel_edge_cases(RT, name, layout):

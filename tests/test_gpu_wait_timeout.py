@@ -71,8 +71,9 @@ def test_expired_wait_is_reported_and_later_launches_skip(env):
         torch.cuda.synchronize(dev)
         assert time.perf_counter() - t0 < 0.5
         assert K.kvlink_device_status() == K.KVLINK_STATUS_WAIT_TIMEOUT
-        if lp.info.n_attn_splits == 0:          # no merge kernel: the output was never written
-            assert int(torch.count_nonzero(out.view(torch.int16)).item()) == 0
+        # split ranges are merged inside the attention kernel, which did nothing: the output
+        # was never written
+        assert int(torch.count_nonzero(out.view(torch.int16)).item()) == 0
     finally:
         K.kvlink_clear_device_status()
     assert K.kvlink_device_status() == 0

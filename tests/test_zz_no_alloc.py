@@ -45,8 +45,13 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(env):
     K, RT = env
     from _gpu_common import check_query
 
+    from _gpu_common import EDGE, custom_batch
+
     dev = torch.device("cuda:0")
-    batch = W.draw_batch(W.get_config(2))       # Llama-1B shape: its plan splits KV ranges
+    # one 6000-token document and 50 fresh rows: 16 long M-tiles on 152 SMs, so the plan cuts
+    # their KV ranges between CTAs and the partials go to the scratch
+    name = "long_single_doc_split_kv"
+    batch = custom_batch(50 + sorted(EDGE).index(name), **EDGE[name])
     lp = RT.LinkedPrefill.from_batch(batch, device=dev)
     info = lp.info
     assert info.n_attn_splits > 0, "the plan must use scratch for this test to mean anything"
