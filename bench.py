@@ -210,7 +210,9 @@ class Workload:
             K.kvlink_linked_prefill_layers_overlapped(self.plan, *self.ptrs, self.ws, self.wsb, self.sh, self.re_sh)
 
     def launches_per_step(self):
-        n_merge = 1 if self.info.n_attn_splits > 0 else 0
+        # the persistent attention merges cut KV ranges itself; the one-kernel path needs the
+        # merge kernel after it
+        n_merge = 1 if self.one_kernel and self.info.n_attn_splits > 0 else 0
         per_layer = 1 if self.one_kernel else 2 if self.path == "two-kernel-serial" else 3
         return self.L * (per_layer + n_merge)
 

@@ -42,31 +42,6 @@ constexpr float kRescaleThreshold = 8.0f;         // log2 units: rescale O when 
 
 constexpr uint32_t kTmemCols = 512;
 
-// Shared-memory and TMEM layout of the kernels that stream K and V tiles of a
-// materialised linked cache through two TMA rings (Q, NK K stages, NV V stages).
-template <int D>
-struct TcCfg {
-    static constexpr int ATOMS = D / 64;                 // 128-byte swizzle atoms along head_dim
-    static constexpr int NK = (D == 128) ? 3 : 5;        // K ring stages
-    static constexpr int NV = (D == 128) ? 3 : 5;        // V ring stages
-    static constexpr int NB = 3;                         // S/P buffers in TMEM
-    static constexpr uint32_t ATOM_BYTES = 128 * 128;    // [128 rows][64 bf16]
-    static constexpr uint32_t Q_BYTES = ATOMS * ATOM_BYTES;
-    static constexpr uint32_t KV_BYTES = ATOMS * ATOM_BYTES;
-    static constexpr uint32_t OFF_Q = 0;
-    static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
-    static constexpr uint32_t OFF_V = OFF_K + NK * KV_BYTES;
-    static constexpr uint32_t OFF_BAR = OFF_V + NV * KV_BYTES;
-    // q_full, k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB], p_full[NB], o_done[NB], drain x2
-    static constexpr int N_BARS = 1 + 2 * NK + 2 * NV + 3 * NB + 2;
-    static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
-    // TMEM columns: S/P buffers then the O accumulator
-    static constexpr uint32_t TMEM_S = 0;                // buffer b at b * 128
-    static constexpr uint32_t TMEM_O = NB * kAttnBN;
-    static_assert(TMEM_O + D <= kTmemCols, "TMEM budget");
-    static_assert(SMEM_BYTES <= 232448, "shared memory budget");
-};
-
 // Wait for phase `parity` of `bar`; false if another role aborted or the time limit passed.
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag,
                                          int32_t* status, uint64_t limit_ns = kWaitLimitNs) {
@@ -133,89 +108,6 @@ __device__ __forceinline__ uint64_t exp2_poly2(uint64_t x2) {
     const float ra = __int_as_float(__float_as_int(pa) + (int)((uint32_t)__float_as_int(ta) << 23));
     const float rb = __int_as_float(__float_as_int(pb) + (int)((uint32_t)__float_as_int(tb) << 23));
     return f2_pack(ra, rb);
-}
-
-// TMA producer loop for one ring (K or V) of a materialised linked cache: the n key tiles
-// of the item's list, rows ctx0 + 128 * item_tile(it, kv_tile0 + j) .. of its KV head.
-template <int STAGES, int ATOMS>
-__device__ __forceinline__ void produce_ring(uint8_t* ring, uint32_t stage_bytes, const CUtensorMap* map,
-                                             uint64_t* full, uint64_t* empty, int n, const AttnItem& it,
-                                             int ctx0, volatile int32_t* abort_flag, int32_t* status) {
-    using namespace sm100;
-    int issued = 0;
-    for (int j = 0; j < n; ++j) {
-        const int st = j % STAGES;
-        if (!wait_bar(empty + st, ((j / STAGES) & 1) ^ 1, abort_flag, status)) break;
-        const int row = ctx0 + item_tile(it, it.kv_tile0 + j) * kAttnBN;
-        mbar_arrive_expect_tx(full + st, stage_bytes);
-#pragma unroll
-        for (int a = 0; a < ATOMS; ++a)
-            tma_load_3d(ring + st * stage_bytes + a * (128 * 128), map, a * 64, it.kv_head, row, full + st);
-        issued = j + 1;
-    }
-    // no copy may still be in flight when the CTA leaves
-    for (int j = issued - STAGES > 0 ? issued - STAGES : 0; j < issued; ++j)
-        drain_bar(full + j % STAGES, (j / STAGES) & 1, status);
-}
-
-// Two MMA-issuing threads, one for S_j = Q K_j^T and one for O += P_i V_i.  A thread that
-// waits on an mbarrier right after its own tcgen05.commit was seen to stall until its MMAs
-// had drained (~400 cycles per tile with one issuer doing both); with two issuers each
-// waits only on its own work while the other keeps the tensor pipe fed.  S_j goes into S
-// buffer j % NB once PV_{j-NB} has read that buffer; PV_i reads P_i from TMEM and V_i
-// MN-major from shared memory.
-template <int D, int NK, int NB>
-__device__ __forceinline__ void mma_s_role(uint8_t* smem, uint32_t off_q, uint32_t off_k, uint32_t kv_bytes,
-                                           uint32_t atom_bytes, uint32_t tmem_s, int n_tiles, uint64_t* bar_q_full,
-                                           uint64_t* bar_k_full, uint64_t* bar_k_empty, uint64_t* bar_s_full,
-                                           uint64_t* bar_o_done, uint64_t* bar_drain, volatile int32_t* abort_flag,
-                                           int32_t* status) {
-    using namespace sm100;
-    constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kAttnBN, 0, 0);
-    const uint32_t sQ = smem_u32(smem + off_q);
-    bool ok = wait_bar(bar_q_full, 0, abort_flag, status);
-    for (int j = 0; ok && j < n_tiles; ++j) {
-        const int sk = j % NK, b = j % NB;
-        if (!(ok = wait_bar(bar_k_full + sk, (j / NK) & 1, abort_flag, status))) break;
-        if (j >= NB && !(ok = wait_bar(bar_o_done + b, ((j - NB) / NB) & 1, abort_flag, status))) break;
-        tc_fence_after();
-        const uint32_t sK = smem_u32(smem + off_k + sk * kv_bytes);
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t koff = (kk >> 2) * atom_bytes + (kk & 3) * 32;
-            mma_bf16_ss(tmem_s + b * kAttnBN, sdesc_sw128(sQ + koff, 16, 1024), sdesc_sw128(sK + koff, 16, 1024),
-                        idesc_qk, kk > 0 ? 1u : 0u);
-        }
-        mma_commit(bar_s_full + b);
-        mma_commit(bar_k_empty + sk);
-    }
-    mma_commit(bar_drain);
-    drain_bar(bar_drain, 0, status);
-}
-
-template <int D, int NV, int NB>
-__device__ __forceinline__ void mma_pv_role(uint8_t* smem, uint32_t off_v, uint32_t kv_bytes, uint32_t atom_bytes,
-                                            uint32_t tmem_s, uint32_t tmem_o, int n_tiles, uint64_t* bar_v_full,
-                                            uint64_t* bar_v_empty, uint64_t* bar_p_full, uint64_t* bar_o_done,
-                                            uint64_t* bar_drain, volatile int32_t* abort_flag, int32_t* status) {
-    using namespace sm100;
-    constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, 0, 1);
-    for (int i = 0; i < n_tiles; ++i) {
-        const int b = i % NB, sv = i % NV;
-        if (!wait_bar(bar_p_full + b, (i / NB) & 1, abort_flag, status)) break;
-        if (!wait_bar(bar_v_full + sv, (i / NV) & 1, abort_flag, status)) break;
-        tc_fence_after();
-        const uint32_t sV = smem_u32(smem + off_v + sv * kv_bytes);
-        const uint32_t pcol = tmem_s + b * kAttnBN;
-#pragma unroll
-        for (int kk = 0; kk < kAttnBN / 16; ++kk)
-            mma_bf16_ts(tmem_o, pcol + kk * 8, sdesc_sw128(sV + kk * 16 * 128, atom_bytes, 1024), idesc_pv,
-                        (i > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(bar_o_done + b);
-        mma_commit(bar_v_empty + sv);
-    }
-    mma_commit(bar_drain);
-    drain_bar(bar_drain, 0, status);
 }
 
 // Softmax over the key tiles of one item, run by warps 0-3 (threadIdx.x = tile row).  TMEM

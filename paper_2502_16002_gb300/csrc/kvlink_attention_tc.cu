@@ -1,34 +1,29 @@
 // Suffix attention on the tcgen05 tensor cores (Sec. 2.3, "inference").
 //
-// Work item = one M-tile of up to 128 rows (up to 128/G fresh tokens x the G
-// query heads that share one KV head) of one query, over a range of 128-key
-// tiles of that query's linked cache (cache-row order; in the links-at-end layout the
-// cached rows and the fresh rows at the end form two runs).  Rows are (token, head)
-// pairs, so the G heads of a GQA group share every K/V tile load.
+// Work item = one M-tile of up to 128 rows (up to 128/G fresh tokens x the G query heads
+// that share one KV head) of one query, over a range of 128-key tiles of that query's linked
+// cache (cache-row order; in the links-at-end layout the cached rows and the fresh rows at
+// the end form two runs).  Rows are (token, head) pairs, so the G heads of a GQA group share
+// every K/V tile load.  The kernel is persistent: one CTA per SM runs the list of items the
+// plan gave it (see the comment before PtCfg for the warp roles).
 //
-// Warp roles (256 threads, one CTA per SM, 512 TMEM columns):
-//   warps 0-3  softmax + epilogue; thread r owns row r = TMEM lane r
-//   warp 4     TMA: Q once, then K tiles into an NK-stage ring
-//   warp 5     TMEM allocation and the thread issuing the S = Q K^T MMAs
-//   warp 6     TMA: V tiles into an NV-stage ring
-//   warp 7     the thread issuing the O += P V MMAs
 // Per KV tile j (TMEM: three S/P buffers of 128 columns, then O):
 //   S_j = Q K_j^T           tcgen05.mma SMEM x SMEM -> S buffer j%3
 //   P_j = exp2(S_j c - m)   softmax warps: TMEM -> registers -> bf16 P written back
 //                           over the first 64 columns of the same buffer
 //   O  += P_j V_j           tcgen05.mma TMEM x SMEM (P from TMEM, V read MN-major)
-// S_j is issued only after PV_{j-3} has finished reading the buffer, so up to
-// three tiles are in flight and the softmax never waits on a PV except to
-// rescale O.  S and PV come from two issuing threads (see mma_s_role).  The running max m is raised only when it grows by more than 2^8,
-// so that rescale is rare.  The mask keeps the cache rows holding positions up to
-// the row's own (a threshold pair per row, see softmax_role) and is evaluated only on
-// tiles that reach past the rows every row of the tile sees.  Items whose KV range was split write
-// unnormalised partials (O, m, l) to the workspace; attn_merge_kernel combines them.
+// S_j is issued only after PV_{j-3} has finished reading the buffer, so up to three tiles
+// are in flight and the softmax never waits on a PV except to rescale O.  S and PV come from
+// two issuing threads: a thread that waits on an mbarrier right after its own tcgen05.commit
+// was seen to stall until its MMAs had drained.  The running max m is raised only when it
+// grows by more than 2^8, so the rescale is rare.  The mask keeps the cache rows holding
+// positions up to the row's own and is evaluated only on tiles that reach past the rows every
+// row of the tile sees.
 //
 // Every mbarrier wait is bounded in time.  On expiry the kernel records
-// kAttnStatusWaitTimeout in its status word, the other roles leave their loops,
-// the producer and MMA threads wait (bounded) for their own in-flight copies and
-// MMAs, TMEM is freed and the CTA returns.
+// kAttnStatusWaitTimeout in its status word, the other roles leave their loops, the producer
+// and MMA threads wait (bounded) for their own in-flight copies and MMAs, TMEM is freed and
+// the CTA returns.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -43,115 +38,12 @@ using namespace sm100;
 
 static __device__ int32_t g_attn_status;
 
-constexpr int kTcThreads = 256;
 constexpr int kPvWarp = 7;
 constexpr int kSoftmaxWarps = 4;
 constexpr int kTmaKWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kTmaVWarp = 6;
 
-
-template <int D, int G>
-__global__ void __launch_bounds__(kTcThreads, 1)
-    attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                   const __grid_constant__ CUtensorMap tm_v, DevicePlan P, __nv_bfloat16* __restrict__ out,
-                   float* __restrict__ ws, int h_q, float scale_log2) {
-    using C = TcCfg<D>;
-    constexpr int NK = C::NK, NV = C::NV, NB = C::NB;
-    extern __shared__ uint8_t smem_raw[];
-    const uint32_t raw_addr = smem_u32(smem_raw);
-    uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
-
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
-    uint64_t* bar_q_full = bars;
-    uint64_t* bar_k_full = bar_q_full + 1;
-    uint64_t* bar_k_empty = bar_k_full + NK;
-    uint64_t* bar_v_full = bar_k_empty + NK;
-    uint64_t* bar_v_empty = bar_v_full + NV;
-    uint64_t* bar_s_full = bar_v_empty + NV;
-    uint64_t* bar_p_full = bar_s_full + NB;
-    uint64_t* bar_o_done = bar_p_full + NB;
-    uint64_t* bar_drain = bar_o_done + NB;
-    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + C::N_BARS);
-    volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(tmem_holder + 1);
-
-    const AttnItem it = P.items[blockIdx.x];
-    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int n_tiles = it.kv_tile1 - it.kv_tile0;
-
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < C::N_BARS; ++i) {
-            const bool p_full = bars + i >= bar_p_full && bars + i < bar_p_full + NB;
-            mbar_init(bars + i, p_full ? kSoftmaxWarps : 1);
-        }
-        // after a recorded failure, later launches skip their work instead of waiting out their bounds
-        *abort_flag = *reinterpret_cast<volatile int32_t*>(&g_attn_status) != 0 ? 1 : 0;
-#ifdef KVLINK_DEBUG_CHECKS
-        if (!*abort_flag && !item_in_bounds(it, P)) {
-            atomicCAS(&g_attn_status, 0, kAttnStatusBadIndex);
-            *abort_flag = 1;
-        }
-#endif
-        fence_mbar_init();
-    }
-    if (warp == kMmaWarp) {
-        tmem_alloc(tmem_holder, kTmemCols);
-        tmem_relinquish();
-    }
-    if (warp == kTmaKWarp && lane == 0) {
-        prefetch_tensormap(&tm_q);
-        prefetch_tensormap(&tm_k);
-        prefetch_tensormap(&tm_v);
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *tmem_holder;
-    const bool skip = *abort_flag != 0;  // written before the barrier: uniform across the CTA
-    const int ctx0 = skip ? 0 : (int)P.cu_ctx[it.query];
-
-    if (skip) {
-        // nothing issued: fall through to the teardown
-    } else if (warp == kTmaKWarp) {
-        // ------------------------------------------------------------ Q, then the K ring
-        if (lane == 0) {
-            const int q_row0 = P.cu_fresh[it.query] + it.tok0;
-            mbar_arrive_expect_tx(bar_q_full, C::Q_BYTES);
-#pragma unroll
-            for (int a = 0; a < C::ATOMS; ++a)
-                tma_load_3d(smem + C::OFF_Q + a * C::ATOM_BYTES, &tm_q, a * 64, it.kv_head * G, q_row0, bar_q_full);
-            produce_ring<NK, C::ATOMS>(smem + C::OFF_K, C::KV_BYTES, &tm_k, bar_k_full, bar_k_empty, n_tiles, it,
-                                       ctx0, abort_flag, &g_attn_status);
-            drain_bar(bar_q_full, 0, &g_attn_status);
-        }
-    } else if (warp == kTmaVWarp) {
-        // ------------------------------------------------------------ the V ring
-        if (lane == 0)
-            produce_ring<NV, C::ATOMS>(smem + C::OFF_V, C::KV_BYTES, &tm_v, bar_v_full, bar_v_empty, n_tiles, it,
-                                       ctx0, abort_flag, &g_attn_status);
-    } else if (warp == kMmaWarp) {
-        if (lane == 0)
-            mma_s_role<D, NK, NB>(smem, C::OFF_Q, C::OFF_K, C::KV_BYTES, C::ATOM_BYTES, tmem + C::TMEM_S, n_tiles,
-                                  bar_q_full, bar_k_full, bar_k_empty, bar_s_full, bar_o_done, bar_drain, abort_flag,
-                                  &g_attn_status);
-    } else if (warp == kPvWarp) {
-        if (lane == 0)
-            mma_pv_role<D, NV, NB>(smem, C::OFF_V, C::KV_BYTES, C::ATOM_BYTES, tmem + C::TMEM_S, tmem + C::TMEM_O,
-                                   n_tiles, bar_v_full, bar_v_empty, bar_p_full, bar_o_done, bar_drain + 1,
-                                   abort_flag, &g_attn_status);
-    } else {
-        // ------------------------------------------------------------ softmax + epilogue (warps 0-3)
-        softmax_role<D, G, NB>(it, P, tmem + C::TMEM_S, tmem + C::TMEM_O, n_tiles, bar_s_full, bar_p_full,
-                               bar_o_done, abort_flag, &g_attn_status, out, ws, h_q, scale_log2);
-    }
-
-    tc_fence_before();
-    __syncthreads();
-    if (warp == kMmaWarp) {
-        tc_fence_after();
-        tmem_dealloc(tmem, kTmemCols);
-    }
-}
 
 // ------------------------------------------------------------------------------------------
 // Persistent form: one CTA per SM runs its list of items (the plan's per-CTA schedule) back to
@@ -180,8 +72,8 @@ static_assert(kPtThreads * 168 <= 65536, "launch register budget");
 static_assert(128 * (kPtSoftmaxRegs + kPtIdleRegs + 168) <= kPtThreads * 168, "register split");
 
 // Shared memory: two Q buffers (the next item's Q lands while the current item runs), the K
-// ring and the V ring (one stage fewer than the one-item kernel's for head_dim 128: a V tile
-// is needed a softmax later than its K tile), m and l of one item, a flag, the barriers.
+// ring and the V ring (one stage shorter than the K ring for head_dim 128: a V tile is needed
+// a softmax later than its K tile), m and l of one item, a flag, the barriers.
 template <int D>
 struct PtCfg {
     static constexpr int ATOMS = D / 64;
@@ -536,29 +428,18 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uin
 
 template <int D, int G>
 static cudaError_t launch_tc_dg(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv,
-                                const DevicePlan& P, int n_items, int n_ctas, int n_merges, void* out, float* ws,
-                                int h_q, float scale_log2, cudaStream_t stream) {
+                                const DevicePlan& P, int n_ctas, void* out, float* ws, int h_q, float scale_log2,
+                                cudaStream_t stream) {
     static std::atomic<uint64_t> attr_set{0};
     cudaError_t ea = once_per_device(attr_set, [] {
-        cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)TcCfg<D>::SMEM_BYTES);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(attn_tc_persistent_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)PtCfg<D>::SMEM_BYTES);
-        return e;
+        return cudaFuncSetAttribute(attn_tc_persistent_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)PtCfg<D>::SMEM_BYTES);
     });
     if (ea != cudaSuccess) return ea;
-    if (n_items > 0 && n_ctas > 0) {       // split ranges are merged inside the kernel
+    // cut ranges are merged inside the kernel: nothing follows it
+    if (n_ctas > 0)
         attn_tc_persistent_kernel<D, G><<<n_ctas, kPtThreads, PtCfg<D>::SMEM_BYTES, stream>>>(
             mq, mk, mv, P, (__nv_bfloat16*)out, ws, h_q, scale_log2);
-        return cudaGetLastError();
-    }
-    if (n_items > 0)
-        attn_tc_kernel<D, G><<<n_items, kTcThreads, TcCfg<D>::SMEM_BYTES, stream>>>(
-            mq, mk, mv, P, (__nv_bfloat16*)out, ws, h_q, scale_log2);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    if (n_merges > 0) attn_merge_kernel<D><<<n_merges, 256, 0, stream>>>(P, ws, (__nv_bfloat16*)out, h_q, G);
     return cudaGetLastError();
 }
 
@@ -574,7 +455,7 @@ cudaError_t launch_attn_merge(const DevicePlan& P, int n_merges, const float* ws
 }
 
 // Returns 0, or KVLINK_ECUDA / KVLINK_EUNSUPPORTED.
-// n_ctas > 0: the persistent kernel over the plan's per-CTA schedule; 0: one CTA per item.
+// The persistent kernel over the plan's per-CTA schedule (n_ctas CTAs).
 int launch_attention_tc(const DevicePlan& P, int n_items, int n_ctas, int n_merges, int n_fresh, int64_t ctx_rows,
                         int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err) {
@@ -589,8 +470,7 @@ int launch_attention_tc(const DevicePlan& P, int n_items, int n_ctas, int n_merg
     float* w = (float*)ws;
     cudaError_t e = cudaErrorInvalidValue;
 #define KVLINK_TC_CASE(DD, GG)                                                                         \
-    if (head_dim == DD && G == GG) e = launch_tc_dg<DD, GG>(mq, mk, mv, P, n_items, n_ctas, n_merges, out, w, h_q, \
-                                                            sl2, stream);
+    if (head_dim == DD && G == GG) e = launch_tc_dg<DD, GG>(mq, mk, mv, P, n_ctas, out, w, h_q, sl2, stream);
     KVLINK_TC_CASE(128, 1) KVLINK_TC_CASE(128, 2) KVLINK_TC_CASE(128, 4) KVLINK_TC_CASE(128, 8)
     KVLINK_TC_CASE(128, 16) KVLINK_TC_CASE(64, 1) KVLINK_TC_CASE(64, 2) KVLINK_TC_CASE(64, 4)
     KVLINK_TC_CASE(64, 8) KVLINK_TC_CASE(64, 16)
