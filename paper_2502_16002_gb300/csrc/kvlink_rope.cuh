@@ -7,8 +7,10 @@
 // then be off by many bf16 ulps.  The delta table therefore holds cos and sin as
 // unevaluated float pairs hi + lo (about 48 significant bits, split from the
 // fp64 values) and the products are formed with their exact FMA rounding
-// errors, so the fp32 result carries an absolute error near 2^-47 |x| and rounds
-// to within one bf16 ulp of the correctly rounded fp64 rotation.
+// errors (the error-free TwoProduct transformation of Dekker, in its FMA form as
+// used by Ogita, Rump and Oishi for compensated dot products), so the fp32 result
+// carries an absolute error near 2^-47 |x| and rounds to within one bf16 ulp of
+// the correctly rounded fp64 rotation.
 #pragma once
 
 #include <cuda_bf16.h>
