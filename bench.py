@@ -364,6 +364,56 @@ class Workload:
                 "note": "every layer's document pool in pinned host memory, read over NVLink-C2C by the "
                         "re-encode (kvlink_linked_prefill_layers_host_pool); fresh rows resident in HBM"}
 
+    def zero_copy_leg(self, args, world, local_rank):
+        """The same step with zero-copy values (cache_v NULL): the re-encode writes keys only and
+        the attention reads every value row where it is (pool rows, v_new); and the two kernels
+        of one layer timed alone, launch by launch."""
+        import torch
+        K, sh = self.K, self.sh
+        ptrs = list(self.ptrs)
+        ptrs[6] = None
+
+        def step():
+            K.kvlink_linked_prefill_layers_overlapped(self.plan, *ptrs, self.ws, self.wsb, sh, self.re_sh)
+
+        for _ in range(args.warmup):
+            step()
+        torch.cuda.synchronize(self.dev)
+        ms, clocks = self.timed_steps(args.steps, world, args.clock_ms, local_rank, step)
+        n = min(args.steps, 20) * self.L
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n)]
+        torch.cuda.synchronize(self.dev)
+        for j, (a, b_, c) in enumerate(ev):
+            l = j % self.L
+            a.record(self.stream)
+            K.kvlink_reencode_concat(self.plan, self.pool_k[l].data_ptr(), None, self.ck[l].data_ptr(), None, sh)
+            b_.record(self.stream)
+            K.kvlink_suffix_attention_pool_values(self.plan, self.q[l].data_ptr(), None, self.vn[l].data_ptr(),
+                                                  self.pool_v[l].data_ptr(), self.ck[l].data_ptr(),
+                                                  self.out[l].data_ptr(), self.ws, self.wsb, sh)
+            c.record(self.stream)
+        torch.cuda.synchronize(self.dev)
+        assert K.kvlink_device_status() == 0
+        t_re = float(np.mean([a.elapsed_time(b_) for a, b_, _ in ev])) * 1e-3
+        t_at = float(np.mean([b_.elapsed_time(c) for _, b_, c in ev])) * 1e-3
+        cnt = algorithmic_counts(self.batch, self.info)
+        peaks = _peaks()
+        re_bytes = cnt["reencode_bytes"] // 2          # keys only: half of the K+V figure
+        at_tfs = cnt["attn_flops"] / t_at / 1e12
+        return {"value": round(whole_job_us_per_query(ms, self.cfg.batch, world), 3), "unit": UNIT,
+                "ms_per_step": round(ms, 4), "steps": args.steps, "clocks": clocks,
+                "reencode_keys_us_per_launch": round(t_re * 1e6, 2),
+                "reencode_keys_GB_per_s": round(re_bytes / t_re / 1e9, 1),
+                "reencode_keys_frac_hbm": round(re_bytes / t_re / 1e9 / peaks["hbm_gbs"], 4),
+                "reencode_keys_algorithmic_bytes": int(re_bytes),
+                "attention_pool_values_us_per_launch": round(t_at * 1e6, 2),
+                "attention_pool_values_TFLOP_per_s": round(at_tfs, 2),
+                "attention_pool_values_frac_bf16_burst": round(at_tfs / peaks["bf16_tflops"], 4),
+                "launches_per_step": 3 * self.L,
+                "note": "kvlink_linked_prefill_layers_overlapped with cache_v NULL: keys re-encoded into "
+                        "the linked cache, values read by the attention from the pool and v_new (no "
+                        "value copy); the line's value keeps the linked value cache"}
+
     def config(self, world):
         cfg, info = self.cfg, self.info
         return {"workload": cfg.name, "index": cfg.index, "batch_per_gpu": cfg.batch, "layers": self.L,
@@ -462,6 +512,10 @@ def run_ours(args, rank, world, local_rank, cfg_index, main=True):
     t_re, t_at, t_re_all = wl.kernel_pass(min(args.steps, 20) if main else min(args.steps, 5))
     roof, kernels = wl.roofline(t_re, t_at, t_re_all, _peaks())
 
+    zero_copy = None
+    if not args.no_zero_copy and not wl.one_kernel and args.layout == "interleaved":
+        zero_copy = wl.zero_copy_leg(args, world, local_rank)
+
     e2e = host_pool = None
     if main and not args.no_e2e and not wl.one_kernel and args.layout == "interleaved":
         e2e = run_e2e(wl, args, world)
@@ -479,6 +533,7 @@ def run_ours(args, rank, world, local_rank, cfg_index, main=True):
         "per_rank_us_per_query": round(ms_per_step * 1e3 / wl.cfg.batch, 3),
         "gpu_launches": int(args.steps * wl.launches_per_step()),
         "clocks": clocks,
+        "zero_copy_values": zero_copy,
     }
     if main:
         res["sustained"] = sustained
@@ -568,6 +623,8 @@ def main():
     ap.add_argument("--clock-ms", type=int, default=50, help="nvidia-smi sampling interval")
     ap.add_argument("--no-host-pool", action="store_true",
                     help="skip the leg with the document pool in pinned host memory")
+    ap.add_argument("--no-zero-copy", action="store_true",
+                    help="skip the leg with zero-copy values (cache_v NULL)")
     ap.add_argument("--no-sustained", action="store_true",
                     help="skip the run of at least a second that gives the clock record many samples")
     args = ap.parse_args()

@@ -224,6 +224,9 @@ int kvlink_plan_upload(kvlink_plan_t* plan, double theta, void* d_buf, size_t by
  * The pool entries, their global offsets (pos) and theta come from the plan.
  * d_pool_k/d_pool_v: one layer of the pool (contiguous or paged as described);
  * d_cache_k/d_cache_v: one layer of the linked cache, [ctx_rows][h_kv][D].
+ * d_cache_v may be NULL (zero-copy values): only the keys are re-encoded and written, and
+ * d_pool_v is not read (may be NULL); the attention then reads the values where they are
+ * (kvlink_suffix_attention_pool_values).
  * Fresh (link/question) slots are left untouched.  Errors: EINVAL, ECUDA. */
 int kvlink_reencode_concat(const kvlink_plan_t* plan, const void* d_pool_k, const void* d_pool_v,
                            void* d_cache_k, void* d_cache_v, kvlink_stream_t stream);
@@ -251,6 +254,25 @@ int kvlink_suffix_attention(const kvlink_plan_t* plan, const void* d_q, const vo
                             const void* d_v_new, void* d_cache_k, void* d_cache_v, void* d_out,
                             void* d_workspace, size_t workspace_bytes, kvlink_stream_t stream);
 
+/* kvlink_suffix_attention with zero-copy values (Sec. 2.3, "inference": the cached values
+ * are concatenated unchanged, so they need not be copied): the same keys, mask and output,
+ * with every value row read where it already is instead of from a linked cache:
+ *   value of cache row j = pool_v[src(j)] for a prefix or document position,
+ *                          v_new[src(j)]  for a fresh (link or question) row,
+ * src the plan's source table (kvlink_plan_get_sources: kind KVLINK_SRC_POOL or
+ * KVLINK_SRC_FRESH, row).  Runs of 8 cache rows whose sources are 8 consecutive rows of one
+ * tensor are read as 8-row TMA boxes, the other rows one by one.
+ * d_q, d_k_new, d_out: as for kvlink_suffix_attention; d_k_new may be NULL when the fresh keys
+ * are already in d_cache_k (only keys are placed; d_cache_k holds keys only).
+ * d_v_new: [n_fresh][h_kv][D], required.  d_pool_v: one layer of the pool's values (the
+ * tensor kvlink_reencode_concat reads, contiguous or paged), required.
+ * The output equals kvlink_suffix_attention's bit for bit on the same keys and values (same
+ * tiles, same order of operations).  Errors: EINVAL, ECAPACITY, EUNSUPPORTED, ECUDA. */
+int kvlink_suffix_attention_pool_values(const kvlink_plan_t* plan, const void* d_q, const void* d_k_new,
+                                        const void* d_v_new, const void* d_pool_v, void* d_cache_k,
+                                        void* d_out, void* d_workspace, size_t workspace_bytes,
+                                        kvlink_stream_t stream);
+
 /* The same computation as kvlink_suffix_attention on the CUDA cores: one CTA per
  * (fresh row, KV head) streams the row's visible keys with an online softmax in
  * fp32; no tensor cores, no workspace.  A second, independent GPU implementation
@@ -273,7 +295,9 @@ int kvlink_rope_fresh(const kvlink_plan_t* plan, void* d_q, void* d_k_new, kvlin
 
 /* One layer of the linked prefill: kvlink_reencode_concat with the fresh-row
  * placement fused into the same launch, then the suffix attention.  Same arguments
- * and errors as the two calls it chains. */
+ * and errors as the two calls it chains.  d_cache_v NULL selects zero-copy values: the
+ * re-encode writes keys only and the attention is kvlink_suffix_attention_pool_values
+ * (same output bits). */
 int kvlink_linked_prefill(const kvlink_plan_t* plan, const void* d_pool_k, const void* d_pool_v,
                           const void* d_q, const void* d_k_new, const void* d_v_new,
                           void* d_cache_k, void* d_cache_v, void* d_out,
@@ -301,7 +325,8 @@ int kvlink_linked_prefill_fused(const kvlink_plan_t* plan, const void* d_pool_k,
 
 /* Re-encode + concat (Sec. 2.2, Sec. 2.1) of the document caches of n_layers layers in
  * one launch: the same result as kvlink_reencode_concat(plan, pool_k[l], pool_v[l],
- * cache_k[l], cache_v[l]) for every layer l, bit for bit.  The precomputed document
+ * cache_k[l], cache_v[l]) for every layer l, bit for bit (d_cache_v itself NULL: keys only
+ * in every layer, d_pool_v not read).  The precomputed document
  * caches do not depend on the forward pass of the fresh rows, so a prefill can rotate
  * every layer's caches before its first layer runs, in one launch instead of one per
  * layer (the fresh rows are then placed per layer by kvlink_suffix_attention with
@@ -317,7 +342,7 @@ int kvlink_reencode_concat_layers(const kvlink_plan_t* plan, int32_t n_layers, c
  * one call, with the same results, bit for bit, as kvlink_linked_prefill(plan,
  * pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l], out[l], ...)
  * for every layer l in order, which is what it enqueues.  Each argument is a HOST array
- * of n_layers device pointers.  One workspace serves all layers (they run in stream
+ * of n_layers device pointers; d_cache_v itself may be NULL (zero-copy values in every layer).  One workspace serves all layers (they run in stream
  * order).  Every pointer is checked before the first launch.  Errors: as
  * kvlink_linked_prefill. */
 int kvlink_linked_prefill_layers(const kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
@@ -334,7 +359,8 @@ int kvlink_linked_prefill_layers(const kvlink_plan_t* plan, int32_t n_layers, co
  * re-encode of later layers fills the SMs that the attention of earlier layers leaves
  * idle (the ends of its grid, the gaps between launches).  When the call returns,
  * `stream` is ordered after all of its work.  The plan keeps the events it uses: calls
- * with one plan must not run concurrently.  Errors: as kvlink_linked_prefill_layers;
+ * with one plan must not run concurrently.  d_cache_v NULL: zero-copy values in every layer,
+ * as for kvlink_linked_prefill_layers.  Errors: as kvlink_linked_prefill_layers;
  * EINVAL also when the two streams are the same. */
 int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
                                             const void* const* d_pool_v, const void* const* d_q,
@@ -365,7 +391,8 @@ int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* plan, int32_t n_layer
  * output copy).  The chain links calls
  * of this function only: other work that touches the same buffers in between (another
  * entry point, the caller's kernels) must be ordered by the caller, e.g. by making
- * copy_in_stream wait for it.  The four streams must be distinct.  Errors: as
+ * copy_in_stream wait for it.  The four streams must be distinct.  d_cache_v NULL: zero-copy
+ * values in every layer, as for kvlink_linked_prefill_layers.  Errors: as
  * kvlink_linked_prefill_layers; EINVAL also for a NULL host pointer or repeated
  * streams. */
 int kvlink_linked_prefill_layers_host(kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
@@ -399,8 +426,10 @@ int kvlink_reencode_concat_host_pool(const kvlink_plan_t* plan, const void* h_po
  * n_layers page-locked host pointers; the other arrays as for
  * kvlink_linked_prefill_layers_overlapped.  When the call returns, `stream` is ordered after
  * all of its work.  The plan keeps the events it uses: calls with one plan must not run
- * concurrently.  Errors: as kvlink_linked_prefill_layers_overlapped; EINVAL also for a pool
- * pointer that is not page-locked host memory, or when the two streams are the same. */
+ * concurrently.  The values are loaded into d_cache_v (required here: a host pool's values
+ * are not read by the attention in place).  Errors: as
+ * kvlink_linked_prefill_layers_overlapped; EINVAL also for a pool pointer that is not
+ * page-locked host memory, or when the two streams are the same. */
 int kvlink_linked_prefill_layers_host_pool(kvlink_plan_t* plan, int32_t n_layers, const void* const* h_pool_k,
                                            const void* const* h_pool_v, const void* const* d_q,
                                            const void* const* d_k_new, const void* const* d_v_new,

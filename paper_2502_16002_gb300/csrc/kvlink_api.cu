@@ -31,7 +31,7 @@ void launch_attention_simt(const DevicePlan& P, int n_fresh, int head_dim, int h
                            const void* q, const void* cache_k, const void* cache_v, void* out,
                            cudaStream_t stream);
 int launch_attention_tc(const DevicePlan& P, int n_items, int n_ctas, int n_merges, int n_fresh, int64_t ctx_rows,
-                        int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
+                        int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const ValueSource& vs,
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err);
 int read_attention_status(int32_t* status);
 int clear_attention_status();
@@ -351,8 +351,9 @@ int kvlink_reencode_concat(const kvlink_plan_t* p, const void* pool_k, const voi
                            void* cache_k, void* cache_v, kvlink_stream_t stream) {
     int rc = check_plan(p);
     if (rc) return rc;
-    if (!pool_k || !pool_v || !cache_k || !cache_v) return KVLINK_EINVAL;
-    if (!aligned16(pool_k) || !aligned16(pool_v) || !aligned16(cache_k) || !aligned16(cache_v))
+    // cache_v NULL: keys only (zero-copy values); pool_v is then not read
+    if (!pool_k || !cache_k || (cache_v && !pool_v)) return KVLINK_EINVAL;
+    if (!aligned16(pool_k) || !aligned16(cache_k) || (cache_v && (!aligned16(pool_v) || !aligned16(cache_v))))
         return KVLINK_EINVAL;
     launch_reencode(p->dev, 0, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, pool_k, pool_v, nullptr,
                     nullptr, cache_k, cache_v, (cudaStream_t)stream);
@@ -370,10 +371,19 @@ int kvlink_reencode_concat_layers(const kvlink_plan_t* p, int32_t n_layers, cons
                                   kvlink_stream_t stream) {
     int rc = check_plan(p);
     if (rc) return rc;
-    if (n_layers <= 0 || !pool_k || !pool_v || !cache_k || !cache_v) return KVLINK_EINVAL;
-    if (!all_aligned(n_layers, pool_k) || !all_aligned(n_layers, pool_v) ||
-        !all_aligned(n_layers, (const void* const*)cache_k) || !all_aligned(n_layers, (const void* const*)cache_v))
+    // cache_v NULL: keys only for every layer (zero-copy values); pool_v is then not read
+    if (n_layers <= 0 || !pool_k || !cache_k || (cache_v && !pool_v)) return KVLINK_EINVAL;
+    if (!all_aligned(n_layers, pool_k) || !all_aligned(n_layers, (const void* const*)cache_k) ||
+        (cache_v && (!all_aligned(n_layers, pool_v) || !all_aligned(n_layers, (const void* const*)cache_v))))
         return KVLINK_EINVAL;
+    std::vector<const void*> no_pool_v;
+    std::vector<void*> no_cache_v;
+    if (!cache_v) {
+        no_pool_v.assign((size_t)n_layers, nullptr);
+        no_cache_v.assign((size_t)n_layers, nullptr);
+        pool_v = no_pool_v.data();
+        cache_v = no_cache_v.data();
+    }
     launch_reencode_layers(p->dev, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, n_layers, pool_k, pool_v,
                            cache_k, cache_v, (cudaStream_t)stream);
     return check_launch("reencode_kernel (layers)");
@@ -386,20 +396,28 @@ static int place_fresh(const kvlink_plan_t* p, const void* k_new, const void* v_
     return check_launch("place_fresh_kernel");
 }
 
-static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k, void* cache_v,
+// vs.cache_v NULL: zero-copy values, read from vs.pool_v and vs.v_new
+static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k, const ValueSource& vs,
                             void* out, void* ws, size_t ws_bytes, cudaStream_t s) {
-    if (!q || !cache_k || !cache_v || !out) return KVLINK_EINVAL;
-    if (!aligned16(q) || !aligned16(cache_k) || !aligned16(cache_v) || !aligned16(out))
+    if (!q || !cache_k || !out) return KVLINK_EINVAL;
+    if (!aligned16(q) || !aligned16(cache_k) || !aligned16(out)) return KVLINK_EINVAL;
+    if (vs.cache_v ? !aligned16(vs.cache_v)
+                   : (!vs.pool_v || !vs.v_new || !aligned16(vs.pool_v) || !aligned16(vs.v_new)))
         return KVLINK_EINVAL;
     if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
     if (ws && !aligned16(ws)) return KVLINK_EINVAL;
     cudaError_t err = cudaSuccess;
     const int rc = launch_attention_tc(p->dev, (int)p->items.size(), (int)p->cu_sched.size() - 1,
                                        (int)p->merges.size(), p->cu_fresh.back(),
-                                       p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out,
+                                       p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, vs, out,
                                        ws, s, &err);
     if (rc == KVLINK_ECUDA) return cuda_fail(err, "suffix attention launch");
     return rc;
+}
+
+// the values of the linked cache, or (cache_v NULL) where they are
+static ValueSource values(void* cache_v, const void* pool_v, const void* v_new) {
+    return cache_v ? ValueSource{cache_v, nullptr, nullptr} : ValueSource{nullptr, pool_v, v_new};
 }
 
 int kvlink_suffix_attention(const kvlink_plan_t* p, const void* q, const void* k_new, const void* v_new,
@@ -415,7 +433,22 @@ int kvlink_suffix_attention(const kvlink_plan_t* p, const void* q, const void* k
         rc = place_fresh(p, k_new, v_new, cache_k, cache_v, s);
         if (rc) return rc;
     }
-    return attention_common(p, q, cache_k, cache_v, out, ws, ws_bytes, s);
+    return attention_common(p, q, cache_k, values(cache_v, nullptr, nullptr), out, ws, ws_bytes, s);
+}
+
+int kvlink_suffix_attention_pool_values(const kvlink_plan_t* p, const void* q, const void* k_new,
+                                        const void* v_new, const void* pool_v, void* cache_k, void* out, void* ws,
+                                        size_t ws_bytes, kvlink_stream_t stream) {
+    int rc = check_plan(p);
+    if (rc) return rc;
+    if (!v_new || !pool_v || !cache_k) return KVLINK_EINVAL;
+    if (k_new && !aligned16(k_new)) return KVLINK_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (k_new) {
+        rc = place_fresh(p, k_new, nullptr, cache_k, nullptr, s);
+        if (rc) return rc;
+    }
+    return attention_common(p, q, cache_k, values(nullptr, pool_v, v_new), out, ws, ws_bytes, s);
 }
 
 int kvlink_suffix_attention_simt(const kvlink_plan_t* p, const void* q, const void* k_new, const void* v_new,
@@ -440,15 +473,17 @@ int kvlink_linked_prefill(const kvlink_plan_t* p, const void* pool_k, const void
                           void* ws, size_t ws_bytes, kvlink_stream_t stream) {
     int rc = check_plan(p);
     if (rc) return rc;
-    if (!pool_k || !pool_v || !k_new || !v_new || !cache_k || !cache_v) return KVLINK_EINVAL;
-    if (!aligned16(pool_k) || !aligned16(pool_v) || !aligned16(k_new) || !aligned16(v_new))
+    // cache_v NULL: zero-copy values (keys re-encoded, values read where they are)
+    if (!pool_k || !pool_v || !k_new || !v_new || !cache_k) return KVLINK_EINVAL;
+    if (!aligned16(pool_k) || !aligned16(pool_v) || !aligned16(k_new) || !aligned16(v_new) ||
+        (cache_v && !aligned16(cache_v)))
         return KVLINK_EINVAL;
     cudaStream_t s = (cudaStream_t)stream;
     launch_reencode(p->dev, 0, (int)p->chunks.size(), p->head_dim, p->h_kv, p->num_sms, pool_k, pool_v, k_new,
                     v_new, cache_k, cache_v, s);
     rc = check_launch("reencode_kernel (fused)");
     if (rc) return rc;
-    return attention_common(p, q, cache_k, cache_v, out, ws, ws_bytes, s);
+    return attention_common(p, q, cache_k, values(cache_v, pool_v, v_new), out, ws, ws_bytes, s);
 }
 
 int kvlink_linked_prefill_fused(const kvlink_plan_t* p, const void* pool_k, const void* pool_v, const void* q,
@@ -477,8 +512,8 @@ int kvlink_linked_prefill_layers(const kvlink_plan_t* p, int32_t n_layers, const
                                  void* const* out, void* ws, size_t ws_bytes, kvlink_stream_t stream) {
     int rc = check_plan(p);
     if (rc) return rc;
-    if (n_layers <= 0 || !pool_k || !pool_v || !q || !k_new || !v_new || !cache_k || !cache_v || !out)
-        return KVLINK_EINVAL;
+    // cache_v NULL: zero-copy values in every layer
+    if (n_layers <= 0 || !pool_k || !pool_v || !q || !k_new || !v_new || !cache_k || !out) return KVLINK_EINVAL;
     // every argument is checked before the first launch
     if (!all_aligned(n_layers, q) || !all_aligned(n_layers, k_new) || !all_aligned(n_layers, v_new) ||
         !all_aligned(n_layers, (const void* const*)out))
@@ -486,14 +521,15 @@ int kvlink_linked_prefill_layers(const kvlink_plan_t* p, int32_t n_layers, const
     if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
     if (ws && !aligned16(ws)) return KVLINK_EINVAL;
     if (!all_aligned(n_layers, pool_k) || !all_aligned(n_layers, pool_v) ||
-        !all_aligned(n_layers, (const void* const*)cache_k) || !all_aligned(n_layers, (const void* const*)cache_v))
+        !all_aligned(n_layers, (const void* const*)cache_k) ||
+        (cache_v && !all_aligned(n_layers, (const void* const*)cache_v)))
         return KVLINK_EINVAL;
     // per layer, one re-encode launch that also places the fresh rows, then the suffix
     // attention.  (Re-encoding every layer's documents in one launch first streams at the
     // same rate and then needs a separate fresh-row launch per layer: slower.)
     for (int l = 0; l < n_layers; ++l) {
-        rc = kvlink_linked_prefill(p, pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l], cache_v[l],
-                                   out[l], ws, ws_bytes, stream);
+        rc = kvlink_linked_prefill(p, pool_k[l], pool_v[l], q[l], k_new[l], v_new[l], cache_k[l],
+                                   cache_v ? cache_v[l] : nullptr, out[l], ws, ws_bytes, stream);
         if (rc) return rc;
     }
     return KVLINK_OK;
@@ -507,12 +543,13 @@ int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* p, int32_t n_layers, 
                                             kvlink_stream_t reencode_stream) {
     int rc = check_plan(p);
     if (rc) return rc;
-    if (n_layers <= 0 || !pool_k || !pool_v || !q || !k_new || !v_new || !cache_k || !cache_v || !out)
-        return KVLINK_EINVAL;
+    // cache_v NULL: zero-copy values in every layer
+    if (n_layers <= 0 || !pool_k || !pool_v || !q || !k_new || !v_new || !cache_k || !out) return KVLINK_EINVAL;
     if (stream == reencode_stream) return KVLINK_EINVAL;
     // every argument is checked before the first launch
     if (!all_aligned(n_layers, pool_k) || !all_aligned(n_layers, pool_v) ||
-        !all_aligned(n_layers, (const void* const*)cache_k) || !all_aligned(n_layers, (const void* const*)cache_v) ||
+        !all_aligned(n_layers, (const void* const*)cache_k) ||
+        (cache_v && !all_aligned(n_layers, (const void* const*)cache_v)) ||
         !all_aligned(n_layers, q) || !all_aligned(n_layers, k_new) || !all_aligned(n_layers, v_new) ||
         !all_aligned(n_layers, (const void* const*)out))
         return KVLINK_EINVAL;
@@ -529,7 +566,7 @@ int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* p, int32_t n_layers, 
     if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_overlapped: stream order");
     for (int l = 0; l < n_layers; ++l) {
         launch_reencode(p->dev, 0, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, pool_k[l], pool_v[l],
-                        nullptr, nullptr, cache_k[l], cache_v[l], r);
+                        nullptr, nullptr, cache_k[l], cache_v ? cache_v[l] : nullptr, r);
         rc = check_launch("reencode_kernel (overlapped)");
         if (rc) return rc;
         e = cudaEventRecord(ev[l], r);
@@ -540,9 +577,10 @@ int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* p, int32_t n_layers, 
     for (int l = 0; l < n_layers; ++l) {
         e = cudaStreamWaitEvent(s, ev[l], 0);
         if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_overlapped: wait");
-        rc = place_fresh(p, k_new[l], v_new[l], cache_k[l], cache_v[l], s);
+        void* cv = cache_v ? cache_v[l] : nullptr;
+        rc = place_fresh(p, k_new[l], v_new[l], cache_k[l], cv, s);
         if (rc) return rc;
-        rc = attention_common(p, q[l], cache_k[l], cache_v[l], out[l], ws, ws_bytes, s);
+        rc = attention_common(p, q[l], cache_k[l], values(cv, pool_v[l], v_new[l]), out[l], ws, ws_bytes, s);
         if (rc) return rc;
     }
     return KVLINK_OK;
@@ -557,8 +595,9 @@ int kvlink_linked_prefill_layers_host(kvlink_plan_t* p, int32_t n_layers, const 
                                       kvlink_stream_t copy_in_stream, kvlink_stream_t copy_out_stream) {
     int rc = check_plan(p);
     if (rc) return rc;
+    // cache_v NULL: zero-copy values in every layer
     if (n_layers <= 0 || !pool_k || !pool_v || !h_q || !h_k_new || !h_v_new || !q || !k_new || !v_new ||
-        !cache_k || !cache_v || !out || !h_out)
+        !cache_k || !out || !h_out)
         return KVLINK_EINVAL;
     if (stream == reencode_stream || stream == copy_in_stream || stream == copy_out_stream ||
         reencode_stream == copy_in_stream || reencode_stream == copy_out_stream || copy_in_stream == copy_out_stream)
@@ -566,7 +605,7 @@ int kvlink_linked_prefill_layers_host(kvlink_plan_t* p, int32_t n_layers, const 
     auto cv = [](void* const* a) { return (const void* const*)a; };
     if (!all_aligned(n_layers, pool_k) || !all_aligned(n_layers, pool_v) || !all_aligned(n_layers, cv(q)) ||
         !all_aligned(n_layers, cv(k_new)) || !all_aligned(n_layers, cv(v_new)) || !all_aligned(n_layers, cv(cache_k)) ||
-        !all_aligned(n_layers, cv(cache_v)) || !all_aligned(n_layers, cv(out)))
+        (cache_v && !all_aligned(n_layers, cv(cache_v))) || !all_aligned(n_layers, cv(out)))
         return KVLINK_EINVAL;
     for (int l = 0; l < n_layers; ++l)
         if (!h_q[l] || !h_k_new[l] || !h_v_new[l] || !h_out[l]) return KVLINK_EINVAL;
@@ -601,7 +640,7 @@ int kvlink_linked_prefill_layers_host(kvlink_plan_t* p, int32_t n_layers, const 
         if (chained && (e = cudaStreamWaitEvent(r, ev_c[l], 0)) != cudaSuccess)
             return cuda_fail(e, "linked_prefill_layers_host: wait");
         launch_reencode(p->dev, 0, p->n_chunks_cached, p->head_dim, p->h_kv, p->num_sms, pool_k[l], pool_v[l],
-                        nullptr, nullptr, cache_k[l], cache_v[l], r);
+                        nullptr, nullptr, cache_k[l], cache_v ? cache_v[l] : nullptr, r);
         rc = check_launch("reencode_kernel (host path)");
         if (rc) return rc;
         if ((e = cudaEventRecord(ev_re[l], r)) != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host");
@@ -620,9 +659,10 @@ int kvlink_linked_prefill_layers_host(kvlink_plan_t* p, int32_t n_layers, const 
         if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev_re[l], 0);
         if (e == cudaSuccess && chained) e = cudaStreamWaitEvent(s, ev_o[l], 0);
         if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host: inputs");
-        rc = place_fresh(p, k_new[l], v_new[l], cache_k[l], cache_v[l], s);
+        void* cvl = cache_v ? cache_v[l] : nullptr;
+        rc = place_fresh(p, k_new[l], v_new[l], cache_k[l], cvl, s);
         if (rc) return rc;
-        rc = attention_common(p, q[l], cache_k[l], cache_v[l], out[l], ws, ws_bytes, s);
+        rc = attention_common(p, q[l], cache_k[l], values(cvl, pool_v[l], v_new[l]), out[l], ws, ws_bytes, s);
         if (rc) return rc;
         // the output back to the host
         e = cudaEventRecord(ev_c[l], s);
@@ -703,7 +743,7 @@ int kvlink_linked_prefill_layers_host_pool(kvlink_plan_t* p, int32_t n_layers, c
         if (e != cudaSuccess) return cuda_fail(e, "linked_prefill_layers_host_pool: wait");
         rc = place_fresh(p, k_new[l], v_new[l], cache_k[l], cache_v[l], s);
         if (rc) return rc;
-        rc = attention_common(p, q[l], cache_k[l], cache_v[l], out[l], ws, ws_bytes, s);
+        rc = attention_common(p, q[l], cache_k[l], values(cache_v[l], nullptr, nullptr), out[l], ws, ws_bytes, s);
         if (rc) return rc;
     }
     return KVLINK_OK;

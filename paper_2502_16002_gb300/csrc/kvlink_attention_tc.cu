@@ -67,18 +67,23 @@ constexpr int kTmaVWarp = 6;
 // 56 and the softmax warpgroup rises to 240 (240 + 56 + 168 per SM sub-partition).
 constexpr int kPtThreads = 384;
 constexpr int kPtEpiWarp0 = 8;
-constexpr uint32_t kPtSoftmaxRegs = 240, kPtIdleRegs = 56;
+// With zero-copy values the V warp gathers rows and keeps the next tile's records, so that
+// warpgroup keeps 96 (240 + 96 + 168 = 3 x 168: the whole launch budget).
+constexpr uint32_t kPtSoftmaxRegs = 240, kPtIdleRegs = 56, kPtIdleRegsZv = 96;
 static_assert(kPtThreads * 168 <= 65536, "launch register budget");
 static_assert(128 * (kPtSoftmaxRegs + kPtIdleRegs + 168) <= kPtThreads * 168, "register split");
+static_assert(128 * (kPtSoftmaxRegs + kPtIdleRegsZv + 168) <= kPtThreads * 168, "register split (zero-copy values)");
 
 // Shared memory: two Q buffers (the next item's Q lands while the current item runs), the K
 // ring and the V ring (one stage shorter than the K ring for head_dim 128: a V tile is needed
-// a softmax later than its K tile), m and l of one item, a flag, the barriers.
-template <int D>
+// a softmax later than its K tile), m and l of one item, a flag, the barriers.  With zero-copy
+// values (ZV) the rings trade places: the value tiles come from the pool, partly row by row,
+// and need the longer lead.
+template <int D, bool ZV = false>
 struct PtCfg {
     static constexpr int ATOMS = D / 64;
-    static constexpr int NK = (D == 128) ? 3 : 5;
-    static constexpr int NV = (D == 128) ? 2 : 4;
+    static constexpr int NK = (D == 128) ? (ZV ? 2 : 3) : (ZV ? 4 : 5);
+    static constexpr int NV = (D == 128) ? (ZV ? 3 : 2) : (ZV ? 5 : 4);
     static constexpr int NB = 3;
     static constexpr uint32_t ATOM_BYTES = 128 * 128;
     static constexpr uint32_t Q_BYTES = ATOMS * ATOM_BYTES, KV_BYTES = ATOMS * ATOM_BYTES;
@@ -134,12 +139,236 @@ __device__ __forceinline__ void epilogue_item(const AttnItem& it, const DevicePl
                        out + ((int64_t)(P.cu_fresh[mg.query] + tok) * h_q + mg.kv_head * G + (r % G)) * D);
 }
 
-template <int D, int G>
+// Zero-copy values: the V tiles are read where the values are (the pool's rows for the prefix
+// and document positions, v_new for the fresh rows) in the cache-row order of the key tiles,
+// so the linked cache needs no value rows.  The whole V warp runs it.  Per 8 cache rows the
+// plan's group table says whether their sources are 8 consecutive rows of one tensor; those
+// groups are TMA copies landing 1024-byte aligned in the 128-byte swizzled layout the PV MMA
+// reads, a run of groups that continue one another in naturally aligned boxes of 8 to 128 rows
+// (lane = group + 16 x atom; the first group of a box issues it).  The rows of the other groups
+// (a segment boundary inside, or past the query's end) the warp copies 16 bytes at a time with
+// cp.async (lane = 16-byte chunk of a row), or zero-fills.
+// The warp keeps the tables a tile ahead: the items' entries 32 at a time (one item per lane),
+// and the group entries and source records of the next tile, loaded while the current tile is
+// issued and first used a tile later.  Per tile it issues the row copies first and the boxes
+// second; lane 0 raises the stage's byte count for the boxes before they are issued.  A stage
+// without row copies is published at once (lane 0 arrives; the boxes complete it).  A stage with
+// row copies is published after the next tile has been issued, when its copies have landed:
+// every lane waits for them and fences them into the async proxy, then lane 0 arrives.  That
+// arrival waits for the next stage to come free, i.e. for the PV MMA NV - 1 tiles back, so the
+// value ring is deeper here (NV >= 3) than with a linked value cache.  (With two stages the
+// deferred arrival made each PV MMA wait for the one before it; publishing only after the
+// copies' own latency left each stage a copy latency late.)
+struct PoolValues {
+    const __nv_bfloat16* pool_v;   // [pool_rows][h_kv][D]
+    const __nv_bfloat16* v_new;    // [n_fresh][h_kv][D]
+    int h_kv;
+};
+
+// Source tensors of the value copies: boxes of 8 << h rows (h = 0..4: 8 to 128 rows) over the
+// pool (src 0) and v_new (src 1).  Passed as one kernel parameter.
+constexpr int kVBoxSizes = 5;
+struct ValueMaps {
+    CUtensorMap m[2][kVBoxSizes];
+};
+
+template <int D, int NV>
+__device__ __forceinline__ void pool_values_role(const DevicePlan& P, const PoolValues& V, const ValueMaps* M,
+                                                 uint8_t* smem_v, int first, int n_mine, uint64_t* bar_v_full,
+                                                 uint64_t* bar_v_empty, volatile int32_t* abort_flag,
+                                                 int32_t* status) {
+    constexpr int ATOMS = D / 64;
+    constexpr uint32_t ATOM_BYTES = 128 * 128, KV_BYTES = ATOMS * ATOM_BYTES, GROUP_BYTES = ATOMS * 8 * 128;
+    constexpr int N_GRP = kAttnBN / 8;      // 16 groups per tile
+    constexpr int CPR = D / 8;              // 16-byte chunks per row
+    constexpr int RPP = 32 / CPR;           // rows per warp pass
+    constexpr int RPL = kAttnBN / 32;       // records per lane
+    static_assert(N_GRP * ATOMS <= 32 && 8 % RPP == 0 && N_GRP == 16, "V warp split");
+    const int lane = threadIdx.x % 32, ch = lane % CPR;
+    const uint32_t v_base = smem_u32(smem_v);
+    const int64_t row_elems = (int64_t)V.h_kv * D;
+
+    // The tables of this CTA's items, one item per lane, 32 items per load: an item's entry
+    // (its schedule index, then the item, then its query's offsets) is a chain of dependent
+    // loads, paid once per 32 items instead of at every item change.
+    int l_head = 0, l_t0 = 0, l_n = 0, l_a = 0, l_b = 0, l_npos = 0, l_gbase = 0, l_ngrp = 0;
+    int64_t l_ctx0 = 0;
+    auto load_items = [&](int k0) {
+        const int k = k0 + lane;
+        if (k < n_mine) {
+            const AttnItem it = P.items[P.sched[first + k]];
+            l_head = it.kv_head;
+            l_t0 = it.kv_tile0;
+            l_n = it.kv_tile1 - it.kv_tile0;
+            l_a = it.a_tiles;
+            l_b = it.b_tile0;
+            l_ctx0 = P.cu_ctx[it.query];
+            l_npos = (int)(P.cu_ctx[it.query + 1] - l_ctx0);
+            l_gbase = P.cu_grp[it.query];
+            l_ngrp = P.cu_grp[it.query + 1] - l_gbase;
+        }
+    };
+    // the tile after the current one: tile jn of item kn, and what the warp loaded for it (raw:
+    // the loads are first used a tile later, so their latency overlaps the current tile)
+    int kn = 0, jn = 0;
+    int headn = 0, t0n = 0, nn = 0, an = 0, bn = 0, n_posn = 0, gbasen = 0, n_grpn = 0;
+    int64_t ctx0n = 0;
+    int key0n = 0;
+    int32_t gwn = -1;
+    int2 srcn[RPL];
+    auto item_info = [&](int k) {
+        if (k % 32 == 0) load_items(k);
+        const int src = k % 32;
+        headn = __shfl_sync(0xffffffffu, l_head, src);
+        t0n = __shfl_sync(0xffffffffu, l_t0, src);
+        nn = __shfl_sync(0xffffffffu, l_n, src);
+        an = __shfl_sync(0xffffffffu, l_a, src);
+        bn = __shfl_sync(0xffffffffu, l_b, src);
+        ctx0n = __shfl_sync(0xffffffffu, l_ctx0, src);
+        n_posn = __shfl_sync(0xffffffffu, l_npos, src);
+        gbasen = __shfl_sync(0xffffffffu, l_gbase, src);
+        n_grpn = __shfl_sync(0xffffffffu, l_ngrp, src);
+    };
+    // group entries and source records (kind, row; row -1 past the query's end) of tile jn
+    auto prefetch = [&]() {
+        const int v = t0n + jn;   // the item's key-tile list entry (item_tile)
+        key0n = (v < an ? v : bn + (v - an)) * kAttnBN;
+        const int m0 = key0n / 8;
+        gwn = -1;
+        if (lane < N_GRP && m0 + lane < n_grpn) gwn = __ldg(P.grp_src + gbasen + m0 + lane);
+#pragma unroll
+        for (int t = 0; t < RPL; ++t) {
+            const int pos = key0n + lane + 32 * t;
+            srcn[t] = make_int2(0, -1);
+            if (pos < n_posn) srcn[t] = __ldg(reinterpret_cast<const int2*>(P.src_row + ctx0n + pos));
+        }
+    };
+
+    bool have = n_mine > 0;
+    if (have) {
+        item_info(0);
+        prefetch();
+    }
+    int g = 0;                 // tiles issued
+    bool pend = false;         // tile g - 1 has row copies and is not yet published
+    static_assert(NV >= 3, "the deferred publication needs three value stages");
+    while (have) {
+        // the current tile is the prefetched one
+        const int kv_head = headn;
+        int32_t gw = gwn;
+        int32_t rec[RPL];      // kGrpFresh | row, or -1 (zero-filled)
+#pragma unroll
+        for (int t = 0; t < RPL; ++t) {
+            const int2 e = srcn[t];
+            rec[t] = e.y < 0 ? -1 : (e.y | (e.x == KVLINK_SRC_FRESH ? kGrpFresh : 0));
+#ifdef KVLINK_DEBUG_CHECKS
+            if (e.y >= (e.x == KVLINK_SRC_FRESH ? (int64_t)P.n_fresh : P.pool_rows)) {
+                atomicCAS(status, 0, kAttnStatusBadIndex);
+                rec[t] = -1;   // zero-filled instead
+            }
+#endif
+        }
+#ifdef KVLINK_DEBUG_CHECKS
+        if (gw >= 0 && (gw & kGrpRowMask) + 8 > ((gw & kGrpFresh) ? (int64_t)P.n_fresh : P.pool_rows)) {
+            atomicCAS(status, 0, kAttnStatusBadIndex);
+            gw = -1;   // its rows take the per-row path, whose records are checked above
+        }
+#endif
+        // advance and start the next tile's loads
+        if (++jn >= nn) {
+            jn = 0;
+            if (++kn < n_mine) item_info(kn);
+            else have = false;
+        }
+        if (have) prefetch();
+
+        const int st = g % NV;
+        if (!warp_wait(bar_v_empty + st, ((g / NV) & 1) ^ 1, abort_flag, status)) break;
+        const uint32_t by_tma = __ballot_sync(0xffffffffu, gw >= 0);   // lanes >= N_GRP hold -1
+        const uint32_t by_row = ~by_tma & ((1u << N_GRP) - 1);
+        // Runs of groups whose rows continue one another go in naturally aligned boxes of 1, 2,
+        // 4, 8 or 16 groups: a block of 2^h groups starting at a multiple of 2^h is one box when
+        // every group in it is a TMA group and each continues the one before.
+        const int32_t prev = __shfl_up_sync(0xffffffffu, gw, 1);
+        const uint32_t cont = __ballot_sync(0xffffffffu, lane < N_GRP && lane > 0 && gw >= 0 && gw == prev + 8);
+        // the row copies first (one commit group per tile), then the boxes
+        const uint32_t sv_addr = v_base + st * KV_BYTES;
+        const int64_t col = (int64_t)kv_head * D + 8 * ch;   // this lane's chunk within a row
+        for (uint32_t rest = by_row; rest != 0; rest &= rest - 1) {
+            const int m = __ffs(rest) - 1;
+#pragma unroll
+            for (int p = 0; p < 8 / RPP; ++p) {
+                const int r0 = m * 8 + p * RPP;          // a multiple of RPP: the rows' records
+                const int t = r0 / 32;                   // sit in slot t of every lane
+                int32_t mine = rec[0];
+#pragma unroll
+                for (int u = 1; u < RPL; ++u)
+                    if (t == u) mine = rec[u];
+                const int r = r0 + lane / CPR;
+                const int32_t e = __shfl_sync(0xffffffffu, mine, r % 32);
+                const uint32_t dst =
+                    sv_addr + (uint32_t)(ch >> 3) * ATOM_BYTES + (uint32_t)r * 128u + ((uint32_t)((ch & 7) ^ (r & 7)) << 4);
+                if (e >= 0)
+                    cp_async16(dst, ((e & kGrpFresh) ? V.v_new : V.pool_v) + (int64_t)(e & kGrpRowMask) * row_elems + col);
+                else
+                    st_shared_zero16(dst);
+            }
+        }
+        cp_async_commit();
+        uint8_t* sv = smem_v + st * KV_BYTES;
+        if (lane == 0) mbar_expect_tx(bar_v_full + st, (uint32_t)__popc(by_tma) * GROUP_BYTES);
+        __syncwarp();
+        {
+            const int m = lane % N_GRP, a = lane / N_GRP;
+            // the largest whole block holding group m
+            int h = 0;
+#pragma unroll
+            for (int hh = 1; hh < kVBoxSizes; ++hh) {
+                const int n = 1 << hh, b0 = m & ~(n - 1);
+                const uint32_t blk = ((1u << n) - 1u) << b0;
+                const uint32_t inner = blk & ~(1u << b0);         // groups that must continue
+                if ((by_tma & blk) == blk && (cont & inner) == inner) h = hh;
+            }
+            const int32_t gm = __shfl_sync(0xffffffffu, gw, m);
+            if (a < ATOMS && gm >= 0 && (m & ((1 << h) - 1)) == 0)
+                tma_load_3d(sv + a * ATOM_BYTES + m * 8 * 128, &M->m[(gm & kGrpFresh) ? 1 : 0][h], a * 64, kv_head,
+                            gm & kGrpRowMask, bar_v_full + st);
+        }
+        // The previous tile's row copies have had this tile's issue time to land: publish that
+        // stage (fence into the async proxy, lane 0 arrives); a tile without row copies is
+        // published at once.  With NV >= 3 stages the deferred arrival waits only for the PV MMA
+        // NV - 1 tiles back, which its own PV follows anyway.
+        if (pend) {
+            cp_async_wait<1>();
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_v_full + (g - 1) % NV);
+        }
+        pend = by_row != 0;
+        if (!pend) {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_v_full + st);
+        }
+        ++g;
+    }
+    if (pend) {
+        cp_async_wait<0>();
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar_v_full + (g - 1) % NV);
+    }
+    // no copy may still be in flight when the CTA leaves
+    if (lane == 0)
+        for (int gg = g - NV > 0 ? g - NV : 0; gg < g; ++gg) drain_bar(bar_v_full + gg % NV, (gg / NV) & 1, status);
+}
+
+template <int D, int G, bool ZV>
 __global__ void __launch_bounds__(kPtThreads, 1)
     attn_tc_persistent_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                              const __grid_constant__ CUtensorMap tm_v, DevicePlan P,
-                              __nv_bfloat16* __restrict__ out, float* __restrict__ ws, int h_q, float scale_log2) {
-    using C = PtCfg<D>;
+                              const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ ValueMaps vmaps,
+                              DevicePlan P, const PoolValues V, __nv_bfloat16* __restrict__ out,
+                              float* __restrict__ ws, int h_q, float scale_log2) {
+    using C = PtCfg<D, ZV>;
     constexpr int NK = C::NK, NV = C::NV, NB = C::NB;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
@@ -206,6 +435,8 @@ __global__ void __launch_bounds__(kPtThreads, 1)
         prefetch_tensormap(&tm_q);
         prefetch_tensormap(&tm_k);
         prefetch_tensormap(&tm_v);
+        if (ZV)
+            for (int i = 0; i < 2 * kVBoxSizes; ++i) prefetch_tensormap(&vmaps.m[i / kVBoxSizes][i % kVBoxSizes]);
     }
     tc_fence_before();
     __syncthreads();
@@ -216,7 +447,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
     if (skip) {
         // nothing issued: fall through to the teardown
     } else if (warp >= kSoftmaxWarps && warp < kPtEpiWarp0) {
-        setmaxnreg_dec<kPtIdleRegs>();
+        setmaxnreg_dec<ZV ? kPtIdleRegsZv : kPtIdleRegs>();
         if (warp == kTmaKWarp && lane == 0) {
             // ------------------------------------------------ Q of every item, and the K ring
             int g = 0, q_issued = 0;
@@ -248,6 +479,11 @@ __global__ void __launch_bounds__(kPtThreads, 1)
             for (int gg = g - NK > 0 ? g - NK : 0; gg < g; ++gg) drain_bar(bar_k_full + gg % NK, (gg / NK) & 1, status);
             for (int k = q_issued - 2 > 0 ? q_issued - 2 : 0; k < q_issued; ++k)
                 drain_bar(bar_q_full + (k & 1), (k >> 1) & 1, status);
+        } else if (warp == kTmaVWarp && ZV) {
+            // ------------------------------------------------ the V ring, values where they are
+            if constexpr (ZV)
+                pool_values_role<D, NV>(P, V, &vmaps, smem + C::OFF_V, first, n_mine, bar_v_full, bar_v_empty,
+                                        abort_flag, status);
         } else if (warp == kTmaVWarp && lane == 0) {
             // ------------------------------------------------ the V ring
             int g = 0;
@@ -426,20 +662,20 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uin
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D, int G>
+template <int D, int G, bool ZV>
 static cudaError_t launch_tc_dg(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv,
-                                const DevicePlan& P, int n_ctas, void* out, float* ws, int h_q, float scale_log2,
-                                cudaStream_t stream) {
+                                const ValueMaps& vm, const DevicePlan& P, const PoolValues& V, int n_ctas, void* out,
+                                float* ws, int h_q, float scale_log2, cudaStream_t stream) {
     static std::atomic<uint64_t> attr_set{0};
     cudaError_t ea = once_per_device(attr_set, [] {
-        return cudaFuncSetAttribute(attn_tc_persistent_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)PtCfg<D>::SMEM_BYTES);
+        return cudaFuncSetAttribute(attn_tc_persistent_kernel<D, G, ZV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)PtCfg<D, ZV>::SMEM_BYTES);
     });
     if (ea != cudaSuccess) return ea;
     // cut ranges are merged inside the kernel: nothing follows it
     if (n_ctas > 0)
-        attn_tc_persistent_kernel<D, G><<<n_ctas, kPtThreads, PtCfg<D>::SMEM_BYTES, stream>>>(
-            mq, mk, mv, P, (__nv_bfloat16*)out, ws, h_q, scale_log2);
+        attn_tc_persistent_kernel<D, G, ZV><<<n_ctas, kPtThreads, PtCfg<D, ZV>::SMEM_BYTES, stream>>>(
+            mq, mk, mv, vm, P, V, (__nv_bfloat16*)out, ws, h_q, scale_log2);
     return cudaGetLastError();
 }
 
@@ -455,22 +691,40 @@ cudaError_t launch_attn_merge(const DevicePlan& P, int n_merges, const float* ws
 }
 
 // Returns 0, or KVLINK_ECUDA / KVLINK_EUNSUPPORTED.
-// The persistent kernel over the plan's per-CTA schedule (n_ctas CTAs).
+// The persistent kernel over the plan's per-CTA schedule (n_ctas CTAs); values from the linked
+// cache (vs.cache_v), or where they are (vs.cache_v NULL: vs.pool_v and vs.v_new, through
+// 8-row TMA boxes).
 int launch_attention_tc(const DevicePlan& P, int n_items, int n_ctas, int n_merges, int n_fresh, int64_t ctx_rows,
-                        int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
+                        int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const ValueSource& vs,
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err) {
     const int G = h_q / h_kv;
-    CUtensorMap mq, mk, mv;
+    const bool zv = vs.cache_v == nullptr;
+    CUtensorMap mq, mk, mv;      // values: the linked cache (zero-copy values: vm)
+    ValueMaps vm{};              // zero-copy values: pool / v_new in boxes of 8 .. 128 rows
     const uint32_t box_tok = (uint32_t)(kAttnBM / G);
     if (!make_map_3d(&mq, q, (uint64_t)head_dim, (uint64_t)h_q, (uint64_t)n_fresh, 64, (uint32_t)G, box_tok) ||
-        !make_map_3d(&mk, cache_k, (uint64_t)head_dim, (uint64_t)h_kv, (uint64_t)ctx_rows, 64, 1, kAttnBN) ||
-        !make_map_3d(&mv, cache_v, (uint64_t)head_dim, (uint64_t)h_kv, (uint64_t)ctx_rows, 64, 1, kAttnBN))
+        !make_map_3d(&mk, cache_k, (uint64_t)head_dim, (uint64_t)h_kv, (uint64_t)ctx_rows, 64, 1, kAttnBN))
         return KVLINK_EUNSUPPORTED;
+    if (!zv) {
+        if (!make_map_3d(&mv, vs.cache_v, (uint64_t)head_dim, (uint64_t)h_kv, (uint64_t)ctx_rows, 64, 1, kAttnBN))
+            return KVLINK_EUNSUPPORTED;
+    } else {
+        mv = mk;   // unused
+        const uint64_t D = (uint64_t)head_dim, H = (uint64_t)h_kv;
+        const uint64_t rows[2] = {(uint64_t)P.pool_rows, (uint64_t)n_fresh};
+        const void* base[2] = {vs.pool_v, vs.v_new};
+        for (int src = 0; src < 2; ++src)
+            for (int h = 0; h < kVBoxSizes; ++h)
+                if (!make_map_3d(&vm.m[src][h], base[src], D, H, rows[src], 64, 1, 8u << h)) return KVLINK_EUNSUPPORTED;
+    }
+    const PoolValues V{(const __nv_bfloat16*)vs.pool_v, (const __nv_bfloat16*)vs.v_new, h_kv};
     const float sl2 = 1.4426950408889634f / sqrtf((float)head_dim);
     float* w = (float*)ws;
     cudaError_t e = cudaErrorInvalidValue;
-#define KVLINK_TC_CASE(DD, GG)                                                                         \
-    if (head_dim == DD && G == GG) e = launch_tc_dg<DD, GG>(mq, mk, mv, P, n_ctas, out, w, h_q, sl2, stream);
+#define KVLINK_TC_CASE(DD, GG)                                                                              \
+    if (head_dim == DD && G == GG)                                                                          \
+        e = zv ? launch_tc_dg<DD, GG, true>(mq, mk, mv, vm, P, V, n_ctas, out, w, h_q, sl2, stream)         \
+               : launch_tc_dg<DD, GG, false>(mq, mk, mv, vm, P, V, n_ctas, out, w, h_q, sl2, stream);
     KVLINK_TC_CASE(128, 1) KVLINK_TC_CASE(128, 2) KVLINK_TC_CASE(128, 4) KVLINK_TC_CASE(128, 8)
     KVLINK_TC_CASE(128, 16) KVLINK_TC_CASE(64, 1) KVLINK_TC_CASE(64, 2) KVLINK_TC_CASE(64, 4)
     KVLINK_TC_CASE(64, 8) KVLINK_TC_CASE(64, 16)

@@ -141,6 +141,15 @@ struct DevicePlan {
     unsigned long long* merge_count;   // [n_merges], in the plan buffer (written by the kernel)
     int32_t n_merges;
 };
+// Where the suffix attention reads the values.  cache_v non-NULL: the linked cache's value
+// rows, [ctx_rows][h_kv][D].  cache_v NULL (zero-copy values): every value row where it
+// already is, pool_v [pool_rows][h_kv][D] for the prefix and document positions and v_new
+// [n_fresh][h_kv][D] for the fresh rows, found through the plan's source and group tables.
+struct ValueSource {
+    const void* cache_v;
+    const void* pool_v;
+    const void* v_new;
+};
 constexpr int32_t kGrpFresh = 1 << 30;
 constexpr int32_t kGrpRowMask = kGrpFresh - 1;
 

@@ -31,7 +31,7 @@ void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head
 void launch_place_fresh(const int32_t* d_fresh_dst, int n_fresh, int64_t ctx_rows, int row_bytes,
                         const void* k_new, const void* v_new, void* cache_k, void* cache_v, cudaStream_t stream);
 int launch_attention_tc(const DevicePlan& P, int n_items, int n_ctas, int n_merges, int n_fresh, int64_t ctx_rows,
-                        int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const void* cache_v,
+                        int head_dim, int h_q, int h_kv, const void* q, const void* cache_k, const ValueSource& vs,
                         void* out, void* ws, cudaStream_t stream, cudaError_t* err);
 }  // namespace kvlink
 
@@ -88,8 +88,8 @@ extern "C" int kvlink_suffix_attention_noalloc(const kvlink_plan_t* p, const voi
     cudaError_t err = cudaSuccess;
     rc = kvlink::launch_attention_tc(p->dev, (int)p->items.size(), (int)p->cu_sched.size() - 1,
                                      (int)p->merges.size(), p->cu_fresh.back(),
-                                     p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k, cache_v, out, ws, s,
-                                     &err);
+                                     p->cu_ctx.back(), p->head_dim, p->h_q, p->h_kv, q, cache_k,
+                                     kvlink::ValueSource{cache_v, nullptr, nullptr}, out, ws, s, &err);
     if (rc == KVLINK_ECUDA) return kvlink::record_cuda_error(err, "suffix attention launch (noalloc)");
     return rc;
 }

@@ -56,7 +56,7 @@ void launch_rope_table(const kvlink_segment_t* d_seg, int n_seg, float4* d_rope,
 // --------------------------------------------------------------------------
 // A3 + A4: persistent re-encode/copy through a shared-memory ring.
 // --------------------------------------------------------------------------
-constexpr int kCopyConsumers = 128;                  // 4 warps rotate keys in shared memory
+constexpr int kCopyConsumers = 256;                  // 8 warps rotate keys in shared memory
 constexpr int kCopyThreads = 32 + kCopyConsumers;    // + 1 producer warp
 constexpr int kCopyStages = 3;
 constexpr uint64_t kCopyWaitLimitNs = 2000000000ull;
@@ -67,10 +67,14 @@ constexpr int32_t kCopyStatusBadIndex = 0x22;   // a table entry out of bounds
 
 static __device__ int32_t g_copy_status;
 
+// WV: a stage holds a unit's keys then its values (3 stages); keys only (zero-copy values):
+// the same 192 KB as 6 stages of keys, so as many bytes stay in flight.
+template <bool WV>
 struct CopySmem {
-    static constexpr uint32_t STAGE = 2 * kCopyStageBytes;   // K then V
-    static constexpr uint32_t OFF_BAR = kCopyStages * STAGE;
-    static constexpr uint32_t BYTES = OFF_BAR + 2 * kCopyStages * 8 + 16 + 128;
+    static constexpr int NST = WV ? kCopyStages : 2 * kCopyStages;
+    static constexpr uint32_t STAGE = WV ? 2 * kCopyStageBytes : kCopyStageBytes;
+    static constexpr uint32_t OFF_BAR = NST * STAGE;
+    static constexpr uint32_t BYTES = OFF_BAR + 2 * NST * 8 + 16 + 128;
 };
 
 __device__ __forceinline__ bool copy_wait(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
@@ -113,26 +117,30 @@ constexpr int kMaxLayersPerLaunch = 64;     // 2 KB of kernel parameters
 // range [n*b/grid, n*(b+1)/grid), n = n_layers * n_chunks, in groups of consecutive
 // chunks that read the same source rows (same layer, same tensor, same first row and
 // length), loading each group's rows once.  The one-layer launches take the chunks in
-// linked-cache order (consecutive chunks never share rows); the all-layer launch takes
+// linked-cache order, where consecutive chunks read other rows (but for a document retrieved
+// twice in a row with no link tokens between), so there a group is one chunk and the next
+// chunk's entry is loaded a group ahead; the all-layer launch takes
 // the document chunks sorted by pool row, so every destination of a document that
 // several queries retrieved follows the first and its rows are loaded once per layer.
 // (One layer is bound by the cache writes, which do not shrink; over all layers the
 // saved reads pay: measured 1607 -> 1314 us for 32 layers of the Llama-8B batch-8
 // workload, while grouping one layer's chunks moved its time from 50 to 53 us.)
 // Producer (warp 0, one thread): bulk-loads a group's K rows and V rows into a stage.
-// Consumers (warps 1-4), per chunk of the group: document keys are read from the stage,
+// Consumers (warps 1-8), per chunk of the group: document keys are read from the stage,
 // rotated by the chunk's delta in registers (each thread keeps a fixed (head, j0) slot
 // and its eight double-float cos/sin pairs) and written with 16-byte global stores;
 // one thread bulk-stores the values (and the keys of prefix and fresh chunks, which are
 // not rotated) straight from the stage.  The stage is freed once the group's stores
-// have read it and every consumer has passed the next group's barrier.
+// have read it and every consumer has passed the next group's barrier.  With zero-copy
+// values (WV false, the linked cache has no value rows) only keys are loaded and stored,
+// and the same shared memory holds twice as many stages.
 __device__ __forceinline__ bool same_source(const CopyChunk& a, int la, const CopyChunk& b, int lb) {
     const bool fa = a.kind == KVLINK_SEG_LINK || a.kind == KVLINK_SEG_QUESTION;
     const bool fb = b.kind == KVLINK_SEG_LINK || b.kind == KVLINK_SEG_QUESTION;
     return la == lb && fa == fb && a.src_row == b.src_row && a.n == b.n;
 }
 
-template <int D, int MAXL>
+template <int D, int MAXL, bool WV>
 __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     const CopyChunk* __restrict__ chunks, int n_chunks, int n_layers, const float4* __restrict__ rope, int h_kv,
     const LayerPtrs<MAXL> L, const __nv_bfloat16* __restrict__ k_new, const __nv_bfloat16* __restrict__ v_new,
@@ -141,9 +149,9 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + ((128u - (raw_addr & 127u)) & 127u);
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + CopySmem::OFF_BAR);
-    uint64_t* empty = full + kCopyStages;
-    volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(empty + kCopyStages);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + CopySmem<WV>::OFF_BAR);
+    uint64_t* empty = full + CopySmem<WV>::NST;
+    volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(empty + CopySmem<WV>::NST);
 
     const int64_t n_units = (int64_t)n_chunks * n_layers;
     const int c_begin = (int)(n_units * blockIdx.x / gridDim.x);
@@ -164,7 +172,7 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     };
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < kCopyStages; ++i) {
+        for (int i = 0; i < CopySmem<WV>::NST; ++i) {
             mbar_init(full + i, 1);
             mbar_init(empty + i, 1);
         }
@@ -196,25 +204,30 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
         // ------------------------------------------------------------ producer
         if (threadIdx.x == 0) {
             int issued = 0;
+            // one-layer launches: a group is one unit, and the next unit's entry is loaded while
+            // this one waits for its stage
+            CopyChunk ch_next{};
+            if (MAXL == 1 && c_begin < c_end) ch_next = chunks[c_begin];
             for (int c = c_begin, g = 0; c < c_end; ++g) {
                 const int layer = layer_of(c);
-                const CopyChunk ch = chunks[c - layer * n_chunks];
-                const int st = g % kCopyStages;
-                if (!copy_wait(empty + st, ((g / kCopyStages) & 1) ^ 1, abort_flag)) break;
+                const CopyChunk ch = MAXL == 1 ? ch_next : chunks[c - layer * n_chunks];
+                if (MAXL == 1 && c + 1 < c_end) ch_next = chunks[c + 1];
+                const int st = g % CopySmem<WV>::NST;
+                if (!copy_wait(empty + st, ((g / CopySmem<WV>::NST) & 1) ^ 1, abort_flag)) break;
                 const bool fresh = ch.kind == KVLINK_SEG_LINK || ch.kind == KVLINK_SEG_QUESTION;
                 const __nv_bfloat16* sk = (fresh ? k_new : L.pool_k[layer]) + ch.src_row * row_elems;
-                const __nv_bfloat16* sv = (fresh ? v_new : L.pool_v[layer]) + ch.src_row * row_elems;
+                const __nv_bfloat16* sv = WV ? (fresh ? v_new : L.pool_v[layer]) + ch.src_row * row_elems : nullptr;
                 const uint32_t bytes = (uint32_t)ch.n * row_bytes;
-                uint8_t* stage = smem + st * CopySmem::STAGE;
-                mbar_arrive_expect_tx(full + st, 2 * bytes);
+                uint8_t* stage = smem + st * CopySmem<WV>::STAGE;
+                mbar_arrive_expect_tx(full + st, WV ? 2 * bytes : bytes);
                 bulk_load(stage, sk, bytes, full + st);
-                bulk_load(stage + kCopyStageBytes, sv, bytes, full + st);
+                if (WV) bulk_load(stage + kCopyStageBytes, sv, bytes, full + st);
                 issued = g + 1;
-                c = group_end(c, layer, ch);
+                c = MAXL == 1 ? c + 1 : group_end(c, layer, ch);
             }
             // no load may still be in flight when the CTA leaves
-            for (int i = issued - kCopyStages > 0 ? issued - kCopyStages : 0; i < issued; ++i)
-                copy_drain(full + i % kCopyStages, (i / kCopyStages) & 1);
+            for (int i = issued - CopySmem<WV>::NST > 0 ? issued - CopySmem<WV>::NST : 0; i < issued; ++i)
+                copy_drain(full + i % CopySmem<WV>::NST, (i / CopySmem<WV>::NST) & 1);
         }
         return;
     }
@@ -231,21 +244,26 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
     const uint32_t lo_off = (uint32_t)(head * D + j0) * 2;
     int cur_table = -1;
     float4 cs[8];
+    // one-layer launches: a group is one unit (consecutive units never read the same rows), and
+    // the next unit's entry is loaded a group ahead, so its latency overlaps this group's work
+    CopyChunk ch_next{};
+    if (MAXL == 1 && c_begin < c_end) ch_next = chunks[c_begin];
     for (int c = c_begin, g = 0; c < c_end; ++g) {
         const int layer = layer_of(c);
-        const CopyChunk ch0 = chunks[c - layer * n_chunks];
-        const int c1 = group_end(c, layer, ch0);
-        const int st = g % kCopyStages;
-        const bool loaded = copy_wait(full + st, (g / kCopyStages) & 1, abort_flag);
+        const CopyChunk ch0 = MAXL == 1 ? ch_next : chunks[c - layer * n_chunks];
+        if (MAXL == 1 && c + 1 < c_end) ch_next = chunks[c + 1];
+        const int c1 = MAXL == 1 ? c + 1 : group_end(c, layer, ch0);
+        const int st = g % CopySmem<WV>::NST;
+        const bool loaded = copy_wait(full + st, (g / CopySmem<WV>::NST) & 1, abort_flag);
         // Every consumer is done with the previous group, and all of them take one decision:
         // the producer may raise the abort flag at any moment (its own wait ran out), so each
         // consumer's read of the flag could differ; the barrier ORs them, so either all 128
         // leave the loop or none does, and no consumer is left waiting at the next barrier.
         if (named_bar_any(1, kCopyConsumers, !loaded || *abort_flag != 0)) break;
-        const uint8_t* stage = smem + st * CopySmem::STAGE;
+        const uint8_t* stage = smem + st * CopySmem<WV>::STAGE;
         const uint32_t bytes = (uint32_t)ch0.n * row_bytes;
         for (int cc = c; cc < c1; ++cc) {
-            const CopyChunk ch = chunks[cc - layer * n_chunks];
+            const CopyChunk ch = MAXL == 1 ? ch0 : chunks[cc - layer * n_chunks];
             if (ch.kind == KVLINK_SEG_DOC) {
                 if (ch.table != cur_table) {
                     const float4* t = rope + (int64_t)ch.table * (D / 2) + j0;
@@ -266,32 +284,44 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
             } else if (tc == 0) {
                 bulk_store(L.cache_k[layer] + ch.dst_row * row_elems, stage, bytes);
             }
-            if (tc == 0) bulk_store(L.cache_v[layer] + ch.dst_row * row_elems, stage + kCopyStageBytes, bytes);
+            if (WV && tc == 0) bulk_store(L.cache_v[layer] + ch.dst_row * row_elems, stage + kCopyStageBytes, bytes);
         }
         if (tc == 0) {
             bulk_commit();
             bulk_wait_read<1>();  // the previous group's stores have read their stage
-            if (g > 0) mbar_arrive(empty + (g - 1) % kCopyStages);
+            if (g > 0) mbar_arrive(empty + (g - 1) % CopySmem<WV>::NST);
         }
         c = c1;
     }
     if (tc == 0) bulk_wait<0>();
 }
 
+template <int D, int MAXL, bool WV>
+static void launch_reencode_wv(const CopyChunk* ch, int n_chunks, int n_layers, const float4* rope, int h_kv,
+                               int num_sms, const LayerPtrs<MAXL>& L, const void* k_new, const void* v_new,
+                               const CopyBounds& bounds, cudaStream_t stream) {
+    // a failure here surfaces as the launch error, which the caller checks
+    static std::atomic<uint64_t> attr{0};
+    once_per_device(attr, [] {
+        return cudaFuncSetAttribute(reencode_kernel<D, MAXL, WV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)CopySmem<WV>::BYTES);
+    });
+    const int64_t n_units = (int64_t)n_chunks * n_layers;
+    const int grid = n_units < num_sms ? (int)n_units : num_sms;
+    reencode_kernel<D, MAXL, WV><<<grid, kCopyThreads, CopySmem<WV>::BYTES, stream>>>(
+        ch, n_chunks, n_layers, rope, h_kv, L, (const __nv_bfloat16*)k_new, (const __nv_bfloat16*)v_new, bounds);
+}
+
+// values copied when the linked cache has value rows (every layer's, or none: zero-copy values)
 template <int D, int MAXL>
 static void launch_reencode_t(const CopyChunk* ch, int n_chunks, int n_layers, const float4* rope, int h_kv,
                               int num_sms, const LayerPtrs<MAXL>& L, const void* k_new, const void* v_new,
                               const CopyBounds& bounds, cudaStream_t stream) {
-    // a failure here surfaces as the launch error, which the caller checks
-    static std::atomic<uint64_t> attr{0};
-    once_per_device(attr, [] {
-        return cudaFuncSetAttribute(reencode_kernel<D, MAXL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)CopySmem::BYTES);
-    });
-    const int64_t n_units = (int64_t)n_chunks * n_layers;
-    const int grid = n_units < num_sms ? (int)n_units : num_sms;
-    reencode_kernel<D, MAXL><<<grid, kCopyThreads, CopySmem::BYTES, stream>>>(
-        ch, n_chunks, n_layers, rope, h_kv, L, (const __nv_bfloat16*)k_new, (const __nv_bfloat16*)v_new, bounds);
+    if (L.cache_v[0] != nullptr)
+        launch_reencode_wv<D, MAXL, true>(ch, n_chunks, n_layers, rope, h_kv, num_sms, L, k_new, v_new, bounds, stream);
+    else
+        launch_reencode_wv<D, MAXL, false>(ch, n_chunks, n_layers, rope, h_kv, num_sms, L, k_new, v_new, bounds,
+                                           stream);
 }
 
 void launch_reencode(const DevicePlan& P, int chunk_base, int n_chunks, int head_dim, int h_kv, int num_sms,
@@ -464,6 +494,7 @@ __global__ void __launch_bounds__(32 * kPlaceWarps) place_fresh_kernel(const int
     }
 #endif
     const int64_t src = (int64_t)row * row_vec, dst = (int64_t)fresh_dst[row] * row_vec;
+    const bool with_v = cache_v != nullptr;   // NULL: zero-copy values (the attention reads v_new)
     for (int i0 = lane; i0 < row_vec; i0 += 4 * 32) {
         uint4 k[4], v[4];
 #pragma unroll
@@ -471,7 +502,7 @@ __global__ void __launch_bounds__(32 * kPlaceWarps) place_fresh_kernel(const int
             const int i = i0 + u * 32;
             if (i < row_vec) {
                 k[u] = __ldg(k_new + src + i);
-                v[u] = __ldg(v_new + src + i);
+                if (with_v) v[u] = __ldg(v_new + src + i);
             }
         }
 #pragma unroll
@@ -479,7 +510,7 @@ __global__ void __launch_bounds__(32 * kPlaceWarps) place_fresh_kernel(const int
             const int i = i0 + u * 32;
             if (i < row_vec) {
                 cache_k[dst + i] = k[u];
-                cache_v[dst + i] = v[u];
+                if (with_v) cache_v[dst + i] = v[u];
             }
         }
     }

@@ -97,6 +97,7 @@ def _load():
         "kvlink_plan_upload": (C.c_int, [P, C.c_double, V, C.c_size_t, V]),
         "kvlink_reencode_concat": (C.c_int, [P, V, V, V, V, V]),
         "kvlink_suffix_attention": (C.c_int, [P, V, V, V, V, V, V, V, C.c_size_t, V]),
+        "kvlink_suffix_attention_pool_values": (C.c_int, [P, V, V, V, V, V, V, V, C.c_size_t, V]),
         "kvlink_suffix_attention_simt": (C.c_int, [P, V, V, V, V, V, V, V]),
         "kvlink_suffix_attention_noalloc": (C.c_int, [P, V, V, V, V, V, V, V]),
         "kvlink_rope_fresh": (C.c_int, [P, V, V, V]),
@@ -133,7 +134,7 @@ DECLARED = [
     "kvlink_plan_get_sources", "kvlink_linked_prefill_fused", "kvlink_linked_prefill_layers",
     "kvlink_reencode_concat_layers", "kvlink_plan_rebuild", "kvlink_linked_prefill_layers_overlapped",
     "kvlink_linked_prefill_layers_host", "kvlink_reencode_concat_host_pool", "kvlink_linked_prefill_layers_host_pool",
-    "kvlink_selftest_wait_timeout",
+    "kvlink_selftest_wait_timeout", "kvlink_suffix_attention_pool_values",
 ]
 
 # size of the static scratch used by kvlink_suffix_attention_noalloc (include/kvlink.h)
@@ -277,6 +278,13 @@ def kvlink_suffix_attention(plan: Plan, q: int, k_new, v_new, cache_k: int, cach
                                        workspace_bytes, stream), "kvlink_suffix_attention")
 
 
+def kvlink_suffix_attention_pool_values(plan: Plan, q: int, k_new, v_new: int, pool_v: int, cache_k: int, out: int,
+                                        workspace, workspace_bytes: int, stream: int = 0) -> None:
+    """Suffix attention with zero-copy values: value rows read from pool_v and v_new."""
+    _check(lib.kvlink_suffix_attention_pool_values(plan.handle, q, k_new, v_new, pool_v, cache_k, out, workspace,
+                                                   workspace_bytes, stream), "kvlink_suffix_attention_pool_values")
+
+
 def kvlink_suffix_attention_simt(plan: Plan, q: int, k_new, v_new, cache_k: int, cache_v: int, out: int,
                                  stream: int = 0) -> None:
     _check(lib.kvlink_suffix_attention_simt(plan.handle, q, k_new, v_new, cache_k, cache_v, out, stream),
@@ -314,26 +322,37 @@ def _ptr_array(ptrs):
     return arr
 
 
+def _ptr_arrays(n, seqs, optional=()):
+    """HOST arrays of per-layer pointers; a sequence at an index in `optional` may be None
+    (passed as a NULL array: e.g. cache_v for zero-copy values)."""
+    out = []
+    for i, x in enumerate(seqs):
+        if x is None and i in optional:
+            out.append(None)
+            continue
+        a = _ptr_array(x)
+        if len(a) != n:
+            raise ValueError("every per-layer pointer list needs one entry per layer")
+        out.append(C.cast(a, C.c_void_p))
+    return out
+
+
 def kvlink_linked_prefill_layers(plan: Plan, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out,
                                  workspace, workspace_bytes: int, stream: int = 0) -> None:
     """Every argument but the plan, workspace and stream: a sequence of per-layer device pointers."""
     n = len(pool_k)
-    arrs = [_ptr_array(x) for x in (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out)]
-    if any(len(a) != n for a in arrs):
-        raise ValueError("every per-layer pointer list needs one entry per layer")
-    _check(lib.kvlink_linked_prefill_layers(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs], workspace,
-                                            workspace_bytes, stream), "kvlink_linked_prefill_layers")
+    arrs = _ptr_arrays(n, (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out), optional=(6,))
+    _check(lib.kvlink_linked_prefill_layers(plan.handle, n, *arrs, workspace, workspace_bytes, stream),
+           "kvlink_linked_prefill_layers")
 
 
 def kvlink_linked_prefill_layers_overlapped(plan: Plan, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out,
                                             workspace, workspace_bytes: int, stream: int, reencode_stream: int) -> None:
     """As kvlink_linked_prefill_layers, with the re-encode on reencode_stream."""
     n = len(pool_k)
-    arrs = [_ptr_array(x) for x in (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out)]
-    if any(len(a) != n for a in arrs):
-        raise ValueError("every per-layer pointer list needs one entry per layer")
-    _check(lib.kvlink_linked_prefill_layers_overlapped(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs],
-                                                       workspace, workspace_bytes, stream, reencode_stream),
+    arrs = _ptr_arrays(n, (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out), optional=(6,))
+    _check(lib.kvlink_linked_prefill_layers_overlapped(plan.handle, n, *arrs, workspace, workspace_bytes, stream,
+                                                       reencode_stream),
            "kvlink_linked_prefill_layers_overlapped")
 
 
@@ -343,10 +362,8 @@ def kvlink_linked_prefill_layers_host(plan: Plan, pool_k, pool_v, h_q, h_k_new, 
     """Per-layer pointer sequences (h_*: host, the rest device); see include/kvlink.h."""
     n = len(pool_k)
     seqs = (pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new, cache_k, cache_v, out, h_out)
-    arrs = [_ptr_array(x) for x in seqs]
-    if any(len(a) != n for a in arrs):
-        raise ValueError("every per-layer pointer list needs one entry per layer")
-    _check(lib.kvlink_linked_prefill_layers_host(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs], workspace,
+    arrs = _ptr_arrays(n, seqs, optional=(9,))
+    _check(lib.kvlink_linked_prefill_layers_host(plan.handle, n, *arrs, workspace,
                                                  workspace_bytes, stream, reencode_stream, copy_in_stream,
                                                  copy_out_stream), "kvlink_linked_prefill_layers_host")
 
@@ -373,10 +390,8 @@ def kvlink_linked_prefill_layers_host_pool(plan: Plan, h_pool_k, h_pool_v, q, k_
 def kvlink_reencode_concat_layers(plan: Plan, pool_k, pool_v, cache_k, cache_v, stream: int = 0) -> None:
     """Every argument but the plan and stream: a sequence of per-layer device pointers."""
     n = len(pool_k)
-    arrs = [_ptr_array(x) for x in (pool_k, pool_v, cache_k, cache_v)]
-    if any(len(a) != n for a in arrs):
-        raise ValueError("every per-layer pointer list needs one entry per layer")
-    _check(lib.kvlink_reencode_concat_layers(plan.handle, n, *[C.cast(a, C.c_void_p) for a in arrs], stream),
+    arrs = _ptr_arrays(n, (pool_k, pool_v, cache_k, cache_v), optional=(1, 3))
+    _check(lib.kvlink_reencode_concat_layers(plan.handle, n, *arrs, stream),
            "kvlink_reencode_concat_layers")
 
 

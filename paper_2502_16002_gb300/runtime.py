@@ -21,6 +21,16 @@ def bits_from_bf16(t: torch.Tensor) -> np.ndarray:
     return t.detach().contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
 
 
+def _ptr(t):
+    """Device pointer of a tensor, or None (NULL) for None."""
+    return t.data_ptr() if t is not None else None
+
+
+def _ptr_seqs(seqs):
+    """Per-layer pointer lists; a None sequence stays None (a NULL array)."""
+    return [None if seq is None else [t.data_ptr() for t in seq] for seq in seqs]
+
+
 def _stream_handle(stream) -> int:
     if stream is None:
         stream = torch.cuda.current_stream()
@@ -96,8 +106,17 @@ class LinkedPrefill:
 
     # one ABI call each
     def reencode_concat(self, pool_k, pool_v, cache_k, cache_v, stream=None):
-        K.kvlink_reencode_concat(self.plan, pool_k.data_ptr(), pool_v.data_ptr(), cache_k.data_ptr(),
-                                 cache_v.data_ptr(), _stream_handle(stream))
+        """cache_v None: keys only (zero-copy values; pool_v is then not read)."""
+        K.kvlink_reencode_concat(self.plan, pool_k.data_ptr(), _ptr(pool_v), cache_k.data_ptr(),
+                                 _ptr(cache_v), _stream_handle(stream))
+
+    def suffix_attention_pool_values(self, q, k_new, v_new, pool_v, cache_k, out, stream=None):
+        """Suffix attention with zero-copy values: value rows read from pool_v and v_new
+        (k_new None: the fresh keys are already in cache_k)."""
+        K.kvlink_suffix_attention_pool_values(self.plan, q.data_ptr(), _ptr(k_new), v_new.data_ptr(),
+                                              pool_v.data_ptr(), cache_k.data_ptr(), out.data_ptr(),
+                                              self.workspace.data_ptr(), self.workspace.numel(),
+                                              _stream_handle(stream))
 
     def suffix_attention(self, q, k_new, v_new, cache_k, cache_v, out, stream=None):
         K.kvlink_suffix_attention(self.plan, q.data_ptr(),
@@ -120,7 +139,7 @@ class LinkedPrefill:
     def linked_prefill(self, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out, stream=None):
         K.kvlink_linked_prefill(self.plan, pool_k.data_ptr(), pool_v.data_ptr(), q.data_ptr(),
                                 k_new.data_ptr(), v_new.data_ptr(), cache_k.data_ptr(),
-                                cache_v.data_ptr(), out.data_ptr(), self.workspace.data_ptr(),
+                                _ptr(cache_v), out.data_ptr(), self.workspace.data_ptr(),
                                 self.workspace.numel(), _stream_handle(stream))
 
     def linked_prefill_fused(self, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out, stream=None):
@@ -133,8 +152,8 @@ class LinkedPrefill:
                                       self.workspace.data_ptr(), self.workspace.numel(), _stream_handle(stream))
 
     def linked_prefill_layers(self, pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out, stream=None):
-        """All layers in one ABI call (sequences of per-layer tensors)."""
-        ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out)]
+        """All layers in one ABI call (sequences of per-layer tensors; cache_v None: zero-copy values)."""
+        ptrs = _ptr_seqs((pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out))
         K.kvlink_linked_prefill_layers(self.plan, *ptrs, self.workspace.data_ptr(), self.workspace.numel(),
                                        _stream_handle(stream))
 
@@ -143,7 +162,7 @@ class LinkedPrefill:
         """All layers in one ABI call, the re-encode on a second stream (created if not given)."""
         if reencode_stream is None:
             reencode_stream = self._reencode_stream()
-        ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out)]
+        ptrs = _ptr_seqs((pool_k, pool_v, q, k_new, v_new, cache_k, cache_v, out))
         K.kvlink_linked_prefill_layers_overlapped(self.plan, *ptrs, self.workspace.data_ptr(), self.workspace.numel(),
                                                   _stream_handle(stream), _stream_handle(reencode_stream))
 
@@ -172,7 +191,7 @@ class LinkedPrefill:
 
     def reencode_concat_layers(self, pool_k, pool_v, cache_k, cache_v, stream=None):
         """The document caches of all layers in one launch (sequences of per-layer tensors)."""
-        ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, cache_k, cache_v)]
+        ptrs = _ptr_seqs((pool_k, pool_v, cache_k, cache_v))
         K.kvlink_reencode_concat_layers(self.plan, *ptrs, _stream_handle(stream))
 
     def linked_prefill_layers_from_host(self, pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new,
@@ -197,8 +216,7 @@ class LinkedPrefill:
         for seq in (h_q, h_k_new, h_v_new, h_out):
             if not all(t.is_pinned() for t in seq):
                 raise ValueError("host tensors must be pinned")
-        ptrs = [[t.data_ptr() for t in seq] for seq in (pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new,
-                                                      cache_k, cache_v, out, h_out)]
+        ptrs = _ptr_seqs((pool_k, pool_v, h_q, h_k_new, h_v_new, q, k_new, v_new, cache_k, cache_v, out, h_out))
         K.kvlink_linked_prefill_layers_host(self.plan, *ptrs, self.workspace.data_ptr(), self.workspace.numel(),
                                             _stream_handle(s_c), _stream_handle(self._reencode_stream()),
                                             _stream_handle(s_in), _stream_handle(s_out))

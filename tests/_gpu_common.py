@@ -29,7 +29,9 @@ def run_layer(RT, batch, layer, mode="fused", rows=None, layout=0, write_v=True)
     mode: "fused" = kvlink_linked_prefill (re-encode and attention kernels chained),
     "separate" = kvlink_reencode_concat then kvlink_suffix_attention,
     "onekernel" = kvlink_linked_prefill_fused (cache_v not written when write_v is False;
-    its bits are then returned as None)."""
+    its bits are then returned as None), "zero_copy" = kvlink_linked_prefill with cache_v
+    NULL (zero-copy values: keys re-encoded, values read from the pool and v_new; cache_v
+    bits returned as None)."""
     dev = torch.device("cuda:0")
     pk, pv = W.pool_kv(batch, layer)
     q, kn, vn = W.fresh_qkv(batch, layer)
@@ -39,8 +41,12 @@ def run_layer(RT, batch, layer, mode="fused", rows=None, layout=0, write_v=True)
     cv.view(torch.int16).fill_(-1)
     out = torch.full(lp.fresh_shape(batch.cfg.h_q), float("nan"), dtype=torch.bfloat16, device=dev)
     t = {k: RT.bf16_from_bits(v, dev) for k, v in dict(pk=pk, pv=pv, q=q, kn=kn, vn=vn).items()}
+    if mode == "zero_copy":
+        write_v = False
     if mode == "fused":
         lp.linked_prefill(t["pk"], t["pv"], t["q"], t["kn"], t["vn"], ck, cv, out)
+    elif mode == "zero_copy":
+        lp.linked_prefill(t["pk"], t["pv"], t["q"], t["kn"], t["vn"], ck, None, out)
     elif mode == "onekernel":
         lp.linked_prefill_fused(t["pk"], t["pv"], t["q"], t["kn"], t["vn"], ck, cv if write_v else None, out)
     else:

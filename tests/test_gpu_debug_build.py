@@ -5,7 +5,7 @@ destination against the plan's bounds before using it, and record a code in the 
 status word instead of touching memory through a bad entry.  On valid plans the checks
 must never fire and the results must be the release build's, bit for bit: every path
 (per-layer linked prefill, the overlapped all-layers call, split KV ranges and their
-merge, the paged pool, both cache layouts) runs once in a child process bound to the
+merge, the paged pool, both cache layouts, zero-copy values) runs once in a child process bound to the
 debug library and once here with the release library.
 """
 import os
@@ -45,6 +45,8 @@ for cfg_index, layout in {cases!r}:
     lp.linked_prefill_layers_overlapped(pk, pv, q, kn, vn, [c[0] for c in caches], [c[1] for c in caches], outs)
     ck, cv = lp.empty_cache(); o1 = torch.empty_like(q[0])
     lp.linked_prefill(pk[0], pv[0], q[0], kn[0], vn[0], ck, cv, o1)
+    ck2 = lp.empty_cache()[0]; o2 = torch.empty_like(q[0])
+    lp.linked_prefill(pk[0], pv[0], q[0], kn[0], vn[0], ck2, None, o2)     # zero-copy values
     torch.cuda.synchronize()
     assert K.kvlink_device_status() == 0, (cfg_index, layout, K.kvlink_device_status())
     for l in range(n_layers):
@@ -52,6 +54,8 @@ for cfg_index, layout in {cases!r}:
         res[f"{{cfg_index}}_{{layout}}_{{l}}_v"] = RT.bits_from_bf16(caches[l][1])
         res[f"{{cfg_index}}_{{layout}}_{{l}}_o"] = RT.bits_from_bf16(outs[l])
     res[f"{{cfg_index}}_{{layout}}_single_o"] = RT.bits_from_bf16(o1)
+    res[f"{{cfg_index}}_{{layout}}_zero_copy_o"] = RT.bits_from_bf16(o2)
+    assert np.array_equal(res[f"{{cfg_index}}_{{layout}}_zero_copy_o"], res[f"{{cfg_index}}_{{layout}}_single_o"])
 np.savez({out!r}, **res)
 print("ok")
 """
