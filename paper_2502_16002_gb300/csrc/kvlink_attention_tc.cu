@@ -82,20 +82,21 @@ static_assert(128 * (kPtSoftmaxRegs + kPtIdleRegsZv + 168) <= kPtThreads * 168, 
 template <int D, bool ZV = false>
 struct PtCfg {
     static constexpr int ATOMS = D / 64;
+    static constexpr int NQ = 2;
     static constexpr int NK = (D == 128) ? (ZV ? 2 : 3) : (ZV ? 4 : 5);
     static constexpr int NV = (D == 128) ? (ZV ? 3 : 2) : (ZV ? 5 : 4);
     static constexpr int NB = 3;
     static constexpr uint32_t ATOM_BYTES = 128 * 128;
     static constexpr uint32_t Q_BYTES = ATOMS * ATOM_BYTES, KV_BYTES = ATOMS * ATOM_BYTES;
     static constexpr uint32_t OFF_Q = 0;                                // two buffers
-    static constexpr uint32_t OFF_K = OFF_Q + 2 * Q_BYTES;
+    static constexpr uint32_t OFF_K = OFF_Q + NQ * Q_BYTES;
     static constexpr uint32_t OFF_V = OFF_K + NK * KV_BYTES;
     static constexpr uint32_t OFF_STATS = OFF_V + NV * KV_BYTES;        // m[128], l[128] of one item
     static constexpr uint32_t OFF_FLAG = OFF_STATS + 2 * kAttnBM * 4;   // the epilogue's merge decision
     static constexpr uint32_t OFF_BAR = OFF_FLAG + 16;
-    // q_full[2], q_empty[2], k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB],
+    // q_full[NQ], q_empty[NQ], k_full[NK], k_empty[NK], v_full[NV], v_empty[NV], s_full[NB],
     // p_full[NB], o_done[NB], o_full, o_free, st_full, st_empty, drain x2
-    static constexpr int N_BARS = 4 + 2 * NK + 2 * NV + 3 * NB + 6;
+    static constexpr int N_BARS = 2 * NQ + 2 * NK + 2 * NV + 3 * NB + 6;
     static constexpr uint32_t SMEM_BYTES = OFF_BAR + N_BARS * 8 + 16 + 1024;
     static constexpr uint32_t TMEM_S = 0, TMEM_O = NB * kAttnBN;
     static_assert(TMEM_O + D <= kTmemCols, "TMEM budget");
@@ -375,9 +376,10 @@ __global__ void __launch_bounds__(kPtThreads, 1)
     uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
 
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
-    uint64_t* bar_q_full = bars;                 // [2]
-    uint64_t* bar_q_empty = bar_q_full + 2;      // [2]
-    uint64_t* bar_k_full = bar_q_empty + 2;
+    constexpr int NQ = C::NQ;
+    uint64_t* bar_q_full = bars;                 // [NQ]
+    uint64_t* bar_q_empty = bar_q_full + NQ;     // [NQ]
+    uint64_t* bar_k_full = bar_q_empty + NQ;
     uint64_t* bar_k_empty = bar_k_full + NK;
     uint64_t* bar_v_full = bar_k_empty + NK;
     uint64_t* bar_v_empty = bar_v_full + NV;
@@ -455,9 +457,9 @@ __global__ void __launch_bounds__(kPtThreads, 1)
             for (int k = 0; ok && k < n_mine; ++k) {
                 const AttnItem it = P.items[P.sched[first + k]];
                 const int n = it.kv_tile1 - it.kv_tile0, ctx0 = (int)P.cu_ctx[it.query];
-                // Q buffer k % 2, once the S MMAs of item k - 2 have read it
-                const int qb = k & 1;
-                if (!(ok = wait_bar(bar_q_empty + qb, ((k >> 1) & 1) ^ 1, abort_flag, status))) break;
+                // Q buffer k % NQ, once the S MMAs of item k - NQ have read it
+                const int qb = k % NQ;
+                if (!(ok = wait_bar(bar_q_empty + qb, ((k / NQ) & 1) ^ 1, abort_flag, status))) break;
                 mbar_arrive_expect_tx(bar_q_full + qb, C::Q_BYTES);
 #pragma unroll
                 for (int a = 0; a < C::ATOMS; ++a)
@@ -477,8 +479,8 @@ __global__ void __launch_bounds__(kPtThreads, 1)
             }
             // no copy may still be in flight when the CTA leaves
             for (int gg = g - NK > 0 ? g - NK : 0; gg < g; ++gg) drain_bar(bar_k_full + gg % NK, (gg / NK) & 1, status);
-            for (int k = q_issued - 2 > 0 ? q_issued - 2 : 0; k < q_issued; ++k)
-                drain_bar(bar_q_full + (k & 1), (k >> 1) & 1, status);
+            for (int k = q_issued - NQ > 0 ? q_issued - NQ : 0; k < q_issued; ++k)
+                drain_bar(bar_q_full + k % NQ, (k / NQ) & 1, status);
         } else if (warp == kTmaVWarp && ZV) {
             // ------------------------------------------------ the V ring, values where they are
             if constexpr (ZV)
@@ -511,8 +513,8 @@ __global__ void __launch_bounds__(kPtThreads, 1)
             for (int k = 0; ok && k < n_mine; ++k) {
                 const AttnItem it = P.items[P.sched[first + k]];
                 const int n = it.kv_tile1 - it.kv_tile0;
-                const int qb = k & 1;
-                if (!(ok = wait_bar(bar_q_full + qb, (k >> 1) & 1, abort_flag, status))) break;
+                const int qb = k % NQ;
+                if (!(ok = wait_bar(bar_q_full + qb, (k / NQ) & 1, abort_flag, status))) break;
                 const uint32_t sQ = smem_u32(smem + C::OFF_Q + qb * C::Q_BYTES);
                 for (int j = 0; j < n; ++j, ++g) {
                     const int sk = g % NK, b = g % NB;
