@@ -56,7 +56,18 @@ KERNEL_SOURCES = {
     "reencode": ["kvlink_reencode.cu", "kvlink_rope.cuh", "kvlink_sm100.cuh", "kvlink_internal.h",
                  "kvlink_plan.cpp"],
 }
-NCU_TRAFFIC = {}    # (kernel, workload index) -> (bytes per launch, source hash)
+# Captures: `ncu --set full` of one launch per kernel, on runs of this script with one or two
+# layers (each launch does a layer's full work); the zero-copy kernels on workload 3 only.
+NCU_TRAFFIC = {
+    ("attention", 3): (236_843_008 + 7_807_744, "fdb2b68e943dfb12"),
+    ("attention", 4): (269_369_088 + 6_317_824, "fdb2b68e943dfb12"),
+    ("attention", 5): (1_707_568_000 + 59_075_840, "fdb2b68e943dfb12"),
+    ("reencode", 3): (102_327_040 + 113_514_752, "7beb3ba7cc6232e6"),
+    ("attention_pool_values", 3): (174_838_784 + 6_245_888, "fdb2b68e943dfb12"),
+    ("reencode_keys", 3): (40_685_312 + 25_736_704, "7beb3ba7cc6232e6"),
+}
+KERNEL_SOURCES["attention_pool_values"] = KERNEL_SOURCES["attention"]
+KERNEL_SOURCES["reencode_keys"] = KERNEL_SOURCES["reencode"]
 
 
 def source_hash(kernel: str) -> str:
@@ -409,6 +420,8 @@ class Workload:
                 "attention_pool_values_us_per_launch": round(t_at * 1e6, 2),
                 "attention_pool_values_TFLOP_per_s": round(at_tfs, 2),
                 "attention_pool_values_frac_bf16_burst": round(at_tfs / peaks["bf16_tflops"], 4),
+                "reencode_keys_traffic": ncu_traffic("reencode_keys", self.cfg.index),
+                "attention_pool_values_traffic": ncu_traffic("attention_pool_values", self.cfg.index),
                 "launches_per_step": 3 * self.L,
                 "note": "kvlink_linked_prefill_layers_overlapped with cache_v NULL: keys re-encoded into "
                         "the linked cache, values read by the attention from the pool and v_new (no "
