@@ -665,7 +665,8 @@ def main():
     for c in args.extra_configs:
         r = run_ours(args, rank, world, local_rank, c, main=False)
         extra[r["config"]["workload"]] = {k: r[k] for k in ("value", "unit", "ms_per_step", "steps", "config",
-                                                             "roofline", "kernels", "clocks", "gpu_launches")}
+                                                             "roofline", "kernels", "clocks", "gpu_launches",
+                                                             "zero_copy_values")}
     if extra:
         res["workloads"] = extra
     if rank == 0:
