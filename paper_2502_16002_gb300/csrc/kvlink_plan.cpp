@@ -301,8 +301,8 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         }
     }
     // ---- work items and the persistent attention's schedule.
-    // Costs are in half tiles: two per key tile, one for an item's own start and finish.  Two
-    // schedules are built and the one with the shorter estimated time is kept:
+    // Costs are in half tiles: two per key tile, one for an item's own start and finish.  The
+    // schedules below are built and the one with the shorter estimated time is kept:
     //  A  whole M-tiles in launch order, each to the CTA with the least work so far (list
     //     scheduling; also tried longest first over all M-tiles).  The launch order keeps the
     //     M-tiles of one (query, KV head) together, groups with the longest M-tile first, so
@@ -321,6 +321,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     //     the merge (epilogue work that also takes issue slots from the softmax), so B is also
     //     tried with shares 5% and 10% above the mean, where fewer M-tiles are cut.  One long
     //     query (M-tiles of a few hundred key tiles) needs B.
+    //  G  gangs (below): every group whole on one gang of CTAs, for many short M-tiles.
     // Small batches use fewer CTAs (at least kMinShare half tiles each) and never cut a piece
     // under kMinPiece key tiles.
     struct Sched {
@@ -407,6 +408,40 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         return s;
     };
 
+    // G: gangs of S CTAs.  Every (query, KV head) group goes whole to one gang (the gang with
+    // the least work, groups by decreasing work), its M-tiles to the gang's CTAs with the least
+    // work, so the CTAs of a gang run the same group's M-tiles at about the same time and read
+    // its K/V tiles once from DRAM between them (the others hit L2).
+    auto schedule_gang = [&](const std::vector<Tile>& order, int32_t S) {
+        Sched s;
+        s.lists.assign((size_t)n_ctas, {});
+        const int32_t n_gangs = n_ctas / S;
+        std::vector<int64_t> load((size_t)n_ctas, 0);
+        std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> gangs;   // (work, gang)
+        for (int32_t q = 0; q < n_gangs; ++q) gangs.push({0, q});
+        for (size_t i = 0; i < order.size();) {
+            size_t j = i;
+            while (j < order.size() && order[j].b == order[i].b && order[j].g == order[i].g) ++j;
+            const Slot gs = gangs.top();
+            gangs.pop();
+            const int32_t c0 = gs.second * S;
+            for (size_t k = i; k < j; ++k) {
+                int32_t c = c0;
+                for (int32_t x = c0 + 1; x < c0 + S; ++x)
+                    if (load[(size_t)x] < load[(size_t)c]) c = x;
+                s.lists[(size_t)c].push_back((int32_t)s.items.size());
+                s.items.push_back(item_of(order[k], 0, order[k].n_tiles));
+                load[(size_t)c] += 2 * (int64_t)order[k].n_tiles + 1;
+            }
+            int64_t gl = 0;
+            for (int32_t x = c0; x < c0 + S; ++x) gl = std::max(gl, load[(size_t)x]);
+            gangs.push({gl, gs.second});
+            i = j;
+        }
+        s.span = *std::max_element(load.begin(), load.end());
+        return s;
+    };
+
     std::vector<int64_t> longest_in_group((size_t)B * d->h_kv, 0), tiles_in_group((size_t)B * d->h_kv, 0);
     int64_t longest = 0;
     for (const Tile& t : tiles) {
@@ -481,6 +516,27 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
     for (int slack : {0, 5, 10}) {
         Sched capped = schedule_capped(by_group(tiles_in_group, false), slack);
         if (capped.span * 100 < best.span * 97) best = std::move(capped);
+    }
+    // Many short M-tiles per CTA: the list schedules scatter a group's M-tiles over time and the
+    // attention turns DRAM-bound on re-read K/V tiles; gangs of as many CTAs as a group has
+    // M-tiles (at most 8) keep them together.  Taken when the CTAs run at least four M-tiles each
+    // and the gangs' estimated time is within 10 % of the best, which the shared K/V tiles more
+    // than repay: workload 5 (64 queries, 2096 M-tiles of about 23 key tiles, estimate 596
+    // against 562) measured 258.9 against 291.1 us per layer with gangs of 6 (gangs of 2: 298.2,
+    // 4: 259.1, 8: 253.9 with a slower step); forced on workloads 3 and 4 (384 and 160 M-tiles,
+    // estimates 21 % and 121 % above the best) gangs measured 93.8 against 81.9 and 454 against
+    // 226 us.
+    {
+        constexpr int64_t kGangMinItemsPerCta = 4;
+        constexpr int64_t kGangSlackPct = 10;
+        int32_t mt_max = 0;
+        std::vector<int32_t> mt_in_group((size_t)B * d->h_kv, 0);
+        for (const Tile& t : tiles) mt_max = std::max(mt_max, ++mt_in_group[(size_t)t.b * d->h_kv + t.g]);
+        const int32_t S = std::min<int32_t>(mt_max, 8);
+        if (S >= 2 && n_ctas >= 4 * S && (int64_t)tiles.size() >= kGangMinItemsPerCta * (int64_t)n_ctas) {
+            Sched gang = schedule_gang(by_group(tiles_in_group, false), S);
+            if (gang.span * 100 <= best.span * (100 + kGangSlackPct)) best = std::move(gang);
+        }
     }
 
     p->items.swap(best.items);
