@@ -274,7 +274,7 @@ __device__ __forceinline__ void gather_role(const AttnItem& it, const DevicePlan
                         for (int q = 0; q < 8; ++q) cs[q] = __ldg(tb + q);
                         cur_table = e.table;
                     }
-                    rotate8(a, b, cs);
+                    rotate8<false>(a, b, cs);
                     *reinterpret_cast<uint4*>(sk + o_lo) = a;
                     *reinterpret_cast<uint4*>(sk + o_hi) = b;
                 }

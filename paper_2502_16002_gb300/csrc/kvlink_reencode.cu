@@ -276,7 +276,7 @@ __global__ void __launch_bounds__(kCopyThreads, 1) reencode_kernel(
                     const uint8_t* src = stage + (uint32_t)t * row_bytes + lo_off;
                     uint4 a = *reinterpret_cast<const uint4*>(src);
                     uint4 b = *reinterpret_cast<const uint4*>(src + D);
-                    rotate8(a, b, cs);
+                    rotate8<!WV>(a, b, cs);
                     uint8_t* d = dst + (size_t)t * row_bytes;
                     *reinterpret_cast<uint4*>(d) = a;
                     *reinterpret_cast<uint4*>(d + D) = b;
@@ -441,7 +441,7 @@ __global__ void __launch_bounds__(32 * kHostWarps) reencode_host_kernel(
 #pragma unroll
                     for (int i = 0; i < kHostPairsPerLane; ++i)
                         if (has[i] && t0 + u < ch.n) {
-                            if (rot) rotate8(k[u][i][0], k[u][i][1], cs[i]);
+                            if (rot) rotate8<false>(k[u][i][0], k[u][i][1], cs[i]);
                             cache_k[dst + lo_idx[i]] = k[u][i][0];
                             cache_k[dst + lo_idx[i] + D / 16] = k[u][i][1];
                             cache_v[dst + lo_idx[i]] = v[u][i][0];

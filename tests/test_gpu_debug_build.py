@@ -55,7 +55,6 @@ for cfg_index, layout in {cases!r}:
         res[f"{{cfg_index}}_{{layout}}_{{l}}_o"] = RT.bits_from_bf16(outs[l])
     res[f"{{cfg_index}}_{{layout}}_single_o"] = RT.bits_from_bf16(o1)
     res[f"{{cfg_index}}_{{layout}}_zero_copy_o"] = RT.bits_from_bf16(o2)
-    assert np.array_equal(res[f"{{cfg_index}}_{{layout}}_zero_copy_o"], res[f"{{cfg_index}}_{{layout}}_single_o"])
 np.savez({out!r}, **res)
 print("ok")
 """

@@ -4,9 +4,16 @@ Sec. 2.3 ("inference") concatenates the cached values unchanged, so they need no
 copied: with cache_v NULL the re-encode writes keys only and the persistent attention reads
 every value row where it already is (the pool's rows for the prefix and the documents, v_new
 for the link and question rows), through the plan's 8-row group table and row-by-row copies
-at segment boundaries.  The tiles and the order of operations are those of the path with a
-linked value cache, so the output must equal that path's bit for bit; it is also checked
-against the fp64 oracle (max |err| <= 1e-2, mean |err| <= 1e-3; keys within 1 bf16 ulp).
+at segment boundaries.  Checks:
+  - the keys are within one bf16 ulp of the fp64 oracle (the keys-only re-encode rotates with
+    a faster form than the value path, so the two may round a key one ulp apart: within one
+    ulp of each other too);
+  - the attention over those keys equals, bit for bit, the value-cache attention
+    (kvlink_suffix_attention) run on the same keys with the value cache built by the value
+    path: the same tiles and the same order of operations, only the value rows come from
+    elsewhere;
+  - the output is within the attention tolerance of the fp64 oracle (max |err| <= 1e-2,
+    mean |err| <= 1e-3).
 """
 import numpy as np
 import pytest
@@ -16,7 +23,7 @@ import workloads as W
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
-from _gpu_common import EDGE, LAYOUTS, check_query, custom_batch, run_layer  # noqa: E402
+from _gpu_common import EDGE, LAYOUTS, check_query, custom_batch, ulp_distance  # noqa: E402
 
 
 @pytest.fixture(scope="module")
@@ -28,19 +35,34 @@ def RT():
     return runtime
 
 
-def _bits_equal(a, b):
-    """Outputs returned by run_layer (bf16 widened to float64): equal bit for bit."""
-    assert a.shape == b.shape
-    assert np.array_equal(a, b) and np.array_equal(np.signbit(a), np.signbit(b))
-
-
 def _both(RT, batch, layer, layout=0):
-    ref = run_layer(RT, batch, layer, "fused", layout=layout)
-    zc = run_layer(RT, batch, layer, "zero_copy", layout=layout)
-    assert zc[2] is None
-    assert np.array_equal(ref[1], zc[1]), "keys differ from the path with a value cache"
-    _bits_equal(ref[3], zc[3])
-    return zc
+    """One layer with the value cache and with zero-copy values.  Returns what
+    _gpu_common.check_query takes for the zero-copy run (value bits None)."""
+    from paper_2502_16002_gb300 import kvlink as K
+    dev = torch.device("cuda:0")
+    pk, pv = W.pool_kv(batch, layer)
+    q, kn, vn = W.fresh_qkv(batch, layer)
+    t = {k: RT.bf16_from_bits(v, dev) for k, v in dict(pk=pk, pv=pv, q=q, kn=kn, vn=vn).items()}
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev, layout=layout)
+    ck, cv = lp.empty_cache()
+    ck.view(torch.int16).fill_(-1)
+    cv.view(torch.int16).fill_(-1)
+    out = torch.full(lp.fresh_shape(batch.cfg.h_q), float("nan"), dtype=torch.bfloat16, device=dev)
+    lp.linked_prefill(t["pk"], t["pv"], t["q"], t["kn"], t["vn"], ck, cv, out)
+    zk = torch.empty_like(ck)
+    zk.view(torch.int16).fill_(-1)
+    zout = torch.full_like(out, float("nan"))
+    lp.linked_prefill(t["pk"], t["pv"], t["q"], t["kn"], t["vn"], zk, None, zout)
+    # the value-cache attention over the zero-copy keys
+    same = torch.full_like(out, float("nan"))
+    lp.suffix_attention(t["q"], None, None, zk, cv, same)
+    torch.cuda.synchronize(dev)
+    assert K.kvlink_device_status() == 0
+    gk, gz = RT.bits_from_bf16(ck), RT.bits_from_bf16(zk)
+    assert ulp_distance(gk, gz).max() <= 1, "keys more than one ulp from the value path's"
+    assert torch.equal(same.view(torch.int16), zout.view(torch.int16)), "attention differs from the value-cache path"
+    zo = zout.float().cpu().numpy().astype(np.float64)
+    return lp, gz, None, zo, (pk, pv, q, kn, vn)
 
 
 @pytest.mark.parametrize("layout", sorted(LAYOUTS))
@@ -98,7 +120,8 @@ def _layer_tensors(RT, batch, L, dev):
 
 
 def test_overlapped_layers(RT):
-    """The step's call with cache_v NULL: the same keys and outputs as with a value cache."""
+    """The step's call with cache_v NULL: keys within one ulp of the value-cache call's, and per
+    layer the same output bits as the value-cache attention over those keys."""
     batch = W.draw_batch(W.get_config(3))
     dev = torch.device("cuda:0")
     L = 3
@@ -112,11 +135,17 @@ def test_overlapped_layers(RT):
                                             [c[1] for c in caches] if with_v else None, out)
         torch.cuda.synchronize()
         runs.append(([c[0] for c in caches], out))
+        if with_v:
+            values = [c[1] for c in caches]
     from paper_2502_16002_gb300 import kvlink as K
     assert K.kvlink_device_status() == 0
     for layer in range(L):
-        assert torch.equal(runs[0][0][layer].view(torch.int16), runs[1][0][layer].view(torch.int16))
-        assert torch.equal(runs[0][1][layer].view(torch.int16), runs[1][1][layer].view(torch.int16))
+        zk, zout = runs[1][0][layer], runs[1][1][layer]
+        assert ulp_distance(RT.bits_from_bf16(runs[0][0][layer]), RT.bits_from_bf16(zk)).max() <= 1
+        same = torch.full_like(zout, float("nan"))
+        lp.suffix_attention(q[layer], None, None, zk, values[layer], same)
+        torch.cuda.synchronize()
+        assert torch.equal(same.view(torch.int16), zout.view(torch.int16))
 
 
 def test_suffix_attention_pool_values(RT):
@@ -135,8 +164,11 @@ def test_suffix_attention_pool_values(RT):
     out = torch.full_like(ref, float("nan"))
     lp.reencode_concat(pk, None, ck2, None)
     lp.suffix_attention_pool_values(q, kn, vn, pv, ck2, out)
+    # the value-cache attention over the keys-only cache (its fresh rows are placed now)
+    ref = torch.full_like(out, float("nan"))
+    lp.suffix_attention(q, None, None, ck2, cv, ref)
     torch.cuda.synchronize()
-    assert torch.equal(ck.view(torch.int16), ck2.view(torch.int16))
+    assert ulp_distance(RT.bits_from_bf16(ck), RT.bits_from_bf16(ck2)).max() <= 1
     assert torch.equal(ref.view(torch.int16), out.view(torch.int16))
     # fresh keys already in the cache: k_new NULL
     out2 = torch.full_like(ref, float("nan"))
@@ -159,11 +191,14 @@ def test_reencode_layers_keys_only(RT):
     lp.reencode_concat_layers(pk, None, keys, None)
     torch.cuda.synchronize()
     for layer in range(L):
-        assert torch.equal(full[layer][0].view(torch.int16), keys[layer].view(torch.int16))
+        # the keys-only launch rotates with the fast form: within one ulp of the value path's
+        assert ulp_distance(RT.bits_from_bf16(full[layer][0]), RT.bits_from_bf16(keys[layer])).max() <= 1
 
 
 def test_host_path(RT):
-    """kvlink_linked_prefill_layers_host with cache_v NULL: the same outputs on the host."""
+    """kvlink_linked_prefill_layers_host with cache_v NULL: per layer, the output on the host
+    equals the value-cache attention over the call's keys, with the value cache of the same
+    call made with cache_v."""
     batch = W.draw_batch(W.get_config(2))
     dev = torch.device("cuda:0")
     L = 2
@@ -172,7 +207,7 @@ def test_host_path(RT):
     qh = [t.cpu().pin_memory() for t in q]
     kh = [t.cpu().pin_memory() for t in kn]
     vh = [t.cpu().pin_memory() for t in vn]
-    outs = []
+    runs = []
     for with_v in (True, False):
         dq = [torch.empty_like(t) for t in q]
         dk = [torch.empty_like(t) for t in kn]
@@ -182,6 +217,10 @@ def test_host_path(RT):
         hout = [torch.empty(t.shape, dtype=torch.bfloat16).pin_memory() for t in q]
         lp.linked_prefill_layers_from_host(pk, pv, qh, kh, vh, dq, dk, dv, [c[0] for c in caches],
                                            [c[1] for c in caches] if with_v else None, dout, hout)
-        outs.append(hout)
+        runs.append((caches, hout))
     for layer in range(L):
-        assert torch.equal(outs[0][layer].view(torch.int16), outs[1][layer].view(torch.int16))
+        zk, hz = runs[1][0][layer][0], runs[1][1][layer]
+        same = torch.full_like(q[layer], float("nan"))
+        lp.suffix_attention(q[layer], None, None, zk, runs[0][0][layer][1], same)
+        torch.cuda.synchronize()
+        assert torch.equal(same.cpu().view(torch.int16), hz.view(torch.int16))
