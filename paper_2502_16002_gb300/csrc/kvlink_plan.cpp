@@ -331,11 +331,12 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         int32_t n_slots = 0;
         int64_t span = 0;
     };
-    constexpr int64_t kMinShare = 2 * 8 + 1;
+    constexpr int64_t kItemCost = 1;   // half tiles for an item's start and finish (4, 8, 14: no change)
+    constexpr int64_t kMinShare = 2 * 8 + kItemCost;
     constexpr int32_t kMinPiece = 4;
     constexpr int64_t kMergeCost = 14;
     int64_t total = 0;
-    for (const Tile& t : tiles) total += 2 * (int64_t)t.n_tiles + 1;
+    for (const Tile& t : tiles) total += 2 * (int64_t)t.n_tiles + kItemCost;
     const int32_t n_ctas = (int32_t)std::max<int64_t>(1, std::min<int64_t>(num_sms, total / kMinShare));
     using Slot = std::pair<int64_t, int32_t>;      // (work so far, CTA)
     auto item_of = [](const Tile& t, int32_t a, int32_t e) {
@@ -354,7 +355,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
             least.pop();
             s.lists[(size_t)sl.second].push_back((int32_t)s.items.size());
             s.items.push_back(item_of(t, 0, t.n_tiles));
-            const int64_t load = sl.first + 2 * (int64_t)t.n_tiles + 1;
+            const int64_t load = sl.first + 2 * (int64_t)t.n_tiles + kItemCost;
             s.span = std::max(s.span, load);
             least.push({load, sl.second});
         }
@@ -367,7 +368,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         std::vector<int32_t> pieces_on((size_t)n_ctas, 0);
         // the equal share, plus room for the starts of two more pieces and slack_pct percent:
         // with slack, an M-tile is cut only where a CTA would otherwise end well past the mean
-        int64_t share = (total + n_ctas - 1) / n_ctas * (100 + slack_pct) / 100 + 2;
+        int64_t share = (total + n_ctas - 1) / n_ctas * (100 + slack_pct) / 100 + 2 * kItemCost;
         std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> least;
         for (int32_t c = 0; c < n_ctas; ++c) least.push({0, c});
         for (const Tile& t : order) {
@@ -376,11 +377,11 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
             int32_t done = 0;
             while (done < t.n_tiles) {
                 // every CTA full (a cut adds a start the shares did not count): all shares grow
-                while (least.top().first + 3 > share) share += 2;
+                while (least.top().first + kItemCost + 2 > share) share += 2;
                 const Slot sl = least.top();
                 least.pop();
                 const int32_t rest = t.n_tiles - done;
-                int32_t m = (int32_t)std::min<int64_t>(rest, (share - sl.first - 1) / 2);
+                int32_t m = (int32_t)std::min<int64_t>(rest, (share - sl.first - kItemCost) / 2);
                 // no piece under kMinPiece key tiles: the CTA rather runs a little past its share
                 if (m < rest) {
                     if (m < kMinPiece) m = std::min(rest, kMinPiece);
@@ -389,7 +390,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
                 s.lists[(size_t)sl.second].push_back((int32_t)s.items.size());
                 s.items.push_back(item_of(t, done, done + m));
                 ctas.push_back(sl.second);
-                least.push({sl.first + 2 * (int64_t)m + 1, sl.second});
+                least.push({sl.first + 2 * (int64_t)m + kItemCost, sl.second});
                 done += m;
             }
             const int32_t n_split = (int32_t)(s.items.size() - first_piece);
@@ -431,7 +432,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
                     if (load[(size_t)x] < load[(size_t)c]) c = x;
                 s.lists[(size_t)c].push_back((int32_t)s.items.size());
                 s.items.push_back(item_of(order[k], 0, order[k].n_tiles));
-                load[(size_t)c] += 2 * (int64_t)order[k].n_tiles + 1;
+                load[(size_t)c] += 2 * (int64_t)order[k].n_tiles + kItemCost;
             }
             int64_t gl = 0;
             for (int32_t x = c0; x < c0 + S; ++x) gl = std::max(gl, load[(size_t)x]);
@@ -485,7 +486,8 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
         Sched r = best;
         std::vector<int64_t> load((size_t)n_ctas, 0);
         for (int32_t c = 0; c < n_ctas; ++c)
-            for (int32_t i : r.lists[(size_t)c]) load[(size_t)c] += 2 * (int64_t)(r.items[(size_t)i].kv_tile1 - r.items[(size_t)i].kv_tile0) + 1;
+            for (int32_t i : r.lists[(size_t)c])
+                load[(size_t)c] += 2 * (int64_t)(r.items[(size_t)i].kv_tile1 - r.items[(size_t)i].kv_tile0) + kItemCost;
         for (int32_t step = 0; step < n_ctas; ++step) {
             const int32_t hi = (int32_t)(std::max_element(load.begin(), load.end()) - load.begin());
             const int32_t lo = (int32_t)(std::min_element(load.begin(), load.end()) - load.begin());
@@ -508,7 +510,7 @@ int build_plan(const kvlink_batch_desc_t* d, int32_t num_sms, kvlink_plan* p, st
             r.lists[(size_t)lo].push_back((int32_t)r.items.size());
             r.items.push_back(moved);
             load[(size_t)hi] += -2 * (int64_t)x + kMergeCost;
-            load[(size_t)lo] += 2 * (int64_t)x + 1 + kMergeCost;
+            load[(size_t)lo] += 2 * (int64_t)x + kItemCost + kMergeCost;
         }
         r.span = *std::max_element(load.begin(), load.end());
         if (r.span * 100 < best.span * 97) best = std::move(r);
