@@ -59,12 +59,12 @@ KERNEL_SOURCES = {
 # Captures: `ncu --set full` of one launch per kernel, on runs of this script with one or two
 # layers (each launch does a layer's full work); the zero-copy kernels on workload 3 only.
 NCU_TRAFFIC = {
-    ("attention", 3): (236_843_008 + 7_807_744, "fdb2b68e943dfb12"),
-    ("attention", 4): (269_369_088 + 6_317_824, "fdb2b68e943dfb12"),
-    ("attention", 5): (1_707_568_000 + 59_075_840, "fdb2b68e943dfb12"),
-    ("reencode", 3): (102_327_040 + 113_514_752, "7beb3ba7cc6232e6"),
-    ("attention_pool_values", 3): (174_838_784 + 6_245_888, "fdb2b68e943dfb12"),
-    ("reencode_keys", 3): (40_685_312 + 25_736_704, "7beb3ba7cc6232e6"),
+    ("attention", 3): (237_301_760 + 8_349_696, "2227415ce887690a"),
+    ("attention", 4): (283_856_640 + 6_546_176, "2227415ce887690a"),
+    ("attention", 5): (873_828_096 + 56_577_792, "2227415ce887690a"),
+    ("reencode", 3): (102_178_560 + 113_795_072, "d3ba56d5b4506e2b"),
+    ("attention_pool_values", 3): (175_213_056 + 6_225_664, "2227415ce887690a"),
+    ("reencode_keys", 3): (40_691_456 + 25_600_000, "d3ba56d5b4506e2b"),
 }
 KERNEL_SOURCES["attention_pool_values"] = KERNEL_SOURCES["attention"]
 KERNEL_SOURCES["reencode_keys"] = KERNEL_SOURCES["reencode"]
