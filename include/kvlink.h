@@ -201,6 +201,23 @@ int kvlink_plan_get_fresh_positions(const kvlink_plan_t* plan, int32_t* fresh_po
  * Errors: EINVAL, ECAPACITY. */
 int kvlink_plan_get_sources(const kvlink_plan_t* plan, kvlink_source_t* src, int64_t cap);
 
+/* One work item of the persistent suffix attention: the fresh tokens [tok0, tok1) of query
+ * `query` (query-relative) with the query heads of KV head `kv_head` (an M-tile), over the
+ * entries [entry0, entry1) of the M-tile's key-tile list (entry e < a_tiles is key tile e of
+ * the query's linked cache; entry a_tiles + i is key tile b_tile0 + i, the fresh rows at the
+ * end of the links-at-end layout), run by CTA `cta`.  slot >= 0: the item is one piece of a
+ * cut key range and writes a partial result to that workspace slot. */
+typedef struct {
+    int32_t query, kv_head, tok0, tok1;
+    int32_t entry0, entry1, a_tiles, b_tile0;
+    int32_t slot, cta;
+} kvlink_attn_item_t;
+
+/* items: [cap] work items in the order the CTAs run them (CTA 0's list first); one per
+ * scheduled item (n_attn_items of them).  Plan introspection: the schedule is the plan's
+ * business, this exposes it for checks and tuning.  Errors: EINVAL, ECAPACITY. */
+int kvlink_plan_get_attention_items(const kvlink_plan_t* plan, kvlink_attn_item_t* items, int32_t cap);
+
 /* Copy the plan's tables to the caller's device buffer d_buf (>= device_bytes,
  * 256-byte aligned) and build the RoPE delta table there: cos and sin of
  * delta_i * theta^(-2j/D) for every cached document i and j < D/2, with the angle

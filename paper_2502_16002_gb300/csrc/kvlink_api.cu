@@ -264,6 +264,19 @@ int kvlink_plan_get_sources(const kvlink_plan_t* p, kvlink_source_t* src, int64_
     return KVLINK_OK;
 }
 
+int kvlink_plan_get_attention_items(const kvlink_plan_t* p, kvlink_attn_item_t* items, int32_t cap) {
+    if (!p || !items) return KVLINK_EINVAL;
+    if (cap < (int32_t)p->sched.size()) return KVLINK_ECAPACITY;
+    int32_t k = 0;
+    for (size_t c = 0; c + 1 < p->cu_sched.size(); ++c)
+        for (int32_t s = p->cu_sched[c]; s < p->cu_sched[c + 1]; ++s) {
+            const AttnItem& it = p->items[(size_t)p->sched[(size_t)s]];
+            items[k++] = kvlink_attn_item_t{it.query,   it.kv_head,  it.tok0, it.tok1,       it.kv_tile0,
+                                            it.kv_tile1, it.a_tiles, it.b_tile0, it.slot, (int32_t)c};
+        }
+    return KVLINK_OK;
+}
+
 int kvlink_plan_upload(kvlink_plan_t* p, double theta, void* d_buf, size_t bytes, kvlink_stream_t stream) {
     if (!p || !d_buf) return KVLINK_EINVAL;
     if (!(theta > 1.0)) return KVLINK_EINVAL;

@@ -94,6 +94,7 @@ def _load():
         "kvlink_plan_get_offsets": (C.c_int, [P, V, V]),
         "kvlink_plan_get_fresh_positions": (C.c_int, [P, V, C.c_int32]),
         "kvlink_plan_get_sources": (C.c_int, [P, V, C.c_int64]),
+        "kvlink_plan_get_attention_items": (C.c_int, [P, V, C.c_int32]),
         "kvlink_plan_upload": (C.c_int, [P, C.c_double, V, C.c_size_t, V]),
         "kvlink_reencode_concat": (C.c_int, [P, V, V, V, V, V]),
         "kvlink_suffix_attention": (C.c_int, [P, V, V, V, V, V, V, V, C.c_size_t, V]),
@@ -134,7 +135,7 @@ DECLARED = [
     "kvlink_plan_get_sources", "kvlink_linked_prefill_fused", "kvlink_linked_prefill_layers",
     "kvlink_reencode_concat_layers", "kvlink_plan_rebuild", "kvlink_linked_prefill_layers_overlapped",
     "kvlink_linked_prefill_layers_host", "kvlink_reencode_concat_host_pool", "kvlink_linked_prefill_layers_host_pool",
-    "kvlink_selftest_wait_timeout", "kvlink_suffix_attention_pool_values",
+    "kvlink_selftest_wait_timeout", "kvlink_suffix_attention_pool_values", "kvlink_plan_get_attention_items",
 ]
 
 # size of the static scratch used by kvlink_suffix_attention_noalloc (include/kvlink.h)
@@ -259,6 +260,18 @@ def kvlink_plan_get_sources(plan: Plan) -> np.ndarray:
     n = kvlink_plan_get_info(plan).ctx_rows
     out = np.zeros(n, dtype=SOURCE_DTYPE)
     _check(lib.kvlink_plan_get_sources(plan.handle, out.ctypes.data, n), "kvlink_plan_get_sources")
+    return out
+
+
+ATTN_ITEM_DTYPE = np.dtype([(n, np.int32) for n in ("query", "kv_head", "tok0", "tok1", "entry0", "entry1",
+                                                      "a_tiles", "b_tile0", "slot", "cta")])
+
+
+def kvlink_plan_get_attention_items(plan: Plan) -> np.ndarray:
+    """The persistent attention's work items in run order, with the CTA of each."""
+    n = int(kvlink_plan_get_info(plan).n_attn_items)
+    out = np.zeros(n, ATTN_ITEM_DTYPE)
+    _check(lib.kvlink_plan_get_attention_items(plan.handle, out.ctypes.data, n), "kvlink_plan_get_attention_items")
     return out
 
 

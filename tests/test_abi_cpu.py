@@ -167,6 +167,52 @@ def test_attention_work_counts(K, cfg_index):
     assert info.workspace_bytes == info.n_attn_splits * 128 * (cfg.head_dim + 2) * 4
 
 
+@pytest.mark.parametrize("num_sms", [152, 37])
+@pytest.mark.parametrize("cfg_index,layout", [(1, 0), (2, 0), (2, 1), (3, 0), (3, 1), (4, 0), (5, 0)])
+def test_attention_schedule_covers_every_key_tile_once(K, cfg_index, layout, num_sms):
+    """Whatever schedule the plan picks (whole M-tiles, repaired, capped shares, gangs): per
+    (query, KV head) the M-tiles partition the query's fresh tokens; per M-tile the pieces'
+    key-tile entries partition [0, n) with n the tiles the M-tile's last row reaches
+    (interleaved layout: ceil((position + 1) / 128)); every piece runs on exactly one CTA, and
+    exactly the pieces of cut M-tiles write partials, to distinct slots."""
+    batch = W.draw_batch(W.get_config(cfg_index))
+    plan = _plan(K, batch, num_sms=num_sms, layout=layout)
+    info = K.kvlink_plan_get_info(plan)
+    items = K.kvlink_plan_get_attention_items(plan)
+    assert len(items) == info.n_attn_items
+    assert items["cta"].min() >= 0 and items["cta"].max() < info.n_attn_ctas
+    assert np.all(np.diff(items["cta"]) >= 0)          # in run order, CTA by CTA
+    cu_ctx, cu_fresh = K.kvlink_plan_get_offsets(plan)
+    fresh_pos = K.kvlink_plan_get_fresh_positions(plan)
+    mtiles = {}
+    for it in items:
+        key = (int(it["query"]), int(it["kv_head"]), int(it["tok0"]), int(it["tok1"]))
+        mtiles.setdefault(key, []).append(it)
+    slots = []
+    per_group = {}
+    for (b, g, t0, t1), pieces in mtiles.items():
+        per_group.setdefault((b, g), []).append((t0, t1))
+        ranges = sorted((int(p["entry0"]), int(p["entry1"])) for p in pieces)
+        assert ranges[0][0] == 0 and all(r[0] < r[1] for r in ranges)
+        assert all(ranges[i][1] == ranges[i + 1][0] for i in range(len(ranges) - 1))
+        assert len({(int(p["a_tiles"]), int(p["b_tile0"])) for p in pieces}) == 1
+        if layout == 0:
+            last_pos = int(fresh_pos[int(cu_fresh[b]) + t1 - 1])
+            assert ranges[-1][1] == -(-(last_pos + 1) // 128)
+        if len(pieces) > 1:
+            slots += [int(p["slot"]) for p in pieces]
+        else:
+            assert int(pieces[0]["slot"]) == -1
+    assert len(slots) == len(set(slots)) == info.n_attn_splits
+    assert min(slots, default=0) >= 0
+    for b in range(batch.cfg.batch):
+        T = int(cu_fresh[b + 1] - cu_fresh[b])
+        for g in range(batch.cfg.h_kv):
+            spans = sorted(per_group[(b, g)])
+            assert spans[0][0] == 0 and spans[-1][1] == T
+            assert all(spans[i][1] == spans[i + 1][0] for i in range(len(spans) - 1))
+
+
 def test_invalid_arguments_are_rejected_before_launch(K):
     batch = W.draw_batch(W.get_config(1))
     with pytest.raises(K.KvlinkError) as e:
