@@ -483,6 +483,9 @@ __global__ void __launch_bounds__(32 * kPlaceWarps) place_fresh_kernel(const int
                                                                        const uint4* __restrict__ v_new,
                                                                        uint4* __restrict__ cache_k,
                                                                        uint4* __restrict__ cache_v) {
+    // the attention launched after this kernel may start its prologue now (it waits for this
+    // kernel's writes before reading them)
+    asm volatile("griddepcontrol.launch_dependents;");
     // after a recorded failure, later launches skip their work
     if (*reinterpret_cast<volatile int32_t*>(&g_copy_status) != 0) return;
     const int row = blockIdx.x * kPlaceWarps + threadIdx.x / 32, lane = threadIdx.x % 32;
