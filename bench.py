@@ -59,12 +59,12 @@ KERNEL_SOURCES = {
 # Captures: `ncu --set full` of one launch per kernel, on runs of this script with one or two
 # layers (each launch does a layer's full work); the zero-copy kernels on workload 3 only.
 NCU_TRAFFIC = {
-    ("attention", 3): (237_301_760 + 8_349_696, "2227415ce887690a"),
-    ("attention", 4): (283_856_640 + 6_546_176, "2227415ce887690a"),
-    ("attention", 5): (873_828_096 + 56_577_792, "2227415ce887690a"),
-    ("reencode", 3): (102_178_560 + 113_795_072, "d3ba56d5b4506e2b"),
-    ("attention_pool_values", 3): (175_213_056 + 6_225_664, "2227415ce887690a"),
-    ("reencode_keys", 3): (40_691_456 + 25_600_000, "d3ba56d5b4506e2b"),
+    ("attention", 3): (237_865_728 + 7_885_824, "cee90bd7320fd08e"),
+    ("attention", 4): (264_504_832 + 6_526_976, "cee90bd7320fd08e"),
+    ("attention", 5): (873_054_720 + 56_700_672, "cee90bd7320fd08e"),
+    ("reencode", 3): (102_522_112 + 113_229_568, "a171595bc7e10bc7"),
+    ("attention_pool_values", 3): (174_782_720 + 6_285_056, "cee90bd7320fd08e"),
+    ("reencode_keys", 3): (40_695_552 + 25_574_400, "a171595bc7e10bc7"),
 }
 KERNEL_SOURCES["attention_pool_values"] = KERNEL_SOURCES["attention"]
 KERNEL_SOURCES["reencode_keys"] = KERNEL_SOURCES["reencode"]
