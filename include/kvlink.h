@@ -377,7 +377,9 @@ int kvlink_linked_prefill_layers(const kvlink_plan_t* plan, int32_t n_layers, co
  * idle (the ends of its grid, the gaps between launches).  When the call returns,
  * `stream` is ordered after all of its work.  The plan keeps the events it uses: calls
  * with one plan must not run concurrently.  d_cache_v NULL: zero-copy values in every layer,
- * as for kvlink_linked_prefill_layers.  Errors: as kvlink_linked_prefill_layers;
+ * as for kvlink_linked_prefill_layers.  The call may be captured in a CUDA graph on `stream`
+ * (the second stream joins the capture through the plan's events) and the graph replayed with
+ * the same results.  Errors: as kvlink_linked_prefill_layers;
  * EINVAL also when the two streams are the same. */
 int kvlink_linked_prefill_layers_overlapped(kvlink_plan_t* plan, int32_t n_layers, const void* const* d_pool_k,
                                             const void* const* d_pool_v, const void* const* d_q,

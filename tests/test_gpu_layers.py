@@ -189,3 +189,57 @@ def test_host_path_calls_with_different_layer_counts(RT):
     c, *_, h_out = results[-1]
     gk, gv = RT.bits_from_bf16(ck[len(c) - 1]), RT.bits_from_bf16(cv[len(c) - 1])
     check_query(batch, 0, lp, gk, gv, h_out[len(c) - 1].float().numpy().astype(np.float64), raw[c[-1]])
+
+
+@pytest.mark.parametrize("zero_copy", [False, True])
+def test_overlapped_call_replays_from_a_cuda_graph(RT, zero_copy):
+    """The step's call captured once in a CUDA graph (its second stream and events joined into
+    the capture) and replayed: every layer's cache and output equal a direct call's, bit for
+    bit, on two replays (the attention's merge counters keep growing across launches)."""
+    from paper_2502_16002_gb300 import kvlink as K
+    dev = torch.device("cuda:0")
+    batch = W.draw_batch(W.get_config(2))       # workload 2 cuts KV ranges: in-kernel merges
+    L = 3
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    t = {}
+    for name, seq in (("pk", []), ("pv", []), ("q", []), ("kn", []), ("vn", [])):
+        t[name] = seq
+    for layer in range(L):
+        a, b = W.pool_kv(batch, layer)
+        x, y, z = W.fresh_qkv(batch, layer)
+        for name, arr in zip(("pk", "pv", "q", "kn", "vn"), (a, b, x, y, z)):
+            t[name].append(RT.bf16_from_bits(arr, dev))
+
+    def buffers():
+        caches = [_sentinel_cache(lp) for _ in range(L)]
+        outs = [torch.full(lp.fresh_shape(batch.cfg.h_q), float("nan"), dtype=torch.bfloat16, device=dev)
+                for _ in range(L)]
+        return caches, outs
+
+    ref_c, ref_o = buffers()
+    lp.linked_prefill_layers_overlapped(t["pk"], t["pv"], t["q"], t["kn"], t["vn"], [c[0] for c in ref_c],
+                                        None if zero_copy else [c[1] for c in ref_c], ref_o)
+    torch.cuda.synchronize()
+    g_c, g_o = buffers()
+    s = torch.cuda.Stream(dev)
+    re_s = torch.cuda.Stream(dev)
+    s.wait_stream(torch.cuda.current_stream(dev))
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=s):
+        lp.linked_prefill_layers_overlapped(t["pk"], t["pv"], t["q"], t["kn"], t["vn"], [c[0] for c in g_c],
+                                            None if zero_copy else [c[1] for c in g_c], g_o, stream=s,
+                                            reencode_stream=re_s)
+    for _ in range(2):
+        for c, o in zip(g_c, g_o):
+            c[0].view(torch.int16).fill_(-1)
+            c[1].view(torch.int16).fill_(-1)
+            o.fill_(float("nan"))
+        torch.cuda.synchronize()
+        graph.replay()
+        torch.cuda.synchronize()
+        assert K.kvlink_device_status() == 0
+        for layer in range(L):
+            assert torch.equal(ref_c[layer][0].view(torch.int16), g_c[layer][0].view(torch.int16))
+            if not zero_copy:
+                assert torch.equal(ref_c[layer][1].view(torch.int16), g_c[layer][1].view(torch.int16))
+            assert torch.equal(ref_o[layer].view(torch.int16), g_o[layer].view(torch.int16))
