@@ -196,8 +196,8 @@ int kvlink_plan_get_segments(const kvlink_plan_t* plan, kvlink_segment_t* seg, i
 int kvlink_plan_get_offsets(const kvlink_plan_t* plan, int64_t* cu_ctx, int32_t* cu_fresh);
 int kvlink_plan_get_fresh_positions(const kvlink_plan_t* plan, int32_t* fresh_pos, int32_t cap);
 /* src: [cap] sources, one per position of every query (ctx_rows of them), at
- * cu_ctx[b] + position.  With a zero-copy value cache (kvlink_linked_prefill_fused with
- * d_cache_v NULL) this is where each position's value row lives.
+ * cu_ctx[b] + position.  With zero-copy values (d_cache_v NULL in the linked-prefill calls,
+ * kvlink_suffix_attention_pool_values) this is where each position's value row lives.
  * Errors: EINVAL, ECAPACITY. */
 int kvlink_plan_get_sources(const kvlink_plan_t* plan, kvlink_source_t* src, int64_t cap);
 
