@@ -282,6 +282,18 @@ class Workload:
         t_re = float(np.mean([a.elapsed_time(b_) for a, b_, _ in ev])) * 1e-3
         t_at = float(np.mean([b_.elapsed_time(c) for _, b_, c in ev])) * 1e-3
         t_re_all = timed(lambda j: K.kvlink_reencode_concat_layers(self.plan, *self.layer_ptrs, sh), k_steps)
+        # the attention launches back to back over the layers (one event pair around all of them)
+        n_b2b = k_steps * L
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(dev)
+        e0.record(stream)
+        for j in range(n_b2b):
+            l = j % L
+            K.kvlink_suffix_attention(self.plan, self.q[l].data_ptr(), None, None, self.ck[l].data_ptr(),
+                                      self.cv[l].data_ptr(), self.out[l].data_ptr(), self.ws, self.wsb, sh)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        self.t_at_b2b = e0.elapsed_time(e1) * 1e-3 / n_b2b
         assert K.kvlink_device_status() == 0
         return t_re, t_at, t_re_all
 
@@ -293,8 +305,12 @@ class Workload:
         at_tfs = cnt["attn_flops"] / t_at / 1e12
         at_frac = at_tfs / peaks["bf16_tflops"]
         default_path = not self.one_kernel and self.layout == "interleaved"
+        b2b = getattr(self, "t_at_b2b", None)
         attn_entry = {"us_per_launch": round(t_at * 1e6, 2), "TFLOP_per_s": round(at_tfs, 2),
                       "frac_bf16_burst": round(at_frac, 4),
+                      "us_per_launch_back_to_back": round(b2b * 1e6, 2) if b2b else None,
+                      "frac_bf16_burst_back_to_back": round(cnt["attn_flops"] / b2b / 1e12 / peaks["bf16_tflops"], 4)
+                      if b2b else None,
                       "frac_bf16_sustained": round(at_tfs / peaks["bf16_tflops_sustained"], 4),
                       "algorithmic_flops": cnt["attn_flops"],
                       "hbm_bound_us": round(cnt["attn_bytes"] / peaks["hbm_gbs"] / 1e3, 2),
