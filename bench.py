@@ -227,25 +227,38 @@ class Workload:
         per_layer = 1 if self.one_kernel else 2 if self.path == "two-kernel-serial" else 3
         return self.L * (per_layer + n_merge)
 
-    def timed_steps(self, n, world, clock_ms, local_rank, step=None):
+    def timed_steps(self, n, world, clock_ms, local_rank, step=None, per_step=False):
         """ms per step over n steps, CUDA events on the launching stream, barrier and synchronize
-        on both sides, max over ranks; with the clocks sampled during the timed region."""
+        on both sides, max over ranks; with the clocks sampled during the timed region.  With
+        per_step, an event is also recorded between steps and the third value is this rank's
+        per-step distribution (ms: mean, p50, p99, min, max)."""
         import torch
         step = step or self.step
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        mid = [torch.cuda.Event(enable_timing=True) for _ in range(n - 1)] if per_step else []
         with ClockSampler(local_rank, clock_ms) as clk:
             barrier(world)
             torch.cuda.synchronize(self.dev)
             clk.start()
             e0.record(self.stream)
-            for _ in range(n):
+            for i in range(n):
                 step()
+                if per_step and i < n - 1:
+                    mid[i].record(self.stream)
             e1.record(self.stream)
             torch.cuda.synchronize(self.dev)
             clk.stop()
             barrier(world)
         assert self.K.kvlink_device_status() == 0
-        return max_over_ranks(e0.elapsed_time(e1), world, self.dev) / n, clk.summary()
+        ms = max_over_ranks(e0.elapsed_time(e1), world, self.dev) / n
+        if not per_step:
+            return ms, clk.summary()
+        marks = [e0] + mid + [e1]
+        d = np.array([a.elapsed_time(b_) for a, b_ in zip(marks[:-1], marks[1:])])
+        dist = {"mean": round(float(d.mean()), 4), "p50": round(float(np.median(d)), 4),
+                "p99": round(float(np.percentile(d, 99)), 4), "min": round(float(d.min()), 4),
+                "max": round(float(d.max()), 4)}
+        return ms, clk.summary(), dist
 
     def kernel_pass(self, k_steps):
         """The step's kernels timed one launch at a time with events around each call: per layer
@@ -533,10 +546,11 @@ def run_ours(args, rank, world, local_rank, cfg_index, main=True):
     sustained = None
     if main and not args.no_sustained:
         n = int(min(5000, max(args.steps, math.ceil(1.2e3 / max(ms_per_step, 1e-3)))))
-        ms_s, clk_s = wl.timed_steps(n, world, args.clock_ms, local_rank)
+        ms_s, clk_s, dist = wl.timed_steps(n, world, args.clock_ms, local_rank, per_step=True)
         sustained = {"steps": n, "ms_per_step": round(ms_s, 4),
                      "value": round(whole_job_us_per_query(ms_s, wl.cfg.batch, world), 3), "unit": UNIT,
-                     "timed_s": round(n * ms_s / 1e3, 3), "clocks": clk_s}
+                     "timed_s": round(n * ms_s / 1e3, 3), "clocks": clk_s,
+                     "step_ms_distribution": dist}
 
     t_re, t_at, t_re_all = wl.kernel_pass(min(args.steps, 20) if main else min(args.steps, 5))
     roof, kernels = wl.roofline(t_re, t_at, t_re_all, _peaks())
