@@ -449,8 +449,8 @@ class Workload:
                 "attention_pool_values_us_per_launch": round(t_at * 1e6, 2),
                 "attention_pool_values_TFLOP_per_s": round(at_tfs, 2),
                 "attention_pool_values_frac_bf16_burst": round(at_tfs / peaks["bf16_tflops"], 4),
-                "reencode_keys_traffic": ncu_traffic("reencode_keys", self.cfg.index),
-                "attention_pool_values_traffic": ncu_traffic("attention_pool_values", self.cfg.index),
+                "reencode_keys_traffic": ncu_traffic("reencode_keys", self.cfg.index) if self.layout == "interleaved" else None,
+                "attention_pool_values_traffic": ncu_traffic("attention_pool_values", self.cfg.index) if self.layout == "interleaved" else None,
                 "launches_per_step": 3 * self.L,
                 "note": "kvlink_linked_prefill_layers_overlapped with cache_v NULL: keys re-encoded into "
                         "the linked cache, values read by the attention from the pool and v_new (no "
@@ -556,7 +556,7 @@ def run_ours(args, rank, world, local_rank, cfg_index, main=True):
     roof, kernels = wl.roofline(t_re, t_at, t_re_all, _peaks())
 
     zero_copy = None
-    if not args.no_zero_copy and not wl.one_kernel and args.layout == "interleaved":
+    if not args.no_zero_copy and not wl.one_kernel:
         zero_copy = wl.zero_copy_leg(args, world, local_rank)
 
     e2e = host_pool = None

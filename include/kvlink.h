@@ -201,6 +201,18 @@ int kvlink_plan_get_fresh_positions(const kvlink_plan_t* plan, int32_t* fresh_po
  * Errors: EINVAL, ECAPACITY. */
 int kvlink_plan_get_sources(const kvlink_plan_t* plan, kvlink_source_t* src, int64_t cap);
 
+/* Bit set in a value-group entry whose rows are fresh rows (k_new / v_new), not pool rows. */
+#define KVLINK_GROUP_FRESH (1 << 30)
+/* The plan's groups of 8 cache rows, as the zero-copy value path and the one-kernel path
+ * read them.  Query b owns entries cu_grp[b] .. cu_grp[b+1]), one per 8 cache rows
+ * (ceil(rows of b / 8)); entry m covers its cache rows 8m .. 8m+7 and holds the first
+ * source row when those 8 rows come from 8 consecutive rows of one tensor (a pool row, or
+ * KVLINK_GROUP_FRESH | a fresh row): the kernels copy such a group as one tile.  Else -1
+ * (a segment boundary inside, or the query's last, partial group): its rows are copied one
+ * by one.  grp: [cap] host int32, cu_grp: [B+1] host int32, both owned by the caller.
+ * Errors: EINVAL, ECAPACITY (cap below cu_grp[B]). */
+int kvlink_plan_get_value_groups(const kvlink_plan_t* plan, int32_t* grp, int32_t* cu_grp, int64_t cap);
+
 /* One work item of the persistent suffix attention: the fresh tokens [tok0, tok1) of query
  * `query` (query-relative) with the query heads of KV head `kv_head` (an M-tile), over the
  * entries [entry0, entry1) of the M-tile's key-tile list (entry e < a_tiles is key tile e of

@@ -264,6 +264,15 @@ int kvlink_plan_get_sources(const kvlink_plan_t* p, kvlink_source_t* src, int64_
     return KVLINK_OK;
 }
 
+static_assert(KVLINK_GROUP_FRESH == kvlink::kGrpFresh, "value-group fresh bit");
+int kvlink_plan_get_value_groups(const kvlink_plan_t* p, int32_t* grp, int32_t* cu_grp, int64_t cap) {
+    if (!p || !grp || !cu_grp) return KVLINK_EINVAL;
+    if (cap < (int64_t)p->grp_src.size()) return KVLINK_ECAPACITY;
+    std::memcpy(grp, p->grp_src.data(), p->grp_src.size() * sizeof(int32_t));
+    std::memcpy(cu_grp, p->cu_grp.data(), p->cu_grp.size() * sizeof(int32_t));
+    return KVLINK_OK;
+}
+
 int kvlink_plan_get_attention_items(const kvlink_plan_t* p, kvlink_attn_item_t* items, int32_t cap) {
     if (!p || !items) return KVLINK_EINVAL;
     if (cap < (int32_t)p->sched.size()) return KVLINK_ECAPACITY;

@@ -28,6 +28,7 @@ KVLINK_EDEVICE = -6
 KVLINK_SEG_PREFIX, KVLINK_SEG_DOC, KVLINK_SEG_LINK, KVLINK_SEG_QUESTION = 0, 1, 2, 3
 KVLINK_LAYOUT_INTERLEAVED, KVLINK_LAYOUT_LINKS_AT_END = 0, 1
 KVLINK_SRC_POOL, KVLINK_SRC_FRESH = 0, 1
+KVLINK_GROUP_FRESH = 1 << 30
 KVLINK_STATUS_WAIT_TIMEOUT, KVLINK_STATUS_COPY_TIMEOUT = 0x41, 0x21
 KVLINK_STATUS_BAD_INDEX_ATTN, KVLINK_STATUS_BAD_INDEX_COPY = 0x42, 0x22
 
@@ -95,6 +96,7 @@ def _load():
         "kvlink_plan_get_fresh_positions": (C.c_int, [P, V, C.c_int32]),
         "kvlink_plan_get_sources": (C.c_int, [P, V, C.c_int64]),
         "kvlink_plan_get_attention_items": (C.c_int, [P, V, C.c_int32]),
+        "kvlink_plan_get_value_groups": (C.c_int, [P, V, V, C.c_int64]),
         "kvlink_plan_upload": (C.c_int, [P, C.c_double, V, C.c_size_t, V]),
         "kvlink_reencode_concat": (C.c_int, [P, V, V, V, V, V]),
         "kvlink_suffix_attention": (C.c_int, [P, V, V, V, V, V, V, V, C.c_size_t, V]),
@@ -136,6 +138,7 @@ DECLARED = [
     "kvlink_reencode_concat_layers", "kvlink_plan_rebuild", "kvlink_linked_prefill_layers_overlapped",
     "kvlink_linked_prefill_layers_host", "kvlink_reencode_concat_host_pool", "kvlink_linked_prefill_layers_host_pool",
     "kvlink_selftest_wait_timeout", "kvlink_suffix_attention_pool_values", "kvlink_plan_get_attention_items",
+    "kvlink_plan_get_value_groups",
 ]
 
 # size of the static scratch used by kvlink_suffix_attention_noalloc (include/kvlink.h)
@@ -273,6 +276,18 @@ def kvlink_plan_get_attention_items(plan: Plan) -> np.ndarray:
     out = np.zeros(n, ATTN_ITEM_DTYPE)
     _check(lib.kvlink_plan_get_attention_items(plan.handle, out.ctypes.data, n), "kvlink_plan_get_attention_items")
     return out
+
+
+def kvlink_plan_get_value_groups(plan: Plan):
+    """(grp, cu_grp): the 8-row value groups of every query (entry m of query b at
+    cu_grp[b] + m: first source row, with KVLINK_GROUP_FRESH for fresh rows, or -1)."""
+    cu_ctx, _ = kvlink_plan_get_offsets(plan)
+    n = int(np.sum((np.diff(cu_ctx) + 7) // 8))
+    grp = np.zeros(n, np.int32)
+    cu = np.zeros(len(cu_ctx), np.int32)
+    _check(lib.kvlink_plan_get_value_groups(plan.handle, grp.ctypes.data, cu.ctypes.data, n),
+           "kvlink_plan_get_value_groups")
+    return grp, cu
 
 
 def kvlink_plan_upload(plan: Plan, theta: float, d_buf: int, nbytes: int, stream: int = 0) -> None:

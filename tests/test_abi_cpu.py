@@ -148,6 +148,44 @@ def test_sources_and_rows_match_oracle(K, cfg_index, layout):
             assert np.array_equal(rows[p0: p0 + n], int(sg["dst"]) - c0 + np.arange(n))
 
 
+@pytest.mark.parametrize("cfg_index", [1, 2, 3, 4, 5])
+@pytest.mark.parametrize("layout", [0, 1])
+def test_value_groups_match_sources(K, cfg_index, layout):
+    """The 8-row groups that the zero-copy value path (and the one-kernel path) copies as one
+    tile each: an entry holds the first source row exactly when its 8 cache rows read 8
+    consecutive rows of one tensor, flagged fresh for k_new / v_new rows; a group with a
+    segment boundary inside, or a query's last partial group, is -1.  Checked against the
+    per-position sources, which test_sources_and_rows_match_oracle ties to the oracle."""
+    batch = W.draw_batch(W.get_config(cfg_index))
+    plan = _plan(K, batch, layout=layout)
+    src = K.kvlink_plan_get_sources(plan)
+    cu_ctx, _ = K.kvlink_plan_get_offsets(plan)
+    grp, cu = K.kvlink_plan_get_value_groups(plan)
+    # sources in cache-row order (slot is the batch cache row of each position)
+    kind = np.empty(len(src), np.int64)
+    row = np.empty(len(src), np.int64)
+    kind[src["slot"]] = src["kind"]
+    row[src["slot"]] = src["row"]
+    runs = 0
+    for b in range(batch.cfg.batch):
+        c0, C = int(cu_ctx[b]), int(cu_ctx[b + 1] - cu_ctx[b])
+        n = (C + 7) // 8
+        assert cu[b + 1] - cu[b] == n
+        for m in range(n):
+            e = int(grp[cu[b] + m])
+            r = slice(c0 + 8 * m, c0 + 8 * m + 8)
+            whole = 8 * m + 8 <= C
+            run = whole and np.all(kind[r] == kind[r][0]) and np.array_equal(row[r], row[r][0] + np.arange(8))
+            if run:
+                flag = K.KVLINK_GROUP_FRESH if kind[r][0] == K.KVLINK_SRC_FRESH else 0
+                assert e == (int(row[r][0]) | flag), (b, m)
+                runs += 1
+            else:
+                assert e == -1, (b, m)
+    assert cu[-1] == len(grp)
+    assert runs > 0.5 * len(grp)       # documents of 64 to 512 rows: most groups are one tile
+
+
 def _items(K, plan):
     """Attention items and merge groups, read back from the plan's device-buffer image."""
     import paper_2502_16002_gb300.kvlink as KK
