@@ -418,9 +418,11 @@ static int place_fresh(const kvlink_plan_t* p, const void* k_new, const void* v_
     return check_launch("place_fresh_kernel");
 }
 
-// vs.cache_v NULL: zero-copy values, read from vs.pool_v and vs.v_new
-static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k, const ValueSource& vs,
-                            void* out, void* ws, size_t ws_bytes, cudaStream_t s) {
+// The attention's arguments (vs.cache_v NULL: zero-copy values, read from vs.pool_v and
+// vs.v_new).  The entry points that launch something before the attention check them first,
+// so that a call returning an error has launched nothing.
+static int attention_args(const kvlink_plan_t* p, const void* q, const void* cache_k, const ValueSource& vs,
+                          const void* out, const void* ws, size_t ws_bytes) {
     if (!q || !cache_k || !out) return KVLINK_EINVAL;
     if (!aligned16(q) || !aligned16(cache_k) || !aligned16(out)) return KVLINK_EINVAL;
     if (vs.cache_v ? !aligned16(vs.cache_v)
@@ -428,6 +430,13 @@ static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k
         return KVLINK_EINVAL;
     if (p->workspace_bytes > 0 && (!ws || ws_bytes < p->workspace_bytes)) return KVLINK_ECAPACITY;
     if (ws && !aligned16(ws)) return KVLINK_EINVAL;
+    return KVLINK_OK;
+}
+
+static int attention_common(const kvlink_plan_t* p, const void* q, void* cache_k, const ValueSource& vs,
+                            void* out, void* ws, size_t ws_bytes, cudaStream_t s) {
+    const int arc = attention_args(p, q, cache_k, vs, out, ws, ws_bytes);
+    if (arc) return arc;
     cudaError_t err = cudaSuccess;
     const int rc = launch_attention_tc(p->dev, (int)p->items.size(), (int)p->cu_sched.size() - 1,
                                        (int)p->merges.size(), p->cu_fresh.back(),
@@ -450,6 +459,8 @@ int kvlink_suffix_attention(const kvlink_plan_t* p, const void* q, const void* k
     if ((k_new == nullptr) != (v_new == nullptr)) return KVLINK_EINVAL;
     if (k_new && (!aligned16(k_new) || !aligned16(v_new))) return KVLINK_EINVAL;
     if (!cache_k || !cache_v) return KVLINK_EINVAL;
+    rc = attention_args(p, q, cache_k, values(cache_v, nullptr, nullptr), out, ws, ws_bytes);
+    if (rc) return rc;
     cudaStream_t s = (cudaStream_t)stream;
     if (k_new) {
         rc = place_fresh(p, k_new, v_new, cache_k, cache_v, s);
@@ -465,6 +476,8 @@ int kvlink_suffix_attention_pool_values(const kvlink_plan_t* p, const void* q, c
     if (rc) return rc;
     if (!v_new || !pool_v || !cache_k) return KVLINK_EINVAL;
     if (k_new && !aligned16(k_new)) return KVLINK_EINVAL;
+    rc = attention_args(p, q, cache_k, values(nullptr, pool_v, v_new), out, ws, ws_bytes);
+    if (rc) return rc;
     cudaStream_t s = (cudaStream_t)stream;
     if (k_new) {
         rc = place_fresh(p, k_new, nullptr, cache_k, nullptr, s);
@@ -500,10 +513,12 @@ int kvlink_linked_prefill(const kvlink_plan_t* p, const void* pool_k, const void
     if (!aligned16(pool_k) || !aligned16(pool_v) || !aligned16(k_new) || !aligned16(v_new) ||
         (cache_v && !aligned16(cache_v)))
         return KVLINK_EINVAL;
+    rc = attention_args(p, q, cache_k, values(cache_v, pool_v, v_new), out, ws, ws_bytes);
+    if (rc) return rc;
     cudaStream_t s = (cudaStream_t)stream;
     launch_reencode(p->dev, 0, (int)p->chunks.size(), p->head_dim, p->h_kv, p->num_sms, pool_k, pool_v, k_new,
                     v_new, cache_k, cache_v, s);
-    rc = check_launch("reencode_kernel (fused)");
+    rc = check_launch("reencode_kernel (with the fresh rows)");
     if (rc) return rc;
     return attention_common(p, q, cache_k, values(cache_v, pool_v, v_new), out, ws, ws_bytes, s);
 }

@@ -67,6 +67,43 @@ def test_reencode_leaves_fresh_slots_untouched(RT):
     assert not np.any(RT.bits_from_bf16(ck)[lay.kind == O.DOC] == 0x1234)
 
 
+def test_rejected_calls_launch_nothing(RT):
+    """A call that returns an error has launched nothing: the entry points that place the fresh
+    rows (or re-encode the documents) before the attention check the attention's arguments
+    first, so a misaligned q is rejected with the cache left as it was."""
+    from paper_2502_16002_gb300 import kvlink as K
+    batch = W.draw_batch(W.get_config(1))
+    dev = torch.device("cuda:0")
+    pk, pv = W.pool_kv(batch, 0)
+    q, kn, vn = W.fresh_qkv(batch, 0)
+    t = {k: RT.bf16_from_bits(v, dev) for k, v in dict(pk=pk, pv=pv, q=q, kn=kn, vn=vn).items()}
+    lp = RT.LinkedPrefill.from_batch(batch, device=dev)
+    ck, cv = lp.empty_cache()
+    out = torch.zeros(lp.fresh_shape(batch.cfg.h_q), dtype=torch.bfloat16, device=dev)
+    ws, wsb = lp.workspace.data_ptr(), lp.workspace.numel()
+    bad_q = t["q"].data_ptr() + 2                 # not 16-byte aligned
+    kn_p, vn_p, pk_p, pv_p = (t[k].data_ptr() for k in ("kn", "vn", "pk", "pv"))
+    calls = {
+        "kvlink_suffix_attention": lambda: K.kvlink_suffix_attention(
+            lp.plan, bad_q, kn_p, vn_p, ck.data_ptr(), cv.data_ptr(), out.data_ptr(), ws, wsb, 0),
+        "kvlink_suffix_attention_pool_values": lambda: K.kvlink_suffix_attention_pool_values(
+            lp.plan, bad_q, kn_p, vn_p, pv_p, ck.data_ptr(), out.data_ptr(), ws, wsb, 0),
+        "kvlink_linked_prefill": lambda: K.kvlink_linked_prefill(
+            lp.plan, pk_p, pv_p, bad_q, kn_p, vn_p, ck.data_ptr(), cv.data_ptr(), out.data_ptr(), ws, wsb, 0),
+    }
+    for name, call in calls.items():
+        ck.view(torch.int16).fill_(0x1234)
+        cv.view(torch.int16).fill_(0x1234)
+        torch.cuda.synchronize()
+        with pytest.raises(K.KvlinkError) as e:
+            call()
+        assert e.value.code == K.KVLINK_EINVAL, name
+        torch.cuda.synchronize()
+        assert bool(torch.all(ck.view(torch.int16) == 0x1234)), name
+        assert bool(torch.all(cv.view(torch.int16) == 0x1234)), name
+    assert K.kvlink_device_status() == 0
+
+
 # ----------------------------------------------------------------- full-size workloads, sampled
 
 @pytest.mark.parametrize("layer", [0, 31])
